@@ -1,0 +1,216 @@
+/*
+ * ebd.h -- C ABI of the Early-Bird (EB) decoding step on one GB300 GPU.
+ *
+ * One call of ebd_step() performs one denoising step of EB decoding over
+ * the active window of every sequence in a batch (paper arxiv 2609.16450):
+ *
+ *   1. window attention: the window's queries attend bidirectionally to the
+ *      cached prefix keys/values followed by the window's own keys/values
+ *      (Sec. 3 "bidirectional Transformer"; Sec. 6.3 "Effect of KV-Cache
+ *      Configuration", prefix cache at the block boundary);
+ *   2. the LM head l = W_lm h for every window row, reduced on the fly to
+ *      the per-position statistics of the softmax (App. B Eq. app-confidence:
+ *      kappa = max_v p(v); Sec. 5.1: normalized entropy H~ and top-1 token
+ *      x_hat; Sec. 5.2: top-1/top-2 gap Delta); logits never reach memory;
+ *   3. the EB decision (App. E, algorithm "Inference with LBS Block
+ *      Selection and LPS Parallel Commit"): when a sequence has no active
+ *      block, the LBS router (Sec. 5.1, App. C.1 Eq. lbs_feat) scores its
+ *      masked rows and the filters (EOS removal, max gap g_max, min tokens
+ *      L_min with the first-L_B fallback) select the block; the LPS router
+ *      (Sec. 5.2, App. D.1) scores the block's masked rows; the union accept
+ *      rule (kappa >= tau or p_psi > tau_psi), the anti-stall fallback and the
+ *      parallel commit update tokens, mask and block state in place.
+ *
+ * Conventions
+ *   - bf16 tensors are passed as uint16_t bit patterns, row-major, densely
+ *     packed, 16-byte aligned.  Every pointer in ebd_step_args is a DEVICE
+ *     pointer on the handle's device, owned by the caller, except in
+ *     ebd_step_host() (see there).
+ *   - The handle owns the router weights, the folded token-branch table,
+ *     a workspace and a device status word; nothing else is allocated per
+ *     call.  One handle serves one stream at a time; it is not thread-safe.
+ *   - Functions that take a stream only enqueue work (asynchronous); they
+ *     check their arguments on the host first and return an error without
+ *     enqueuing anything when a check fails.  Failures detected on the
+ *     device (a bounded wait that gave up, a non-finite logit statistic, an
+ *     inconsistent row count) are recorded in the status word and reported
+ *     by ebd_sync_status().
+ *   - Supported shapes: d_model % 8 == 0, d_base % 8 == 0, head_dim in
+ *     {64, 128}, n_heads_q % n_heads_kv == 0, 1 <= window rows of a
+ *     sequence <= max_window <= 64, gen_len >= max_window, vocab >= 2,
+ *     rows of a step <= max_rows <= 4096.  Anything else returns
+ *     EBD_ERR_UNSUPPORTED.
+ *   - stream arguments are cudaStream_t values passed as void* (NULL = the
+ *     legacy default stream).
+ */
+#ifndef EBD_H_
+#define EBD_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct ebd_handle ebd_handle;
+
+typedef int32_t ebd_status;
+#define EBD_OK 0
+#define EBD_ERR_INVALID_ARG (-1) /* null pointer, bad size, misalignment    */
+#define EBD_ERR_UNSUPPORTED (-2) /* shape outside the supported set          */
+#define EBD_ERR_CUDA (-3)        /* a CUDA runtime/driver call failed        */
+#define EBD_ERR_TIMEOUT (-4)     /* a device-side bounded wait gave up       */
+#define EBD_ERR_NONFINITE (-5)   /* NaN/Inf logit statistic; row not committed */
+#define EBD_ERR_STATE (-6)       /* call order: e.g. LBS needs a bound W_e   */
+
+/* debug_flags bits (tests only) */
+#define EBD_DEBUG_FORCE_TIMEOUT 1 /* LM-head kernel waits on a barrier that
+                                     nothing completes, with a 20 ms limit */
+
+typedef struct {
+  /* backbone shapes */
+  int32_t d_model;     /* hidden size d                                     */
+  int32_t vocab;       /* |V|                                               */
+  int32_t n_heads_q;   /* query heads Hq                                    */
+  int32_t n_heads_kv;  /* key/value heads Hkv (GQA when < Hq)               */
+  int32_t head_dim;    /* D                                                 */
+  int32_t d_base;      /* width of the frozen token embedding W_e           */
+  /* capacity of the handle */
+  int32_t max_batch;   /* sequences per step                                */
+  int32_t max_window;  /* window rows per sequence (<= 64)                  */
+  int32_t max_rows;    /* window rows per step, all sequences (<= 4096)     */
+  int32_t max_prefix;  /* P_max: second dimension of the K/V cache          */
+  /* EB hyper-parameters (App. F) */
+  int32_t gen_len;     /* L: rows of the LBS positional table E_pos         */
+  int32_t g_max;       /* max gap between consecutive block members (5)     */
+  int32_t l_min;       /* min block size (8 LLaDA/Dream, 16 LLaDA-1.5)      */
+  int32_t l_b;         /* min-tokens fallback block size (32)               */
+  int32_t eos_id;      /* token id removed from LBS candidates              */
+  int32_t lps_enabled; /* 1: union accept with LPS; 0: LBS + threshold only */
+  float tau;           /* confidence threshold (0.9)                        */
+  float tau_psi;       /* LPS acceptance threshold (0.89 / 0.90 / 0.87)     */
+  uint64_t seed;       /* seed of the routers' random init                  */
+  int32_t debug_flags; /* EBD_DEBUG_* (tests); 0 in normal use              */
+  int32_t reserved;
+} ebd_config;
+
+typedef struct {
+  int32_t batch;              /* B <= max_batch                                  */
+  int32_t rows;               /* R = cu_rows[B] <= max_rows (host copy)          */
+  const int32_t* cu_rows;     /* [B+1] window row offsets, cu_rows[0] = 0        */
+  const int32_t* prefix_len;  /* [B] cached prefix length, <= max_prefix         */
+  const int32_t* row_pos;     /* [R] absolute position of each window row,
+                                 strictly increasing within a sequence         */
+  const uint16_t* hidden;     /* [R][d_model] bf16 final hidden states           */
+  const uint16_t* q;          /* [R][Hq][D] bf16 window queries                  */
+  const uint16_t* k_win;      /* [R][Hkv][D] bf16 window keys                    */
+  const uint16_t* v_win;      /* [R][Hkv][D] bf16 window values                  */
+  const uint16_t* k_cache;    /* [B][max_prefix][Hkv][D] bf16 cached prefix keys */
+  const uint16_t* v_cache;    /* [B][max_prefix][Hkv][D] bf16 cached values      */
+  const uint16_t* w_lm;       /* [vocab][d_model] bf16 LM-head weight            */
+  /* decode state, read and updated in place */
+  int32_t* tokens;            /* [R] token ids; committed rows get x_hat         */
+  uint8_t* mask;              /* [R] 1 = [MASK]; committed rows become 0         */
+  uint8_t* in_block;          /* [R] 1 = member of the active block B            */
+  int32_t* blk_meta;          /* [B][2] {b = min position of B, |B| at selection};
+                                 |B| = 0 means no active block                 */
+  /* outputs; any of them may be NULL */
+  float* attn_out;            /* [R][Hq][D] fp32 attention output                */
+  float* conf;                /* [R] kappa                                       */
+  float* entropy;             /* [R] H in nats                                   */
+  float* ent_norm;            /* [R] H~ = H / ln(vocab)                          */
+  float* gap;                 /* [R] Delta = p(top1) - p(top2)                   */
+  int32_t* argmax;            /* [R] x_hat (lowest index on ties)                */
+  float* lbs_logit;           /* [R] O_phi where LBS ran, NaN elsewhere          */
+  float* lps_prob;            /* [R] p_psi where LPS scored, NaN elsewhere       */
+  uint8_t* accepted;          /* [R] 1 = committed this step                     */
+} ebd_step_args;
+
+/* Creates a handle on the current CUDA device: validates *cfg, allocates the
+ * router weights (random-init from cfg->seed, see ebd_router_init_host),
+ * the workspace and the status word.  On failure *out is NULL. */
+ebd_status ebd_create(const ebd_config* cfg, ebd_handle** out);
+
+/* Frees everything the handle owns (never caller memory).  NULL-safe.
+ * Synchronises the device first. */
+void ebd_destroy(ebd_handle* h);
+
+/* Binds the frozen token embedding W_e [vocab][d_base] bf16 (device,
+ * caller-owned; it must stay valid while bound) and folds the LBS token
+ * branch: table[v] = W_tok W_e[v] (App. C.1 "Token branch"; the projection
+ * is linear, so it is applied to every vocabulary row once instead of to the
+ * gathered rows of every step).  Must precede any step in which LBS runs;
+ * ebd_import_weights() re-folds with the bound table.  Enqueued on stream. */
+ebd_status ebd_bind_embedding(ebd_handle* h, const uint16_t* w_emb, void* stream);
+
+/* One EB decoding step (see top of file).  Enqueue only. */
+ebd_status ebd_step(ebd_handle* h, const ebd_step_args* a, void* stream);
+
+/* Same step with the per-step tensors in HOST memory (pinned memory gives
+ * asynchronous copies): cu_rows, prefix_len, row_pos, hidden, q, k_win,
+ * v_win, tokens, mask, in_block, blk_meta and every non-NULL output are
+ * host pointers; w_lm, k_cache and v_cache stay device pointers (resident
+ * model weights and cache).  The handle copies the inputs to its own device
+ * staging, runs the step and copies state and outputs back, all on
+ * `stream`; the host buffers must stay valid until the stream reaches that
+ * point (e.g. ebd_sync_status).  Enqueue only. */
+ebd_status ebd_step_host(ebd_handle* h, const ebd_step_args* a, void* stream);
+
+/* Only the decision (step 3) on caller-provided statistics: reads
+ * a->conf, a->ent_norm, a->gap, a->argmax (device, [R]) as INPUTS, plus
+ * cu_rows, row_pos and the decode state; writes the state, lbs_logit,
+ * lps_prob and accepted.  hidden, q, k/v, w_lm and attn_out are ignored. */
+ebd_status ebd_decide(ebd_handle* h, const ebd_step_args* a, void* stream);
+
+/* Only step 2 (LM head + statistics) for a->rows rows of a->hidden:
+ * writes conf, entropy, ent_norm, gap, argmax (any may be NULL). */
+ebd_status ebd_lm_stats(ebd_handle* h, const ebd_step_args* a, void* stream);
+
+/* Only step 1 (window attention): writes a->attn_out. */
+ebd_status ebd_attention(ebd_handle* h, const ebd_step_args* a, void* stream);
+
+/* Synchronises `stream`, returns the first device-side failure recorded
+ * since the last call (EBD_OK if none) and clears it. */
+ebd_status ebd_sync_status(ebd_handle* h, void* stream);
+
+/* Router weights as one bf16 blob, tensors row-major in this order:
+ * LBS  ent1.w[64][1] ent1.b[64] ent2.w[64][64] ent2.b[64] ent_ln.g[64]
+ *      ent_ln.b[64] tok.w[64][d_base] tok.b[64] comb.w[128][128] comb.b[128]
+ *      pos[gen_len][128], then for l = 0, 1: qkv.w[384][128] qkv.b[384]
+ *      out.w[128][128] out.b[128] ln1.g[128] ln1.b[128] ff1.w[256][128]
+ *      ff1.b[256] ff2.w[128][256] ff2.b[128] ln2.g[128] ln2.b[128],
+ *      head.w[1][128] head.b[1];
+ * LPS  in.w[32][5] in.b[32] in_ln.g[32] in_ln.b[32], then for l = 0, 1:
+ *      ln1.g[32] ln1.b[32] qkv.w[96][32] qkv.b[96] out.w[32][32] out.b[32]
+ *      ln2.g[32] ln2.b[32] ff1.w[64][32] ff1.b[64] ff2.w[32][64] ff2.b[32],
+ *      head.w[1][32] head.b[1].
+ * (qkv rows: query, key, value blocks; head h uses rows h*dh..h*dh+dh-1 of
+ * each block.)  With host == NULL only *bytes is set.  Synchronous. */
+ebd_status ebd_export_weights(const ebd_handle* h, void* host, size_t* bytes);
+ebd_status ebd_import_weights(ebd_handle* h, const void* host, size_t bytes);
+
+/* The random init of ebd_create() computed on the host, without any CUDA
+ * call: Linear weights and biases ~ U(-1/sqrt(fan_in), +1/sqrt(fan_in)),
+ * LayerNorm gains 1 and biases 0, E_pos ~ U(-0.02*sqrt(3), +0.02*sqrt(3)),
+ * from SplitMix64 used as a counter-based generator: with
+ * G = 0x9E3779B97F4A7C15 and mix() the SplitMix64 output function,
+ * key_t = mix(seed ^ ((t+1)*G)) for the t-th tensor of the blob order, and
+ * element i draws u = (mix(key_t + (i+1)*G) >> 40) * 2^-24, then
+ * w = bf16_rne((2u - 1) * bound) in float32.  With host == NULL only
+ * *bytes is set. */
+ebd_status ebd_router_init_host(const ebd_config* cfg, void* host, size_t* bytes);
+
+/* Number of bf16 elements of the weight blob for cfg. */
+size_t ebd_weight_count(const ebd_config* cfg);
+
+/* Last error message of the handle (never NULL; "" if none). */
+const char* ebd_last_error(const ebd_handle* h);
+
+/* Library version string. */
+const char* ebd_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* EBD_H_ */

@@ -1,0 +1,876 @@
+// Host side of the C ABI declared in include/ebd.h.
+#include <cudaTypedefs.h>
+
+#include <cmath>
+#include <cstdio>
+#include <cstring>
+#include <string>
+#include <vector>
+
+#include "ebd.h"
+#include "internal.h"
+
+namespace ebd {
+cudaError_t decide_configure();
+cudaError_t attn_configure();
+cudaError_t lm_configure();
+cudaError_t launch_merge_stats(const float4* part_f, const int* part_i, int rows, int grid,
+                               int V, float inv_log_v, float* conf, float* entropy,
+                               float* ent_norm, float* gap, int* argmax, int* status,
+                               cudaStream_t st);
+}  // namespace ebd
+
+using namespace ebd;
+
+namespace {
+
+constexpr uint64_t kLimitNs = 1000ull * 1000 * 1000;  // 1 s per device-side wait
+constexpr int kMaxSplits = 8;
+
+// ------------------------------------------------------------------ router layout
+struct TensorDesc {
+  std::string name;
+  int rows, cols;  // row-major [rows][cols]; vectors have rows = 1
+  int kind;        // 0 linear (fan_in), 1 ones, 2 zeros, 3 positional
+  int fan_in;
+};
+
+std::vector<TensorDesc> router_layout(int d_base, int gen_len) {
+  std::vector<TensorDesc> t;
+  auto lin = [&](const std::string& n, int o, int i) {
+    t.push_back({n + ".w", o, i, 0, i});
+    t.push_back({n + ".b", 1, o, 0, i});
+  };
+  auto ln = [&](const std::string& n, int d) {
+    t.push_back({n + ".g", 1, d, 1, 0});
+    t.push_back({n + ".b", 1, d, 2, 0});
+  };
+  lin("lbs.ent1", 64, 1);
+  lin("lbs.ent2", 64, 64);
+  ln("lbs.ent_ln", 64);
+  lin("lbs.tok", 64, d_base);
+  lin("lbs.comb", 128, 128);
+  t.push_back({"lbs.pos", gen_len, 128, 3, 0});
+  for (int l = 0; l < 2; ++l) {
+    const std::string p = "lbs.l" + std::to_string(l);
+    lin(p + ".qkv", 384, 128);
+    lin(p + ".out", 128, 128);
+    ln(p + ".ln1", 128);
+    lin(p + ".ff1", 256, 128);
+    lin(p + ".ff2", 128, 256);
+    ln(p + ".ln2", 128);
+  }
+  lin("lbs.head", 1, 128);
+  lin("lps.in", 32, 5);
+  ln("lps.in_ln", 32);
+  for (int l = 0; l < 2; ++l) {
+    const std::string p = "lps.l" + std::to_string(l);
+    ln(p + ".ln1", 32);
+    lin(p + ".qkv", 96, 32);
+    lin(p + ".out", 32, 32);
+    ln(p + ".ln2", 32);
+    lin(p + ".ff1", 64, 32);
+    lin(p + ".ff2", 32, 64);
+  }
+  lin("lps.head", 1, 32);
+  return t;
+}
+
+size_t layout_count(const std::vector<TensorDesc>& t) {
+  size_t n = 0;
+  for (const auto& x : t) n += static_cast<size_t>(x.rows) * x.cols;
+  return n;
+}
+
+// SplitMix64 output function (Steele, Lea & Flood 2014)
+inline uint64_t mix64(uint64_t z) {
+  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+  z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+  return z ^ (z >> 31);
+}
+
+inline uint16_t f32_to_bf16_rne(float f) {
+  uint32_t u;
+  std::memcpy(&u, &f, 4);
+  u += 0x7FFFu + ((u >> 16) & 1u);
+  return static_cast<uint16_t>(u >> 16);
+}
+inline float bf16_to_f32(uint16_t b) {
+  uint32_t u = static_cast<uint32_t>(b) << 16;
+  float f;
+  std::memcpy(&f, &u, 4);
+  return f;
+}
+
+void router_init(uint64_t seed, const std::vector<TensorDesc>& layout, uint16_t* out) {
+  const uint64_t G = 0x9E3779B97F4A7C15ull;
+  size_t off = 0;
+  for (size_t ti = 0; ti < layout.size(); ++ti) {
+    const TensorDesc& t = layout[ti];
+    const size_t n = static_cast<size_t>(t.rows) * t.cols;
+    if (t.kind == 1) {
+      for (size_t i = 0; i < n; ++i) out[off + i] = 0x3F80;
+    } else if (t.kind == 2) {
+      for (size_t i = 0; i < n; ++i) out[off + i] = 0;
+    } else {
+      const float bound = t.kind == 0 ? 1.0f / std::sqrt(static_cast<float>(t.fan_in))
+                                      : 0.02f * std::sqrt(3.0f);
+      const uint64_t key = mix64(seed ^ ((static_cast<uint64_t>(ti) + 1) * G));
+      for (size_t i = 0; i < n; ++i) {
+        const uint64_t z = mix64(key + (static_cast<uint64_t>(i) + 1) * G);
+        const float u = static_cast<float>(z >> 40) * (1.0f / 16777216.0f);
+        const float v = 2.0f * u - 1.0f;
+        out[off + i] = f32_to_bf16_rne(v * bound);
+      }
+    }
+    off += n;
+  }
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 get_encode() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  if (fn == nullptr) {
+    void* ptr = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(ptr);
+  }
+  return fn;
+}
+
+bool encode_bf16(CUtensorMap* m, const void* base, int rank, const uint64_t* dims,
+                 const uint64_t* strides_bytes, const uint32_t* box) {
+  auto fn = get_encode();
+  if (fn == nullptr) return false;
+  cuuint64_t gd[5], gs[4];
+  cuuint32_t bx[5], es[5];
+  for (int i = 0; i < rank; ++i) {
+    gd[i] = dims[i];
+    bx[i] = box[i];
+    es[i] = 1;
+  }
+  for (int i = 0; i < rank - 1; ++i) gs[i] = strides_bytes[i];
+  CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, static_cast<cuuint32_t>(rank),
+                  const_cast<void*>(base), gd, gs, bx, es, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                  CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+}  // namespace
+
+struct ebd_handle {
+  ebd_config cfg{};
+  int device = 0, num_sms = 0;
+  std::string err;
+  std::vector<TensorDesc> layout;
+  std::vector<uint16_t> h_blob;
+  uint16_t* d_blob = nullptr;
+  uint8_t* d_image = nullptr;
+  RouterImage img{};
+  float* d_tok = nullptr;
+  const uint16_t* w_emb = nullptr;
+  float4* part_f = nullptr;
+  int* part_i = nullptr;
+  int grid_lm = 0;
+  float* attn_part = nullptr;
+  int* tickets = nullptr;
+  int attn_splits = 1, attn_max_qtiles = 1;
+  int* d_status = nullptr;
+  uint8_t* staging = nullptr;
+  size_t staging_bytes = 0;
+};
+
+namespace {
+
+ebd_status fail(ebd_handle* h, ebd_status code, const std::string& msg) {
+  if (h) h->err = msg;
+  return code;
+}
+ebd_status cuda_fail(ebd_handle* h, cudaError_t e, const char* what) {
+  return fail(h, EBD_ERR_CUDA, std::string(what) + ": " + cudaGetErrorString(e));
+}
+
+ebd_status validate_config(const ebd_config* c, std::string& why) {
+  auto bad = [&](const char* m) {
+    why = m;
+    return EBD_ERR_UNSUPPORTED;
+  };
+  if (c->d_model <= 0 || c->d_model % 8) return bad("d_model must be a positive multiple of 8");
+  if (c->d_base <= 0 || c->d_base % 8) return bad("d_base must be a positive multiple of 8");
+  if (c->vocab < 2) return bad("vocab must be >= 2");
+  if (c->head_dim != 64 && c->head_dim != 128) return bad("head_dim must be 64 or 128");
+  if (c->n_heads_kv <= 0 || c->n_heads_q <= 0 || c->n_heads_q % c->n_heads_kv)
+    return bad("n_heads_q must be a positive multiple of n_heads_kv");
+  if (c->max_batch <= 0 || c->max_batch > 65535) return bad("max_batch out of range");
+  if (c->max_window <= 0 || c->max_window > kMaxWindow) return bad("max_window must be 1..64");
+  if (c->max_rows <= 0 || c->max_rows > 4096) return bad("max_rows must be 1..4096");
+  if (c->max_prefix < 0) return bad("max_prefix must be >= 0");
+  if (c->gen_len < c->max_window) return bad("gen_len must be >= max_window");
+  if (c->g_max < 0 || c->l_min < 0 || c->l_b < 0) return bad("g_max, l_min, l_b must be >= 0");
+  if (!(c->tau == c->tau) || !(c->tau_psi == c->tau_psi)) return bad("tau/tau_psi is NaN");
+  return EBD_OK;
+}
+
+ebd_status check_device(ebd_handle* h) {
+  int dev = -1;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_fail(h, e, "cudaGetDevice");
+  if (dev != h->device) return fail(h, EBD_ERR_INVALID_ARG, "current device differs from the handle's");
+  return EBD_OK;
+}
+
+// Builds the decision kernel's weight image from the host blob.
+ebd_status upload_router(ebd_handle* h) {
+  const auto& L = h->layout;
+  std::vector<size_t> off(L.size());
+  {
+    size_t o = 0;
+    for (size_t i = 0; i < L.size(); ++i) {
+      off[i] = o;
+      o += static_cast<size_t>(L[i].rows) * L[i].cols;
+    }
+  }
+  auto find = [&](const std::string& n) -> size_t {
+    for (size_t i = 0; i < L.size(); ++i)
+      if (L[i].name == n) return i;
+    return static_cast<size_t>(-1);
+  };
+  std::vector<uint8_t> img;
+  auto align = [&]() { img.resize((img.size() + 255) / 256 * 256); };
+  auto put_f32 = [&](const std::string& n) -> size_t {
+    align();
+    const size_t i = find(n);
+    const size_t cnt = static_cast<size_t>(L[i].rows) * L[i].cols;
+    const size_t at = img.size();
+    img.resize(at + cnt * 4);
+    float* dst = reinterpret_cast<float*>(img.data() + at);
+    for (size_t k = 0; k < cnt; ++k) dst[k] = bf16_to_f32(h->h_blob[off[i] + k]);
+    return at;
+  };
+  // transposed [cols][rows] of a [rows][cols] matrix, bf16 or fp32
+  auto put_t = [&](const std::string& n, bool as_f32) -> size_t {
+    align();
+    const size_t i = find(n);
+    const int R = L[i].rows, C = L[i].cols;
+    const size_t at = img.size();
+    img.resize(at + static_cast<size_t>(R) * C * (as_f32 ? 4 : 2));
+    for (int r = 0; r < R; ++r)
+      for (int c = 0; c < C; ++c) {
+        const uint16_t v = h->h_blob[off[i] + static_cast<size_t>(r) * C + c];
+        if (as_f32)
+          reinterpret_cast<float*>(img.data() + at)[static_cast<size_t>(c) * R + r] = bf16_to_f32(v);
+        else
+          reinterpret_cast<uint16_t*>(img.data() + at)[static_cast<size_t>(c) * R + r] = v;
+      }
+    return at;
+  };
+  auto put_raw = [&](const std::string& n) -> size_t {  // bf16 as stored
+    align();
+    const size_t i = find(n);
+    const size_t cnt = static_cast<size_t>(L[i].rows) * L[i].cols;
+    const size_t at = img.size();
+    img.resize(at + cnt * 2);
+    std::memcpy(img.data() + at, h->h_blob.data() + off[i], cnt * 2);
+    return at;
+  };
+  struct {
+    size_t ent1_w, ent1_b, ent2_b, ent_ln_g, ent_ln_b, tok_b, comb_b, head_w, head_b, ent2_t,
+        comb_t, pos;
+    size_t lq[2][12];
+    size_t in_t, in_b, in_ln_g, in_ln_b, lh_w, lh_b;
+    size_t pq[2][12];
+  } o{};
+  o.ent1_w = put_f32("lbs.ent1.w");
+  o.ent1_b = put_f32("lbs.ent1.b");
+  o.ent2_b = put_f32("lbs.ent2.b");
+  o.ent_ln_g = put_f32("lbs.ent_ln.g");
+  o.ent_ln_b = put_f32("lbs.ent_ln.b");
+  o.tok_b = put_f32("lbs.tok.b");
+  o.comb_b = put_f32("lbs.comb.b");
+  o.head_w = put_f32("lbs.head.w");
+  o.head_b = put_f32("lbs.head.b");
+  o.ent2_t = put_t("lbs.ent2.w", false);
+  o.comb_t = put_t("lbs.comb.w", false);
+  o.pos = put_raw("lbs.pos");
+  for (int l = 0; l < 2; ++l) {
+    const std::string p = "lbs.l" + std::to_string(l);
+    o.lq[l][0] = put_t(p + ".qkv.w", false);
+    o.lq[l][1] = put_t(p + ".out.w", false);
+    o.lq[l][2] = put_t(p + ".ff1.w", false);
+    o.lq[l][3] = put_t(p + ".ff2.w", false);
+    o.lq[l][4] = put_f32(p + ".qkv.b");
+    o.lq[l][5] = put_f32(p + ".out.b");
+    o.lq[l][6] = put_f32(p + ".ff1.b");
+    o.lq[l][7] = put_f32(p + ".ff2.b");
+    o.lq[l][8] = put_f32(p + ".ln1.g");
+    o.lq[l][9] = put_f32(p + ".ln1.b");
+    o.lq[l][10] = put_f32(p + ".ln2.g");
+    o.lq[l][11] = put_f32(p + ".ln2.b");
+  }
+  o.in_t = put_t("lps.in.w", true);
+  o.in_b = put_f32("lps.in.b");
+  o.in_ln_g = put_f32("lps.in_ln.g");
+  o.in_ln_b = put_f32("lps.in_ln.b");
+  o.lh_w = put_f32("lps.head.w");
+  o.lh_b = put_f32("lps.head.b");
+  for (int l = 0; l < 2; ++l) {
+    const std::string p = "lps.l" + std::to_string(l);
+    o.pq[l][0] = put_t(p + ".qkv.w", false);
+    o.pq[l][1] = put_t(p + ".out.w", false);
+    o.pq[l][2] = put_t(p + ".ff1.w", false);
+    o.pq[l][3] = put_t(p + ".ff2.w", false);
+    o.pq[l][4] = put_f32(p + ".qkv.b");
+    o.pq[l][5] = put_f32(p + ".out.b");
+    o.pq[l][6] = put_f32(p + ".ff1.b");
+    o.pq[l][7] = put_f32(p + ".ff2.b");
+    o.pq[l][8] = put_f32(p + ".ln1.g");
+    o.pq[l][9] = put_f32(p + ".ln1.b");
+    o.pq[l][10] = put_f32(p + ".ln2.g");
+    o.pq[l][11] = put_f32(p + ".ln2.b");
+  }
+  align();
+  if (h->d_image) cudaFree(h->d_image);
+  h->d_image = nullptr;
+  cudaError_t e = cudaMalloc(&h->d_image, img.size());
+  if (e != cudaSuccess) return cuda_fail(h, e, "cudaMalloc(router image)");
+  e = cudaMemcpy(h->d_image, img.data(), img.size(), cudaMemcpyHostToDevice);
+  if (e != cudaSuccess) return cuda_fail(h, e, "cudaMemcpy(router image)");
+  e = cudaMemcpy(h->d_blob, h->h_blob.data(), h->h_blob.size() * 2, cudaMemcpyHostToDevice);
+  if (e != cudaSuccess) return cuda_fail(h, e, "cudaMemcpy(router blob)");
+  uint8_t* B = h->d_image;
+  auto F = [&](size_t x) { return reinterpret_cast<const float*>(B + x); };
+  auto H = [&](size_t x) { return reinterpret_cast<const __nv_bfloat16*>(B + x); };
+  RouterImage& w = h->img;
+  w.ent1_w = F(o.ent1_w); w.ent1_b = F(o.ent1_b); w.ent2_b = F(o.ent2_b);
+  w.ent_ln_g = F(o.ent_ln_g); w.ent_ln_b = F(o.ent_ln_b); w.tok_b = F(o.tok_b);
+  w.comb_b = F(o.comb_b); w.head_w = F(o.head_w); w.head_b = F(o.head_b);
+  w.ent2_t = H(o.ent2_t); w.comb_t = H(o.comb_t); w.pos = H(o.pos);
+  for (int l = 0; l < 2; ++l) {
+    w.lbs[l] = {H(o.lq[l][0]), H(o.lq[l][1]), H(o.lq[l][2]), H(o.lq[l][3]), F(o.lq[l][4]),
+                F(o.lq[l][5]), F(o.lq[l][6]), F(o.lq[l][7]), F(o.lq[l][8]), F(o.lq[l][9]),
+                F(o.lq[l][10]), F(o.lq[l][11])};
+    w.lps[l] = {H(o.pq[l][0]), H(o.pq[l][1]), H(o.pq[l][2]), H(o.pq[l][3]), F(o.pq[l][4]),
+                F(o.pq[l][5]), F(o.pq[l][6]), F(o.pq[l][7]), F(o.pq[l][8]), F(o.pq[l][9]),
+                F(o.pq[l][10]), F(o.pq[l][11])};
+  }
+  w.in_t = F(o.in_t); w.in_b = F(o.in_b); w.in_ln_g = F(o.in_ln_g); w.in_ln_b = F(o.in_ln_b);
+  w.lps_head_w = F(o.lh_w); w.lps_head_b = F(o.lh_b);
+  w.tok_table = h->d_tok;
+  return EBD_OK;
+}
+
+ebd_status fold(ebd_handle* h, cudaStream_t st) {
+  if (h->w_emb == nullptr) return EBD_OK;
+  size_t tok_off = 0;
+  for (const auto& t : h->layout) {
+    if (t.name == "lbs.tok.w") break;
+    tok_off += static_cast<size_t>(t.rows) * t.cols;
+  }
+  cudaError_t e = launch_fold_tok(reinterpret_cast<const __nv_bfloat16*>(h->d_blob + tok_off),
+                                  reinterpret_cast<const __nv_bfloat16*>(h->w_emb), h->d_tok,
+                                  h->cfg.vocab, h->cfg.d_base, st);
+  if (e != cudaSuccess) return cuda_fail(h, e, "fold kernel");
+  return EBD_OK;
+}
+
+ebd_status check_args(ebd_handle* h, const ebd_step_args* a, bool need_attn, bool need_lm,
+                      bool need_state) {
+  if (a == nullptr) return fail(h, EBD_ERR_INVALID_ARG, "args is NULL");
+  const ebd_config& c = h->cfg;
+  if (a->batch < 0 || a->batch > c.max_batch) return fail(h, EBD_ERR_INVALID_ARG, "batch out of range");
+  if (a->rows < 0 || a->rows > c.max_rows) return fail(h, EBD_ERR_INVALID_ARG, "rows out of range");
+  if (a->rows > a->batch * c.max_window)
+    return fail(h, EBD_ERR_INVALID_ARG, "rows exceed batch * max_window");
+  if (need_state) {
+    if (!a->cu_rows || !a->row_pos || !a->tokens || !a->mask || !a->in_block || !a->blk_meta)
+      return fail(h, EBD_ERR_INVALID_ARG, "cu_rows/row_pos/tokens/mask/in_block/blk_meta must be set");
+  }
+  if (need_lm) {
+    if (!a->hidden || !a->w_lm) return fail(h, EBD_ERR_INVALID_ARG, "hidden and w_lm must be set");
+    if (!aligned(a->hidden, 16) || !aligned(a->w_lm, 16))
+      return fail(h, EBD_ERR_INVALID_ARG, "hidden and w_lm must be 16-byte aligned");
+  }
+  if (need_attn) {
+    if (!a->cu_rows || !a->prefix_len || !a->q || !a->k_win || !a->v_win || !a->attn_out ||
+        (c.max_prefix > 0 && (!a->k_cache || !a->v_cache)))
+      return fail(h, EBD_ERR_INVALID_ARG, "attention needs cu_rows, prefix_len, q, k/v and attn_out");
+    if (!aligned(a->k_win, 16) || !aligned(a->v_win, 16) || !aligned(a->q, 16) ||
+        !aligned(a->attn_out, 16) ||
+        (c.max_prefix > 0 && (!aligned(a->k_cache, 16) || !aligned(a->v_cache, 16))))
+      return fail(h, EBD_ERR_INVALID_ARG, "q/k/v/attn_out must be 16-byte aligned");
+  }
+  return EBD_OK;
+}
+
+ebd_status run_attention(ebd_handle* h, const ebd_step_args* a, cudaStream_t st) {
+  const ebd_config& c = h->cfg;
+  const int D = c.head_dim, Hkv = c.n_heads_kv;
+  CUtensorMap kc, vc, kw, vw;
+  const uint64_t R = static_cast<uint64_t>(a->rows);
+  const uint64_t Pm = static_cast<uint64_t>(c.max_prefix > 0 ? c.max_prefix : 1);
+  const void* kcp = c.max_prefix > 0 ? a->k_cache : a->k_win;  // any valid pointer if no cache
+  const void* vcp = c.max_prefix > 0 ? a->v_cache : a->v_win;
+  {
+    const uint64_t dims[4] = {static_cast<uint64_t>(D), static_cast<uint64_t>(Hkv), Pm,
+                              static_cast<uint64_t>(c.max_prefix > 0 ? a->batch : 1)};
+    const uint64_t str[3] = {static_cast<uint64_t>(D) * 2, static_cast<uint64_t>(Hkv) * D * 2,
+                             Pm * Hkv * D * 2};
+    const uint32_t box[4] = {64, 1, 64, 1};
+    if (!encode_bf16(&kc, kcp, 4, dims, str, box) || !encode_bf16(&vc, vcp, 4, dims, str, box))
+      return fail(h, EBD_ERR_CUDA, "cuTensorMapEncodeTiled (K/V cache) failed");
+  }
+  {
+    const uint64_t dims[3] = {static_cast<uint64_t>(D), static_cast<uint64_t>(Hkv), R};
+    const uint64_t str[2] = {static_cast<uint64_t>(D) * 2, static_cast<uint64_t>(Hkv) * D * 2};
+    const uint32_t box[3] = {64, 1, 64};
+    if (!encode_bf16(&kw, a->k_win, 3, dims, str, box) || !encode_bf16(&vw, a->v_win, 3, dims, str, box))
+      return fail(h, EBD_ERR_CUDA, "cuTensorMapEncodeTiled (window K/V) failed");
+  }
+  AttnParams p{};
+  p.B = a->batch;
+  p.Hq = c.n_heads_q;
+  p.Hkv = Hkv;
+  p.D = D;
+  p.group = c.n_heads_q / Hkv;
+  p.max_prefix = c.max_prefix;
+  p.max_qtiles = h->attn_max_qtiles;
+  p.splits = h->attn_splits;
+  p.cu_rows = a->cu_rows;
+  p.prefix_len = a->prefix_len;
+  p.q = reinterpret_cast<const __nv_bfloat16*>(a->q);
+  p.out = a->attn_out;
+  p.part = h->attn_part;
+  p.tickets = h->tickets;
+  p.status = h->d_status;
+  p.limit_ns = kLimitNs;
+  cudaError_t e = launch_attention(kc, vc, kw, vw, p, st);
+  if (e != cudaSuccess) return cuda_fail(h, e, "attention launch");
+  return EBD_OK;
+}
+
+ebd_status run_lm(ebd_handle* h, const ebd_step_args* a, cudaStream_t st) {
+  const ebd_config& c = h->cfg;
+  CUtensorMap tw;
+  {
+    const uint64_t dims[2] = {static_cast<uint64_t>(c.d_model), static_cast<uint64_t>(c.vocab)};
+    const uint64_t str[1] = {static_cast<uint64_t>(c.d_model) * 2};
+    const uint32_t box[2] = {64, 64};
+    if (!encode_bf16(&tw, a->w_lm, 2, dims, str, box))
+      return fail(h, EBD_ERR_CUDA, "cuTensorMapEncodeTiled (W_lm) failed");
+  }
+  for (int g0 = 0; g0 < a->rows; g0 += kMaxGroupRows) {
+    const int rows = a->rows - g0 < kMaxGroupRows ? a->rows - g0 : kMaxGroupRows;
+    LmParams p{};
+    lm_plan(p, rows, c.vocab, c.d_model, h->num_sms);
+    if (p.stages < 2) return fail(h, EBD_ERR_UNSUPPORTED, "LM head: shared memory plan failed");
+    p.row0 = g0;
+    p.part_f = h->part_f;
+    p.part_i = h->part_i;
+    p.status = h->d_status;
+    p.limit_ns = kLimitNs;
+    p.force_timeout = (c.debug_flags & EBD_DEBUG_FORCE_TIMEOUT) ? 1 : 0;
+    CUtensorMap th;
+    const uint64_t dims[2] = {static_cast<uint64_t>(c.d_model), static_cast<uint64_t>(a->rows)};
+    const uint64_t str[1] = {static_cast<uint64_t>(c.d_model) * 2};
+    const uint32_t box[2] = {64, static_cast<uint32_t>(p.nb)};
+    if (!encode_bf16(&th, a->hidden, 2, dims, str, box))
+      return fail(h, EBD_ERR_CUDA, "cuTensorMapEncodeTiled (hidden) failed");
+    cudaError_t e = launch_lm_stats(tw, th, p, st);
+    if (e != cudaSuccess) return cuda_fail(h, e, "LM-head launch");
+  }
+  return EBD_OK;
+}
+
+DecideParams decide_params(ebd_handle* h, const ebd_step_args* a, int features_in) {
+  const ebd_config& c = h->cfg;
+  DecideParams p{};
+  p.B = a->batch;
+  p.V = c.vocab;
+  p.grid_lm = h->grid_lm;
+  p.features_in = features_in;
+  p.gen_len = c.gen_len;
+  p.g_max = c.g_max;
+  p.l_min = c.l_min;
+  p.l_b = c.l_b;
+  p.eos_id = c.eos_id;
+  p.lps_enabled = c.lps_enabled;
+  p.tau = c.tau;
+  p.tau_psi = c.tau_psi;
+  p.inv_log_v = static_cast<float>(1.0 / std::log(static_cast<double>(c.vocab)));
+  p.cu_rows = a->cu_rows;
+  p.row_pos = a->row_pos;
+  p.part_f = h->part_f;
+  p.part_i = h->part_i;
+  p.tokens = a->tokens;
+  p.mask = a->mask;
+  p.in_block = a->in_block;
+  p.blk_meta = a->blk_meta;
+  p.conf = a->conf;
+  p.entropy = a->entropy;
+  p.ent_norm = a->ent_norm;
+  p.gap = a->gap;
+  p.argmax = a->argmax;
+  p.lbs_logit = a->lbs_logit;
+  p.lps_prob = a->lps_prob;
+  p.accepted = a->accepted;
+  p.status = h->d_status;
+  p.rows_expected = a->rows;
+  p.w = h->img;
+  return p;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* ebd_version(void) { return "ebd 0.1 (sm_103a)"; }
+
+size_t ebd_weight_count(const ebd_config* cfg) {
+  if (cfg == nullptr || cfg->d_base <= 0 || cfg->gen_len <= 0) return 0;
+  return layout_count(router_layout(cfg->d_base, cfg->gen_len));
+}
+
+ebd_status ebd_router_init_host(const ebd_config* cfg, void* host, size_t* bytes) {
+  if (cfg == nullptr || bytes == nullptr) return EBD_ERR_INVALID_ARG;
+  if (cfg->d_base <= 0 || cfg->gen_len <= 0) return EBD_ERR_UNSUPPORTED;
+  const auto layout = router_layout(cfg->d_base, cfg->gen_len);
+  const size_t need = layout_count(layout) * 2;
+  if (host == nullptr) {
+    *bytes = need;
+    return EBD_OK;
+  }
+  if (*bytes < need) return EBD_ERR_INVALID_ARG;
+  router_init(cfg->seed, layout, static_cast<uint16_t*>(host));
+  *bytes = need;
+  return EBD_OK;
+}
+
+ebd_status ebd_create(const ebd_config* cfg, ebd_handle** out) {
+  if (out == nullptr) return EBD_ERR_INVALID_ARG;
+  *out = nullptr;
+  if (cfg == nullptr) return EBD_ERR_INVALID_ARG;
+  std::string why;
+  ebd_status s = validate_config(cfg, why);
+  if (s != EBD_OK) {
+    std::fprintf(stderr, "ebd_create: %s\n", why.c_str());
+    return s;
+  }
+  ebd_handle* h = new ebd_handle();
+  h->cfg = *cfg;
+  auto bail = [&](ebd_status code) {
+    std::fprintf(stderr, "ebd_create: %s\n", h->err.c_str());
+    ebd_destroy(h);
+    return code;
+  };
+  cudaError_t e = cudaGetDevice(&h->device);
+  if (e != cudaSuccess) return bail(cuda_fail(h, e, "cudaGetDevice"));
+  e = cudaDeviceGetAttribute(&h->num_sms, cudaDevAttrMultiProcessorCount, h->device);
+  if (e != cudaSuccess) return bail(cuda_fail(h, e, "cudaDeviceGetAttribute"));
+  int cc_major = 0, cc_minor = 0;
+  cudaDeviceGetAttribute(&cc_major, cudaDevAttrComputeCapabilityMajor, h->device);
+  cudaDeviceGetAttribute(&cc_minor, cudaDevAttrComputeCapabilityMinor, h->device);
+  if (cc_major != 10 || cc_minor != 3)
+    return bail(fail(h, EBD_ERR_UNSUPPORTED, "this build targets sm_103a (GB300) only"));
+  if (get_encode() == nullptr)
+    return bail(fail(h, EBD_ERR_CUDA, "cuTensorMapEncodeTiled is unavailable"));
+  if ((e = lm_configure()) != cudaSuccess) return bail(cuda_fail(h, e, "LM-head attributes"));
+  if ((e = attn_configure()) != cudaSuccess) return bail(cuda_fail(h, e, "attention attributes"));
+  if ((e = decide_configure()) != cudaSuccess) return bail(cuda_fail(h, e, "decision attributes"));
+
+  h->layout = router_layout(cfg->d_base, cfg->gen_len);
+  h->h_blob.resize(layout_count(h->layout));
+  router_init(cfg->seed, h->layout, h->h_blob.data());
+  if ((e = cudaMalloc(&h->d_blob, h->h_blob.size() * 2)) != cudaSuccess)
+    return bail(cuda_fail(h, e, "cudaMalloc(router blob)"));
+  if ((e = cudaMalloc(&h->d_tok, static_cast<size_t>(cfg->vocab) * 64 * 4)) != cudaSuccess)
+    return bail(cuda_fail(h, e, "cudaMalloc(token table)"));
+  if ((s = upload_router(h)) != EBD_OK) return bail(s);
+
+  // LM-head partials: one state per (row, CTA)
+  h->grid_lm = h->num_sms < (cfg->vocab + kUnit - 1) / kUnit ? h->num_sms
+                                                             : (cfg->vocab + kUnit - 1) / kUnit;
+  const size_t np = static_cast<size_t>(cfg->max_rows) * h->grid_lm;
+  if ((e = cudaMalloc(&h->part_f, np * sizeof(float4))) != cudaSuccess)
+    return bail(cuda_fail(h, e, "cudaMalloc(partials)"));
+  if ((e = cudaMalloc(&h->part_i, np * sizeof(int))) != cudaSuccess)
+    return bail(cuda_fail(h, e, "cudaMalloc(partials)"));
+  // attention split-KV workspace
+  {
+    const int group = cfg->n_heads_q / cfg->n_heads_kv;
+    h->attn_max_qtiles = (cfg->max_window * group + 63) / 64;
+    const int slots = cfg->max_batch * cfg->n_heads_kv * h->attn_max_qtiles;
+    const int nch = (cfg->max_prefix + kAttnChunk - 1) / kAttnChunk + 1;
+    int splits = (2 * h->num_sms + slots - 1) / slots;
+    if (splits > kMaxSplits) splits = kMaxSplits;
+    if (splits > nch) splits = nch;
+    if (splits < 1) splits = 1;
+    h->attn_splits = splits;
+    if (splits > 1) {
+      const size_t bytes = static_cast<size_t>(slots) * splits * 64 * (cfg->head_dim + 2) * 4;
+      if ((e = cudaMalloc(&h->attn_part, bytes)) != cudaSuccess)
+        return bail(cuda_fail(h, e, "cudaMalloc(attention partials)"));
+    }
+    if ((e = cudaMalloc(&h->tickets, static_cast<size_t>(slots) * sizeof(int))) != cudaSuccess)
+      return bail(cuda_fail(h, e, "cudaMalloc(tickets)"));
+    if ((e = cudaMemset(h->tickets, 0, static_cast<size_t>(slots) * sizeof(int))) != cudaSuccess)
+      return bail(cuda_fail(h, e, "cudaMemset(tickets)"));
+  }
+  if ((e = cudaMalloc(&h->d_status, sizeof(int))) != cudaSuccess)
+    return bail(cuda_fail(h, e, "cudaMalloc(status)"));
+  if ((e = cudaMemset(h->d_status, 0, sizeof(int))) != cudaSuccess)
+    return bail(cuda_fail(h, e, "cudaMemset(status)"));
+  // staging for ebd_step_host
+  {
+    const size_t R = cfg->max_rows, B = cfg->max_batch;
+    const size_t d = cfg->d_model, Hq = cfg->n_heads_q, Hkv = cfg->n_heads_kv, D = cfg->head_dim;
+    size_t bytes = 0;
+    auto add = [&](size_t n) { bytes += (n + 255) / 256 * 256; };
+    add((B + 1) * 4); add(B * 4); add(R * 4); add(R * d * 2); add(R * Hq * D * 2);
+    add(R * Hkv * D * 2); add(R * Hkv * D * 2); add(R * 4); add(R); add(R); add(B * 8);
+    add(R * Hq * D * 4); for (int i = 0; i < 6; ++i) add(R * 4); add(R * 4); add(R);
+    h->staging_bytes = bytes;
+    if ((e = cudaMalloc(&h->staging, bytes)) != cudaSuccess)
+      return bail(cuda_fail(h, e, "cudaMalloc(staging)"));
+  }
+  if ((e = cudaDeviceSynchronize()) != cudaSuccess) return bail(cuda_fail(h, e, "create"));
+  *out = h;
+  return EBD_OK;
+}
+
+void ebd_destroy(ebd_handle* h) {
+  if (h == nullptr) return;
+  int prev = -1;
+  cudaGetDevice(&prev);
+  if (prev != h->device) cudaSetDevice(h->device);
+  cudaDeviceSynchronize();
+  cudaFree(h->d_blob);
+  cudaFree(h->d_image);
+  cudaFree(h->d_tok);
+  cudaFree(h->part_f);
+  cudaFree(h->part_i);
+  cudaFree(h->attn_part);
+  cudaFree(h->tickets);
+  cudaFree(h->d_status);
+  cudaFree(h->staging);
+  if (prev >= 0 && prev != h->device) cudaSetDevice(prev);
+  delete h;
+}
+
+const char* ebd_last_error(const ebd_handle* h) { return h ? h->err.c_str() : "null handle"; }
+
+ebd_status ebd_bind_embedding(ebd_handle* h, const uint16_t* w_emb, void* stream) {
+  if (h == nullptr) return EBD_ERR_INVALID_ARG;
+  ebd_status s = check_device(h);
+  if (s != EBD_OK) return s;
+  if (w_emb == nullptr || !aligned(w_emb, 16))
+    return fail(h, EBD_ERR_INVALID_ARG, "w_emb must be a 16-byte aligned device pointer");
+  h->w_emb = w_emb;
+  return fold(h, static_cast<cudaStream_t>(stream));
+}
+
+ebd_status ebd_export_weights(const ebd_handle* h, void* host, size_t* bytes) {
+  if (h == nullptr || bytes == nullptr) return EBD_ERR_INVALID_ARG;
+  const size_t need = h->h_blob.size() * 2;
+  if (host == nullptr) {
+    *bytes = need;
+    return EBD_OK;
+  }
+  if (*bytes < need) return EBD_ERR_INVALID_ARG;
+  std::memcpy(host, h->h_blob.data(), need);
+  *bytes = need;
+  return EBD_OK;
+}
+
+ebd_status ebd_import_weights(ebd_handle* h, const void* host, size_t bytes) {
+  if (h == nullptr || host == nullptr) return EBD_ERR_INVALID_ARG;
+  if (bytes != h->h_blob.size() * 2) return fail(h, EBD_ERR_INVALID_ARG, "weight blob size mismatch");
+  ebd_status s = check_device(h);
+  if (s != EBD_OK) return s;
+  cudaError_t e = cudaDeviceSynchronize();
+  if (e != cudaSuccess) return cuda_fail(h, e, "import");
+  std::memcpy(h->h_blob.data(), host, bytes);
+  if ((s = upload_router(h)) != EBD_OK) return s;
+  if ((s = fold(h, nullptr)) != EBD_OK) return s;
+  e = cudaDeviceSynchronize();
+  if (e != cudaSuccess) return cuda_fail(h, e, "import");
+  return EBD_OK;
+}
+
+ebd_status ebd_step(ebd_handle* h, const ebd_step_args* a, void* stream) {
+  if (h == nullptr) return EBD_ERR_INVALID_ARG;
+  ebd_status s = check_device(h);
+  if (s != EBD_OK) return s;
+  const bool attn = a != nullptr && a->attn_out != nullptr;
+  if ((s = check_args(h, a, attn, true, true)) != EBD_OK) return s;
+  if (h->w_emb == nullptr) return fail(h, EBD_ERR_STATE, "bind the token embedding first");
+  if (a->rows == 0 || a->batch == 0) return EBD_OK;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  if (attn && (s = run_attention(h, a, st)) != EBD_OK) return s;
+  if ((s = run_lm(h, a, st)) != EBD_OK) return s;
+  DecideParams p = decide_params(h, a, 0);
+  cudaError_t e = launch_decide(p, st);
+  if (e != cudaSuccess) return cuda_fail(h, e, "decision launch");
+  return EBD_OK;
+}
+
+ebd_status ebd_decide(ebd_handle* h, const ebd_step_args* a, void* stream) {
+  if (h == nullptr) return EBD_ERR_INVALID_ARG;
+  ebd_status s = check_device(h);
+  if (s != EBD_OK) return s;
+  if ((s = check_args(h, a, false, false, true)) != EBD_OK) return s;
+  if (!a->conf || !a->ent_norm || !a->gap || !a->argmax)
+    return fail(h, EBD_ERR_INVALID_ARG, "conf/ent_norm/gap/argmax inputs must be set");
+  if (h->w_emb == nullptr) return fail(h, EBD_ERR_STATE, "bind the token embedding first");
+  if (a->rows == 0 || a->batch == 0) return EBD_OK;
+  DecideParams p = decide_params(h, a, 1);
+  p.entropy = nullptr;
+  cudaError_t e = launch_decide(p, static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(h, e, "decision launch");
+  return EBD_OK;
+}
+
+ebd_status ebd_lm_stats(ebd_handle* h, const ebd_step_args* a, void* stream) {
+  if (h == nullptr) return EBD_ERR_INVALID_ARG;
+  ebd_status s = check_device(h);
+  if (s != EBD_OK) return s;
+  if ((s = check_args(h, a, false, true, false)) != EBD_OK) return s;
+  if (a->rows == 0) return EBD_OK;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  if ((s = run_lm(h, a, st)) != EBD_OK) return s;
+  const float inv = static_cast<float>(1.0 / std::log(static_cast<double>(h->cfg.vocab)));
+  cudaError_t e = launch_merge_stats(h->part_f, h->part_i, a->rows, h->grid_lm, h->cfg.vocab, inv,
+                                     a->conf, a->entropy, a->ent_norm, a->gap, a->argmax,
+                                     h->d_status, st);
+  if (e != cudaSuccess) return cuda_fail(h, e, "merge launch");
+  return EBD_OK;
+}
+
+ebd_status ebd_attention(ebd_handle* h, const ebd_step_args* a, void* stream) {
+  if (h == nullptr) return EBD_ERR_INVALID_ARG;
+  ebd_status s = check_device(h);
+  if (s != EBD_OK) return s;
+  if ((s = check_args(h, a, true, false, false)) != EBD_OK) return s;
+  if (a->rows == 0 || a->batch == 0) return EBD_OK;
+  return run_attention(h, a, static_cast<cudaStream_t>(stream));
+}
+
+ebd_status ebd_step_host(ebd_handle* h, const ebd_step_args* a, void* stream) {
+  if (h == nullptr) return EBD_ERR_INVALID_ARG;
+  ebd_status s = check_device(h);
+  if (s != EBD_OK) return s;
+  if (a == nullptr) return fail(h, EBD_ERR_INVALID_ARG, "args is NULL");
+  if (a->batch < 0 || a->batch > h->cfg.max_batch || a->rows < 0 || a->rows > h->cfg.max_rows)
+    return fail(h, EBD_ERR_INVALID_ARG, "batch/rows out of range");
+  if (!a->cu_rows || !a->prefix_len || !a->row_pos || !a->hidden || !a->tokens || !a->mask ||
+      !a->in_block || !a->blk_meta || !a->w_lm)
+    return fail(h, EBD_ERR_INVALID_ARG, "missing host input");
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const ebd_config& c = h->cfg;
+  const size_t R = a->rows, B = a->batch, RM = c.max_rows, BM = c.max_batch;
+  const size_t d = c.d_model, Hq = c.n_heads_q, Hkv = c.n_heads_kv, D = c.head_dim;
+  uint8_t* p = h->staging;
+  auto take = [&](size_t n) {
+    uint8_t* q = p;
+    p += (n + 255) / 256 * 256;
+    return q;
+  };
+  ebd_step_args g = *a;
+  int32_t* cu = reinterpret_cast<int32_t*>(take((BM + 1) * 4));
+  int32_t* pl = reinterpret_cast<int32_t*>(take(BM * 4));
+  int32_t* rp = reinterpret_cast<int32_t*>(take(RM * 4));
+  uint16_t* hid = reinterpret_cast<uint16_t*>(take(RM * d * 2));
+  uint16_t* q = reinterpret_cast<uint16_t*>(take(RM * Hq * D * 2));
+  uint16_t* kw = reinterpret_cast<uint16_t*>(take(RM * Hkv * D * 2));
+  uint16_t* vw = reinterpret_cast<uint16_t*>(take(RM * Hkv * D * 2));
+  int32_t* tok = reinterpret_cast<int32_t*>(take(RM * 4));
+  uint8_t* msk = take(RM);
+  uint8_t* ib = take(RM);
+  int32_t* meta = reinterpret_cast<int32_t*>(take(BM * 8));
+  float* ao = reinterpret_cast<float*>(take(RM * Hq * D * 4));
+  float* f[6];
+  for (int i = 0; i < 6; ++i) f[i] = reinterpret_cast<float*>(take(RM * 4));
+  int32_t* am = reinterpret_cast<int32_t*>(take(RM * 4));
+  uint8_t* acc = take(RM);
+  auto h2d = [&](void* dst, const void* src, size_t n) {
+    return n == 0 || src == nullptr ? cudaSuccess
+                                    : cudaMemcpyAsync(dst, src, n, cudaMemcpyHostToDevice, st);
+  };
+  auto d2h = [&](void* dst, const void* src, size_t n) {
+    return n == 0 || dst == nullptr ? cudaSuccess
+                                    : cudaMemcpyAsync(dst, src, n, cudaMemcpyDeviceToHost, st);
+  };
+  cudaError_t e = cudaSuccess;
+  const bool attn = a->attn_out != nullptr;
+  auto chk = [&](cudaError_t x) {
+    if (e == cudaSuccess) e = x;
+  };
+  chk(h2d(cu, a->cu_rows, (B + 1) * 4));
+  chk(h2d(pl, a->prefix_len, B * 4));
+  chk(h2d(rp, a->row_pos, R * 4));
+  chk(h2d(hid, a->hidden, R * d * 2));
+  if (attn) {
+    chk(h2d(q, a->q, R * Hq * D * 2));
+    chk(h2d(kw, a->k_win, R * Hkv * D * 2));
+    chk(h2d(vw, a->v_win, R * Hkv * D * 2));
+  }
+  chk(h2d(tok, a->tokens, R * 4));
+  chk(h2d(msk, a->mask, R));
+  chk(h2d(ib, a->in_block, R));
+  chk(h2d(meta, a->blk_meta, B * 8));
+  if (e != cudaSuccess) return cuda_fail(h, e, "host-to-device copy");
+  g.cu_rows = cu; g.prefix_len = pl; g.row_pos = rp; g.hidden = hid;
+  g.q = attn ? q : nullptr; g.k_win = attn ? kw : nullptr; g.v_win = attn ? vw : nullptr;
+  g.tokens = tok; g.mask = msk; g.in_block = ib; g.blk_meta = meta;
+  g.attn_out = attn ? ao : nullptr;
+  g.conf = a->conf ? f[0] : nullptr;
+  g.entropy = a->entropy ? f[1] : nullptr;
+  g.ent_norm = a->ent_norm ? f[2] : nullptr;
+  g.gap = a->gap ? f[3] : nullptr;
+  g.lbs_logit = a->lbs_logit ? f[4] : nullptr;
+  g.lps_prob = a->lps_prob ? f[5] : nullptr;
+  g.argmax = a->argmax ? am : nullptr;
+  g.accepted = a->accepted ? acc : nullptr;
+  if ((s = ebd_step(h, &g, stream)) != EBD_OK) return s;
+  chk(d2h(a->tokens, tok, R * 4));
+  chk(d2h(a->mask, msk, R));
+  chk(d2h(a->in_block, ib, R));
+  chk(d2h(a->blk_meta, meta, B * 8));
+  if (attn) chk(d2h(a->attn_out, ao, R * Hq * D * 4));
+  chk(d2h(a->conf, f[0], R * 4));
+  chk(d2h(a->entropy, f[1], R * 4));
+  chk(d2h(a->ent_norm, f[2], R * 4));
+  chk(d2h(a->gap, f[3], R * 4));
+  chk(d2h(a->lbs_logit, f[4], R * 4));
+  chk(d2h(a->lps_prob, f[5], R * 4));
+  chk(d2h(a->argmax, am, R * 4));
+  chk(d2h(a->accepted, acc, R));
+  if (e != cudaSuccess) return cuda_fail(h, e, "device-to-host copy");
+  return EBD_OK;
+}
+
+ebd_status ebd_sync_status(ebd_handle* h, void* stream) {
+  if (h == nullptr) return EBD_ERR_INVALID_ARG;
+  ebd_status s = check_device(h);
+  if (s != EBD_OK) return s;
+  cudaError_t e = cudaStreamSynchronize(static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(h, e, "stream synchronize");
+  int v = 0;
+  if ((e = cudaMemcpy(&v, h->d_status, sizeof(int), cudaMemcpyDeviceToHost)) != cudaSuccess)
+    return cuda_fail(h, e, "status read");
+  if (v != 0) {
+    cudaMemset(h->d_status, 0, sizeof(int));
+    const int group = h->cfg.n_heads_q / h->cfg.n_heads_kv;
+    const int slots = h->cfg.max_batch * h->cfg.n_heads_kv * ((h->cfg.max_window * group + 63) / 64);
+    cudaMemset(h->tickets, 0, static_cast<size_t>(slots) * sizeof(int));
+    cudaDeviceSynchronize();
+    h->err = "device reported status " + std::to_string(v);
+  }
+  return v;
+}
+
+}  // extern "C"

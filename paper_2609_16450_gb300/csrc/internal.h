@@ -1,0 +1,107 @@
+// Launch parameters shared by the host side of the library and its kernels.
+#pragma once
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <cstdint>
+
+#include "ebd.h"
+
+namespace ebd {
+
+constexpr int kMaxWindow = 64;        // window rows per sequence
+constexpr int kUnit = 64;             // vocabulary rows per work unit of the LM head
+constexpr int kLmThreads = 192;       // TMA warp, MMA warp, 4 epilogue warps
+constexpr int kMaxGroupRows = 512;    // rows per LM-head launch (TMEM: 512 columns)
+constexpr int kDecideCluster = 8;     // CTAs per sequence in the decision kernel
+constexpr int kDecideThreads = 256;
+constexpr int kAttnThreads = 128;
+constexpr int kAttnChunk = 64;        // keys per K/V tile
+constexpr int kAttnStages = 3;
+
+// ------------------------------------------------------------------ LM head
+struct LmParams {
+  int V, d;                 // vocabulary, hidden size
+  int row0, rows;           // rows [row0, row0 + rows) of this launch
+  int nb, nsub, n_pad;      // MMA N per sub-tile, sub-tiles, padded N = nb * nsub
+  int n_units;              // ceil(V / 64)
+  int grid;                 // CTAs (partials per row)
+  int nkb;                  // ceil(d / 64) k-blocks
+  int stages, nbuf, acc_stride, tmem_cols;
+  uint32_t off_a, off_b, off_t, off_st, off_bar, smem_bytes;
+  float4* part_f;           // [R][grid] (max, sum exp, sum exp*(l-max), second logit)
+  int* part_i;              // [R][grid] argmax
+  int* status;
+  uint64_t limit_ns;
+  int force_timeout;
+};
+
+// ------------------------------------------------------------------ attention
+struct AttnParams {
+  int B, Hq, Hkv, D, group;
+  int max_prefix;
+  int max_qtiles, splits;
+  const int* cu_rows;
+  const int* prefix_len;
+  const __nv_bfloat16* q;   // [R][Hq][D]
+  float* out;               // [R][Hq][D]
+  float* part;              // [B*Hkv*max_qtiles*splits][64][D+2]
+  int* tickets;             // [B*Hkv*max_qtiles]
+  int* status;
+  uint64_t limit_ns;
+};
+
+// ------------------------------------------------------------------ routers
+// Device image of the router weights used by the decision kernel: matrices
+// transposed to [in][out] bf16, vectors fp32.
+struct LbsLayer {
+  const __nv_bfloat16 *qkv_t, *out_t, *ff1_t, *ff2_t;  // [128][384] [128][128] [128][256] [256][128]
+  const float *qkv_b, *out_b, *ff1_b, *ff2_b, *ln1_g, *ln1_b, *ln2_g, *ln2_b;
+};
+struct LpsLayer {
+  const __nv_bfloat16 *qkv_t, *out_t, *ff1_t, *ff2_t;  // [32][96] [32][32] [32][64] [64][32]
+  const float *qkv_b, *out_b, *ff1_b, *ff2_b, *ln1_g, *ln1_b, *ln2_g, *ln2_b;
+};
+struct RouterImage {
+  // LBS
+  const float *ent1_w, *ent1_b, *ent2_b, *ent_ln_g, *ent_ln_b, *tok_b, *comb_b, *head_w, *head_b;
+  const __nv_bfloat16 *ent2_t, *comb_t, *pos;  // [64][64] [128][128] [L][128]
+  LbsLayer lbs[2];
+  // LPS
+  const float *in_t, *in_b, *in_ln_g, *in_ln_b, *lps_head_w, *lps_head_b;  // in_t: [5][32]
+  LpsLayer lps[2];
+  const float* tok_table;  // [V][64] = W_tok W_e[v] (no bias)
+};
+
+struct DecideParams {
+  int B, V, grid_lm;        // grid_lm: LM-head partials per row
+  int features_in;          // 1: conf/ent_norm/gap/argmax are inputs
+  int gen_len, g_max, l_min, l_b, eos_id, lps_enabled;
+  float tau, tau_psi, inv_log_v;
+  const int* cu_rows;
+  const int* row_pos;
+  const float4* part_f;
+  const int* part_i;
+  int* tokens;
+  uint8_t* mask;
+  uint8_t* in_block;
+  int* blk_meta;
+  float *conf, *entropy, *ent_norm, *gap, *lbs_logit, *lps_prob;
+  int* argmax;
+  uint8_t* accepted;
+  int* status;
+  int rows_expected;
+  RouterImage w;
+};
+
+// host launchers (defined next to their kernels)
+cudaError_t launch_lm_stats(const CUtensorMap& tmap_w, const CUtensorMap& tmap_h,
+                            const LmParams& p, cudaStream_t st);
+void lm_plan(LmParams& p, int rows, int V, int d, int num_sms);
+cudaError_t launch_attention(const CUtensorMap& kc, const CUtensorMap& vc, const CUtensorMap& kw,
+                             const CUtensorMap& vw, const AttnParams& p, cudaStream_t st);
+cudaError_t launch_decide(const DecideParams& p, cudaStream_t st);
+cudaError_t launch_fold_tok(const __nv_bfloat16* w_tok, const __nv_bfloat16* w_emb, float* table,
+                            int V, int d_base, cudaStream_t st);
+
+}  // namespace ebd

@@ -1,0 +1,333 @@
+// Window attention: the active window's queries attend, without a mask, to
+// the sequence's cached prefix keys followed by the window's own keys
+// (bidirectional dLLM, Sec. 3; prefix cache at the block boundary, Sec. 6.3).
+//   O = softmax(Q K^T / sqrt(D)) V, fp32 output.
+//
+// Grid: (key split, query tile, sequence x kv head).  A query tile is 64 rows
+// of (query head of the kv group, window row); each of the 4 warps owns 16
+// rows.  K/V tiles of 64 keys are staged by TMA (128-byte swizzle) through a
+// 3-stage ring; Q K^T runs on mma.sync bf16 with fp32 accumulation; the
+// probabilities are split into a bf16 high part and a bf16 remainder so that
+// P V keeps ~16 mantissa bits.  Splits of the key range combine their
+// (max, sum, O) partials in the last CTA to finish (atomic ticket).
+#include "internal.h"
+#include "ptx.cuh"
+
+namespace ebd {
+
+namespace {
+
+constexpr int kStageBytes = 4 * 8192;  // K and V, two 64-dim halves each
+
+__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2,
+                                        uint32_t& r3) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+               : "r"(addr));
+}
+__device__ __forceinline__ void ldsm_x4_t(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2,
+                                          uint32_t& r3) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+               : "r"(addr));
+}
+__device__ __forceinline__ void mma_bf16(float (&d)[4], const uint32_t (&a)[4], uint32_t b0,
+                                         uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, "
+      "{%8,%9}, {%0,%1,%2,%3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+// split x = hi + lo with hi = bf16(x), lo = bf16(x - hi)
+__device__ __forceinline__ void split2(float x, float y, uint32_t& hi, uint32_t& lo) {
+  __nv_bfloat162 h = __floats2bfloat162_rn(x, y);
+  const float2 hf = __bfloat1622float2(h);
+  __nv_bfloat162 l = __floats2bfloat162_rn(x - hf.x, y - hf.y);
+  hi = *reinterpret_cast<uint32_t*>(&h);
+  lo = *reinterpret_cast<uint32_t*>(&l);
+}
+// byte offset of 16-byte chunk `c` (0..7) of row `r` in a 128B-swizzled tile
+__device__ __forceinline__ uint32_t swz(int r, int c) {
+  return static_cast<uint32_t>(r * 128 + ((c ^ (r & 7)) << 4));
+}
+
+}  // namespace
+
+template <int D>
+__global__ void __launch_bounds__(kAttnThreads)
+    attn_kernel(const __grid_constant__ CUtensorMap tm_kc, const __grid_constant__ CUtensorMap tm_vc,
+                const __grid_constant__ CUtensorMap tm_kw, const __grid_constant__ CUtensorMap tm_vw,
+                const AttnParams p) {
+  constexpr int NH = D / 64;   // 64-dim halves
+  constexpr int KS = D / 16;   // k-steps of Q K^T
+  constexpr int NT = D / 8;    // n-tiles of the output
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + kAttnStages * kStageBytes);
+  __shared__ int s_flag;
+
+  const int split = blockIdx.x, qt = blockIdx.y, bg = blockIdx.z;
+  const int b = bg / p.Hkv, g = bg - b * p.Hkv;
+  const int r0 = p.cu_rows[b];
+  const int wb = p.cu_rows[b + 1] - r0;
+  const int m_total = wb * p.group;
+  if (wb <= 0 || wb > kMaxWindow || qt * 64 >= m_total) return;
+  int P = p.prefix_len[b];
+  P = P < 0 ? 0 : (P > p.max_prefix ? p.max_prefix : P);
+  const int ncc = (P + kAttnChunk - 1) / kAttnChunk;
+  const int nch = ncc + 1;
+  const int c0 = static_cast<int>((static_cast<long long>(split) * nch) / p.splits);
+  const int c1 = static_cast<int>((static_cast<long long>(split + 1) * nch) / p.splits);
+  const int nmy = c1 - c0;
+
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  if (tid == 0) {
+    for (int s = 0; s < kAttnStages; ++s) mbar_init(&full[s], 1);
+    fence_mbar_init();
+    s_flag = 0;
+  }
+  __syncthreads();
+
+  auto issue = [&](int i) {
+    const int s = i % kAttnStages;
+    const int c = c0 + i;
+    uint8_t* kd = smem + s * kStageBytes;
+    uint8_t* vd = kd + 2 * 8192;
+    mbar_arrive_expect_tx(&full[s], 2u * NH * 8192u);
+#pragma unroll
+    for (int hf = 0; hf < NH; ++hf) {
+      if (c < ncc) {
+        tma_load_4d(kd + hf * 8192, &tm_kc, &full[s], hf * 64, g, c * kAttnChunk, b);
+        tma_load_4d(vd + hf * 8192, &tm_vc, &full[s], hf * 64, g, c * kAttnChunk, b);
+      } else {
+        tma_load_3d(kd + hf * 8192, &tm_kw, &full[s], hf * 64, g, r0);
+        tma_load_3d(vd + hf * 8192, &tm_vw, &full[s], hf * 64, g, r0);
+      }
+    }
+  };
+  if (tid == 0)
+    for (int i = 0; i < nmy && i < kAttnStages; ++i) issue(i);
+
+  // query fragments of this warp's 16 rows
+  const int mrow_lo = qt * 64 + warp * 16 + (lane >> 2);
+  const int mrow_hi = mrow_lo + 8;
+  auto qptr = [&](int m) -> const __nv_bfloat16* {
+    if (m >= m_total) return nullptr;
+    const int hl = m / wb, r = m - hl * wb;
+    return p.q + (static_cast<size_t>(r0 + r) * p.Hq + g * p.group + hl) * D;
+  };
+  const __nv_bfloat16* q_lo = qptr(mrow_lo);
+  const __nv_bfloat16* q_hi = qptr(mrow_hi);
+  const bool warp_active = qt * 64 + warp * 16 < m_total;
+  uint32_t qf[KS][4];
+#pragma unroll
+  for (int ks = 0; ks < KS; ++ks) {
+    const int c = ks * 16 + 2 * (lane & 3);
+    qf[ks][0] = q_lo ? *reinterpret_cast<const uint32_t*>(q_lo + c) : 0u;
+    qf[ks][1] = q_hi ? *reinterpret_cast<const uint32_t*>(q_hi + c) : 0u;
+    qf[ks][2] = q_lo ? *reinterpret_cast<const uint32_t*>(q_lo + c + 8) : 0u;
+    qf[ks][3] = q_hi ? *reinterpret_cast<const uint32_t*>(q_hi + c + 8) : 0u;
+  }
+
+  float o[NT][4];
+#pragma unroll
+  for (int t = 0; t < NT; ++t) o[t][0] = o[t][1] = o[t][2] = o[t][3] = 0.f;
+  float m_lo = -INFINITY, m_hi = -INFINITY, l_lo = 0.f, l_hi = 0.f;
+  const float sl2 = 1.4426950408889634f / sqrtf(static_cast<float>(D));  // log2(e)/sqrt(D)
+
+  bool failed = false;
+  for (int i = 0; i < nmy; ++i) {
+    const int s = i % kAttnStages;
+    const bool ok = mbar_wait(&full[s], static_cast<uint32_t>(i / kAttnStages) & 1u, p.limit_ns,
+                              nullptr);
+    if (__syncthreads_or(!ok)) {
+      failed = true;
+      if (tid == 0) {
+        atomicCAS(p.status, 0, EBD_ERR_TIMEOUT);
+        for (int j = i; j < nmy && j < i + kAttnStages; ++j)
+          mbar_wait(&full[j % kAttnStages], static_cast<uint32_t>(j / kAttnStages) & 1u,
+                    p.limit_ns, nullptr);
+      }
+      break;
+    }
+    const int c = c0 + i;
+    const int nvalid = c < ncc ? min(kAttnChunk, P - c * kAttnChunk) : wb;
+    const uint32_t kbase = smem_u32(smem + s * kStageBytes);
+    const uint32_t vbase = kbase + 2 * 8192;
+    if (warp_active) {
+      float sc[8][4];
+#pragma unroll
+      for (int t = 0; t < 8; ++t) sc[t][0] = sc[t][1] = sc[t][2] = sc[t][3] = 0.f;
+      const int mi = lane >> 3, rr = lane & 7;
+#pragma unroll
+      for (int ks = 0; ks < KS; ++ks) {
+        const int hf = ks >> 2;
+        const int cidx = (ks & 3) * 2;
+#pragma unroll
+        for (int np = 0; np < 4; ++np) {
+          const int key = np * 16 + (mi >> 1) * 8 + rr;
+          const uint32_t addr = kbase + hf * 8192 + swz(key, cidx + (mi & 1));
+          uint32_t b0, b1, b2, b3;
+          ldsm_x4(addr, b0, b1, b2, b3);
+          mma_bf16(sc[2 * np], qf[ks], b0, b1);
+          mma_bf16(sc[2 * np + 1], qf[ks], b2, b3);
+        }
+      }
+      float mx_lo = -INFINITY, mx_hi = -INFINITY;
+#pragma unroll
+      for (int t = 0; t < 8; ++t) {
+        const int k0 = t * 8 + 2 * (lane & 3);
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const int key = k0 + (e & 1);
+          const float v = key < nvalid ? sc[t][e] * sl2 : -INFINITY;
+          sc[t][e] = v;
+        }
+        mx_lo = fmaxf(mx_lo, fmaxf(sc[t][0], sc[t][1]));
+        mx_hi = fmaxf(mx_hi, fmaxf(sc[t][2], sc[t][3]));
+      }
+#pragma unroll
+      for (int off = 1; off <= 2; off <<= 1) {
+        mx_lo = fmaxf(mx_lo, __shfl_xor_sync(0xffffffffu, mx_lo, off));
+        mx_hi = fmaxf(mx_hi, __shfl_xor_sync(0xffffffffu, mx_hi, off));
+      }
+      const float mn_lo = fmaxf(m_lo, mx_lo), mn_hi = fmaxf(m_hi, mx_hi);
+      const float al_lo = exp2f(m_lo - mn_lo), al_hi = exp2f(m_hi - mn_hi);
+      m_lo = mn_lo;
+      m_hi = mn_hi;
+      float sum_lo = 0.f, sum_hi = 0.f;
+#pragma unroll
+      for (int t = 0; t < 8; ++t) {
+        sc[t][0] = exp2f(sc[t][0] - mn_lo);
+        sc[t][1] = exp2f(sc[t][1] - mn_lo);
+        sc[t][2] = exp2f(sc[t][2] - mn_hi);
+        sc[t][3] = exp2f(sc[t][3] - mn_hi);
+        sum_lo += sc[t][0] + sc[t][1];
+        sum_hi += sc[t][2] + sc[t][3];
+      }
+#pragma unroll
+      for (int off = 1; off <= 2; off <<= 1) {
+        sum_lo += __shfl_xor_sync(0xffffffffu, sum_lo, off);
+        sum_hi += __shfl_xor_sync(0xffffffffu, sum_hi, off);
+      }
+      l_lo = l_lo * al_lo + sum_lo;
+      l_hi = l_hi * al_hi + sum_hi;
+#pragma unroll
+      for (int t = 0; t < NT; ++t) {
+        o[t][0] *= al_lo;
+        o[t][1] *= al_lo;
+        o[t][2] *= al_hi;
+        o[t][3] *= al_hi;
+      }
+      // O += P V, P split into bf16 high and low parts
+#pragma unroll
+      for (int kk = 0; kk < 4; ++kk) {
+        uint32_t ah[4], al[4];
+        split2(sc[2 * kk][0], sc[2 * kk][1], ah[0], al[0]);
+        split2(sc[2 * kk][2], sc[2 * kk][3], ah[1], al[1]);
+        split2(sc[2 * kk + 1][0], sc[2 * kk + 1][1], ah[2], al[2]);
+        split2(sc[2 * kk + 1][2], sc[2 * kk + 1][3], ah[3], al[3]);
+#pragma unroll
+        for (int dp = 0; dp < D / 16; ++dp) {
+          const int hf = dp >> 2;
+          const int key = kk * 16 + (mi & 1) * 8 + rr;
+          const int chunk = (dp & 3) * 2 + (mi >> 1);
+          const uint32_t addr = vbase + hf * 8192 + swz(key, chunk);
+          uint32_t b0, b1, b2, b3;
+          ldsm_x4_t(addr, b0, b1, b2, b3);
+          mma_bf16(o[2 * dp], ah, b0, b1);
+          mma_bf16(o[2 * dp], al, b0, b1);
+          mma_bf16(o[2 * dp + 1], ah, b2, b3);
+          mma_bf16(o[2 * dp + 1], al, b2, b3);
+        }
+      }
+    }
+    __syncthreads();
+    if (tid == 0 && i + kAttnStages < nmy) issue(i + kAttnStages);
+  }
+  if (failed) return;
+
+  // ------------------------------------------------------------ output / partials
+  auto out_row = [&](int m) -> float* {
+    const int hl = m / wb, r = m - hl * wb;
+    return p.out + (static_cast<size_t>(r0 + r) * p.Hq + g * p.group + hl) * D;
+  };
+  if (p.splits == 1) {
+    if (warp_active) {
+      const float il = l_lo > 0.f ? 1.0f / l_lo : 0.f, ih = l_hi > 0.f ? 1.0f / l_hi : 0.f;
+#pragma unroll
+      for (int t = 0; t < NT; ++t) {
+        const int d = t * 8 + 2 * (lane & 3);
+        if (mrow_lo < m_total)
+          *reinterpret_cast<float2*>(out_row(mrow_lo) + d) = make_float2(o[t][0] * il, o[t][1] * il);
+        if (mrow_hi < m_total)
+          *reinterpret_cast<float2*>(out_row(mrow_hi) + d) = make_float2(o[t][2] * ih, o[t][3] * ih);
+      }
+    }
+    return;
+  }
+  const int slot = (bg * p.max_qtiles + qt);
+  float* part = p.part + (static_cast<size_t>(slot) * p.splits + split) * 64 * (D + 2);
+  if (warp_active) {
+    const int ml = warp * 16 + (lane >> 2), mh = ml + 8;
+#pragma unroll
+    for (int t = 0; t < NT; ++t) {
+      const int d = t * 8 + 2 * (lane & 3);
+      *reinterpret_cast<float2*>(part + ml * (D + 2) + d) = make_float2(o[t][0], o[t][1]);
+      *reinterpret_cast<float2*>(part + mh * (D + 2) + d) = make_float2(o[t][2], o[t][3]);
+    }
+    if ((lane & 3) == 0) {
+      part[ml * (D + 2) + D] = m_lo;
+      part[ml * (D + 2) + D + 1] = l_lo;
+      part[mh * (D + 2) + D] = m_hi;
+      part[mh * (D + 2) + D + 1] = l_hi;
+    }
+  }
+  __threadfence();
+  __syncthreads();
+  if (tid == 0) s_flag = (atomicAdd(&p.tickets[slot], 1) == p.splits - 1);
+  __syncthreads();
+  if (!s_flag) return;
+  __threadfence();
+  const float* base = p.part + static_cast<size_t>(slot) * p.splits * 64 * (D + 2);
+  const int rows_here = min(64, m_total - qt * 64);
+  for (int it = tid; it < rows_here * D; it += blockDim.x) {
+    const int mr = it / D, d = it - mr * D;
+    float M = -INFINITY;
+    for (int sp = 0; sp < p.splits; ++sp)
+      M = fmaxf(M, base[(static_cast<size_t>(sp) * 64 + mr) * (D + 2) + D]);
+    float L = 0.f, acc = 0.f;
+    for (int sp = 0; sp < p.splits; ++sp) {
+      const float* pr = base + (static_cast<size_t>(sp) * 64 + mr) * (D + 2);
+      const float ms = pr[D];
+      if (ms == -INFINITY) continue;
+      const float wgt = exp2f(ms - M);
+      L += wgt * pr[D + 1];
+      acc += wgt * pr[d];
+    }
+    out_row(qt * 64 + mr)[d] = L > 0.f ? acc / L : 0.f;
+  }
+  if (tid == 0) p.tickets[slot] = 0;
+}
+
+cudaError_t attn_configure() {
+  const int bytes = kAttnStages * kStageBytes + 1024 + 64;
+  cudaError_t e = cudaFuncSetAttribute(attn_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+  if (e != cudaSuccess) return e;
+  return cudaFuncSetAttribute(attn_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+}
+
+cudaError_t launch_attention(const CUtensorMap& kc, const CUtensorMap& vc, const CUtensorMap& kw,
+                             const CUtensorMap& vw, const AttnParams& p, cudaStream_t st) {
+  const dim3 grid(p.splits, p.max_qtiles, p.B * p.Hkv);
+  const int bytes = kAttnStages * kStageBytes + 1024 + 64;
+  if (p.D == 64)
+    attn_kernel<64><<<grid, kAttnThreads, bytes, st>>>(kc, vc, kw, vw, p);
+  else
+    attn_kernel<128><<<grid, kAttnThreads, bytes, st>>>(kc, vc, kw, vw, p);
+  return cudaGetLastError();
+}
+
+}  // namespace ebd

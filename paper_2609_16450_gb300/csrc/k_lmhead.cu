@@ -1,0 +1,364 @@
+// LM head fused with the softmax statistics of every window row.
+//
+// For each window row r and vocabulary entry v the logit is
+// l[r][v] = sum_k h[r][k] W[v][k]; the kernel never stores it.  Each CTA owns a
+// contiguous range of 64-row vocabulary units and keeps, per window row, the
+// online-softmax state over the vocabulary it has seen:
+//   m  = max logit,  S = sum exp(l - m),  T = sum exp(l - m) (l - m),
+//   l2 = second largest logit (duplicates count),  idx = argmax (lowest).
+// The decision kernel merges the per-CTA states into kappa = 1/S,
+// H = ln S - T/S, Delta = (1 - exp(l2 - m)) / S and x_hat = idx, i.e. the
+// statistics of App. B (Eq. app-confidence), Sec. 5.1 and Sec. 5.2.
+//
+// Tensor-core mapping (swap-AB): the vocabulary tile is the MMA's M = 128
+// (A = W rows, K-major, streamed by TMA with an evict-first L2 policy), the
+// window rows are N (B = hidden rows, K-major), the fp32 accumulator lives
+// in TMEM as 128 lanes (vocabulary) x N columns (rows).  Warp 0 issues TMA,
+// warp 1 issues tcgen05.mma, warps 2..5 drain TMEM and run the statistics.
+#include <climits>
+
+#include "internal.h"
+#include "ptx.cuh"
+
+namespace ebd {
+
+namespace {
+
+constexpr uint32_t kATile = 128 * 128;  // 128 rows x 64 bf16
+constexpr int kTLd = 132;               // transpose buffer row stride (floats)
+constexpr uint32_t kTBytes = 32 * kTLd * 4;
+
+__device__ __forceinline__ void state_merge(float& m, float& s, float& t, float& l2, int& idx,
+                                            float bm, float bs, float bt, float bl2, int bidx) {
+  if (bm > m || (bm == m && bidx < idx)) {
+    float x;
+    int xi;
+    x = m; m = bm; bm = x;
+    x = s; s = bs; bs = x;
+    x = t; t = bt; bt = x;
+    x = l2; l2 = bl2; bl2 = x;
+    xi = idx; idx = bidx; bidx = xi;
+  }
+  l2 = fmaxf(l2, bm);
+  if (bm == -INFINITY) return;  // the other side is empty
+  const float dl = bm - m;      // <= 0
+  const float sc = __expf(dl);
+  t = t + sc * (bt + dl * bs);
+  s = s + sc * bs;
+}
+
+__device__ __forceinline__ bool named_barrier_and(uint32_t id, uint32_t n, bool pred) {
+  uint32_t r;
+  asm volatile(
+      "{\n .reg .pred p, q;\n setp.ne.u32 p, %1, 0;\n bar.red.and.pred q, %2, %3, p;\n"
+      " selp.u32 %0, 1, 0, q;\n}\n"
+      : "=r"(r)
+      : "r"((uint32_t)pred), "r"(id), "r"(n)
+      : "memory");
+  return r != 0;
+}
+
+__device__ __forceinline__ void record_error(int* status, volatile int* abort, int code) {
+  *abort = 1;
+  atomicCAS(status, 0, code);
+}
+
+}  // namespace
+
+__global__ void __launch_bounds__(kLmThreads, 1)
+    lm_stats_kernel(const __grid_constant__ CUtensorMap tmap_w,
+                    const __grid_constant__ CUtensorMap tmap_h, const LmParams p) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  uint8_t* sA = smem + p.off_a;
+  uint8_t* sB = smem + p.off_b;
+  float* sT = reinterpret_cast<float*>(smem + p.off_t);
+  float* st_m = reinterpret_cast<float*>(smem + p.off_st);
+  float* st_s = st_m + p.n_pad;
+  float* st_t = st_s + p.n_pad;
+  float* st_l2 = st_t + p.n_pad;
+  int* st_i = reinterpret_cast<int*>(st_l2 + p.n_pad);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + p.off_bar);
+  uint64_t* full = bars;
+  uint64_t* empty = bars + p.stages;
+  uint64_t* acc_full = bars + 2 * p.stages;
+  uint64_t* acc_empty = acc_full + 2;
+  uint64_t* drain = acc_empty + 2;
+  uint64_t* dummy = drain + 1;
+  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(dummy + 1);
+  volatile int* abort = reinterpret_cast<volatile int*>(tmem_holder + 1);
+
+  const int tid = threadIdx.x;
+  const int warp = __shfl_sync(0xffffffffu, tid / 32, 0);
+  const int lane = tid & 31;
+  const int cta = blockIdx.x;
+
+  if (tid == 0) {
+    for (int s = 0; s < p.stages; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&acc_full[b], 1);
+      mbar_init(&acc_empty[b], 128);
+    }
+    mbar_init(drain, 1);
+    mbar_init(dummy, 1);
+    *abort = 0;
+    fence_mbar_init();
+    tma_prefetch_desc(&tmap_w);
+    tma_prefetch_desc(&tmap_h);
+  }
+  if (warp == 1) tmem_alloc(tmem_holder, p.tmem_cols);
+  if (tid >= 64) {
+    for (int r = tid - 64; r < p.n_pad; r += 128) {
+      st_m[r] = -INFINITY;
+      st_s[r] = 0.f;
+      st_t[r] = 0.f;
+      st_l2[r] = -INFINITY;
+      st_i[r] = INT_MAX;
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_holder;
+
+  const int u0 = static_cast<int>((static_cast<long long>(cta) * p.n_units) / p.grid);
+  const int u1 = static_cast<int>((static_cast<long long>(cta + 1) * p.n_units) / p.grid);
+  const uint32_t b_stage = static_cast<uint32_t>(p.n_pad) * 128u;
+
+  if (warp == 0) {
+    // ------------------------------------------------------------ TMA producer
+    if (lane == 0) {
+      const uint64_t pol_w = l2_policy_evict_first();
+      const uint64_t pol_h = l2_policy_evict_last();
+      int it = 0;
+      bool ok = true;
+      for (int u = u0; u < u1 && ok; u += 2) {
+        const int nu = min(2, u1 - u);
+        for (int kb = 0; kb < p.nkb; ++kb) {
+          const int s = it % p.stages;
+          const uint32_t ph = static_cast<uint32_t>(it / p.stages) & 1u;
+          if (!mbar_wait(&empty[s], ph ^ 1u, p.limit_ns, abort)) {
+            ok = false;
+            break;
+          }
+          mbar_arrive_expect_tx(&full[s], static_cast<uint32_t>(nu) * kUnit * 128u + b_stage);
+          for (int ui = 0; ui < nu; ++ui)
+            tma_load_2d(sA + s * kATile + ui * (kUnit * 128), &tmap_w, &full[s], kb * 64,
+                        (u + ui) * kUnit, pol_w);
+          for (int sb = 0; sb < p.nsub; ++sb)
+            tma_load_2d(sB + s * b_stage + sb * p.nb * 128, &tmap_h, &full[s], kb * 64,
+                        p.row0 + sb * p.nb, pol_h);
+          ++it;
+        }
+      }
+      if (!ok) {
+        if (!*abort) record_error(p.status, abort, EBD_ERR_TIMEOUT);
+        // let the copies already in flight land before the CTA can exit
+        for (int j = max(0, it - p.stages); j < it; ++j)
+          mbar_wait(&full[j % p.stages], static_cast<uint32_t>(j / p.stages) & 1u, p.limit_ns,
+                    nullptr);
+      }
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------------------ MMA issuer
+    if (lane == 0) {
+      const uint32_t idesc = umma_idesc_bf16(128, static_cast<uint32_t>(p.nb));
+      int it = 0, c = 0;
+      bool ok = true;
+      for (int u = u0; u < u1 && ok; u += 2, ++c) {
+        const int buf = c % p.nbuf;
+        const uint32_t bph = static_cast<uint32_t>(c / p.nbuf) & 1u;
+        if (!mbar_wait(&acc_empty[buf], bph ^ 1u, p.limit_ns, abort)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t d0 = tmem_base + static_cast<uint32_t>(buf * p.acc_stride);
+        for (int kb = 0; kb < p.nkb; ++kb) {
+          const int s = it % p.stages;
+          const uint32_t ph = static_cast<uint32_t>(it / p.stages) & 1u;
+          if (!mbar_wait(&full[s], ph, p.limit_ns, abort)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t a_addr = smem_u32(sA + s * kATile);
+          const uint32_t b_addr = smem_u32(sB + s * b_stage);
+#pragma unroll
+          for (int kk = 0; kk < 4; ++kk) {
+            const uint64_t ad = umma_desc_sw128(a_addr + kk * 32);
+            for (int sb = 0; sb < p.nsub; ++sb) {
+              const uint64_t bd = umma_desc_sw128(b_addr + sb * p.nb * 128 + kk * 32);
+              umma_bf16(d0 + static_cast<uint32_t>(sb * p.nb), ad, bd, idesc,
+                        (kb | kk) != 0 ? 1u : 0u);
+            }
+          }
+          umma_commit(&empty[s]);
+          ++it;
+        }
+        if (!ok) break;
+        umma_commit(&acc_full[buf]);
+      }
+      if (!ok) {
+        if (!*abort) record_error(p.status, abort, EBD_ERR_TIMEOUT);
+        umma_commit(drain);  // completes once every MMA issued so far is done
+        mbar_wait(drain, 0, p.limit_ns, nullptr);
+      }
+    }
+  } else {
+    // ------------------------------------------------------------ epilogue
+    const int et = tid - 64;         // 0..127
+    const int quad = warp & 3;       // TMEM lane quadrant this warp may read
+    const int lanev = quad * 32 + lane;
+    bool ok = true;
+    if (p.force_timeout) {
+      ok = mbar_wait(dummy, 0, 20ull * 1000 * 1000, nullptr);
+      ok = named_barrier_and(1, 128, ok);
+      if (!ok && et == 0) record_error(p.status, abort, EBD_ERR_TIMEOUT);
+    }
+    int c = 0;
+    for (int u = u0; u < u1 && ok; u += 2, ++c) {
+      const int nu = min(2, u1 - u);
+      const int valid = min(nu * kUnit, p.V - u * kUnit);
+      const int buf = c % p.nbuf;
+      const uint32_t bph = static_cast<uint32_t>(c / p.nbuf) & 1u;
+      bool w = mbar_wait(&acc_full[buf], bph, p.limit_ns, abort);
+      ok = named_barrier_and(1, 128, w);
+      if (!ok) {
+        if (et == 0 && !*abort) record_error(p.status, abort, EBD_ERR_TIMEOUT);
+        break;
+      }
+      tc_fence_after();
+      const int vbase = u * kUnit;
+      for (int cc = 0; cc < p.n_pad; cc += 32) {
+        float v[32];
+        const uint32_t taddr = tmem_base + (static_cast<uint32_t>(quad * 32) << 16) +
+                               static_cast<uint32_t>(buf * p.acc_stride + cc);
+        if (p.n_pad - cc >= 32)
+          tmem_ld_32x32b_x32(taddr, v);
+        else
+          tmem_ld_32x32b_x16(taddr, v);
+        if (cc + 32 >= p.n_pad) {
+          tc_fence_before();
+          mbar_arrive(&acc_empty[buf]);
+        }
+        const bool lv = lanev < valid;
+#pragma unroll
+        for (int j = 0; j < 32; ++j) sT[j * kTLd + lanev] = lv ? v[j] : -INFINITY;
+        named_barrier(1, 128);
+        {
+          const int j = et >> 2, q = et & 3;
+          float x[32];
+#pragma unroll
+          for (int i = 0; i < 32; ++i) x[i] = sT[j * kTLd + q + 4 * i];
+          float m = -INFINITY, l2 = -INFINITY;
+          int idx = INT_MAX;
+#pragma unroll
+          for (int i = 0; i < 32; ++i) {
+            if (x[i] > m) {
+              l2 = m;
+              m = x[i];
+              idx = vbase + q + 4 * i;
+            } else if (x[i] > l2) {
+              l2 = x[i];
+            }
+          }
+          float s = 0.f, t = 0.f;
+          if (m != -INFINITY) {
+#pragma unroll
+            for (int i = 0; i < 32; ++i) {
+              const float dl = x[i] - m;
+              const float e = __expf(dl);
+              s += e;
+              if (e > 0.f) t = fmaf(e, dl, t);  // masked lanes: e = 0, dl = -inf
+            }
+          }
+#pragma unroll
+          for (int off = 1; off <= 2; off <<= 1) {
+            const float bm = __shfl_xor_sync(0xffffffffu, m, off);
+            const float bs = __shfl_xor_sync(0xffffffffu, s, off);
+            const float bt = __shfl_xor_sync(0xffffffffu, t, off);
+            const float bl = __shfl_xor_sync(0xffffffffu, l2, off);
+            const int bi = __shfl_xor_sync(0xffffffffu, idx, off);
+            state_merge(m, s, t, l2, idx, bm, bs, bt, bl, bi);
+          }
+          const int r = cc + j;
+          if (q == 0 && r < p.n_pad) {
+            float M = st_m[r], S = st_s[r], T = st_t[r], L2 = st_l2[r];
+            int I = st_i[r];
+            state_merge(M, S, T, L2, I, m, s, t, l2, idx);
+            st_m[r] = M;
+            st_s[r] = S;
+            st_t[r] = T;
+            st_l2[r] = L2;
+            st_i[r] = I;
+          }
+        }
+        named_barrier(1, 128);
+      }
+    }
+    if (ok) {
+      for (int r = et; r < p.rows; r += 128) {
+        const size_t o = static_cast<size_t>(p.row0 + r) * p.grid + cta;
+        p.part_f[o] = make_float4(st_m[r], st_s[r], st_t[r], st_l2[r]);
+        p.part_i[o] = st_i[r];
+      }
+    }
+  }
+
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem_base, p.tmem_cols);
+  }
+}
+
+void lm_plan(LmParams& p, int rows, int V, int d, int num_sms) {
+  p.V = V;
+  p.d = d;
+  p.rows = rows;
+  p.nsub = (rows + 255) / 256;
+  if (p.nsub < 1) p.nsub = 1;
+  p.nb = ((rows + p.nsub - 1) / p.nsub + 15) / 16 * 16;
+  if (p.nb < 16) p.nb = 16;
+  p.n_pad = p.nb * p.nsub;
+  p.acc_stride = (p.n_pad + 31) / 32 * 32;
+  p.nbuf = (2 * p.acc_stride <= 512) ? 2 : 1;
+  int cols = p.nbuf * p.acc_stride;
+  int tc = 32;
+  while (tc < cols) tc <<= 1;
+  p.tmem_cols = tc;
+  p.n_units = (V + kUnit - 1) / kUnit;
+  p.grid = num_sms < p.n_units ? num_sms : p.n_units;
+  p.nkb = (d + 63) / 64;
+  const uint32_t stage = kATile + static_cast<uint32_t>(p.n_pad) * 128u;
+  const uint32_t st_bytes = static_cast<uint32_t>(p.n_pad) * 20u;
+  const uint32_t tail = kTBytes + ((st_bytes + 7) / 8 * 8) + (2 * 8 + 6) * 8 + 16;
+  const uint32_t budget = 232448u - 1024u - tail;
+  int stages = static_cast<int>(budget / stage);
+  if (stages > 8) stages = 8;
+  p.stages = stages;
+  p.off_a = 0;
+  p.off_b = p.off_a + static_cast<uint32_t>(stages) * kATile;
+  p.off_t = p.off_b + static_cast<uint32_t>(stages) * static_cast<uint32_t>(p.n_pad) * 128u;
+  p.off_st = p.off_t + kTBytes;
+  p.off_bar = (p.off_st + st_bytes + 7) / 8 * 8;
+  p.smem_bytes = p.off_bar + static_cast<uint32_t>(2 * stages + 6) * 8u + 16u + 1024u;
+}
+
+cudaError_t lm_configure() {
+  return cudaFuncSetAttribute(lm_stats_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              232448);
+}
+
+cudaError_t launch_lm_stats(const CUtensorMap& tmap_w, const CUtensorMap& tmap_h,
+                            const LmParams& p, cudaStream_t st) {
+  lm_stats_kernel<<<p.grid, kLmThreads, p.smem_bytes, st>>>(tmap_w, tmap_h, p);
+  return cudaGetLastError();
+}
+
+}  // namespace ebd
