@@ -1,0 +1,539 @@
+#!/usr/bin/env python
+"""Benchmark of one Early-Bird decoding step (window attention, LM head with
+fused softmax statistics, EB decision) on GB300.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--config llada8b]
+                    [--state select|inblock] [--impl ours|reference]
+
+Prints ONE JSON line.  The default workload is the LLaDA-8B-shaped step
+(batch 1, hidden 4096, vocab 126464, 32x128 MHA, cached prefix 512, window
+32 with 24 masked rows, no active block so the LBS router runs).  `value` is
+window positions scored per second; `ms_per_step` the device time of one
+step (CUDA events around a CUDA-graph replay of ebd_step, L2 flushed by a
+256 MB write before every timed step, decode state restored outside the
+timed interval).  Multi-GPU runs are independent replicas (one process per
+GPU, no collective on the data path): value = rows of all ranks / max time.
+"""
+from __future__ import annotations
+
+import argparse
+import ctypes
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+
+METRIC = "µs/step & positions/s at LLaDA-8B shape; % of HBM/tensor roofline"
+UNIT = "positions/s"
+FALLBACK_HBM_GBS = 6800.0
+FALLBACK_BF16_TFLOPS = 1900.0
+
+
+# ----------------------------------------------------------------------------- helpers
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(p) as f:
+            d = json.load(f)
+        return (float(d["hbm_gbs"]), float(d["bf16_tflops"]),
+                float(d.get("bf16_tflops_sustained", d["bf16_tflops"])), "measured")
+    except Exception:
+        return FALLBACK_HBM_GBS, FALLBACK_BF16_TFLOPS, 1700.0, "fallback"
+
+
+def shape_for(name):
+    import synth
+    if name in synth.SHAPES:
+        return synth.SHAPES[name]
+    if name.startswith("sweep_"):
+        for s in synth.sweep_points():
+            if s.name == name:
+                return s
+    raise SystemExit(f"unknown config {name}")
+
+
+def workload_text(sh, state):
+    import synth
+    w = synth.window_sizes(sh)
+    return (f"{sh.name} decoding step: batch {sh.batch}, hidden {sh.d_model}, vocab {sh.vocab}, "
+            f"{sh.n_heads_q}q/{sh.n_heads_kv}kv heads x {sh.head_dim}, cached prefix {sh.prefix}, "
+            f"window rows {int(w.sum())} ({'no active block: LBS runs' if state == 'select' else 'active block'})")
+
+
+def lm_kernel_hash():
+    h = hashlib.sha256()
+    for f in ("k_lmhead.cu", "ptx.cuh", "internal.h"):
+        with open(os.path.join(ROOT, "paper_2609_16450_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def profiled_traffic(workload):
+    """DRAM bytes per LM-head launch from a committed ncu summary, or None if
+    the kernel changed since the counters were taken."""
+    p = os.path.join(ROOT, "profiles", f"lm_head_{workload}.json")
+    try:
+        with open(p) as f:
+            d = json.load(f)
+        if d.get("kernel_sha") != lm_kernel_hash():
+            return None
+        return float(d["dram_bytes_per_launch"])
+    except Exception:
+        return None
+
+
+class ClockSampler:
+    """Samples SM clock, power and clock-event reasons through NVML while the
+    timed region runs (read-only queries)."""
+
+    REASONS = {0x4: "sw_power_cap", 0x8: "hw_slowdown", 0x20: "sw_thermal_slowdown",
+               0x40: "hw_thermal_slowdown", 0x80: "hw_power_brake_slowdown", 0x1: "gpu_idle",
+               0x2: "applications_clocks_setting", 0x10: "sync_boost"}
+
+    def __init__(self, uuid: str, period_s: float = 0.002):
+        self.samples = []
+        self.max_mhz = None
+        self.err = None
+        self.period = period_s
+        self._stop = threading.Event()
+        self._t = None
+        try:
+            nv = ctypes.CDLL("libnvidia-ml.so.1")
+            if nv.nvmlInit_v2() != 0:
+                raise RuntimeError("nvmlInit failed")
+            h = ctypes.c_void_p()
+            if nv.nvmlDeviceGetHandleByUUID(("GPU-" + uuid).encode(), ctypes.byref(h)) != 0:
+                raise RuntimeError("nvmlDeviceGetHandleByUUID failed")
+            mx = ctypes.c_uint()
+            nv.nvmlDeviceGetMaxClockInfo(h, 1, ctypes.byref(mx))
+            self.max_mhz = int(mx.value)
+            self.nv, self.h = nv, h
+        except Exception as e:  # no NVML: no clock record
+            self.nv = None
+            self.err = str(e)
+
+    def _run(self):
+        nv, h = self.nv, self.h
+        mhz, reasons, mw = ctypes.c_uint(), ctypes.c_ulonglong(), ctypes.c_uint()
+        while not self._stop.is_set():
+            nv.nvmlDeviceGetClockInfo(h, 1, ctypes.byref(mhz))
+            r = nv.nvmlDeviceGetCurrentClocksEventReasons(h, ctypes.byref(reasons))
+            if r != 0:
+                nv.nvmlDeviceGetCurrentClocksThrottleReasons(h, ctypes.byref(reasons))
+            nv.nvmlDeviceGetPowerUsage(h, ctypes.byref(mw))
+            self.samples.append((int(mhz.value), int(reasons.value), mw.value / 1000.0))
+            time.sleep(self.period)
+
+    def start(self):
+        if self.nv is not None:
+            self._t = threading.Thread(target=self._run, daemon=True)
+            self._t.start()
+
+    def stop(self):
+        if self._t is not None:
+            self._stop.set()
+            self._t.join()
+
+    def summary(self):
+        if not self.samples:
+            return {"sm_mhz": None, "sm_max_mhz": self.max_mhz, "reasons": [],
+                    "samples": 0, "note": self.err or "no samples"}
+        mhz = [s[0] for s in self.samples]
+        bits = 0
+        for s in self.samples:
+            bits |= s[1]
+        reasons = sorted(v for k, v in self.REASONS.items() if bits & k and k != 0x1)
+        return {"sm_mhz": statistics.median(mhz), "sm_max_mhz": self.max_mhz,
+                "reasons": reasons, "samples": len(mhz),
+                "power_w_max": round(max(s[2] for s in self.samples), 1)}
+
+
+# ----------------------------------------------------------------------------- work model
+def step_work(sh, rows, masked, grid_lm, lbs_runs):
+    """Algorithmic bytes and flops of one step (each input read once)."""
+    d, V, Hq, Hkv, D = sh.d_model, sh.vocab, sh.n_heads_q, sh.n_heads_kv, sh.head_dim
+    import synth
+    w = synth.window_sizes(sh)
+    keys = int(sum(sh.prefix + int(x) for x in w))
+    lm_bytes = V * d * 2 + rows * d * 2 + rows * grid_lm * 20
+    lm_flops = 2 * rows * d * V
+    attn_bytes = keys * Hkv * D * 2 * 2 + rows * Hq * D * 2 + rows * Hq * D * 4
+    attn_flops = 4 * sum(int(x) * (sh.prefix + int(x)) for x in w) * Hq * D
+    dec_bytes = rows * grid_lm * 20 + rows * 40
+    if lbs_runs:
+        dec_bytes += 2 * (613761 - 262208) + masked * 64 * 4
+    return dict(lm_bytes=lm_bytes, lm_flops=lm_flops, attn_bytes=attn_bytes,
+                attn_flops=attn_flops, step_bytes=lm_bytes + attn_bytes + dec_bytes,
+                step_flops=lm_flops + attn_flops)
+
+
+# ----------------------------------------------------------------------------- our arm
+def run_ours(args, rank, world, local_rank):
+    import torch
+    torch.cuda.set_device(local_rank)
+    from paper_2609_16450_gb300 import build as B
+    if rank == 0 or world == 1:
+        B.build()
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+    B.build()
+    from paper_2609_16450_gb300 import _ebd as E
+    from paper_2609_16450_gb300 import runtime as rt
+    import synth
+
+    sh = shape_for(args.config)
+    inp = synth.make_step_inputs(sh)
+    if args.state == "inblock":
+        synth.preset_in_block(inp, 20)
+    w = rt.upload_weights(inp)
+    h = rt.Handle(rt.config_for(sh), w.w_emb)
+    if args.w_layout == "packed":
+        w = rt.pack_weights(h, w)  # one-time tiling of W_lm (model load)
+    ds = rt.DeviceStep(inp, w, attention=True)
+    stream = torch.cuda.Stream()
+    sid = stream.cuda_stream
+    args_c = ds.args()
+    E.check(E.ebd_profile_enable(h.h, True), h.h)
+    flush = torch.empty(256 * 1024 * 1024 // 4, dtype=torch.float32, device="cuda")
+    torch.cuda.synchronize()
+
+    graph = None
+    if not args.no_graph:
+        with torch.cuda.stream(stream):
+            E.check(E.ebd_step(h.h, args_c, sid), h.h)  # warm once outside capture
+        torch.cuda.synchronize()
+        ds.restore_state()
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph, stream=stream):
+            E.check(E.ebd_step(h.h, args_c, stream.cuda_stream), h.h)
+        torch.cuda.synchronize()
+
+    def one_step():
+        if graph is not None:
+            graph.replay()
+        else:
+            E.check(E.ebd_step(h.h, args_c, sid), h.h)
+
+    with torch.cuda.stream(stream):
+        for _ in range(args.warmup):
+            ds.restore_state()
+            one_step()
+    torch.cuda.synchronize()
+    if h.sync_status(sid) != 0:
+        raise SystemExit(f"device status after warm-up: {E.ebd_last_error(h.h)}")
+
+    sampler = ClockSampler(str(torch.cuda.get_device_properties(local_rank).uuid))
+    ev0 = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    ev1 = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    kern = []
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+    torch.cuda.synchronize()
+    sampler.start()
+    t_wall = time.perf_counter()
+    with torch.cuda.stream(stream):
+        for i in range(args.steps):
+            ds.restore_state()
+            flush.fill_(float(i))
+            ev0[i].record(stream)
+            one_step()
+            ev1[i].record(stream)
+            stream.synchronize()
+            s, ms = E.ebd_profile_read(h.h)
+            if s != 0:
+                raise SystemExit(f"ebd_profile_read: {E.ebd_last_error(h.h)}")
+            kern.append(ms)
+    torch.cuda.synchronize()
+    t_wall = time.perf_counter() - t_wall
+    if world > 1:
+        dist.barrier()
+    sampler.stop()
+    status = h.sync_status(sid)
+    if status != 0:
+        raise SystemExit(f"device status {status}: {E.ebd_last_error(h.h)}")
+    step_ms = [a.elapsed_time(b) for a, b in zip(ev0, ev1)]
+    mean_ms = float(np.mean(step_ms))
+    if world > 1:
+        t = torch.tensor([mean_ms], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        mean_ms = float(t.item())
+    kern = np.array(kern)
+    k_attn, k_lm, k_dec = (float(np.mean(kern[:, i])) for i in range(3))
+
+    # end to end through ebd_step_host: pinned host inputs in, results out
+    e2e = None
+    if not args.skip_e2e:
+        e2e = run_e2e(args, h, ds, inp, sh, stream, world)
+    out = dict(sh=sh, inp=inp, rows=inp.rows, masked=int(inp.mask.sum()), mean_ms=mean_ms,
+               step_ms=step_ms, k_attn=k_attn, k_lm=k_lm, k_dec=k_dec, grid_lm=None,
+               clocks=sampler.summary(), e2e=e2e, t_wall=t_wall,
+               lbs_runs=args.state == "select")
+    out["launches_per_step"] = 2 + (inp.rows + 511) // 512
+    out["fetch"] = ds.fetch()
+    h_sms = torch.cuda.get_device_properties(local_rank).multi_processor_count
+    out["grid_lm"] = min(h_sms, (sh.vocab + 63) // 64)
+    out["num_sms"] = h_sms
+    h.close()
+    return out
+
+
+def run_e2e(args, h, ds, inp, sh, stream, world):
+    """Same step through ebd_step_host: every step copies its inputs from
+    pinned host memory and its results back inside the timed interval."""
+    import torch
+    from paper_2609_16450_gb300 import _ebd as E
+    R, Hq, Hkv, D = inp.rows, sh.n_heads_q, sh.n_heads_kv, sh.head_dim
+    pin = lambda a: torch.from_numpy(np.ascontiguousarray(a)).pin_memory()  # noqa: E731
+    host_in = dict(cu_rows=pin(inp.cu_rows.astype(np.int32)),
+                   prefix_len=pin(inp.prefix_len.astype(np.int32)),
+                   row_pos=pin(inp.row_pos.astype(np.int32)),
+                   hidden=pin(inp.hidden.view(np.int16)), q=pin(inp.q.view(np.int16)),
+                   k_win=pin(inp.k_win.view(np.int16)), v_win=pin(inp.v_win.view(np.int16)))
+    st0 = dict(tokens=inp.tokens.astype(np.int32), mask=inp.mask.astype(np.uint8),
+               in_block=inp.in_block.astype(np.uint8), blk_meta=inp.blk_meta.astype(np.int32))
+    host_state = {k: pin(v) for k, v in st0.items()}
+    host_out = dict(attn_out=torch.empty((R, Hq, D), dtype=torch.float32).pin_memory())
+    for k in ("conf", "entropy", "ent_norm", "gap", "lbs_logit", "lps_prob"):
+        host_out[k] = torch.empty(R, dtype=torch.float32).pin_memory()
+    host_out["argmax"] = torch.empty(R, dtype=torch.int32).pin_memory()
+    host_out["accepted"] = torch.empty(R, dtype=torch.uint8).pin_memory()
+    a = E.ebd_step_args()
+    a.batch, a.rows = sh.batch, R
+    for k, t in {**host_in, **host_state, **host_out}.items():
+        setattr(a, k, t.data_ptr())
+    a.k_cache, a.v_cache, a.w_lm = ds.k_cache.data_ptr(), ds.v_cache.data_ptr(), \
+        ds.weights.w_lm.data_ptr()
+    a.w_lm_layout = ds.weights.layout
+    h2d = sum(t.numel() * t.element_size() for t in host_in.values()) + \
+        sum(t.numel() * t.element_size() for t in host_state.values())
+    d2h = sum(t.numel() * t.element_size() for t in host_state.values()) + \
+        sum(t.numel() * t.element_size() for t in host_out.values())
+    sid = stream.cuda_stream
+    E.check(E.ebd_profile_enable(h.h, False), h.h)
+
+    def reset():
+        for k, v in st0.items():
+            host_state[k].numpy()[...] = v
+
+    for _ in range(max(1, args.warmup)):
+        reset()
+        E.check(E.ebd_step_host(h.h, a, sid), h.h)
+        stream.synchronize()
+    flush = torch.empty(256 * 1024 * 1024 // 4, dtype=torch.float32, device="cuda")
+    times = []
+    with torch.cuda.stream(stream):
+        for i in range(args.steps):
+            reset()
+            flush.fill_(float(i))
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            E.check(E.ebd_step_host(h.h, a, sid), h.h)
+            e1.record(stream)
+            stream.synchronize()
+            times.append(e0.elapsed_time(e1))
+    if h.sync_status(sid) != 0:
+        raise SystemExit("device status after e2e")
+    mean_ms = float(np.mean(times))
+    if world > 1:
+        import torch.distributed as dist
+        t = torch.tensor([mean_ms], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        mean_ms = float(t.item())
+    return dict(mean_ms=mean_ms, h2d=int(h2d), d2h=int(d2h))
+
+
+# ----------------------------------------------------------------------------- oracle arm
+def oracle_step_sample(sh, inp, budget_s):
+    """Times the CPU oracle on the step's inputs: full steps until budget_s
+    has passed (at least one).  Returns (positions/s, steps, seconds)."""
+    from oracle import ebd_oracle as o
+    import synth
+    W = o.weights_f64(synth.router_weights(sh.seed, sh.d_base, sh.gen_len))
+    prm = o.DecisionParams(tau=sh.tau, tau_psi=sh.tau_psi, l_min=sh.l_min, l_b=sh.l_b,
+                           g_max=sh.g_max, eos_id=sh.eos_id, lps_enabled=bool(sh.lps_enabled))
+    n, t0 = 0, time.perf_counter()
+    while True:
+        o.step(inp, W, prm)
+        n += 1
+        el = time.perf_counter() - t0
+        if el >= budget_s:
+            break
+    return inp.rows * n / el, n, el
+
+
+def run_reference(args, rank, world):
+    """The CPU oracle as the reference arm: rank 0 only."""
+    if rank != 0:
+        return
+    import synth
+    sh = shape_for(args.config)
+    inp = synth.make_step_inputs(sh)
+    if args.state == "inblock":
+        synth.preset_in_block(inp, 20)
+    from oracle import ebd_oracle as o
+    W = o.weights_f64(synth.router_weights(sh.seed, sh.d_base, sh.gen_len))
+    prm = o.DecisionParams(tau=sh.tau, tau_psi=sh.tau_psi, l_min=sh.l_min, l_b=sh.l_b,
+                           g_max=sh.g_max, eos_id=sh.eos_id, lps_enabled=bool(sh.lps_enabled))
+    # size each step's sample so that warm-up + timed steps fit in ~150 s
+    t0 = time.perf_counter()
+    o.step(inp, W, prm)
+    t_full = time.perf_counter() - t0
+    budget = 150.0 / max(1, args.steps + args.warmup)
+    rows = inp.rows
+    if t_full > budget:
+        rows = max(1, int(inp.rows * budget / t_full))
+    sub = inp if rows == inp.rows else _row_sample(inp, rows)
+    for _ in range(args.warmup):
+        o.step(sub, W, prm)
+    times = []
+    for _ in range(args.steps):
+        t0 = time.perf_counter()
+        o.step(sub, W, prm)
+        times.append(time.perf_counter() - t0)
+    ms = 1000.0 * float(np.mean(times))
+    value = rows / (ms / 1000.0)
+    cores = os.cpu_count()
+    sample = (f"oracle step on {rows} of {inp.rows} window rows of {sh.name} per timed step"
+              if rows != inp.rows else f"full oracle step of {sh.name} ({inp.rows} rows)")
+    line = {"impl": "reference", "metric": METRIC, "value": round(value, 3), "unit": UNIT,
+            "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": round(ms, 3), "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": workload_text(sh, args.state), "state": args.state},
+            "cpu_baseline": {"value": round(value, 3), "unit": UNIT, "cores": cores,
+                             "kind": "oracle", "sample": sample},
+            "e2e": {"value": round(value, 3), "unit": UNIT, "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line))
+
+
+def _row_sample(inp, rows):
+    """First `rows` window rows of the single-sequence step (bounded sample)."""
+    import copy
+    s = copy.copy(inp)
+    s.cu_rows = np.array([0, rows], np.int32)
+    s.row_pos = inp.row_pos[:rows]
+    for k in ("hidden", "q", "k_win", "v_win", "tokens", "mask", "in_block"):
+        setattr(s, k, getattr(inp, k)[:rows])
+    return s
+
+
+# ----------------------------------------------------------------------------- main
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--config", default="llada8b")
+    ap.add_argument("--state", choices=["select", "inblock"], default="select")
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--skip-cpu", action="store_true", help="omit the cpu_baseline leg")
+    ap.add_argument("--skip-e2e", action="store_true", help="omit the end-to-end leg")
+    ap.add_argument("--no-graph", action="store_true", help="launch ebd_step without a graph")
+    ap.add_argument("--cpu-budget", type=float, default=12.0)
+    ap.add_argument("--w-layout", choices=["packed", "rowmajor"], default="packed",
+                    help="W_lm tiled once by ebd_pack_lm_head (default) or row-major")
+    args = ap.parse_args()
+    args.warmup = max(args.warmup, 3)
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.impl == "reference":
+        run_reference(args, rank, world)
+        return
+    import torch
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local_rank)
+        dist.init_process_group("nccl")
+    r = run_ours(args, rank, world, local_rank)
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+    if rank != 0:
+        if world > 1:
+            dist.destroy_process_group()
+        return
+
+    sh = r["sh"]
+    hbm, bf16, bf16_sus, peak_src = load_peaks()
+    wk = step_work(sh, r["rows"], r["masked"], r["grid_lm"], r["lbs_runs"])
+    t_lm = r["k_lm"] / 1000.0
+    lm_hbm_t = wk["lm_bytes"] / (hbm * 1e9)
+    lm_tc_t = wk["lm_flops"] / (bf16 * 1e12)
+    if lm_hbm_t >= lm_tc_t:
+        roof = {"bound": "hbm", "achieved": round(wk["lm_bytes"] / t_lm / 1e9, 1),
+                "peak": hbm, "unit": "GB/s"}
+    else:
+        roof = {"bound": "tensor", "achieved": round(wk["lm_flops"] / t_lm / 1e12, 1),
+                "peak": bf16, "unit": "TFLOP/s"}
+    roof["frac"] = round(roof["achieved"] / roof["peak"], 4)
+    roof["traffic"] = profiled_traffic(sh.name)
+    roof["kernel"] = "lm_stats_kernel (LM head + online softmax statistics)"
+    roof["algorithmic"] = {"bytes": wk["lm_bytes"], "flops": wk["lm_flops"]}
+    roof["peak_source"] = f"{peak_src} (MEASURED_PEAKS.json)" if peak_src == "measured" else "fallback"
+    t_step = r["mean_ms"] / 1000.0
+    t_roof = max(wk["step_bytes"] / (hbm * 1e9), wk["step_flops"] / (bf16 * 1e12))
+    value = r["rows"] * world / t_step
+    line = {
+        "metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(r["mean_ms"], 5),
+        "us_per_step": round(r["mean_ms"] * 1000, 2),
+        "us_per_step_p10_p50_p90": [round(float(np.percentile(r["step_ms"], q)) * 1000, 2)
+                                    for q in (10, 50, 90)],
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic (seeded; LLaDA-8B/Dream-7B shapes, random-init routers)",
+        "config": {"workload": workload_text(sh, args.state), "state": args.state,
+                   "rows": r["rows"], "masked": r["masked"],
+                   "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
+                   "l2": "flushed before every timed step (256 MB write); W_lm (1 GB) > L2",
+                   "launch": "cuda_graph" if not args.no_graph else "stream",
+                   "w_lm": ("64x64 tiles, unit-major (ebd_pack_lm_head, once at load)"
+                            if args.w_layout == "packed" else "row-major [V][d]")},
+        "roofline": roof,
+        "step_roofline": {"bytes": wk["step_bytes"], "flops": wk["step_flops"],
+                          "t_roofline_us": round(t_roof * 1e6, 2),
+                          "frac": round(t_roof / t_step, 4),
+                          "peak_hbm_gbs": hbm, "peak_bf16_tflops": bf16},
+        "kernels_us": {"attention": round(r["k_attn"] * 1000, 2),
+                       "lm_head": round(r["k_lm"] * 1000, 2),
+                       "decision": round(r["k_dec"] * 1000, 2)},
+        "decision_share": round(r["k_dec"] / max(1e-9, r["mean_ms"]), 4),
+        "gpu_launches": int(r["launches_per_step"] * args.steps),
+        "clocks": r["clocks"],
+    }
+    if r["e2e"] is not None:
+        e = r["e2e"]
+        line["e2e"] = {"value": round(r["rows"] * world / (e["mean_ms"] / 1000.0), 1),
+                       "unit": UNIT, "h2d_bytes_per_step": e["h2d"],
+                       "d2h_bytes_per_step": e["d2h"], "ms_per_step": round(e["mean_ms"], 4),
+                       "api": "ebd_step_host"}
+    if not args.skip_cpu and world == 1:
+        v, n, el = oracle_step_sample(sh, r["inp"], args.cpu_budget)
+        line["cpu_baseline"] = {"value": round(v, 3), "unit": UNIT, "cores": os.cpu_count(),
+                                "kind": "oracle",
+                                "sample": f"{n} full oracle steps of {sh.name} "
+                                          f"({r['rows']} rows each) in {el:.1f} s"}
+    print(json.dumps(line))
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

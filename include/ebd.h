@@ -125,6 +125,10 @@ typedef struct {
   float* lbs_logit;           /* [R] O_phi where LBS ran, NaN elsewhere          */
   float* lps_prob;            /* [R] p_psi where LPS scored, NaN elsewhere       */
   uint8_t* accepted;          /* [R] 1 = committed this step                     */
+  int32_t w_lm_layout;        /* 0: w_lm is [vocab][d_model] row-major;
+                                 1: w_lm is the tiled copy written by
+                                 ebd_pack_lm_head()                           */
+  int32_t reserved;
 } ebd_step_args;
 
 /* Creates a handle on the current CUDA device: validates *cfg, allocates the
@@ -143,6 +147,20 @@ void ebd_destroy(ebd_handle* h);
  * gathered rows of every step).  Must precede any step in which LBS runs;
  * ebd_import_weights() re-folds with the bound table.  Enqueued on stream. */
 ebd_status ebd_bind_embedding(ebd_handle* h, const uint16_t* w_emb, void* stream);
+
+/* Size in bytes of the tiled LM-head weight written by ebd_pack_lm_head():
+ * ceil(vocab/64) * ceil(d_model/64) tiles of 64 x 64 bf16. */
+size_t ebd_lm_head_packed_bytes(const ebd_config* cfg);
+
+/* Writes W_lm ([vocab][d_model] bf16, device) into the tiled layout the LM
+ * head streams fastest: tile (u, k) holds rows 64u..64u+63 and columns
+ * 64k..64k+63, row-major; tiles ordered u-major, so the 64-row block of the
+ * vocabulary that one work unit reads is one contiguous run of memory.
+ * Rows and columns past the matrix are zero.  w_packed is a caller-owned
+ * device buffer of ebd_lm_head_packed_bytes() bytes, 16-byte aligned.  A
+ * one-time transform (model load); enqueued on stream. */
+ebd_status ebd_pack_lm_head(ebd_handle* h, const uint16_t* w_lm, uint16_t* w_packed,
+                            void* stream);
 
 /* One EB decoding step (see top of file).  Enqueue only. */
 ebd_status ebd_step(ebd_handle* h, const ebd_step_args* a, void* stream);
@@ -203,6 +221,14 @@ ebd_status ebd_router_init_host(const ebd_config* cfg, void* host, size_t* bytes
 
 /* Number of bf16 elements of the weight blob for cfg. */
 size_t ebd_weight_count(const ebd_config* cfg);
+
+/* Per-kernel timing of ebd_step: with on != 0 every later ebd_step records
+ * CUDA events on its stream before the first kernel and after the window
+ * attention, the LM head and the decision (also inside a captured graph).
+ * ebd_profile_read waits for the last recorded event and writes the three
+ * durations in milliseconds to ms[0..2] (attention, LM head, decision). */
+ebd_status ebd_profile_enable(ebd_handle* h, int on);
+ebd_status ebd_profile_read(ebd_handle* h, float* ms);
 
 /* Last error message of the handle (never NULL; "" if none). */
 const char* ebd_last_error(const ebd_handle* h);

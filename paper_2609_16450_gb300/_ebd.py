@@ -45,13 +45,15 @@ class ebd_step_args(Structure):
                 ("blk_meta", c_void_p), ("attn_out", c_void_p), ("conf", c_void_p),
                 ("entropy", c_void_p), ("ent_norm", c_void_p), ("gap", c_void_p),
                 ("argmax", c_void_p), ("lbs_logit", c_void_p), ("lps_prob", c_void_p),
-                ("accepted", c_void_p)]
+                ("accepted", c_void_p), ("w_lm_layout", c_int32), ("reserved", c_int32)]
 
 
 EXPORTS = ["ebd_create", "ebd_destroy", "ebd_bind_embedding", "ebd_step", "ebd_step_host",
            "ebd_decide", "ebd_lm_stats", "ebd_attention", "ebd_sync_status",
            "ebd_export_weights", "ebd_import_weights", "ebd_router_init_host",
-           "ebd_weight_count", "ebd_last_error", "ebd_version"]
+           "ebd_weight_count", "ebd_lm_head_packed_bytes", "ebd_pack_lm_head",
+           "ebd_profile_enable", "ebd_profile_read", "ebd_last_error",
+           "ebd_version"]
 
 _lib = None
 
@@ -85,6 +87,11 @@ def load(path: str = LIB_PATH):
     lib.ebd_weight_count.restype = c_size_t
     lib.ebd_last_error.argtypes = [c_void_p]
     lib.ebd_last_error.restype = c_char_p
+    lib.ebd_lm_head_packed_bytes.argtypes = [P(ebd_config)]
+    lib.ebd_lm_head_packed_bytes.restype = c_size_t
+    lib.ebd_pack_lm_head.argtypes = [c_void_p, c_void_p, c_void_p, c_void_p]
+    lib.ebd_profile_enable.argtypes = [c_void_p, c_int32]
+    lib.ebd_profile_read.argtypes = [c_void_p, P(c_float)]
     lib.ebd_version.argtypes = []
     lib.ebd_version.restype = c_char_p
     for fn in EXPORTS:
@@ -171,6 +178,25 @@ def ebd_router_init_host(cfg: ebd_config):
 
 def ebd_weight_count(cfg: ebd_config) -> int:
     return int(load().ebd_weight_count(ctypes.byref(cfg)))
+
+
+def ebd_lm_head_packed_bytes(cfg: ebd_config) -> int:
+    return int(load().ebd_lm_head_packed_bytes(ctypes.byref(cfg)))
+
+
+def ebd_pack_lm_head(h, w_lm_ptr: int, w_packed_ptr: int, stream: int = 0) -> int:
+    return load().ebd_pack_lm_head(h, c_void_p(w_lm_ptr), c_void_p(w_packed_ptr), c_void_p(stream))
+
+
+def ebd_profile_enable(h, on: bool) -> int:
+    return load().ebd_profile_enable(h, 1 if on else 0)
+
+
+def ebd_profile_read(h):
+    """Returns (status, [attention_ms, lm_head_ms, decision_ms])."""
+    ms = (c_float * 3)()
+    s = load().ebd_profile_read(h, ms)
+    return s, [float(x) for x in ms]
 
 
 def ebd_last_error(h) -> str:

@@ -9,6 +9,7 @@
 
 #include "ebd.h"
 #include "internal.h"
+#include "router_image.h"
 
 namespace ebd {
 cudaError_t decide_configure();
@@ -25,7 +26,7 @@ using namespace ebd;
 namespace {
 
 constexpr uint64_t kLimitNs = 1000ull * 1000 * 1000;  // 1 s per device-side wait
-constexpr int kMaxSplits = 8;
+constexpr int kMaxSplits = kMaxAttnSplits;
 
 // ------------------------------------------------------------------ router layout
 struct TensorDesc {
@@ -161,6 +162,17 @@ bool encode_bf16(CUtensorMap* m, const void* base, int rank, const uint64_t* dim
 
 bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
 
+// Event record that also executes when the stream is being captured into a
+// CUDA graph (an external event-record node rather than a dependency edge).
+cudaError_t record(cudaEvent_t ev, cudaStream_t st) {
+  cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+  cudaError_t e = cudaStreamIsCapturing(st, &cs);
+  if (e != cudaSuccess) return e;
+  if (cs == cudaStreamCaptureStatusActive)
+    return cudaEventRecordWithFlags(ev, st, cudaEventRecordExternal);
+  return cudaEventRecord(ev, st);
+}
+
 }  // namespace
 
 struct ebd_handle {
@@ -178,11 +190,14 @@ struct ebd_handle {
   int* part_i = nullptr;
   int grid_lm = 0;
   float* attn_part = nullptr;
+  float* attn_part_ml = nullptr;
   int* tickets = nullptr;
   int attn_splits = 1, attn_max_qtiles = 1;
   int* d_status = nullptr;
   uint8_t* staging = nullptr;
   size_t staging_bytes = 0;
+  cudaEvent_t ev[4] = {nullptr, nullptr, nullptr, nullptr};
+  int profile = 0;
 };
 
 namespace {
@@ -224,8 +239,9 @@ ebd_status check_device(ebd_handle* h) {
   return EBD_OK;
 }
 
-// Builds the decision kernel's weight image from the host blob.
+// Builds the decision kernel's weight image (router_image.h) from the blob.
 ebd_status upload_router(ebd_handle* h) {
+  using namespace rimg;
   const auto& L = h->layout;
   std::vector<size_t> off(L.size());
   {
@@ -235,132 +251,130 @@ ebd_status upload_router(ebd_handle* h) {
       o += static_cast<size_t>(L[i].rows) * L[i].cols;
     }
   }
-  auto find = [&](const std::string& n) -> size_t {
+  auto T = [&](const std::string& n) -> const TensorDesc& {
+    for (size_t i = 0; i < L.size(); ++i)
+      if (L[i].name == n) return L[i];
+    return L[0];
+  };
+  auto idx = [&](const std::string& n) -> size_t {
     for (size_t i = 0; i < L.size(); ++i)
       if (L[i].name == n) return i;
-    return static_cast<size_t>(-1);
+    return 0;
   };
-  std::vector<uint8_t> img;
-  auto align = [&]() { img.resize((img.size() + 255) / 256 * 256); };
-  auto put_f32 = [&](const std::string& n) -> size_t {
-    align();
-    const size_t i = find(n);
-    const size_t cnt = static_cast<size_t>(L[i].rows) * L[i].cols;
-    const size_t at = img.size();
-    img.resize(at + cnt * 4);
-    float* dst = reinterpret_cast<float*>(img.data() + at);
-    for (size_t k = 0; k < cnt; ++k) dst[k] = bf16_to_f32(h->h_blob[off[i] + k]);
-    return at;
+  // element (r, c) of tensor n as bf16 bits / float
+  auto at = [&](const std::string& n, int r, int c) -> uint16_t {
+    const size_t i = idx(n);
+    return h->h_blob[off[i] + static_cast<size_t>(r) * L[i].cols + c];
   };
-  // transposed [cols][rows] of a [rows][cols] matrix, bf16 or fp32
-  auto put_t = [&](const std::string& n, bool as_f32) -> size_t {
-    align();
-    const size_t i = find(n);
-    const int R = L[i].rows, C = L[i].cols;
-    const size_t at = img.size();
-    img.resize(at + static_cast<size_t>(R) * C * (as_f32 ? 4 : 2));
-    for (int r = 0; r < R; ++r)
-      for (int c = 0; c < C; ++c) {
-        const uint16_t v = h->h_blob[off[i] + static_cast<size_t>(r) * C + c];
-        if (as_f32)
-          reinterpret_cast<float*>(img.data() + at)[static_cast<size_t>(c) * R + r] = bf16_to_f32(v);
-        else
-          reinterpret_cast<uint16_t*>(img.data() + at)[static_cast<size_t>(c) * R + r] = v;
+  auto atf = [&](const std::string& n, int r, int c) { return bf16_to_f32(at(n, r, c)); };
+  (void)T;
+  std::vector<uint16_t> lbs(static_cast<size_t>(kRanks) * LBS_W_ELEMS, 0);
+  std::vector<uint16_t> lps(LPS_W_ELEMS, 0);
+  std::vector<float> vec(static_cast<size_t>(kRanks) * V_ELEMS, 0.f);
+  const int gen_len = h->cfg.gen_len;
+  for (int r = 0; r < kRanks; ++r) {
+    uint16_t* w = lbs.data() + static_cast<size_t>(r) * LBS_W_ELEMS;
+    float* v = vec.data() + static_cast<size_t>(r) * V_ELEMS;
+    for (int k = 0; k < 64; ++k)
+      for (int o = 0; o < 64; ++o) w[W_ENT2 + k * 64 + o] = at("lbs.ent2.w", o, k);
+    for (int k = 0; k < 128; ++k)
+      for (int o = 0; o < kCombSlice; ++o)
+        w[W_COMB + k * kCombSlice + o] = at("lbs.comb.w", kCombSlice * r + o, k);
+    for (int j = 0; j < kPosRows; ++j)
+      for (int o = 0; o < kCombSlice; ++o)
+        w[W_POS + j * kCombSlice + o] = j < gen_len ? at("lbs.pos", j, kCombSlice * r + o) : 0;
+    for (int l = 0; l < 2; ++l) {
+      const std::string pre = "lbs.l" + std::to_string(l);
+      uint16_t* wl = w + W_LAYER0 + l * W_LAYER_STRIDE;
+      float* vl = v + V_LAYER0 + l * V_LAYER_STRIDE;
+      for (int k = 0; k < 128; ++k) {
+        for (int o = 0; o < kQkvSlice; ++o)
+          wl[WL_QKV + k * kQkvSlice + o] = at(pre + ".qkv.w", kQkvSlice * r + o, k);
+        for (int o = 0; o < kOutSlice; ++o)
+          wl[WL_OUT + k * kOutSlice + o] = at(pre + ".out.w", kOutSlice * r + o, k);
+        for (int o = 0; o < kFf1Slice; ++o)
+          wl[WL_FF1 + k * kFf1Slice + o] = at(pre + ".ff1.w", kFf1Slice * r + o, k);
       }
-    return at;
-  };
-  auto put_raw = [&](const std::string& n) -> size_t {  // bf16 as stored
-    align();
-    const size_t i = find(n);
-    const size_t cnt = static_cast<size_t>(L[i].rows) * L[i].cols;
-    const size_t at = img.size();
-    img.resize(at + cnt * 2);
-    std::memcpy(img.data() + at, h->h_blob.data() + off[i], cnt * 2);
-    return at;
-  };
-  struct {
-    size_t ent1_w, ent1_b, ent2_b, ent_ln_g, ent_ln_b, tok_b, comb_b, head_w, head_b, ent2_t,
-        comb_t, pos;
-    size_t lq[2][12];
-    size_t in_t, in_b, in_ln_g, in_ln_b, lh_w, lh_b;
-    size_t pq[2][12];
-  } o{};
-  o.ent1_w = put_f32("lbs.ent1.w");
-  o.ent1_b = put_f32("lbs.ent1.b");
-  o.ent2_b = put_f32("lbs.ent2.b");
-  o.ent_ln_g = put_f32("lbs.ent_ln.g");
-  o.ent_ln_b = put_f32("lbs.ent_ln.b");
-  o.tok_b = put_f32("lbs.tok.b");
-  o.comb_b = put_f32("lbs.comb.b");
-  o.head_w = put_f32("lbs.head.w");
-  o.head_b = put_f32("lbs.head.b");
-  o.ent2_t = put_t("lbs.ent2.w", false);
-  o.comb_t = put_t("lbs.comb.w", false);
-  o.pos = put_raw("lbs.pos");
-  for (int l = 0; l < 2; ++l) {
-    const std::string p = "lbs.l" + std::to_string(l);
-    o.lq[l][0] = put_t(p + ".qkv.w", false);
-    o.lq[l][1] = put_t(p + ".out.w", false);
-    o.lq[l][2] = put_t(p + ".ff1.w", false);
-    o.lq[l][3] = put_t(p + ".ff2.w", false);
-    o.lq[l][4] = put_f32(p + ".qkv.b");
-    o.lq[l][5] = put_f32(p + ".out.b");
-    o.lq[l][6] = put_f32(p + ".ff1.b");
-    o.lq[l][7] = put_f32(p + ".ff2.b");
-    o.lq[l][8] = put_f32(p + ".ln1.g");
-    o.lq[l][9] = put_f32(p + ".ln1.b");
-    o.lq[l][10] = put_f32(p + ".ln2.g");
-    o.lq[l][11] = put_f32(p + ".ln2.b");
+      for (int hh = 0; hh < kFf1Slice; ++hh)
+        for (int o = 0; o < 128; ++o)
+          wl[WL_FF2 + hh * 128 + o] = at(pre + ".ff2.w", o, kFf1Slice * r + hh);
+      for (int o = 0; o < kQkvSlice; ++o) vl[VL_QKVB + o] = atf(pre + ".qkv.b", 0, kQkvSlice * r + o);
+      for (int o = 0; o < kOutSlice; ++o) vl[VL_OUTB + o] = atf(pre + ".out.b", 0, kOutSlice * r + o);
+      for (int o = 0; o < kFf1Slice; ++o) vl[VL_FF1B + o] = atf(pre + ".ff1.b", 0, kFf1Slice * r + o);
+      for (int o = 0; o < kOutSlice; ++o) vl[VL_FF2B + o] = atf(pre + ".ff2.b", 0, kOutSlice * r + o);
+      for (int o = 0; o < 128; ++o) {
+        vl[VL_LN1G + o] = atf(pre + ".ln1.g", 0, o);
+        vl[VL_LN1B + o] = atf(pre + ".ln1.b", 0, o);
+        vl[VL_LN2G + o] = atf(pre + ".ln2.g", 0, o);
+        vl[VL_LN2B + o] = atf(pre + ".ln2.b", 0, o);
+      }
+    }
+    for (int o = 0; o < 64; ++o) {
+      v[V_ENT1W + o] = atf("lbs.ent1.w", o, 0);
+      v[V_ENT1B + o] = atf("lbs.ent1.b", 0, o);
+      v[V_ENT2B + o] = atf("lbs.ent2.b", 0, o);
+      v[V_ENTLNG + o] = atf("lbs.ent_ln.g", 0, o);
+      v[V_ENTLNB + o] = atf("lbs.ent_ln.b", 0, o);
+      v[V_TOKB + o] = atf("lbs.tok.b", 0, o);
+    }
+    for (int o = 0; o < 128; ++o) v[V_HEADW + o] = atf("lbs.head.w", 0, o);
+    v[V_HEADB] = atf("lbs.head.b", 0, 0);
+    for (int o = 0; o < kCombSlice; ++o) v[V_COMBB + o] = atf("lbs.comb.b", 0, kCombSlice * r + o);
+    // LPS vectors (every rank holds them; rank 0 uses them)
+    float* vp = v + V_LPS;
+    for (int k = 0; k < 5; ++k)
+      for (int o = 0; o < 32; ++o) vp[VP_INT + k * 32 + o] = atf("lps.in.w", o, k);
+    for (int o = 0; o < 32; ++o) {
+      vp[VP_INB + o] = atf("lps.in.b", 0, o);
+      vp[VP_INLNG + o] = atf("lps.in_ln.g", 0, o);
+      vp[VP_INLNB + o] = atf("lps.in_ln.b", 0, o);
+      vp[VP_HEADW + o] = atf("lps.head.w", 0, o);
+    }
+    vp[VP_HEADB] = atf("lps.head.b", 0, 0);
+    for (int l = 0; l < 2; ++l) {
+      const std::string pre = "lps.l" + std::to_string(l);
+      float* vl = vp + VP_LAYER0 + l * VP_LAYER_STRIDE;
+      for (int o = 0; o < 32; ++o) {
+        vl[VPL_LN1G + o] = atf(pre + ".ln1.g", 0, o);
+        vl[VPL_LN1B + o] = atf(pre + ".ln1.b", 0, o);
+        vl[VPL_OUTB + o] = atf(pre + ".out.b", 0, o);
+        vl[VPL_LN2G + o] = atf(pre + ".ln2.g", 0, o);
+        vl[VPL_LN2B + o] = atf(pre + ".ln2.b", 0, o);
+        vl[VPL_FF2B + o] = atf(pre + ".ff2.b", 0, o);
+      }
+      for (int o = 0; o < 96; ++o) vl[VPL_QKVB + o] = atf(pre + ".qkv.b", 0, o);
+      for (int o = 0; o < 64; ++o) vl[VPL_FF1B + o] = atf(pre + ".ff1.b", 0, o);
+    }
   }
-  o.in_t = put_t("lps.in.w", true);
-  o.in_b = put_f32("lps.in.b");
-  o.in_ln_g = put_f32("lps.in_ln.g");
-  o.in_ln_b = put_f32("lps.in_ln.b");
-  o.lh_w = put_f32("lps.head.w");
-  o.lh_b = put_f32("lps.head.b");
   for (int l = 0; l < 2; ++l) {
-    const std::string p = "lps.l" + std::to_string(l);
-    o.pq[l][0] = put_t(p + ".qkv.w", false);
-    o.pq[l][1] = put_t(p + ".out.w", false);
-    o.pq[l][2] = put_t(p + ".ff1.w", false);
-    o.pq[l][3] = put_t(p + ".ff2.w", false);
-    o.pq[l][4] = put_f32(p + ".qkv.b");
-    o.pq[l][5] = put_f32(p + ".out.b");
-    o.pq[l][6] = put_f32(p + ".ff1.b");
-    o.pq[l][7] = put_f32(p + ".ff2.b");
-    o.pq[l][8] = put_f32(p + ".ln1.g");
-    o.pq[l][9] = put_f32(p + ".ln1.b");
-    o.pq[l][10] = put_f32(p + ".ln2.g");
-    o.pq[l][11] = put_f32(p + ".ln2.b");
+    const std::string pre = "lps.l" + std::to_string(l);
+    uint16_t* wl = lps.data() + l * PL_STRIDE;
+    for (int k = 0; k < 32; ++k) {
+      for (int o = 0; o < 96; ++o) wl[PL_QKV + k * 96 + o] = at(pre + ".qkv.w", o, k);
+      for (int o = 0; o < 32; ++o) wl[PL_OUT + k * 32 + o] = at(pre + ".out.w", o, k);
+      for (int o = 0; o < 64; ++o) wl[PL_FF1 + k * 64 + o] = at(pre + ".ff1.w", o, k);
+    }
+    for (int k = 0; k < 64; ++k)
+      for (int o = 0; o < 32; ++o) wl[PL_FF2 + k * 32 + o] = at(pre + ".ff2.w", o, k);
   }
-  align();
+  const size_t b_lbs = lbs.size() * 2, b_lps = lps.size() * 2, b_vec = vec.size() * 4;
+  const size_t o_lps = (b_lbs + 255) / 256 * 256;
+  const size_t o_vec = o_lps + (b_lps + 255) / 256 * 256;
+  const size_t total = o_vec + b_vec;
   if (h->d_image) cudaFree(h->d_image);
   h->d_image = nullptr;
-  cudaError_t e = cudaMalloc(&h->d_image, img.size());
+  cudaError_t e = cudaMalloc(&h->d_image, total);
   if (e != cudaSuccess) return cuda_fail(h, e, "cudaMalloc(router image)");
-  e = cudaMemcpy(h->d_image, img.data(), img.size(), cudaMemcpyHostToDevice);
-  if (e != cudaSuccess) return cuda_fail(h, e, "cudaMemcpy(router image)");
+  if ((e = cudaMemcpy(h->d_image, lbs.data(), b_lbs, cudaMemcpyHostToDevice)) != cudaSuccess ||
+      (e = cudaMemcpy(h->d_image + o_lps, lps.data(), b_lps, cudaMemcpyHostToDevice)) != cudaSuccess ||
+      (e = cudaMemcpy(h->d_image + o_vec, vec.data(), b_vec, cudaMemcpyHostToDevice)) != cudaSuccess)
+    return cuda_fail(h, e, "cudaMemcpy(router image)");
   e = cudaMemcpy(h->d_blob, h->h_blob.data(), h->h_blob.size() * 2, cudaMemcpyHostToDevice);
   if (e != cudaSuccess) return cuda_fail(h, e, "cudaMemcpy(router blob)");
-  uint8_t* B = h->d_image;
-  auto F = [&](size_t x) { return reinterpret_cast<const float*>(B + x); };
-  auto H = [&](size_t x) { return reinterpret_cast<const __nv_bfloat16*>(B + x); };
-  RouterImage& w = h->img;
-  w.ent1_w = F(o.ent1_w); w.ent1_b = F(o.ent1_b); w.ent2_b = F(o.ent2_b);
-  w.ent_ln_g = F(o.ent_ln_g); w.ent_ln_b = F(o.ent_ln_b); w.tok_b = F(o.tok_b);
-  w.comb_b = F(o.comb_b); w.head_w = F(o.head_w); w.head_b = F(o.head_b);
-  w.ent2_t = H(o.ent2_t); w.comb_t = H(o.comb_t); w.pos = H(o.pos);
-  for (int l = 0; l < 2; ++l) {
-    w.lbs[l] = {H(o.lq[l][0]), H(o.lq[l][1]), H(o.lq[l][2]), H(o.lq[l][3]), F(o.lq[l][4]),
-                F(o.lq[l][5]), F(o.lq[l][6]), F(o.lq[l][7]), F(o.lq[l][8]), F(o.lq[l][9]),
-                F(o.lq[l][10]), F(o.lq[l][11])};
-    w.lps[l] = {H(o.pq[l][0]), H(o.pq[l][1]), H(o.pq[l][2]), H(o.pq[l][3]), F(o.pq[l][4]),
-                F(o.pq[l][5]), F(o.pq[l][6]), F(o.pq[l][7]), F(o.pq[l][8]), F(o.pq[l][9]),
-                F(o.pq[l][10]), F(o.pq[l][11])};
-  }
-  w.in_t = F(o.in_t); w.in_b = F(o.in_b); w.in_ln_g = F(o.in_ln_g); w.in_ln_b = F(o.in_ln_b);
-  w.lps_head_w = F(o.lh_w); w.lps_head_b = F(o.lh_b);
-  w.tok_table = h->d_tok;
+  h->img.lbs_w = reinterpret_cast<const __nv_bfloat16*>(h->d_image);
+  h->img.lps_w = reinterpret_cast<const __nv_bfloat16*>(h->d_image + o_lps);
+  h->img.vec = reinterpret_cast<const float*>(h->d_image + o_vec);
+  h->img.tok_table = h->d_tok;
   return EBD_OK;
 }
 
@@ -392,6 +406,8 @@ ebd_status check_args(ebd_handle* h, const ebd_step_args* a, bool need_attn, boo
   }
   if (need_lm) {
     if (!a->hidden || !a->w_lm) return fail(h, EBD_ERR_INVALID_ARG, "hidden and w_lm must be set");
+    if (a->w_lm_layout != 0 && a->w_lm_layout != 1)
+      return fail(h, EBD_ERR_INVALID_ARG, "w_lm_layout must be 0 or 1");
     if (!aligned(a->hidden, 16) || !aligned(a->w_lm, 16))
       return fail(h, EBD_ERR_INVALID_ARG, "hidden and w_lm must be 16-byte aligned");
   }
@@ -445,6 +461,7 @@ ebd_status run_attention(ebd_handle* h, const ebd_step_args* a, cudaStream_t st)
   p.q = reinterpret_cast<const __nv_bfloat16*>(a->q);
   p.out = a->attn_out;
   p.part = h->attn_part;
+  p.part_ml = h->attn_part_ml;
   p.tickets = h->tickets;
   p.status = h->d_status;
   p.limit_ns = kLimitNs;
@@ -456,9 +473,13 @@ ebd_status run_attention(ebd_handle* h, const ebd_step_args* a, cudaStream_t st)
 ebd_status run_lm(ebd_handle* h, const ebd_step_args* a, cudaStream_t st) {
   const ebd_config& c = h->cfg;
   CUtensorMap tw;
+  const bool packed = a->w_lm_layout == 1;
   {
-    const uint64_t dims[2] = {static_cast<uint64_t>(c.d_model), static_cast<uint64_t>(c.vocab)};
-    const uint64_t str[1] = {static_cast<uint64_t>(c.d_model) * 2};
+    const uint64_t units = (static_cast<uint64_t>(c.vocab) + kUnit - 1) / kUnit;
+    const uint64_t nkb = (static_cast<uint64_t>(c.d_model) + 63) / 64;
+    const uint64_t dims[2] = {packed ? 64ull : static_cast<uint64_t>(c.d_model),
+                              packed ? units * nkb * 64 : static_cast<uint64_t>(c.vocab)};
+    const uint64_t str[1] = {packed ? 128ull : static_cast<uint64_t>(c.d_model) * 2};
     const uint32_t box[2] = {64, 64};
     if (!encode_bf16(&tw, a->w_lm, 2, dims, str, box))
       return fail(h, EBD_ERR_CUDA, "cuTensorMapEncodeTiled (W_lm) failed");
@@ -469,6 +490,7 @@ ebd_status run_lm(ebd_handle* h, const ebd_step_args* a, cudaStream_t st) {
     lm_plan(p, rows, c.vocab, c.d_model, h->num_sms);
     if (p.stages < 2) return fail(h, EBD_ERR_UNSUPPORTED, "LM head: shared memory plan failed");
     p.row0 = g0;
+    p.packed = packed ? 1 : 0;
     p.part_f = h->part_f;
     p.part_i = h->part_i;
     p.status = h->d_status;
@@ -614,6 +636,7 @@ ebd_status ebd_create(const ebd_config* cfg, ebd_handle** out) {
       const size_t bytes = static_cast<size_t>(slots) * splits * 64 * (cfg->head_dim + 2) * 4;
       if ((e = cudaMalloc(&h->attn_part, bytes)) != cudaSuccess)
         return bail(cuda_fail(h, e, "cudaMalloc(attention partials)"));
+      h->attn_part_ml = h->attn_part + static_cast<size_t>(slots) * splits * 64 * cfg->head_dim;
     }
     if ((e = cudaMalloc(&h->tickets, static_cast<size_t>(slots) * sizeof(int))) != cudaSuccess)
       return bail(cuda_fail(h, e, "cudaMalloc(tickets)"));
@@ -637,6 +660,9 @@ ebd_status ebd_create(const ebd_config* cfg, ebd_handle** out) {
     if ((e = cudaMalloc(&h->staging, bytes)) != cudaSuccess)
       return bail(cuda_fail(h, e, "cudaMalloc(staging)"));
   }
+  for (int i = 0; i < 4; ++i)
+    if ((e = cudaEventCreate(&h->ev[i])) != cudaSuccess)
+      return bail(cuda_fail(h, e, "cudaEventCreate"));
   if ((e = cudaDeviceSynchronize()) != cudaSuccess) return bail(cuda_fail(h, e, "create"));
   *out = h;
   return EBD_OK;
@@ -657,6 +683,8 @@ void ebd_destroy(ebd_handle* h) {
   cudaFree(h->tickets);
   cudaFree(h->d_status);
   cudaFree(h->staging);
+  for (int i = 0; i < 4; ++i)
+    if (h->ev[i]) cudaEventDestroy(h->ev[i]);
   if (prev >= 0 && prev != h->device) cudaSetDevice(prev);
   delete h;
 }
@@ -701,6 +729,28 @@ ebd_status ebd_import_weights(ebd_handle* h, const void* host, size_t bytes) {
   return EBD_OK;
 }
 
+size_t ebd_lm_head_packed_bytes(const ebd_config* cfg) {
+  if (cfg == nullptr || cfg->vocab <= 0 || cfg->d_model <= 0) return 0;
+  const size_t units = (static_cast<size_t>(cfg->vocab) + kUnit - 1) / kUnit;
+  const size_t nkb = (static_cast<size_t>(cfg->d_model) + 63) / 64;
+  return units * nkb * 64 * 64 * 2;
+}
+
+ebd_status ebd_pack_lm_head(ebd_handle* h, const uint16_t* w_lm, uint16_t* w_packed,
+                            void* stream) {
+  if (h == nullptr) return EBD_ERR_INVALID_ARG;
+  ebd_status s = check_device(h);
+  if (s != EBD_OK) return s;
+  if (w_lm == nullptr || w_packed == nullptr || !aligned(w_lm, 16) || !aligned(w_packed, 16))
+    return fail(h, EBD_ERR_INVALID_ARG, "w_lm and w_packed must be 16-byte aligned device pointers");
+  (void)cudaGetLastError();
+  cudaError_t e = launch_pack_lm(reinterpret_cast<const __nv_bfloat16*>(w_lm),
+                                 reinterpret_cast<__nv_bfloat16*>(w_packed), h->cfg.vocab,
+                                 h->cfg.d_model, static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(h, e, "pack launch");
+  return EBD_OK;
+}
+
 ebd_status ebd_step(ebd_handle* h, const ebd_step_args* a, void* stream) {
   if (h == nullptr) return EBD_ERR_INVALID_ARG;
   ebd_status s = check_device(h);
@@ -710,11 +760,21 @@ ebd_status ebd_step(ebd_handle* h, const ebd_step_args* a, void* stream) {
   if (h->w_emb == nullptr) return fail(h, EBD_ERR_STATE, "bind the token embedding first");
   if (a->rows == 0 || a->batch == 0) return EBD_OK;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
+  (void)cudaGetLastError();  // a stale error of an earlier unrelated call is not ours
+  cudaError_t e0 = cudaSuccess;
+  if (h->profile && (e0 = record(h->ev[0], st)) != cudaSuccess)
+    return cuda_fail(h, e0, "profile event");
   if (attn && (s = run_attention(h, a, st)) != EBD_OK) return s;
+  if (h->profile && (e0 = record(h->ev[1], st)) != cudaSuccess)
+    return cuda_fail(h, e0, "profile event");
   if ((s = run_lm(h, a, st)) != EBD_OK) return s;
+  if (h->profile && (e0 = record(h->ev[2], st)) != cudaSuccess)
+    return cuda_fail(h, e0, "profile event");
   DecideParams p = decide_params(h, a, 0);
   cudaError_t e = launch_decide(p, st);
   if (e != cudaSuccess) return cuda_fail(h, e, "decision launch");
+  if (h->profile && (e0 = record(h->ev[3], st)) != cudaSuccess)
+    return cuda_fail(h, e0, "profile event");
   return EBD_OK;
 }
 
@@ -850,6 +910,23 @@ ebd_status ebd_step_host(ebd_handle* h, const ebd_step_args* a, void* stream) {
   chk(d2h(a->argmax, am, R * 4));
   chk(d2h(a->accepted, acc, R));
   if (e != cudaSuccess) return cuda_fail(h, e, "device-to-host copy");
+  return EBD_OK;
+}
+
+ebd_status ebd_profile_enable(ebd_handle* h, int on) {
+  if (h == nullptr) return EBD_ERR_INVALID_ARG;
+  h->profile = on ? 1 : 0;
+  return EBD_OK;
+}
+
+ebd_status ebd_profile_read(ebd_handle* h, float* ms) {
+  if (h == nullptr || ms == nullptr) return EBD_ERR_INVALID_ARG;
+  cudaError_t e = cudaEventSynchronize(h->ev[3]);
+  if (e != cudaSuccess) return cuda_fail(h, e, "cudaEventSynchronize");
+  for (int i = 0; i < 3; ++i) {
+    e = cudaEventElapsedTime(&ms[i], h->ev[i], h->ev[i + 1]);
+    if (e != cudaSuccess) return cuda_fail(h, e, "cudaEventElapsedTime");
+  }
   return EBD_OK;
 }
 

@@ -18,6 +18,7 @@ constexpr int kDecideThreads = 256;
 constexpr int kAttnThreads = 128;
 constexpr int kAttnChunk = 64;        // keys per K/V tile
 constexpr int kAttnStages = 3;
+constexpr int kMaxAttnSplits = 8;
 
 // ------------------------------------------------------------------ LM head
 struct LmParams {
@@ -26,7 +27,9 @@ struct LmParams {
   int nb, nsub, n_pad;      // MMA N per sub-tile, sub-tiles, padded N = nb * nsub
   int n_units;              // ceil(V / 64)
   int grid;                 // CTAs (partials per row)
-  int nkb;                  // ceil(d / 64) k-blocks
+  int nkb;                  // ceil(d / 64) k-blocks of 64 columns
+  int kbs, nks;             // k-blocks per pipeline stage, stages per vocabulary chunk
+  int packed;               // W is tiled: tile (unit, k-block) at row (unit*nkb + kb)*64
   int stages, nbuf, acc_stride, tmem_cols;
   uint32_t off_a, off_b, off_t, off_st, off_bar, smem_bytes;
   float4* part_f;           // [R][grid] (max, sum exp, sum exp*(l-max), second logit)
@@ -45,32 +48,20 @@ struct AttnParams {
   const int* prefix_len;
   const __nv_bfloat16* q;   // [R][Hq][D]
   float* out;               // [R][Hq][D]
-  float* part;              // [B*Hkv*max_qtiles*splits][64][D+2]
+  float* part;              // [B*Hkv*max_qtiles*splits][64][D] unnormalised O
+  float* part_ml;           // [B*Hkv*max_qtiles*splits][64][2] (max, sum) in log2 units
   int* tickets;             // [B*Hkv*max_qtiles]
   int* status;
   uint64_t limit_ns;
 };
 
 // ------------------------------------------------------------------ routers
-// Device image of the router weights used by the decision kernel: matrices
-// transposed to [in][out] bf16, vectors fp32.
-struct LbsLayer {
-  const __nv_bfloat16 *qkv_t, *out_t, *ff1_t, *ff2_t;  // [128][384] [128][128] [128][256] [256][128]
-  const float *qkv_b, *out_b, *ff1_b, *ff2_b, *ln1_g, *ln1_b, *ln2_g, *ln2_b;
-};
-struct LpsLayer {
-  const __nv_bfloat16 *qkv_t, *out_t, *ff1_t, *ff2_t;  // [32][96] [32][32] [32][64] [64][32]
-  const float *qkv_b, *out_b, *ff1_b, *ff2_b, *ln1_g, *ln1_b, *ln2_g, *ln2_b;
-};
+// Device image of the router weights (layout in router_image.h).
 struct RouterImage {
-  // LBS
-  const float *ent1_w, *ent1_b, *ent2_b, *ent_ln_g, *ent_ln_b, *tok_b, *comb_b, *head_w, *head_b;
-  const __nv_bfloat16 *ent2_t, *comb_t, *pos;  // [64][64] [128][128] [L][128]
-  LbsLayer lbs[2];
-  // LPS
-  const float *in_t, *in_b, *in_ln_g, *in_ln_b, *lps_head_w, *lps_head_b;  // in_t: [5][32]
-  LpsLayer lps[2];
-  const float* tok_table;  // [V][64] = W_tok W_e[v] (no bias)
+  const __nv_bfloat16* lbs_w;  // [8 ranks][LBS_W_ELEMS]
+  const __nv_bfloat16* lps_w;  // [LPS_W_ELEMS]
+  const float* vec;            // [8 ranks][V_ELEMS]
+  const float* tok_table;      // [V][64] = W_tok W_e[v] (no bias)
 };
 
 struct DecideParams {
@@ -101,6 +92,8 @@ void lm_plan(LmParams& p, int rows, int V, int d, int num_sms);
 cudaError_t launch_attention(const CUtensorMap& kc, const CUtensorMap& vc, const CUtensorMap& kw,
                              const CUtensorMap& vw, const AttnParams& p, cudaStream_t st);
 cudaError_t launch_decide(const DecideParams& p, cudaStream_t st);
+cudaError_t launch_pack_lm(const __nv_bfloat16* w, __nv_bfloat16* out, int V, int d,
+                           cudaStream_t st);
 cudaError_t launch_fold_tok(const __nv_bfloat16* w_tok, const __nv_bfloat16* w_emb, float* table,
                             int V, int d_base, cudaStream_t st);
 

@@ -269,20 +269,20 @@ __global__ void __launch_bounds__(kAttnThreads)
     return;
   }
   const int slot = (bg * p.max_qtiles + qt);
-  float* part = p.part + (static_cast<size_t>(slot) * p.splits + split) * 64 * (D + 2);
+  // partials: O rows [slot][split][64][D] and (max, sum) [slot][split][64][2]
+  float* po = p.part + (static_cast<size_t>(slot) * p.splits + split) * 64 * D;
+  float* pml = p.part_ml + (static_cast<size_t>(slot) * p.splits + split) * 64 * 2;
   if (warp_active) {
     const int ml = warp * 16 + (lane >> 2), mh = ml + 8;
 #pragma unroll
     for (int t = 0; t < NT; ++t) {
       const int d = t * 8 + 2 * (lane & 3);
-      *reinterpret_cast<float2*>(part + ml * (D + 2) + d) = make_float2(o[t][0], o[t][1]);
-      *reinterpret_cast<float2*>(part + mh * (D + 2) + d) = make_float2(o[t][2], o[t][3]);
+      *reinterpret_cast<float2*>(po + ml * D + d) = make_float2(o[t][0], o[t][1]);
+      *reinterpret_cast<float2*>(po + mh * D + d) = make_float2(o[t][2], o[t][3]);
     }
     if ((lane & 3) == 0) {
-      part[ml * (D + 2) + D] = m_lo;
-      part[ml * (D + 2) + D + 1] = l_lo;
-      part[mh * (D + 2) + D] = m_hi;
-      part[mh * (D + 2) + D + 1] = l_hi;
+      *reinterpret_cast<float2*>(pml + ml * 2) = make_float2(m_lo, l_lo);
+      *reinterpret_cast<float2*>(pml + mh * 2) = make_float2(m_hi, l_hi);
     }
   }
   __threadfence();
@@ -291,23 +291,42 @@ __global__ void __launch_bounds__(kAttnThreads)
   __syncthreads();
   if (!s_flag) return;
   __threadfence();
-  const float* base = p.part + static_cast<size_t>(slot) * p.splits * 64 * (D + 2);
+  // last CTA of the slot: per-row split weights, then a weighted sum of the
+  // splits' O rows with independent vector loads
+  __shared__ float s_w[64][kMaxAttnSplits];
+  const float* bo = p.part + static_cast<size_t>(slot) * p.splits * 64 * D;
+  const float* bml = p.part_ml + static_cast<size_t>(slot) * p.splits * 64 * 2;
   const int rows_here = min(64, m_total - qt * 64);
-  for (int it = tid; it < rows_here * D; it += blockDim.x) {
-    const int mr = it / D, d = it - mr * D;
+  for (int r = tid; r < rows_here; r += blockDim.x) {
     float M = -INFINITY;
-    for (int sp = 0; sp < p.splits; ++sp)
-      M = fmaxf(M, base[(static_cast<size_t>(sp) * 64 + mr) * (D + 2) + D]);
-    float L = 0.f, acc = 0.f;
+    for (int sp = 0; sp < p.splits; ++sp) M = fmaxf(M, bml[(sp * 64 + r) * 2]);
+    float L = 0.f;
     for (int sp = 0; sp < p.splits; ++sp) {
-      const float* pr = base + (static_cast<size_t>(sp) * 64 + mr) * (D + 2);
-      const float ms = pr[D];
-      if (ms == -INFINITY) continue;
-      const float wgt = exp2f(ms - M);
-      L += wgt * pr[D + 1];
-      acc += wgt * pr[d];
+      const float2 v = *reinterpret_cast<const float2*>(bml + (sp * 64 + r) * 2);
+      const float wgt = v.x == -INFINITY ? 0.f : exp2f(v.x - M);
+      s_w[r][sp] = wgt;
+      L += wgt * v.y;
     }
-    out_row(qt * 64 + mr)[d] = L > 0.f ? acc / L : 0.f;
+    const float inv = L > 0.f ? 1.0f / L : 0.f;
+    for (int sp = 0; sp < p.splits; ++sp) s_w[r][sp] *= inv;
+  }
+  __syncthreads();
+  constexpr int D4 = D / 4;
+  for (int it = tid; it < rows_here * D4; it += blockDim.x) {
+    const int r = it / D4, d = (it - r * D4) * 4;
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+    for (int sp = 0; sp < kMaxAttnSplits; ++sp) {
+      if (sp < p.splits) {
+        const float4 v = __ldcg(reinterpret_cast<const float4*>(bo + (static_cast<size_t>(sp) * 64 + r) * D + d));
+        const float wgt = s_w[r][sp];
+        acc.x = fmaf(wgt, v.x, acc.x);
+        acc.y = fmaf(wgt, v.y, acc.y);
+        acc.z = fmaf(wgt, v.z, acc.z);
+        acc.w = fmaf(wgt, v.w, acc.w);
+      }
+    }
+    *reinterpret_cast<float4*>(out_row(qt * 64 + r) + d) = acc;
   }
   if (tid == 0) p.tickets[slot] = 0;
 }

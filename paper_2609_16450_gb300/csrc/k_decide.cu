@@ -21,6 +21,7 @@
 
 #include "internal.h"
 #include "ptx.cuh"
+#include "router_image.h"
 
 namespace cg = cooperative_groups;
 
@@ -28,26 +29,36 @@ namespace ebd {
 
 namespace {
 
-constexpr int W = kMaxWindow;       // rows per sequence
-constexpr int LDZ = 132;            // z / zp row stride
-constexpr int LDX = 260;            // X row stride (concat 128 or FFN 256)
-constexpr int LDKV = 68;            // kv row stride: k in [0,32), v in [32,64)
-constexpr int LDQ = 36;             // q row stride
-constexpr int LDS = 68;             // attention scores row stride
+using namespace rimg;
 
-struct Smem {
-  float z[W * LDZ];
-  float zp[W * LDZ];
-  float X[W * LDX];
-  float kv[W * LDKV];
-  float q[W * LDQ];
-  float S[W * LDS];
-  // per-row data of the sequence
+constexpr int W = kMaxWindow;  // rows per sequence
+constexpr int LDZ = 132;       // residual stream / [e;t] / attention concat
+constexpr int LDKV = 68;       // k in [0,32), v in [32,64)
+constexpr int LDQ = 36;
+constexpr int LDS = 68;
+// activation pool (floats), LBS phase
+constexpr int P_Z = 0;                  // [64][132] residual stream z
+constexpr int P_X = P_Z + W * LDZ;      // [64][132] [e;t] | concat | FFN partial inbox [8][64][16]
+constexpr int P_KV = P_X + W * LDZ;     // [64][68]  k,v of this CTA's head | FFN hidden [64][36]
+constexpr int P_Q = P_KV + W * LDKV;    // [32][36]  queries of this CTA's half
+constexpr int P_S = P_Q + 32 * LDQ;     // [32][68]  attention scores
+constexpr int POOL = P_S + 32 * LDS;    // 24576 floats
+// activation pool, LPS phase (rank 0)
+constexpr int L_Z = 0, L_Y = 2304, L_F = 4608, L_QKV = 5120, L_ATT = 11520, L_SC = 13824,
+              L_H = 18176;
+static_assert(L_H + W * 68 <= POOL, "LPS pool layout");
+static_assert(8 * W * 16 <= W * LDZ, "FFN partial inbox");
+
+struct __align__(16) Smem {
+  __nv_bfloat16 w[LBS_W_ELEMS];   // this rank's LBS weight slices
+  __nv_bfloat16 lw[LPS_W_ELEMS];  // LPS weights (rank 0)
+  float v[V_ELEMS];               // vectors
+  float pool[POOL];
   float f_conf[W], f_ent[W], f_gap[W], f_O[W], f_p[W];
-  int f_arg[W], f_pos[W], f_tok[W];
-  int Mrows[W], Brows[W], BMrows[W];
+  int f_arg[W], f_pos[W], f_tok[W], Mrows[W], Brows[W], BMrows[W];
   uint8_t f_mask[W], f_ib[W], f_acc[W], f_bad[W];
-  int nM, nB, nBM, meta_b, meta_s, n_rows, r0, run_lbs, bad_seq;
+  int nM, nBM, meta_b, meta_s, n_rows, r0, run_lbs, bad_seq, wait_fail;
+  uint64_t bar;
 };
 
 __device__ __forceinline__ float gelu(float x) {
@@ -65,52 +76,59 @@ __device__ __forceinline__ float warp_max(float v) {
   return v;
 }
 
-__device__ __forceinline__ float bf(const __nv_bfloat16 x) { return __bfloat162float(x); }
+__device__ __forceinline__ void bulk_copy(void* smem_dst, const void* gsrc, uint32_t bytes,
+                                          uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::
+          "r"(smem_u32(smem_dst)),
+      "l"(gsrc), "r"(bytes), "r"(smem_u32(bar))
+      : "memory");
+}
 
-// out(j, o) = bias[o0 + o] + sum_k in[j][k] * Wt[k][o0 + o] for j < n and
-// o < Os (Os even); Wt is [K][O] bf16.  epi(j, o, value) consumes results.
+// out(j, o) = bias[o] + sum_k in[j][k] * Wt[k][o] for j < n, o < Os (Os even);
+// Wt is shared-memory bf16 [K][ldw].  epi(j, o, value) consumes the result.
 template <class Epi>
 __device__ __forceinline__ void gemm_rows(const float* in, int ldi, int n, int K,
-                                          const __nv_bfloat16* Wt, int O, int o0, int Os,
+                                          const __nv_bfloat16* Wt, int ldw, int Os,
                                           const float* bias, Epi epi) {
   const int pairs = Os >> 1;
+  const int ldw2 = ldw >> 1;
   for (int it = threadIdx.x; it < n * pairs; it += blockDim.x) {
     const int j = it / pairs, pr = it - j * pairs;
-    const int o = o0 + 2 * pr;
-    float a0 = bias ? bias[o] : 0.f, a1 = bias ? bias[o + 1] : 0.f;
+    float a0 = bias ? bias[2 * pr] : 0.f, a1 = bias ? bias[2 * pr + 1] : 0.f;
     const float* x = in + j * ldi;
-    const __nv_bfloat162* w = reinterpret_cast<const __nv_bfloat162*>(Wt + o);
-    const int O2 = O >> 1;
+    const __nv_bfloat162* w = reinterpret_cast<const __nv_bfloat162*>(Wt) + pr;
     int k = 0;
+#pragma unroll 2
     for (; k + 4 <= K; k += 4) {
       const float4 xv = *reinterpret_cast<const float4*>(x + k);
-      const float2 w0 = __bfloat1622float2(w[(k + 0) * O2]);
-      const float2 w1 = __bfloat1622float2(w[(k + 1) * O2]);
-      const float2 w2 = __bfloat1622float2(w[(k + 2) * O2]);
-      const float2 w3 = __bfloat1622float2(w[(k + 3) * O2]);
+      const float2 w0 = __bfloat1622float2(w[(k + 0) * ldw2]);
+      const float2 w1 = __bfloat1622float2(w[(k + 1) * ldw2]);
+      const float2 w2 = __bfloat1622float2(w[(k + 2) * ldw2]);
+      const float2 w3 = __bfloat1622float2(w[(k + 3) * ldw2]);
       a0 = fmaf(xv.x, w0.x, a0); a1 = fmaf(xv.x, w0.y, a1);
       a0 = fmaf(xv.y, w1.x, a0); a1 = fmaf(xv.y, w1.y, a1);
       a0 = fmaf(xv.z, w2.x, a0); a1 = fmaf(xv.z, w2.y, a1);
       a0 = fmaf(xv.w, w3.x, a0); a1 = fmaf(xv.w, w3.y, a1);
     }
     for (; k < K; ++k) {
-      const float2 wk = __bfloat1622float2(w[k * O2]);
+      const float2 wk = __bfloat1622float2(w[k * ldw2]);
       a0 = fmaf(x[k], wk.x, a0);
       a1 = fmaf(x[k], wk.y, a1);
     }
-    epi(j, o - o0, a0);
-    epi(j, o - o0 + 1, a1);
+    epi(j, 2 * pr, a0);
+    epi(j, 2 * pr + 1, a1);
   }
 }
 
-// LayerNorm over `dim` (multiple of 32, <= 128) of rows j < n; warp per row.
+// LayerNorm (eps 1e-5) over `dim` (32, 64 or 128) of rows j < n; warp per row.
 __device__ __forceinline__ void layer_norm_rows(const float* src, int lds, float* dst, int ldd,
                                                 int n, int dim, const float* g, const float* b) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int nw = blockDim.x >> 5;
   const int per = dim >> 5;
   for (int j = warp; j < n; j += nw) {
-    float v[4];
+    float v[4] = {0.f, 0.f, 0.f, 0.f};
     float s = 0.f;
     for (int c = 0; c < per; ++c) {
       v[c] = src[j * lds + lane + 32 * c];
@@ -130,8 +148,8 @@ __device__ __forceinline__ void layer_norm_rows(const float* src, int lds, float
   }
 }
 
-// Multi-head self-attention core for queries qs[i] (i < nq) over keys/values
-// of rows k < n; head width dh; writes o(i, d) through epi.
+// Scaled dot-product attention of queries qs[i] (i < nq) over keys/values
+// k < n (head width dh); writes o(i, d) through epi.  S: [nq][LDS] scratch.
 template <class Epi>
 __device__ __forceinline__ void attend(const float* qs, int ldq, const float* ks, const float* vs,
                                        int ldkv, int nq, int n, int dh, float* S, Epi epi) {
@@ -183,16 +201,19 @@ __device__ __forceinline__ void merge_state(float& m, float& s, float& t, float&
 }
 
 // ----------------------------------------------------------------- LPS (rank 0)
-__device__ void lps_forward(Smem& sm, const DecideParams& p, int n) {
-  const RouterImage& w = p.w;
-  float* zL = sm.z;        // [n][36]
-  float* yL = sm.zp;       // [n][36]
-  float* fL = sm.zp + W * 36;  // features [n][8]
-  float* qkv = sm.X;       // [n][100]
-  float* att = sm.kv;      // [n][36]
-  float* h64 = sm.S;       // [n][68]
+// Sec. 5.2 / App. D.1: Linear(5->32) -> LayerNorm -> GELU, two pre-norm blocks
+// (4 heads, FFN 64, GELU), head Linear(32->1); p_psi = sigmoid(O).
+__device__ void lps_forward(Smem& sm, int n) {
+  float* P = sm.pool;
+  float* zL = P + L_Z;
+  float* yL = P + L_Y;
+  float* fL = P + L_F;
+  float* qkv = P + L_QKV;
+  float* att = P + L_ATT;
+  float* sc = P + L_SC;
+  float* h64 = P + L_H;
+  const float* V = sm.v + V_LPS;
   constexpr int LD = 36, LDQKV = 100;
-  // features: (kappa, H~, Delta, rho, pos)
   const float rho = static_cast<float>(sm.nBM) / static_cast<float>(sm.meta_s);
   for (int i = threadIdx.x; i < n; i += blockDim.x) {
     const int r = sm.BMrows[i];
@@ -203,15 +224,14 @@ __device__ void lps_forward(Smem& sm, const DecideParams& p, int n) {
     fL[i * 8 + 4] = static_cast<float>(sm.f_pos[r] - sm.meta_b) / static_cast<float>(sm.meta_s);
   }
   __syncthreads();
-  // input embedding: Linear(5 -> 32) -> LayerNorm -> GELU
   for (int it = threadIdx.x; it < n * 32; it += blockDim.x) {
     const int i = it >> 5, o = it & 31;
-    float a = w.in_b[o];
-    for (int k = 0; k < 5; ++k) a = fmaf(fL[i * 8 + k], w.in_t[k * 32 + o], a);
+    float a = V[VP_INB + o];
+    for (int k = 0; k < 5; ++k) a = fmaf(fL[i * 8 + k], V[VP_INT + k * 32 + o], a);
     yL[i * LD + o] = a;
   }
   __syncthreads();
-  layer_norm_rows(yL, LD, zL, LD, n, 32, w.in_ln_g, w.in_ln_b);
+  layer_norm_rows(yL, LD, zL, LD, n, 32, V + VP_INLNG, V + VP_INLNB);
   __syncthreads();
   for (int it = threadIdx.x; it < n * 32; it += blockDim.x) {
     const int i = it >> 5, o = it & 31;
@@ -219,35 +239,33 @@ __device__ void lps_forward(Smem& sm, const DecideParams& p, int n) {
   }
   __syncthreads();
   for (int l = 0; l < 2; ++l) {
-    const LpsLayer& L = w.lps[l];
-    // pre-norm self-attention block
-    layer_norm_rows(zL, LD, yL, LD, n, 32, L.ln1_g, L.ln1_b);
+    const __nv_bfloat16* Wl = sm.lw + l * PL_STRIDE;
+    const float* Vl = V + VP_LAYER0 + l * VP_LAYER_STRIDE;
+    layer_norm_rows(zL, LD, yL, LD, n, 32, Vl + VPL_LN1G, Vl + VPL_LN1B);
     __syncthreads();
-    gemm_rows(yL, LD, n, 32, L.qkv_t, 96, 0, 96, L.qkv_b,
+    gemm_rows(yL, LD, n, 32, Wl + PL_QKV, 96, 96, Vl + VPL_QKVB,
               [&](int j, int o, float v) { qkv[j * LDQKV + o] = v; });
     __syncthreads();
     for (int h = 0; h < 4; ++h) {
-      attend(qkv + 8 * h, LDQKV, qkv + 32 + 8 * h, qkv + 64 + 8 * h, LDQKV, n, n, 8, h64,
+      attend(qkv + 8 * h, LDQKV, qkv + 32 + 8 * h, qkv + 64 + 8 * h, LDQKV, n, n, 8, sc,
              [&](int i, int d, float v) { att[i * LD + 8 * h + d] = v; });
       __syncthreads();
     }
-    gemm_rows(att, LD, n, 32, L.out_t, 32, 0, 32, L.out_b,
+    gemm_rows(att, LD, n, 32, Wl + PL_OUT, 32, 32, Vl + VPL_OUTB,
               [&](int j, int o, float v) { zL[j * LD + o] += v; });
     __syncthreads();
-    // pre-norm feed-forward block
-    layer_norm_rows(zL, LD, yL, LD, n, 32, L.ln2_g, L.ln2_b);
+    layer_norm_rows(zL, LD, yL, LD, n, 32, Vl + VPL_LN2G, Vl + VPL_LN2B);
     __syncthreads();
-    gemm_rows(yL, LD, n, 32, L.ff1_t, 64, 0, 64, L.ff1_b,
-              [&](int j, int o, float v) { h64[j * LDS + o] = gelu(v); });
+    gemm_rows(yL, LD, n, 32, Wl + PL_FF1, 64, 64, Vl + VPL_FF1B,
+              [&](int j, int o, float v) { h64[j * 68 + o] = gelu(v); });
     __syncthreads();
-    gemm_rows(h64, LDS, n, 64, L.ff2_t, 32, 0, 32, L.ff2_b,
+    gemm_rows(h64, 68, n, 64, Wl + PL_FF2, 32, 32, Vl + VPL_FF2B,
               [&](int j, int o, float v) { zL[j * LD + o] += v; });
     __syncthreads();
   }
-  // head Linear(32 -> 1), p = sigmoid(O)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   for (int i = warp; i < n; i += (blockDim.x >> 5)) {
-    const float a = warp_sum(zL[i * LD + lane] * w.lps_head_w[lane]) + w.lps_head_b[0];
+    const float a = warp_sum(zL[i * LD + lane] * V[VP_HEADW + lane]) + V[VP_HEADB];
     if (lane == 0) sm.f_p[sm.BMrows[i]] = 1.0f / (1.0f + expf(-a));
   }
   __syncthreads();
@@ -264,11 +282,20 @@ __global__ void __cluster_dims__(kDecideCluster, 1, 1) __launch_bounds__(kDecide
   const int rank = static_cast<int>(cluster.block_rank());
   const int seq = blockIdx.x / kDecideCluster;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const RouterImage& w = p.w;
+  float* const P = sm.pool;
 
   if (tid == 0) {
+    // weights and vectors of this rank: bulk copies issued first, so they
+    // land while the statistics are merged
+    mbar_init(&sm.bar, 1);
+    fence_mbar_init();
+    const uint32_t wb = LBS_W_ELEMS * 2u, lb = LPS_W_ELEMS * 2u, vb = V_ELEMS * 4u;
+    mbar_arrive_expect_tx(&sm.bar, wb + vb + (rank == 0 ? lb : 0u));
+    bulk_copy(sm.w, p.w.lbs_w + static_cast<size_t>(rank) * LBS_W_ELEMS, wb, &sm.bar);
+    bulk_copy(sm.v, p.w.vec + static_cast<size_t>(rank) * V_ELEMS, vb, &sm.bar);
+    if (rank == 0) bulk_copy(sm.lw, p.w.lps_w, lb, &sm.bar);
     const int r0 = p.cu_rows[seq], r1 = p.cu_rows[seq + 1];
-    int n = r1 - r0;
+    const int n = r1 - r0;
     sm.bad_seq = 0;
     if (p.cu_rows[p.B] != p.rows_expected || n < 0 || n > W || r0 < 0) {
       sm.bad_seq = 1;
@@ -278,13 +305,13 @@ __global__ void __cluster_dims__(kDecideCluster, 1, 1) __launch_bounds__(kDecide
     sm.n_rows = sm.bad_seq ? 0 : n;
     sm.meta_b = p.blk_meta[2 * seq];
     sm.meta_s = p.blk_meta[2 * seq + 1];
+    sm.wait_fail = 0;
   }
   // every CTA of the cluster must be running before any distributed
   // shared-memory access; this also orders the block-level setup above
   cluster.sync();
   const int r0 = sm.r0, nr = sm.n_rows;
 
-  // per-row state (every rank keeps its own copy)
   for (int j = tid; j < nr; j += blockDim.x) {
     sm.f_mask[j] = p.mask[r0 + j];
     sm.f_ib[j] = p.in_block[r0 + j];
@@ -299,11 +326,12 @@ __global__ void __cluster_dims__(kDecideCluster, 1, 1) __launch_bounds__(kDecide
   if (p.features_in) {
     for (int j = tid; j < nr; j += blockDim.x) {
       const float c = p.conf[r0 + j], e = p.ent_norm[r0 + j], g = p.gap[r0 + j];
+      const int a = p.argmax[r0 + j];
       sm.f_conf[j] = c;
       sm.f_ent[j] = e;
       sm.f_gap[j] = g;
-      sm.f_arg[j] = p.argmax[r0 + j];
-      sm.f_bad[j] = !(isfinite(c) && isfinite(e) && isfinite(g));
+      sm.f_arg[j] = a;
+      sm.f_bad[j] = !(isfinite(c) && isfinite(e) && isfinite(g)) || a < 0 || a >= p.V;
     }
   } else {
     // row j is merged by warp (j / 8) of rank (j % 8) and broadcast
@@ -349,6 +377,14 @@ __global__ void __cluster_dims__(kDecideCluster, 1, 1) __launch_bounds__(kDecide
       }
     }
   }
+  // the weight copy must have landed before any use (and before exit)
+  {
+    const bool ok = mbar_wait(&sm.bar, 0, 1000ull * 1000 * 1000, nullptr);
+    if (!ok && tid == 0) {
+      sm.wait_fail = 1;
+      atomicCAS(p.status, 0, EBD_ERR_TIMEOUT);
+    }
+  }
   cluster.sync();
 
   // ---------------------------------------------------------------- 2. masked set
@@ -365,101 +401,119 @@ __global__ void __cluster_dims__(kDecideCluster, 1, 1) __launch_bounds__(kDecide
   // ---------------------------------------------------------------- 3. LBS router
   if (sm.run_lbs) {
     const int n = nM;
-    // 3a. entropy branch F_ent and token branch (every rank, all rows)
+    float* Z = P + P_Z;
+    float* X = P + P_X;
+    float* KV = P + P_KV;
+    float* Q = P + P_Q;
+    float* S = P + P_S;
+    const float* Vv = sm.v;
+    // 3a. entropy branch F_ent and token branch, every rank for all rows
     for (int it = tid; it < n * 64; it += blockDim.x) {
       const int j = it >> 6, o = it & 63;
-      sm.X[j * LDX + o] = gelu(fmaf(w.ent1_w[o], sm.f_ent[sm.Mrows[j]], w.ent1_b[o]));
-      const int tok = sm.f_arg[sm.Mrows[j]];
-      const float tv = (tok >= 0 && tok < p.V) ? w.tok_table[static_cast<size_t>(tok) * 64 + o] : 0.f;
-      sm.zp[j * LDZ + 64 + o] = tv + w.tok_b[o];
+      const int row = sm.Mrows[j];
+      KV[j * LDKV + o] = gelu(fmaf(Vv[V_ENT1W + o], sm.f_ent[row], Vv[V_ENT1B + o]));
+      const int tok = sm.f_arg[row];
+      const float tv =
+          (tok >= 0 && tok < p.V) ? p.w.tok_table[static_cast<size_t>(tok) * 64 + o] : 0.f;
+      X[j * LDZ + 64 + o] = tv + Vv[V_TOKB + o];
     }
     __syncthreads();
-    gemm_rows(sm.X, LDX, n, 64, w.ent2_t, 64, 0, 64, w.ent2_b,
-              [&](int j, int o, float v) { sm.S[j * LDS + o] = v; });
+    gemm_rows(KV, LDKV, n, 64, sm.w + W_ENT2, 64, 64, Vv + V_ENT2B,
+              [&](int j, int o, float v) { X[j * LDZ + o] = v; });
     __syncthreads();
-    layer_norm_rows(sm.S, LDS, sm.zp, LDZ, n, 64, w.ent_ln_g, w.ent_ln_b);
+    layer_norm_rows(X, LDZ, X, LDZ, n, 64, Vv + V_ENTLNG, Vv + V_ENTLNB);
     __syncthreads();
-    // 3b. fusion W_combine [e; t] + E_pos[rank], output slice of this CTA
+    // 3b. fusion W_combine [e; t] + E_pos[rank of the row]: this CTA's 16 outputs
     {
-      const int o0 = 16 * rank;
-      gemm_rows(sm.zp, LDZ, n, 128, w.comb_t, 128, o0, 16, w.comb_b, [&](int j, int o, float v) {
-        const float val = v + bf(w.pos[j * 128 + o0 + o]);
-        for (int rr = 0; rr < kDecideCluster; ++rr)
-          cluster.map_shared_rank(sm.z, rr)[j * LDZ + o0 + o] = val;
-      });
+      const int o0 = kCombSlice * rank;
+      gemm_rows(X, LDZ, n, 128, sm.w + W_COMB, kCombSlice, kCombSlice, Vv + V_COMBB,
+                [&](int j, int o, float v) {
+                  const float val = v + __bfloat162float(sm.w[W_POS + j * kCombSlice + o]);
+                  for (int rr = 0; rr < kDecideCluster; ++rr)
+                    cluster.map_shared_rank(Z, rr)[j * LDZ + o0 + o] = val;
+                });
     }
     cluster.sync();
     // 3c. two post-norm encoder layers
-    const int h = rank >> 1, role = rank & 1;
+    const int hd = rank >> 1, half = rank & 1;
     const int nh = (n + 1) >> 1;
-    const int qa = role == 0 ? 0 : nh, qb = role == 0 ? nh : n;
+    const int qa = half == 0 ? 0 : nh, qb = half == 0 ? nh : n;
     for (int l = 0; l < 2; ++l) {
-      const LbsLayer& L = w.lbs[l];
-      // Q for this CTA's query half; K (role 0) or V (role 1) of head h for all rows
-      gemm_rows(sm.z + qa * LDZ, LDZ, qb - qa, 128, L.qkv_t, 384, 32 * h, 32, L.qkv_b,
-                [&](int j, int o, float v) { sm.q[j * LDQ + o] = v; });
-      {
-        const int cbase = (role == 0 ? 128 : 256) + 32 * h;
-        const int koff = role == 0 ? 0 : 32;
-        float* mine = sm.kv;
-        float* peer = cluster.map_shared_rank(sm.kv, rank ^ 1);
-        gemm_rows(sm.z, LDZ, n, 128, L.qkv_t, 384, cbase, 32, L.qkv_b,
+      const __nv_bfloat16* Wl = sm.w + W_LAYER0 + l * W_LAYER_STRIDE;
+      const float* Vl = Vv + V_LAYER0 + l * V_LAYER_STRIDE;
+      // QKV: this CTA's 48 features for every row, scattered to the CTAs
+      // that attend with them (head h lives in ranks 2h and 2h+1)
+      gemm_rows(Z, LDZ, n, 128, Wl + WL_QKV, kQkvSlice, kQkvSlice, Vl + VL_QKVB,
+                [&](int j, int o, float v) {
+                  const int f = kQkvSlice * rank + o;
+                  const int part = f >> 7, h = (f >> 5) & 3, dd = f & 31;
+                  if (part == 0) {
+                    const int dst = 2 * h + (j >= nh ? 1 : 0);
+                    const int jj = j >= nh ? j - nh : j;
+                    cluster.map_shared_rank(P, dst)[P_Q + jj * LDQ + dd] = v;
+                  } else {
+                    const int col = (part == 1 ? 0 : 32) + dd;
+                    cluster.map_shared_rank(P, 2 * h)[P_KV + j * LDKV + col] = v;
+                    cluster.map_shared_rank(P, 2 * h + 1)[P_KV + j * LDKV + col] = v;
+                  }
+                });
+      cluster.sync();
+      attend(Q, LDQ, KV, KV + 32, LDKV, qb - qa, n, 32, S, [&](int i, int d, float v) {
+        for (int rr = 0; rr < kDecideCluster; ++rr)
+          cluster.map_shared_rank(X, rr)[(qa + i) * LDZ + 32 * hd + d] = v;
+      });
+      cluster.sync();
+      {  // output projection + residual, 16 outputs, written in place into z
+        const int o0 = kOutSlice * rank;
+        gemm_rows(X, LDZ, n, 128, Wl + WL_OUT, kOutSlice, kOutSlice, Vl + VL_OUTB,
                   [&](int j, int o, float v) {
-                    mine[j * LDKV + koff + o] = v;
-                    peer[j * LDKV + koff + o] = v;
+                    const float val = v + Z[j * LDZ + o0 + o];
+                    for (int rr = 0; rr < kDecideCluster; ++rr)
+                      cluster.map_shared_rank(Z, rr)[j * LDZ + o0 + o] = val;
                   });
       }
       cluster.sync();
-      attend(sm.q, LDQ, sm.kv, sm.kv + 32, LDKV, qb - qa, n, 32, sm.S,
-             [&](int i, int d, float v) {
-               for (int rr = 0; rr < kDecideCluster; ++rr)
-                 cluster.map_shared_rank(sm.X, rr)[(qa + i) * LDX + 32 * h + d] = v;
-             });
-      cluster.sync();
-      {  // output projection + residual, slice of 16
-        const int o0 = 16 * rank;
-        gemm_rows(sm.X, LDX, n, 128, L.out_t, 128, o0, 16, L.out_b, [&](int j, int o, float v) {
-          const float val = v + sm.z[j * LDZ + o0 + o];
-          for (int rr = 0; rr < kDecideCluster; ++rr)
-            cluster.map_shared_rank(sm.zp, rr)[j * LDZ + o0 + o] = val;
-        });
-      }
-      cluster.sync();
-      layer_norm_rows(sm.zp, LDZ, sm.z, LDZ, n, 128, L.ln1_g, L.ln1_b);
+      layer_norm_rows(Z, LDZ, Z, LDZ, n, 128, Vl + VL_LN1G, Vl + VL_LN1B);
       __syncthreads();
-      {  // FFN first linear + GELU, slice of 32
-        const int o0 = 32 * rank;
-        gemm_rows(sm.z, LDZ, n, 128, L.ff1_t, 256, o0, 32, L.ff1_b, [&](int j, int o, float v) {
-          const float val = gelu(v);
+      // FFN: hidden units [32r, 32r+32) locally, then the partial second
+      // linear of those units sent to the owners of each 16-output slice
+      float* Hh = KV;  // [n][36]
+      gemm_rows(Z, LDZ, n, 128, Wl + WL_FF1, kFf1Slice, kFf1Slice, Vl + VL_FF1B,
+                [&](int j, int o, float v) { Hh[j * LDQ + o] = gelu(v); });
+      __syncthreads();
+      gemm_rows(Hh, LDQ, n, kFf1Slice, Wl + WL_FF2, 128, 128, nullptr,
+                [&](int j, int o, float v) {
+                  const int owner = o >> 4;
+                  cluster.map_shared_rank(X, owner)[(rank * W + j) * 16 + (o & 15)] = v;
+                });
+      cluster.sync();
+      {  // owner: sum the 8 partials + bias + residual, broadcast its slice
+        const int o0 = kOutSlice * rank;
+        for (int it = tid; it < n * 16; it += blockDim.x) {
+          const int j = it >> 4, oo = it & 15;
+          float a = Vl[VL_FF2B + oo] + Z[j * LDZ + o0 + oo];
+#pragma unroll
+          for (int src = 0; src < kDecideCluster; ++src) a += X[(src * W + j) * 16 + oo];
           for (int rr = 0; rr < kDecideCluster; ++rr)
-            cluster.map_shared_rank(sm.X, rr)[j * LDX + o0 + o] = val;
-        });
+            cluster.map_shared_rank(Z, rr)[j * LDZ + o0 + oo] = a;
+        }
       }
       cluster.sync();
-      {  // FFN second linear + residual, slice of 16
-        const int o0 = 16 * rank;
-        gemm_rows(sm.X, LDX, n, 256, L.ff2_t, 128, o0, 16, L.ff2_b, [&](int j, int o, float v) {
-          const float val = v + sm.z[j * LDZ + o0 + o];
-          for (int rr = 0; rr < kDecideCluster; ++rr)
-            cluster.map_shared_rank(sm.zp, rr)[j * LDZ + o0 + o] = val;
-        });
-      }
-      cluster.sync();
-      layer_norm_rows(sm.zp, LDZ, sm.z, LDZ, n, 128, L.ln2_g, L.ln2_b);
+      layer_norm_rows(Z, LDZ, Z, LDZ, n, 128, Vl + VL_LN2G, Vl + VL_LN2B);
       __syncthreads();
     }
-    // 3d. head Linear(128 -> 1) (rank 0 needs it)
+    // 3d. head Linear(128 -> 1), needed by rank 0
     if (rank == 0) {
       for (int j = warp; j < n; j += (blockDim.x >> 5)) {
         float a = 0.f;
-        for (int c = 0; c < 4; ++c) a += sm.z[j * LDZ + lane + 32 * c] * w.head_w[lane + 32 * c];
-        a = warp_sum(a) + w.head_b[0];
+        for (int c = 0; c < 4; ++c) a += Z[j * LDZ + lane + 32 * c] * Vv[V_HEADW + lane + 32 * c];
+        a = warp_sum(a) + Vv[V_HEADB];
         if (lane == 0) sm.f_O[sm.Mrows[j]] = a;
       }
     }
     __syncthreads();
   }
-  if (rank != 0) return;  // no remote shared-memory access after this point
+  if (rank != 0) return;  // no distributed shared-memory access after this point
 
   // ---------------------------------------------------------------- 4. block selection
   if (tid == 0) {
@@ -500,7 +554,7 @@ __global__ void __cluster_dims__(kDecideCluster, 1, 1) __launch_bounds__(kDecide
   // ---------------------------------------------------------------- 5. LPS + accept + commit
   const int nBM = sm.nBM;
   if (nBM > 0) {
-    if (p.lps_enabled) lps_forward(sm, p, nBM);
+    if (p.lps_enabled) lps_forward(sm, nBM);
     if (tid == 0) {
       int nacc = 0;
       for (int i = 0; i < nBM; ++i) {

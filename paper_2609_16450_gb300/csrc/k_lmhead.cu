@@ -16,6 +16,7 @@
 // in TMEM as 128 lanes (vocabulary) x N columns (rows).  Warp 0 issues TMA,
 // warp 1 issues tcgen05.mma, warps 2..5 drain TMEM and run the statistics.
 #include <climits>
+#include <cstdlib>
 
 #include "internal.h"
 #include "ptx.cuh"
@@ -127,7 +128,9 @@ __global__ void __launch_bounds__(kLmThreads, 1)
 
   const int u0 = static_cast<int>((static_cast<long long>(cta) * p.n_units) / p.grid);
   const int u1 = static_cast<int>((static_cast<long long>(cta + 1) * p.n_units) / p.grid);
-  const uint32_t b_stage = static_cast<uint32_t>(p.n_pad) * 128u;
+  const uint32_t b_sub = static_cast<uint32_t>(p.n_pad) * 128u;  // one k-box of hidden rows
+  const uint32_t a_stage = static_cast<uint32_t>(p.kbs) * kATile;
+  const uint32_t b_stage = static_cast<uint32_t>(p.kbs) * b_sub;
 
   if (warp == 0) {
     // ------------------------------------------------------------ TMA producer
@@ -138,20 +141,31 @@ __global__ void __launch_bounds__(kLmThreads, 1)
       bool ok = true;
       for (int u = u0; u < u1 && ok; u += 2) {
         const int nu = min(2, u1 - u);
-        for (int kb = 0; kb < p.nkb; ++kb) {
+        for (int ks = 0; ks < p.nks; ++ks) {
           const int s = it % p.stages;
           const uint32_t ph = static_cast<uint32_t>(it / p.stages) & 1u;
           if (!mbar_wait(&empty[s], ph ^ 1u, p.limit_ns, abort)) {
             ok = false;
             break;
           }
-          mbar_arrive_expect_tx(&full[s], static_cast<uint32_t>(nu) * kUnit * 128u + b_stage);
+          const int nsubk = min(p.kbs, p.nkb - ks * p.kbs);
+          mbar_arrive_expect_tx(&full[s], static_cast<uint32_t>(nsubk) *
+                                              (static_cast<uint32_t>(nu) * kUnit * 128u + b_sub));
+          uint8_t* a_st = sA + static_cast<size_t>(s) * a_stage;
+          uint8_t* b_st = sB + static_cast<size_t>(s) * b_stage;
+          // one row half at a time, its k-boxes back to back: each W row is
+          // requested as one contiguous run of nsubk * 128 bytes
           for (int ui = 0; ui < nu; ++ui)
-            tma_load_2d(sA + s * kATile + ui * (kUnit * 128), &tmap_w, &full[s], kb * 64,
-                        (u + ui) * kUnit, pol_w);
-          for (int sb = 0; sb < p.nsub; ++sb)
-            tma_load_2d(sB + s * b_stage + sb * p.nb * 128, &tmap_h, &full[s], kb * 64,
-                        p.row0 + sb * p.nb, pol_h);
+            for (int j = 0; j < nsubk; ++j)
+              tma_load_2d(a_st + j * kATile + ui * (kUnit * 128), &tmap_w, &full[s],
+                          p.packed ? 0 : (ks * p.kbs + j) * 64,
+                          p.packed ? ((u + ui) * p.nkb + ks * p.kbs + j) * kUnit
+                                   : (u + ui) * kUnit,
+                          pol_w);
+          for (int j = 0; j < nsubk; ++j)
+            for (int sb = 0; sb < p.nsub; ++sb)
+              tma_load_2d(b_st + j * b_sub + sb * p.nb * 128, &tmap_h, &full[s],
+                          (ks * p.kbs + j) * 64, p.row0 + sb * p.nb, pol_h);
           ++it;
         }
       }
@@ -178,7 +192,7 @@ __global__ void __launch_bounds__(kLmThreads, 1)
         }
         tc_fence_after();
         const uint32_t d0 = tmem_base + static_cast<uint32_t>(buf * p.acc_stride);
-        for (int kb = 0; kb < p.nkb; ++kb) {
+        for (int ks = 0; ks < p.nks; ++ks) {
           const int s = it % p.stages;
           const uint32_t ph = static_cast<uint32_t>(it / p.stages) & 1u;
           if (!mbar_wait(&full[s], ph, p.limit_ns, abort)) {
@@ -186,15 +200,19 @@ __global__ void __launch_bounds__(kLmThreads, 1)
             break;
           }
           tc_fence_after();
-          const uint32_t a_addr = smem_u32(sA + s * kATile);
-          const uint32_t b_addr = smem_u32(sB + s * b_stage);
+          const int nsubk = min(p.kbs, p.nkb - ks * p.kbs);
+          const uint32_t a_addr = smem_u32(sA + static_cast<size_t>(s) * a_stage);
+          const uint32_t b_addr = smem_u32(sB + static_cast<size_t>(s) * b_stage);
+          for (int j = 0; j < nsubk; ++j) {
 #pragma unroll
-          for (int kk = 0; kk < 4; ++kk) {
-            const uint64_t ad = umma_desc_sw128(a_addr + kk * 32);
-            for (int sb = 0; sb < p.nsub; ++sb) {
-              const uint64_t bd = umma_desc_sw128(b_addr + sb * p.nb * 128 + kk * 32);
-              umma_bf16(d0 + static_cast<uint32_t>(sb * p.nb), ad, bd, idesc,
-                        (kb | kk) != 0 ? 1u : 0u);
+            for (int kk = 0; kk < 4; ++kk) {
+              const uint64_t ad = umma_desc_sw128(a_addr + j * kATile + kk * 32);
+              for (int sb = 0; sb < p.nsub; ++sb) {
+                const uint64_t bd =
+                    umma_desc_sw128(b_addr + j * b_sub + sb * p.nb * 128 + kk * 32);
+                umma_bf16(d0 + static_cast<uint32_t>(sb * p.nb), ad, bd, idesc,
+                          (ks | j | kk) != 0 ? 1u : 0u);
+              }
             }
           }
           umma_commit(&empty[s]);
@@ -335,19 +353,68 @@ void lm_plan(LmParams& p, int rows, int V, int d, int num_sms) {
   p.n_units = (V + kUnit - 1) / kUnit;
   p.grid = num_sms < p.n_units ? num_sms : p.n_units;
   p.nkb = (d + 63) / 64;
-  const uint32_t stage = kATile + static_cast<uint32_t>(p.n_pad) * 128u;
   const uint32_t st_bytes = static_cast<uint32_t>(p.n_pad) * 20u;
   const uint32_t tail = kTBytes + ((st_bytes + 7) / 8 * 8) + (2 * 8 + 6) * 8 + 16;
   const uint32_t budget = 232448u - 1024u - tail;
+  // k-boxes (64 columns each) per pipeline stage: longer contiguous runs of
+  // each W row per request, while keeping at least two stages in flight
+  int kbs = 4;
+  if (const char* env = getenv("EBD_LM_KBS")) kbs = atoi(env);
+  if (kbs < 1) kbs = 1;
+  if (kbs > p.nkb) kbs = p.nkb;
+  while (kbs > 1 && budget / (static_cast<uint32_t>(kbs) * (kATile + p.n_pad * 128u)) < 2) --kbs;
+  p.kbs = kbs;
+  p.nks = (p.nkb + kbs - 1) / kbs;
+  const uint32_t stage = static_cast<uint32_t>(kbs) * (kATile + static_cast<uint32_t>(p.n_pad) * 128u);
   int stages = static_cast<int>(budget / stage);
   if (stages > 8) stages = 8;
   p.stages = stages;
   p.off_a = 0;
-  p.off_b = p.off_a + static_cast<uint32_t>(stages) * kATile;
-  p.off_t = p.off_b + static_cast<uint32_t>(stages) * static_cast<uint32_t>(p.n_pad) * 128u;
+  p.off_b = p.off_a + static_cast<uint32_t>(stages) * kbs * kATile;
+  p.off_t = p.off_b + static_cast<uint32_t>(stages) * kbs * static_cast<uint32_t>(p.n_pad) * 128u;
   p.off_st = p.off_t + kTBytes;
   p.off_bar = (p.off_st + st_bytes + 7) / 8 * 8;
   p.smem_bytes = p.off_bar + static_cast<uint32_t>(2 * stages + 6) * 8u + 16u + 1024u;
+}
+
+// Tiled copy of W: out[((u * nkb + k) * 64 + r) * 64 + c] = W[64u + r][64k + c]
+__global__ void __launch_bounds__(256) pack_lm_kernel(const uint4* __restrict__ w,
+                                                      uint4* __restrict__ out, int V, int d,
+                                                      int nkb, long long n_vec) {
+  const long long i = static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x;
+  if (i >= n_vec) return;
+  const int c8 = static_cast<int>(i & 7);          // 8 bf16 per 16-byte vector
+  const long long row = i >> 3;                    // packed row (64 columns)
+  const int r = static_cast<int>(row & 63);
+  const long long tile = row >> 6;
+  const int kb = static_cast<int>(tile % nkb);
+  const long long u = tile / nkb;
+  const long long v = u * 64 + r;
+  const int col = kb * 64 + c8 * 8;
+  uint4 val = make_uint4(0u, 0u, 0u, 0u);
+  if (v < V && col < d) {
+    if (col + 8 <= d && (d % 8) == 0) {
+      val = w[(v * d + col) / 8];
+    } else {
+      const __nv_bfloat16* ws = reinterpret_cast<const __nv_bfloat16*>(w);
+      __nv_bfloat16 t[8];
+      for (int e = 0; e < 8; ++e)
+        t[e] = (col + e < d) ? ws[v * d + col + e] : __float2bfloat16(0.f);
+      val = *reinterpret_cast<uint4*>(t);
+    }
+  }
+  out[i] = val;
+}
+
+cudaError_t launch_pack_lm(const __nv_bfloat16* w, __nv_bfloat16* out, int V, int d,
+                           cudaStream_t st) {
+  const int nkb = (d + 63) / 64;
+  const long long units = (V + 63) / 64;
+  const long long n_vec = units * nkb * 64 * 8;
+  const long long blocks = (n_vec + 255) / 256;
+  pack_lm_kernel<<<static_cast<unsigned>(blocks), 256, 0, st>>>(
+      reinterpret_cast<const uint4*>(w), reinterpret_cast<uint4*>(out), V, d, nkb, n_vec);
+  return cudaGetLastError();
 }
 
 cudaError_t lm_configure() {

@@ -1,0 +1,57 @@
+// Device image of the router weights, laid out for the decision kernel.
+//
+// The LBS encoder is split over the 8 CTAs of a cluster by output features
+// (rank r owns QKV features [48r, 48r+48), projection/combine outputs
+// [16r, 16r+16) and FFN hidden units [32r, 32r+32)).  Each rank's matrices
+// are stored transposed ([in][out], bf16) in one contiguous block, so a CTA
+// loads everything it needs with one bulk copy; vectors are fp32.
+#pragma once
+
+namespace ebd {
+namespace rimg {
+
+constexpr int kRanks = 8;
+constexpr int kQkvSlice = 48, kOutSlice = 16, kFf1Slice = 32, kCombSlice = 16;
+constexpr int kPosRows = 64;  // E_pos rows a window can use
+
+// ---- LBS weights of one rank, bf16 elements
+constexpr int W_ENT2 = 0;         // [64][64]   ent2 (full)
+constexpr int W_COMB = 4096;      // [128][16]  combine slice
+constexpr int W_POS = 6144;       // [64][16]   E_pos slice
+constexpr int W_LAYER0 = 7168;    // two layers of W_LAYER_STRIDE
+constexpr int W_LAYER_STRIDE = 16384;
+constexpr int WL_QKV = 0;         // [128][48]  QKV feature slice
+constexpr int WL_OUT = 6144;      // [128][16]  output projection slice
+constexpr int WL_FF1 = 8192;      // [128][32]  FFN first linear, hidden slice
+constexpr int WL_FF2 = 12288;     // [32][128]  FFN second linear, rows of the hidden slice
+constexpr int LBS_W_ELEMS = W_LAYER0 + 2 * W_LAYER_STRIDE;  // 39936
+
+// ---- LPS weights (one copy), bf16 elements, per layer
+constexpr int PL_QKV = 0;         // [32][96]
+constexpr int PL_OUT = 3072;      // [32][32]
+constexpr int PL_FF1 = 4096;      // [32][64]
+constexpr int PL_FF2 = 6144;      // [64][32]
+constexpr int PL_STRIDE = 8192;
+constexpr int LPS_W_ELEMS = 2 * PL_STRIDE;
+
+// ---- fp32 vectors of one rank
+constexpr int V_ENT1W = 0, V_ENT1B = 64, V_ENT2B = 128, V_ENTLNG = 192, V_ENTLNB = 256;
+constexpr int V_TOKB = 320, V_HEADW = 384, V_HEADB = 512, V_COMBB = 516;
+constexpr int V_LAYER0 = 544, V_LAYER_STRIDE = 624;
+constexpr int VL_QKVB = 0, VL_OUTB = 48, VL_FF1B = 64, VL_FF2B = 96;
+constexpr int VL_LN1G = 112, VL_LN1B = 240, VL_LN2G = 368, VL_LN2B = 496;
+constexpr int V_LPS = 1792;
+constexpr int VP_INT = 0, VP_INB = 160, VP_INLNG = 192, VP_INLNB = 224, VP_HEADW = 256;
+constexpr int VP_HEADB = 288, VP_LAYER0 = 292, VP_LAYER_STRIDE = 352;
+constexpr int VPL_LN1G = 0, VPL_LN1B = 32, VPL_QKVB = 64, VPL_OUTB = 160, VPL_LN2G = 192;
+constexpr int VPL_LN2B = 224, VPL_FF1B = 256, VPL_FF2B = 320;
+constexpr int V_ELEMS = 2800;
+
+static_assert(V_LAYER0 + 2 * V_LAYER_STRIDE <= V_LPS, "vector layout");
+static_assert(V_LPS + VP_LAYER0 + 2 * VP_LAYER_STRIDE <= V_ELEMS, "vector layout");
+static_assert((LBS_W_ELEMS * 2) % 16 == 0 && (LPS_W_ELEMS * 2) % 16 == 0 &&
+                  (V_ELEMS * 4) % 16 == 0,
+              "bulk copies move multiples of 16 bytes");
+
+}  // namespace rimg
+}  // namespace ebd

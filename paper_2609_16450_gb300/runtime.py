@@ -90,10 +90,21 @@ def stream_handle(stream) -> int:
 class DeviceWeights:
     w_lm: torch.Tensor
     w_emb: torch.Tensor
+    layout: int = 0          # 0: row-major W_lm; 1: tiled by ebd_pack_lm_head
 
 
 def upload_weights(inp, device="cuda") -> DeviceWeights:
     return DeviceWeights(w_lm=_dev(inp.w_lm, device), w_emb=_dev(inp.w_emb, device))
+
+
+def pack_weights(h: "Handle", w: DeviceWeights, stream=None) -> DeviceWeights:
+    """Tiled copy of W_lm (one-time); the row-major copy is released."""
+    n = E.ebd_lm_head_packed_bytes(h.cfg)
+    packed = torch.empty(n // 2, dtype=torch.int16, device=w.w_lm.device)
+    E.check(E.ebd_pack_lm_head(h.h, w.w_lm.data_ptr(), packed.data_ptr(), stream_handle(stream)),
+            h.h)
+    torch.cuda.synchronize()
+    return DeviceWeights(w_lm=packed, w_emb=w.w_emb, layout=1)
 
 
 class DeviceStep:
@@ -157,6 +168,7 @@ class DeviceStep:
                      "lbs_logit", "lps_prob", "accepted"):
             setattr(a, name, ptr(getattr(self, name)))
         a.w_lm = self.weights.w_lm.data_ptr()
+        a.w_lm_layout = self.weights.layout
         return a
 
     def fetch(self) -> Dict[str, np.ndarray]:

@@ -26,3 +26,17 @@ def pytest_collection_modifyitems(config, items):
     for it in items:
         if "gpu" in it.keywords:
             it.add_marker(skip)
+
+
+@pytest.fixture(scope="session", autouse=True)
+def _build_library_for_gpu_tests(request):
+    """GPU sessions compile libebd.so for sm_103a first (no-op when fresh)."""
+    try:
+        import torch
+        if not torch.cuda.is_available():
+            return
+    except Exception:
+        return
+    if any("gpu" in it.keywords for it in request.session.items):
+        from paper_2609_16450_gb300 import build
+        build.build()

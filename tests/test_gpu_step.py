@@ -68,9 +68,13 @@ def test_tiny_step(state):
     assert gpu["accepted"].sum() >= 1
 
 
-def test_llada_step():
+@pytest.mark.parametrize("layout", ["rowmajor", "packed"])
+def test_llada_step(layout):
+    from paper_2609_16450_gb300 import runtime as rt
     sh = synth.llada
     inp, w, h = _setup(sh)
+    if layout == "packed":
+        w = rt.pack_weights(h, rt.DeviceWeights(w_lm=w.w_lm, w_emb=w.w_emb))
     for state in ("select", "inblock"):
         inp2 = synth.make_step_inputs(sh)
         if state == "inblock":
