@@ -350,12 +350,12 @@ ebd_status upload_router(ebd_handle* h) {
     const std::string pre = "lps.l" + std::to_string(l);
     uint16_t* wl = lps.data() + l * PL_STRIDE;
     for (int k = 0; k < 32; ++k) {
-      for (int o = 0; o < 96; ++o) wl[PL_QKV + k * 96 + o] = at(pre + ".qkv.w", o, k);
-      for (int o = 0; o < 32; ++o) wl[PL_OUT + k * 32 + o] = at(pre + ".out.w", o, k);
-      for (int o = 0; o < 64; ++o) wl[PL_FF1 + k * 64 + o] = at(pre + ".ff1.w", o, k);
+      for (int o = 0; o < 96; ++o) wl[PL_QKV + k * PL_LDQKV + o] = at(pre + ".qkv.w", o, k);
+      for (int o = 0; o < 32; ++o) wl[PL_OUT + k * PL_LDOUT + o] = at(pre + ".out.w", o, k);
+      for (int o = 0; o < 64; ++o) wl[PL_FF1 + k * PL_LDFF1 + o] = at(pre + ".ff1.w", o, k);
     }
     for (int k = 0; k < 64; ++k)
-      for (int o = 0; o < 32; ++o) wl[PL_FF2 + k * 32 + o] = at(pre + ".ff2.w", o, k);
+      for (int o = 0; o < 32; ++o) wl[PL_FF2 + k * PL_LDFF2 + o] = at(pre + ".ff2.w", o, k);
   }
   const size_t b_lbs = lbs.size() * 2, b_lps = lps.size() * 2, b_vec = vec.size() * 4;
   const size_t o_lps = (b_lbs + 255) / 256 * 256;

@@ -19,34 +19,6 @@ namespace {
 
 constexpr int kStageBytes = 4 * 8192;  // K and V, two 64-dim halves each
 
-__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2,
-                                        uint32_t& r3) {
-  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
-               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
-               : "r"(addr));
-}
-__device__ __forceinline__ void ldsm_x4_t(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2,
-                                          uint32_t& r3) {
-  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
-               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
-               : "r"(addr));
-}
-__device__ __forceinline__ void mma_bf16(float (&d)[4], const uint32_t (&a)[4], uint32_t b0,
-                                         uint32_t b1) {
-  asm volatile(
-      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, "
-      "{%8,%9}, {%0,%1,%2,%3};"
-      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
-      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
-}
-// split x = hi + lo with hi = bf16(x), lo = bf16(x - hi)
-__device__ __forceinline__ void split2(float x, float y, uint32_t& hi, uint32_t& lo) {
-  __nv_bfloat162 h = __floats2bfloat162_rn(x, y);
-  const float2 hf = __bfloat1622float2(h);
-  __nv_bfloat162 l = __floats2bfloat162_rn(x - hf.x, y - hf.y);
-  hi = *reinterpret_cast<uint32_t*>(&h);
-  lo = *reinterpret_cast<uint32_t*>(&l);
-}
 // byte offset of 16-byte chunk `c` (0..7) of row `r` in a 128B-swizzled tile
 __device__ __forceinline__ uint32_t swz(int r, int c) {
   return static_cast<uint32_t>(r * 128 + ((c ^ (r & 7)) << 4));
@@ -225,10 +197,10 @@ __global__ void __launch_bounds__(kAttnThreads)
 #pragma unroll
       for (int kk = 0; kk < 4; ++kk) {
         uint32_t ah[4], al[4];
-        split2(sc[2 * kk][0], sc[2 * kk][1], ah[0], al[0]);
-        split2(sc[2 * kk][2], sc[2 * kk][3], ah[1], al[1]);
-        split2(sc[2 * kk + 1][0], sc[2 * kk + 1][1], ah[2], al[2]);
-        split2(sc[2 * kk + 1][2], sc[2 * kk + 1][3], ah[3], al[3]);
+        split_bf16x2(sc[2 * kk][0], sc[2 * kk][1], ah[0], al[0]);
+        split_bf16x2(sc[2 * kk][2], sc[2 * kk][3], ah[1], al[1]);
+        split_bf16x2(sc[2 * kk + 1][0], sc[2 * kk + 1][1], ah[2], al[2]);
+        split_bf16x2(sc[2 * kk + 1][2], sc[2 * kk + 1][3], ah[3], al[3]);
 #pragma unroll
         for (int dp = 0; dp < D / 16; ++dp) {
           const int hf = dp >> 2;

@@ -11,10 +11,16 @@
 //
 // One thread-block cluster of 8 CTAs per sequence.  The LBS encoder is split
 // across the cluster by output features (and, for attention, by head and
-// query half); every CTA keeps a full copy of the activations and the
-// slices are exchanged through distributed shared memory.  Router matmuls
-// are fp32 FMA on bf16-stored weights.  The LPS router and the decision run
-// in rank 0.
+// query half); every CTA keeps a full copy of the residual stream and the
+// slices are exchanged through distributed shared memory.  The LPS router
+// and the decision run in rank 0.
+//
+// Matrix products run on the tensor cores (mma.sync m16n8k16, bf16 weights,
+// fp32 accumulation).  Every activation that feeds a product is stored once,
+// by the phase that produces it, as a bf16 high part and a bf16 remainder
+// (x = hi + lo to ~16 mantissa bits), so that a product loads its A fragments
+// with ldmatrix and runs two MMAs per k-step.  The kernel is short and
+// latency-bound: phases are kept few and their per-warp chains short.
 #include <cooperative_groups.h>
 
 #include <climits>
@@ -32,39 +38,48 @@ namespace {
 using namespace rimg;
 
 constexpr int W = kMaxWindow;  // rows per sequence
-constexpr int LDZ = 132;       // residual stream / [e;t] / attention concat
-constexpr int LDKV = 68;       // k in [0,32), v in [32,64)
+constexpr int LDZ = 132;       // fp32 residual stream row stride
+constexpr int LDH = 136;       // bf16 hi/lo row stride for 128 columns (conflict-free ldmatrix)
+constexpr int LDKV = 68;       // fp32 k in [0,32), v in [32,64)
 constexpr int LDQ = 36;
 constexpr int LDS = 68;
 // activation pool (floats), LBS phase
-constexpr int P_Z = 0;                  // [64][132] residual stream z
-constexpr int P_X = P_Z + W * LDZ;      // [64][132] [e;t] | concat | FFN partial inbox [8][64][16]
-constexpr int P_KV = P_X + W * LDZ;     // [64][68]  k,v of this CTA's head | FFN hidden [64][36]
-constexpr int P_Q = P_KV + W * LDKV;    // [32][36]  queries of this CTA's half
-constexpr int P_S = P_Q + 32 * LDQ;     // [32][68]  attention scores
-constexpr int POOL = P_S + 32 * LDS;    // 24576 floats
+constexpr int P_Z = 0;                       // [64][132] fp32 residual stream z
+constexpr int P_ZH = P_Z + W * LDZ;          // [64][136] bf16 x2: z as GEMM input (hi, lo)
+constexpr int P_XH = P_ZH + W * LDH;         // [64][136] bf16 x2: [e;t] | concat ; fp32 FFN inbox [8][64][16]
+constexpr int P_KV = P_XH + W * LDH;         // [64][68]  fp32 k,v of this CTA's head | bf16 x2 FFN hidden / F_ent
+constexpr int P_Q = P_KV + W * LDKV;         // [32][36]  fp32 queries of this CTA's half
+constexpr int P_S = P_Q + 32 * LDQ;          // [32][68]  fp32 attention scores
+constexpr int POOL = P_S + 32 * LDS;
+static_assert(8 * W * 16 <= W * LDH, "FFN partial inbox");
+static_assert(W * 72 <= POOL - P_KV, "F_ent hidden hi/lo (spans k/v, q and scores)");
+static_assert(W * LDZ <= W * LDH, "ent2 output scratch in the z hi/lo region");
 // activation pool, LPS phase (rank 0)
-constexpr int L_Z = 0, L_Y = 2304, L_F = 4608, L_QKV = 5120, L_ATT = 11520, L_SC = 13824,
-              L_H = 18176;
-static_assert(L_H + W * 68 <= POOL, "LPS pool layout");
-static_assert(8 * W * 16 <= W * LDZ, "FFN partial inbox");
+constexpr int L_FEAT = 0;                    // [64][8] features
+constexpr int L_Z = 512;                     // [64][36] fp32 residual stream
+constexpr int L_YH = L_Z + W * LDQ;          // [64][40] bf16 x2: LayerNorm output
+constexpr int L_QKV = L_YH + W * 40;         // [64][100] fp32 q | k | v
+constexpr int L_AH = L_QKV + W * 100;        // [64][40] bf16 x2: attention output
+constexpr int L_HH = L_AH + W * 40;          // [64][72] bf16 x2: FFN hidden
+constexpr int L_PROB = L_HH + W * 72;        // [64]
+static_assert(L_PROB + W <= POOL, "LPS pool layout");
 
 struct __align__(16) Smem {
-  __nv_bfloat16 w[LBS_W_ELEMS];   // this rank's LBS weight slices
-  __nv_bfloat16 lw[LPS_W_ELEMS];  // LPS weights (rank 0)
-  float v[V_ELEMS];               // vectors
+  __nv_bfloat16 w[LBS_W_ELEMS];  // this rank's LBS weight slices; later the LPS weights
+  float v[V_ELEMS];              // vectors
   float pool[POOL];
   float f_conf[W], f_ent[W], f_gap[W], f_O[W], f_p[W];
   int f_arg[W], f_pos[W], f_tok[W], Mrows[W], Brows[W], BMrows[W];
   uint8_t f_mask[W], f_ib[W], f_acc[W], f_bad[W];
-  int nM, nBM, meta_b, meta_s, n_rows, r0, run_lbs, bad_seq, wait_fail;
-  uint64_t bar;
+  int nM, nBM, meta_b, meta_s, n_rows, r0, run_lbs, bad_seq, lps_loaded;
+  uint64_t bar;   // vectors (+ LBS weights)
+  uint64_t bar2;  // LPS weights
 };
+static_assert(sizeof(Smem) + 16 <= 232448, "dynamic shared memory of one CTA");
 
 __device__ __forceinline__ float gelu(float x) {
   return 0.5f * x * (1.0f + erff(x * 0.70710678118654752f));
 }
-
 __device__ __forceinline__ float warp_sum(float v) {
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
@@ -85,99 +100,97 @@ __device__ __forceinline__ void bulk_copy(void* smem_dst, const void* gsrc, uint
       : "memory");
 }
 
-// out(j, o) = bias[o] + sum_k in[j][k] * Wt[k][o] for j < n, o < Os (Os even);
-// Wt is shared-memory bf16 [K][ldw].  epi(j, o, value) consumes the result.
+// hi/lo pair of bf16 buffers: hi at base, lo at base + plane (elements)
+struct HL {
+  __nv_bfloat16* p;
+  int ld, plane;
+};
+__device__ __forceinline__ HL hl_at(float* pool_floats, int ld) {
+  return HL{reinterpret_cast<__nv_bfloat16*>(pool_floats), ld, W * ld};
+}
+// stores (x, y) as columns (c, c+1) of row j
+__device__ __forceinline__ void hl_store2(const HL& h, int j, int c, float x, float y) {
+  uint32_t hi, lo;
+  split_bf16x2(x, y, hi, lo);
+  *reinterpret_cast<uint32_t*>(h.p + j * h.ld + c) = hi;
+  *reinterpret_cast<uint32_t*>(h.p + h.plane + j * h.ld + c) = lo;
+}
+__device__ __forceinline__ void hl_store1(const HL& h, int j, int c, float x) {
+  const __nv_bfloat16 hi = __float2bfloat16_rn(x);
+  h.p[j * h.ld + c] = hi;
+  h.p[h.plane + j * h.ld + c] = __float2bfloat16_rn(x - __bfloat162float(hi));
+}
+
+// out(j, o) = sum_k A[j][k] Wt[k][o] for j < n, o < Os, A = hi + lo in
+// shared memory, Wt bf16 [K][ldw].  Each warp owns 16-row x 16-output tiles;
+// epi(j, o, v0, v1) receives the outputs o and o + 1 of row j.
 template <class Epi>
-__device__ __forceinline__ void gemm_rows(const float* in, int ldi, int n, int K,
-                                          const __nv_bfloat16* Wt, int ldw, int Os,
-                                          const float* bias, Epi epi) {
-  const int pairs = Os >> 1;
-  const int ldw2 = ldw >> 1;
-  for (int it = threadIdx.x; it < n * pairs; it += blockDim.x) {
-    const int j = it / pairs, pr = it - j * pairs;
-    float a0 = bias ? bias[2 * pr] : 0.f, a1 = bias ? bias[2 * pr + 1] : 0.f;
-    const float* x = in + j * ldi;
-    const __nv_bfloat162* w = reinterpret_cast<const __nv_bfloat162*>(Wt) + pr;
-    int k = 0;
-#pragma unroll 2
-    for (; k + 4 <= K; k += 4) {
-      const float4 xv = *reinterpret_cast<const float4*>(x + k);
-      const float2 w0 = __bfloat1622float2(w[(k + 0) * ldw2]);
-      const float2 w1 = __bfloat1622float2(w[(k + 1) * ldw2]);
-      const float2 w2 = __bfloat1622float2(w[(k + 2) * ldw2]);
-      const float2 w3 = __bfloat1622float2(w[(k + 3) * ldw2]);
-      a0 = fmaf(xv.x, w0.x, a0); a1 = fmaf(xv.x, w0.y, a1);
-      a0 = fmaf(xv.y, w1.x, a0); a1 = fmaf(xv.y, w1.y, a1);
-      a0 = fmaf(xv.z, w2.x, a0); a1 = fmaf(xv.z, w2.y, a1);
-      a0 = fmaf(xv.w, w3.x, a0); a1 = fmaf(xv.w, w3.y, a1);
+__device__ __forceinline__ void gemm_hl(const HL& A, int n, int K, const __nv_bfloat16* Wt,
+                                        int ldw, int Os, Epi epi) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int g = lane >> 2, t = lane & 3;
+  const int mi = lane >> 3, rr = lane & 7;
+  const int mt = (n + 15) >> 4, np = Os >> 4;
+#pragma unroll 1
+  for (int unit = warp; unit < mt * np; unit += (blockDim.x >> 5)) {
+    const int m0 = (unit / np) * 16, c0 = (unit % np) * 16;
+    float acc[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
+    const uint32_t ah_base =
+        smem_u32(A.p + (m0 + (mi & 1) * 8 + rr) * A.ld + (mi >> 1) * 8);
+    const uint32_t al_base = ah_base + static_cast<uint32_t>(A.plane * 2);
+    const uint32_t w_base = smem_u32(Wt + ((mi & 1) * 8 + rr) * ldw + c0 + (mi >> 1) * 8);
+#pragma unroll 4
+    for (int k0 = 0; k0 < K; k0 += 16) {
+      uint32_t ah[4], al[4], b0, b1, b2, b3;
+      ldsm_x4(ah_base + k0 * 2, ah[0], ah[1], ah[2], ah[3]);
+      ldsm_x4(al_base + k0 * 2, al[0], al[1], al[2], al[3]);
+      ldsm_x4_t(w_base + static_cast<uint32_t>(k0 * ldw * 2), b0, b1, b2, b3);
+      mma_bf16(acc[0], ah, b0, b1);
+      mma_bf16(acc[1], ah, b2, b3);
+      mma_bf16(acc[0], al, b0, b1);
+      mma_bf16(acc[1], al, b2, b3);
     }
-    for (; k < K; ++k) {
-      const float2 wk = __bfloat1622float2(w[k * ldw2]);
-      a0 = fmaf(x[k], wk.x, a0);
-      a1 = fmaf(x[k], wk.y, a1);
+    const int r_lo = m0 + g, r_hi = r_lo + 8;
+#pragma unroll
+    for (int nt = 0; nt < 2; ++nt) {
+      const int o = c0 + nt * 8 + 2 * t;
+      if (r_lo < n) epi(r_lo, o, acc[nt][0], acc[nt][1]);
+      if (r_hi < n) epi(r_hi, o, acc[nt][2], acc[nt][3]);
     }
-    epi(j, 2 * pr, a0);
-    epi(j, 2 * pr + 1, a1);
   }
 }
 
-// LayerNorm (eps 1e-5) over `dim` (32, 64 or 128) of rows j < n; warp per row.
-__device__ __forceinline__ void layer_norm_rows(const float* src, int lds, float* dst, int ldd,
-                                                int n, int dim, const float* g, const float* b) {
+// LayerNorm (eps 1e-5) over `dim` (32, 64 or 128) of rows j < n, warp per
+// row; the result goes to an fp32 buffer (if dst) and/or a hi/lo buffer.
+__device__ __forceinline__ void ln_rows(const float* src, int lds, float* dst, int ldd,
+                                        const HL* hl, int hl_col, int n, int dim, const float* g,
+                                        const float* b) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int nw = blockDim.x >> 5;
   const int per = dim >> 5;
-  for (int j = warp; j < n; j += nw) {
+#pragma unroll 1
+  for (int j = warp; j < n; j += (blockDim.x >> 5)) {
     float v[4] = {0.f, 0.f, 0.f, 0.f};
     float s = 0.f;
-    for (int c = 0; c < per; ++c) {
-      v[c] = src[j * lds + lane + 32 * c];
-      s += v[c];
-    }
+#pragma unroll
+    for (int c = 0; c < 4; ++c)
+      if (c < per) {
+        v[c] = src[j * lds + lane + 32 * c];
+        s += v[c];
+      }
     const float mean = warp_sum(s) / dim;
     float q = 0.f;
-    for (int c = 0; c < per; ++c) {
-      const float d = v[c] - mean;
-      q += d * d;
-    }
+#pragma unroll
+    for (int c = 0; c < 4; ++c)
+      if (c < per) q += (v[c] - mean) * (v[c] - mean);
     const float inv = 1.0f / sqrtf(warp_sum(q) / dim + 1e-5f);
-    for (int c = 0; c < per; ++c) {
-      const int o = lane + 32 * c;
-      dst[j * ldd + o] = (v[c] - mean) * inv * g[o] + b[o];
-    }
-  }
-}
-
-// Scaled dot-product attention of queries qs[i] (i < nq) over keys/values
-// k < n (head width dh); writes o(i, d) through epi.  S: [nq][LDS] scratch.
-template <class Epi>
-__device__ __forceinline__ void attend(const float* qs, int ldq, const float* ks, const float* vs,
-                                       int ldkv, int nq, int n, int dh, float* S, Epi epi) {
-  const float scale = 1.0f / sqrtf(static_cast<float>(dh));
-  for (int it = threadIdx.x; it < nq * n; it += blockDim.x) {
-    const int i = it / n, k = it - i * n;
-    float a = 0.f;
-    for (int d = 0; d < dh; ++d) a = fmaf(qs[i * ldq + d], ks[k * ldkv + d], a);
-    S[i * LDS + k] = a * scale;
-  }
-  __syncthreads();
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  for (int i = warp; i < nq; i += (blockDim.x >> 5)) {
-    const float x0 = lane < n ? S[i * LDS + lane] : -INFINITY;
-    const float x1 = lane + 32 < n ? S[i * LDS + lane + 32] : -INFINITY;
-    const float m = warp_max(fmaxf(x0, x1));
-    const float e0 = lane < n ? expf(x0 - m) : 0.f;
-    const float e1 = lane + 32 < n ? expf(x1 - m) : 0.f;
-    const float inv = 1.0f / warp_sum(e0 + e1);
-    if (lane < n) S[i * LDS + lane] = e0 * inv;
-    if (lane + 32 < n) S[i * LDS + lane + 32] = e1 * inv;
-  }
-  __syncthreads();
-  for (int it = threadIdx.x; it < nq * dh; it += blockDim.x) {
-    const int i = it / dh, d = it - i * dh;
-    float a = 0.f;
-    for (int k = 0; k < n; ++k) a = fmaf(S[i * LDS + k], vs[k * ldkv + d], a);
-    epi(i, d, a);
+#pragma unroll
+    for (int c = 0; c < 4; ++c)
+      if (c < per) {
+        const int o = lane + 32 * c;
+        const float y = (v[c] - mean) * inv * g[o] + b[o];
+        if (dst) dst[j * ldd + o] = y;
+        if (hl) hl_store1(*hl, j, hl_col + o, y);
+      }
   }
 }
 
@@ -200,73 +213,229 @@ __device__ __forceinline__ void merge_state(float& m, float& s, float& t, float&
   s = s + sc * bs;
 }
 
-// ----------------------------------------------------------------- LPS (rank 0)
-// Sec. 5.2 / App. D.1: Linear(5->32) -> LayerNorm -> GELU, two pre-norm blocks
-// (4 heads, FFN 64, GELU), head Linear(32->1); p_psi = sigmoid(O).
-__device__ void lps_forward(Smem& sm, int n) {
-  float* P = sm.pool;
-  float* zL = P + L_Z;
-  float* yL = P + L_Y;
-  float* fL = P + L_F;
-  float* qkv = P + L_QKV;
-  float* att = P + L_ATT;
-  float* sc = P + L_SC;
-  float* h64 = P + L_H;
-  const float* V = sm.v + V_LPS;
-  constexpr int LD = 36, LDQKV = 100;
-  const float rho = static_cast<float>(sm.nBM) / static_cast<float>(sm.meta_s);
-  for (int i = threadIdx.x; i < n; i += blockDim.x) {
-    const int r = sm.BMrows[i];
-    fL[i * 8 + 0] = sm.f_conf[r];
-    fL[i * 8 + 1] = sm.f_ent[r];
-    fL[i * 8 + 2] = sm.f_gap[r];
-    fL[i * 8 + 3] = rho;
-    fL[i * 8 + 4] = static_cast<float>(sm.f_pos[r] - sm.meta_b) / static_cast<float>(sm.meta_s);
-  }
-  __syncthreads();
-  for (int it = threadIdx.x; it < n * 32; it += blockDim.x) {
-    const int i = it >> 5, o = it & 31;
-    float a = V[VP_INB + o];
-    for (int k = 0; k < 5; ++k) a = fmaf(fL[i * 8 + k], V[VP_INT + k * 32 + o], a);
-    yL[i * LD + o] = a;
-  }
-  __syncthreads();
-  layer_norm_rows(yL, LD, zL, LD, n, 32, V + VP_INLNG, V + VP_INLNB);
-  __syncthreads();
-  for (int it = threadIdx.x; it < n * 32; it += blockDim.x) {
-    const int i = it >> 5, o = it & 31;
-    zL[i * LD + o] = gelu(zL[i * LD + o]);
-  }
-  __syncthreads();
-  for (int l = 0; l < 2; ++l) {
-    const __nv_bfloat16* Wl = sm.lw + l * PL_STRIDE;
-    const float* Vl = V + VP_LAYER0 + l * VP_LAYER_STRIDE;
-    layer_norm_rows(zL, LD, yL, LD, n, 32, Vl + VPL_LN1G, Vl + VPL_LN1B);
-    __syncthreads();
-    gemm_rows(yL, LD, n, 32, Wl + PL_QKV, 96, 96, Vl + VPL_QKVB,
-              [&](int j, int o, float v) { qkv[j * LDQKV + o] = v; });
-    __syncthreads();
-    for (int h = 0; h < 4; ++h) {
-      attend(qkv + 8 * h, LDQKV, qkv + 32 + 8 * h, qkv + 64 + 8 * h, LDQKV, n, n, 8, sc,
-             [&](int i, int d, float v) { att[i * LD + 8 * h + d] = v; });
-      __syncthreads();
+// ------------------------------------------------------------------ LBS attention
+// This CTA's query rows [qa, qa + nq) of head hd (width 32) over the n rows'
+// keys/values; the output (hi/lo) goes to every rank's concat buffer.
+__device__ __forceinline__ void lbs_attention(cg::cluster_group& cluster, float* P, int nq, int n,
+                                              int qa, int hd) {
+  const float* Q = P + P_Q;
+  const float* KV = P + P_KV;
+  float* S = P + P_S;
+  const float scale = 0.17677669529663687f;  // 1/sqrt(32)
+#pragma unroll 1
+  for (int it = threadIdx.x; it < nq * n; it += blockDim.x) {
+    const int i = it / n, k = it - i * n;
+    const float4* q4 = reinterpret_cast<const float4*>(Q + i * LDQ);
+    const float4* k4 = reinterpret_cast<const float4*>(KV + k * LDKV);
+    float a0 = 0.f, a1 = 0.f;
+#pragma unroll
+    for (int d = 0; d < 8; d += 2) {
+      const float4 x0 = q4[d], y0 = k4[d], x1 = q4[d + 1], y1 = k4[d + 1];
+      a0 = fmaf(x0.x, y0.x, fmaf(x0.y, y0.y, fmaf(x0.z, y0.z, fmaf(x0.w, y0.w, a0))));
+      a1 = fmaf(x1.x, y1.x, fmaf(x1.y, y1.y, fmaf(x1.z, y1.z, fmaf(x1.w, y1.w, a1))));
     }
-    gemm_rows(att, LD, n, 32, Wl + PL_OUT, 32, 32, Vl + VPL_OUTB,
-              [&](int j, int o, float v) { zL[j * LD + o] += v; });
+    S[i * LDS + k] = (a0 + a1) * scale;
+  }
+  __syncthreads();
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+#pragma unroll 1
+  for (int i = warp; i < nq; i += (blockDim.x >> 5)) {
+    const float x0 = lane < n ? S[i * LDS + lane] : -INFINITY;
+    const float x1 = lane + 32 < n ? S[i * LDS + lane + 32] : -INFINITY;
+    const float m = warp_max(fmaxf(x0, x1));
+    const float e0 = lane < n ? expf(x0 - m) : 0.f;
+    const float e1 = lane + 32 < n ? expf(x1 - m) : 0.f;
+    const float inv = 1.0f / warp_sum(e0 + e1);
+    if (lane < n) S[i * LDS + lane] = e0 * inv;
+    if (lane + 32 < n) S[i * LDS + lane + 32] = e1 * inv;
+  }
+  __syncthreads();
+#pragma unroll 1
+  for (int it = threadIdx.x; it < nq * 16; it += blockDim.x) {
+    const int i = it >> 4, d = 2 * (it & 15);
+    float a0 = 0.f, a1 = 0.f, c0 = 0.f, c1 = 0.f;
+    int k = 0;
+#pragma unroll 2
+    for (; k + 1 < n; k += 2) {
+      const float p0 = S[i * LDS + k], p1 = S[i * LDS + k + 1];
+      const float2 v0 = *reinterpret_cast<const float2*>(KV + k * LDKV + 32 + d);
+      const float2 v1 = *reinterpret_cast<const float2*>(KV + (k + 1) * LDKV + 32 + d);
+      a0 = fmaf(p0, v0.x, a0);
+      a1 = fmaf(p0, v0.y, a1);
+      c0 = fmaf(p1, v1.x, c0);
+      c1 = fmaf(p1, v1.y, c1);
+    }
+    if (k < n) {
+      const float p0 = S[i * LDS + k];
+      const float2 v0 = *reinterpret_cast<const float2*>(KV + k * LDKV + 32 + d);
+      a0 = fmaf(p0, v0.x, a0);
+      a1 = fmaf(p0, v0.y, a1);
+    }
+    uint32_t hi, lo;
+    split_bf16x2(a0 + c0, a1 + c1, hi, lo);
+    const int off = (qa + i) * LDH + 32 * hd + d;
+#pragma unroll 1
+    for (int r = 0; r < kDecideCluster; ++r) {
+      __nv_bfloat16* X = reinterpret_cast<__nv_bfloat16*>(cluster.map_shared_rank(P + P_XH, r));
+      *reinterpret_cast<uint32_t*>(X + off) = hi;
+      *reinterpret_cast<uint32_t*>(X + W * LDH + off) = lo;
+    }
+  }
+}
+
+// ------------------------------------------------------------------ LPS (rank 0)
+// One attention unit: 16 query rows [m0, m0+16) of head h (width 8) over the
+// n keys; qkv: [n][100] fp32 (q | k | v); the output goes to hi/lo columns
+// 8h..8h+7 of `out`.
+__device__ __forceinline__ void lps_attention_unit(const float* qkv, int n, int m0, int h,
+                                                   const HL& out) {
+  const int lane = threadIdx.x & 31, g = lane >> 2, t = lane & 3;
+  const int r_lo = m0 + g, r_hi = r_lo + 8;
+  uint32_t qh[4], ql[4];
+  {
+    float2 q0 = make_float2(0.f, 0.f), q1 = make_float2(0.f, 0.f);
+    if (r_lo < n) q0 = *reinterpret_cast<const float2*>(qkv + r_lo * 100 + 8 * h + 2 * t);
+    if (r_hi < n) q1 = *reinterpret_cast<const float2*>(qkv + r_hi * 100 + 8 * h + 2 * t);
+    split_bf16x2(q0.x, q0.y, qh[0], ql[0]);
+    split_bf16x2(q1.x, q1.y, qh[1], ql[1]);
+    qh[2] = qh[3] = ql[2] = ql[3] = 0u;  // head width 8: upper k half is zero
+  }
+  const int nkb = (n + 7) >> 3;
+  float s[8][4];
+  float mx0 = -INFINITY, mx1 = -INFINITY;
+#pragma unroll
+  for (int kb = 0; kb < 8; ++kb) {
+    s[kb][0] = s[kb][1] = s[kb][2] = s[kb][3] = -INFINITY;
+    if (kb < nkb) {
+      const int key = 8 * kb + g;
+      const float2 kk = key < n ? *reinterpret_cast<const float2*>(qkv + key * 100 + 32 + 8 * h + 2 * t)
+                                : make_float2(0.f, 0.f);
+      uint32_t bh, bl;
+      split_bf16x2(kk.x, kk.y, bh, bl);
+      float a[4] = {0.f, 0.f, 0.f, 0.f};
+      mma_bf16(a, qh, bh, 0u);
+      mma_bf16(a, qh, bl, 0u);
+      mma_bf16(a, ql, bh, 0u);
+      const int c = 8 * kb + 2 * t;
+      s[kb][0] = c < n ? a[0] * 0.35355339059327373f : -INFINITY;  // 1/sqrt(8)
+      s[kb][1] = c + 1 < n ? a[1] * 0.35355339059327373f : -INFINITY;
+      s[kb][2] = c < n ? a[2] * 0.35355339059327373f : -INFINITY;
+      s[kb][3] = c + 1 < n ? a[3] * 0.35355339059327373f : -INFINITY;
+      mx0 = fmaxf(mx0, fmaxf(s[kb][0], s[kb][1]));
+      mx1 = fmaxf(mx1, fmaxf(s[kb][2], s[kb][3]));
+    }
+  }
+  mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 1));
+  mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 2));
+  mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 1));
+  mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 2));
+  float l0 = 0.f, l1 = 0.f;
+#pragma unroll
+  for (int kb = 0; kb < 8; ++kb) {
+    s[kb][0] = expf(s[kb][0] - mx0);
+    s[kb][1] = expf(s[kb][1] - mx0);
+    s[kb][2] = expf(s[kb][2] - mx1);
+    s[kb][3] = expf(s[kb][3] - mx1);
+    l0 += s[kb][0] + s[kb][1];
+    l1 += s[kb][2] + s[kb][3];
+  }
+  l0 += __shfl_xor_sync(0xffffffffu, l0, 1);
+  l0 += __shfl_xor_sync(0xffffffffu, l0, 2);
+  l1 += __shfl_xor_sync(0xffffffffu, l1, 1);
+  l1 += __shfl_xor_sync(0xffffffffu, l1, 2);
+  float o[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    if (16 * j < n) {
+      uint32_t ph[4], pl[4];
+      split_bf16x2(s[2 * j][0], s[2 * j][1], ph[0], pl[0]);
+      split_bf16x2(s[2 * j][2], s[2 * j][3], ph[1], pl[1]);
+      split_bf16x2(s[2 * j + 1][0], s[2 * j + 1][1], ph[2], pl[2]);
+      split_bf16x2(s[2 * j + 1][2], s[2 * j + 1][3], ph[3], pl[3]);
+      float v[4];
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const int key = 16 * j + (e >> 1) * 8 + 2 * t + (e & 1);
+        v[e] = key < n ? qkv[key * 100 + 64 + 8 * h + g] : 0.f;
+      }
+      uint32_t b0h, b0l, b1h, b1l;
+      split_bf16x2(v[0], v[1], b0h, b0l);
+      split_bf16x2(v[2], v[3], b1h, b1l);
+      mma_bf16(o, ph, b0h, b1h);
+      mma_bf16(o, ph, b0l, b1l);
+      mma_bf16(o, pl, b0h, b1h);
+    }
+  }
+  const float i0 = 1.0f / l0, i1 = 1.0f / l1;
+  if (r_lo < n) hl_store2(out, r_lo, 8 * h + 2 * t, o[0] * i0, o[1] * i0);
+  if (r_hi < n) hl_store2(out, r_hi, 8 * h + 2 * t, o[2] * i1, o[3] * i1);
+}
+
+// LPS (Sec. 5.2 / App. D.1): Linear(5->32) -> LayerNorm -> GELU, two pre-norm
+// blocks (4 heads of width 8, FFN 64, GELU), head Linear(32->1), p = sigmoid.
+// Over the n (<= 64) masked rows of the block (features at P + L_FEAT);
+// p_psi of row i -> P[L_PROB + i].  Called by the whole CTA.
+__device__ __noinline__ void lps_forward(float* P, int n, const __nv_bfloat16* Wlps,
+                                         const float* V) {
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const float* feats = P + L_FEAT;
+  float* Z = P + L_Z;
+  float* QKV = P + L_QKV;
+  const HL Y = hl_at(P + L_YH, 40);
+  const HL At = hl_at(P + L_AH, 40);
+  const HL Hh = hl_at(P + L_HH, 72);
+  float* Yf = P + L_QKV;  // fp32 scratch for the input layer (before QKV is used)
+#pragma unroll 1
+  for (int it = tid; it < n * 32; it += blockDim.x) {  // Linear(5 -> 32)
+    const int r = it >> 5, c = it & 31;
+    float a = V[VP_INB + c];
+#pragma unroll
+    for (int k = 0; k < 5; ++k) a = fmaf(feats[r * 8 + k], V[VP_INT + k * 32 + c], a);
+    Yf[r * LDQ + c] = a;
+  }
+  __syncthreads();
+  ln_rows(Yf, LDQ, Z, LDQ, nullptr, 0, n, 32, V + VP_INLNG, V + VP_INLNB);
+  __syncthreads();
+#pragma unroll 1
+  for (int it = tid; it < n * 32; it += blockDim.x) Z[(it >> 5) * LDQ + (it & 31)] = gelu(Z[(it >> 5) * LDQ + (it & 31)]);
+  __syncthreads();
+#pragma unroll 1
+  for (int l = 0; l < 2; ++l) {
+    const __nv_bfloat16* Wl = Wlps + l * PL_STRIDE;
+    const float* Vl = V + VP_LAYER0 + l * VP_LAYER_STRIDE;
+    ln_rows(Z, LDQ, nullptr, 0, &Y, 0, n, 32, Vl + VPL_LN1G, Vl + VPL_LN1B);
     __syncthreads();
-    layer_norm_rows(zL, LD, yL, LD, n, 32, Vl + VPL_LN2G, Vl + VPL_LN2B);
+    gemm_hl(Y, n, 32, Wl + PL_QKV, PL_LDQKV, 96, [&](int j, int o, float a, float b) {
+      *reinterpret_cast<float2*>(QKV + j * 100 + o) = make_float2(a + Vl[VPL_QKVB + o], b + Vl[VPL_QKVB + o + 1]);
+    });
     __syncthreads();
-    gemm_rows(yL, LD, n, 32, Wl + PL_FF1, 64, 64, Vl + VPL_FF1B,
-              [&](int j, int o, float v) { h64[j * 68 + o] = gelu(v); });
+    const int mt = (n + 15) >> 4;
+#pragma unroll 1
+    for (int u = warp; u < 4 * mt; u += (blockDim.x >> 5)) lps_attention_unit(QKV, n, 16 * (u >> 2), u & 3, At);
     __syncthreads();
-    gemm_rows(h64, 68, n, 64, Wl + PL_FF2, 32, 32, Vl + VPL_FF2B,
-              [&](int j, int o, float v) { zL[j * LD + o] += v; });
+    gemm_hl(At, n, 32, Wl + PL_OUT, PL_LDOUT, 32, [&](int j, int o, float a, float b) {
+      float2* z = reinterpret_cast<float2*>(Z + j * LDQ + o);
+      const float2 zz = *z;
+      *z = make_float2(zz.x + (a + Vl[VPL_OUTB + o]), zz.y + (b + Vl[VPL_OUTB + o + 1]));
+    });
+    __syncthreads();
+    ln_rows(Z, LDQ, nullptr, 0, &Y, 0, n, 32, Vl + VPL_LN2G, Vl + VPL_LN2B);
+    __syncthreads();
+    gemm_hl(Y, n, 32, Wl + PL_FF1, PL_LDFF1, 64, [&](int j, int o, float a, float b) {
+      hl_store2(Hh, j, o, gelu(a + Vl[VPL_FF1B + o]), gelu(b + Vl[VPL_FF1B + o + 1]));
+    });
+    __syncthreads();
+    gemm_hl(Hh, n, 64, Wl + PL_FF2, PL_LDFF2, 32, [&](int j, int o, float a, float b) {
+      float2* z = reinterpret_cast<float2*>(Z + j * LDQ + o);
+      const float2 zz = *z;
+      *z = make_float2(zz.x + (a + Vl[VPL_FF2B + o]), zz.y + (b + Vl[VPL_FF2B + o + 1]));
+    });
     __syncthreads();
   }
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+#pragma unroll 1
   for (int i = warp; i < n; i += (blockDim.x >> 5)) {
-    const float a = warp_sum(zL[i * LD + lane] * V[VP_HEADW + lane]) + V[VP_HEADB];
-    if (lane == 0) sm.f_p[sm.BMrows[i]] = 1.0f / (1.0f + expf(-a));
+    const float a = warp_sum(Z[i * LDQ + lane] * V[VP_HEADW + lane]) + V[VP_HEADB];
+    if (lane == 0) P[L_PROB + i] = 1.0f / (1.0f + expf(-a));
   }
   __syncthreads();
 }
@@ -286,14 +455,26 @@ __global__ void __cluster_dims__(kDecideCluster, 1, 1) __launch_bounds__(kDecide
 
   if (tid == 0) {
     // weights and vectors of this rank: bulk copies issued first, so they
-    // land while the statistics are merged
+    // land while the statistics are merged.  With no active block the LBS
+    // weights are needed (every rank); otherwise only rank 0 needs the LPS
+    // weights, which then go straight into the weight region.
     mbar_init(&sm.bar, 1);
+    mbar_init(&sm.bar2, 1);
     fence_mbar_init();
-    const uint32_t wb = LBS_W_ELEMS * 2u, lb = LPS_W_ELEMS * 2u, vb = V_ELEMS * 4u;
-    mbar_arrive_expect_tx(&sm.bar, wb + vb + (rank == 0 ? lb : 0u));
-    bulk_copy(sm.w, p.w.lbs_w + static_cast<size_t>(rank) * LBS_W_ELEMS, wb, &sm.bar);
+    sm.meta_b = p.blk_meta[2 * seq];
+    sm.meta_s = p.blk_meta[2 * seq + 1];
+    const bool lbs_possible = sm.meta_s == 0;
+    const uint32_t wb = LBS_W_ELEMS * 2u, vb = V_ELEMS * 4u;
+    mbar_arrive_expect_tx(&sm.bar, vb + (lbs_possible ? wb : 0u));
     bulk_copy(sm.v, p.w.vec + static_cast<size_t>(rank) * V_ELEMS, vb, &sm.bar);
-    if (rank == 0) bulk_copy(sm.lw, p.w.lps_w, lb, &sm.bar);
+    if (lbs_possible)
+      bulk_copy(sm.w, p.w.lbs_w + static_cast<size_t>(rank) * LBS_W_ELEMS, wb, &sm.bar);
+    sm.lps_loaded = 0;
+    if (!lbs_possible && rank == 0 && p.lps_enabled) {
+      mbar_arrive_expect_tx(&sm.bar2, LPS_W_ELEMS * 2u);
+      bulk_copy(sm.w, p.w.lps_w, LPS_W_ELEMS * 2u, &sm.bar2);
+      sm.lps_loaded = 1;
+    }
     const int r0 = p.cu_rows[seq], r1 = p.cu_rows[seq + 1];
     const int n = r1 - r0;
     sm.bad_seq = 0;
@@ -303,15 +484,13 @@ __global__ void __cluster_dims__(kDecideCluster, 1, 1) __launch_bounds__(kDecide
     }
     sm.r0 = r0;
     sm.n_rows = sm.bad_seq ? 0 : n;
-    sm.meta_b = p.blk_meta[2 * seq];
-    sm.meta_s = p.blk_meta[2 * seq + 1];
-    sm.wait_fail = 0;
   }
   // every CTA of the cluster must be running before any distributed
   // shared-memory access; this also orders the block-level setup above
   cluster.sync();
   const int r0 = sm.r0, nr = sm.n_rows;
 
+#pragma unroll 1
   for (int j = tid; j < nr; j += blockDim.x) {
     sm.f_mask[j] = p.mask[r0 + j];
     sm.f_ib[j] = p.in_block[r0 + j];
@@ -324,6 +503,7 @@ __global__ void __cluster_dims__(kDecideCluster, 1, 1) __launch_bounds__(kDecide
 
   // ---------------------------------------------------------------- 1. statistics
   if (p.features_in) {
+#pragma unroll 1
     for (int j = tid; j < nr; j += blockDim.x) {
       const float c = p.conf[r0 + j], e = p.ent_norm[r0 + j], g = p.gap[r0 + j];
       const int a = p.argmax[r0 + j];
@@ -335,14 +515,22 @@ __global__ void __cluster_dims__(kDecideCluster, 1, 1) __launch_bounds__(kDecide
     }
   } else {
     // row j is merged by warp (j / 8) of rank (j % 8) and broadcast
+#pragma unroll 1
     for (int j = warp * kDecideCluster + rank; j < nr; j += kDecideCluster * (blockDim.x >> 5)) {
       const size_t base = static_cast<size_t>(r0 + j) * p.grid_lm;
       float m = -INFINITY, s = 0.f, t = 0.f, l2 = -INFINITY;
       int idx = INT_MAX;
-      for (int g = lane; g < p.grid_lm; g += 32) {
-        const float4 f = p.part_f[base + g];
-        merge_state(m, s, t, l2, idx, f.x, f.y, f.z, f.w, p.part_i[base + g]);
+      float4 fv[8];
+      int iv[8];
+#pragma unroll
+      for (int c = 0; c < 8; ++c) {  // independent loads first (partials per lane <= 8)
+        const int g = lane + 32 * c;
+        fv[c] = g < p.grid_lm ? p.part_f[base + g] : make_float4(-INFINITY, 0.f, 0.f, -INFINITY);
+        iv[c] = g < p.grid_lm ? p.part_i[base + g] : INT_MAX;
       }
+#pragma unroll
+      for (int c = 0; c < 8; ++c)
+        merge_state(m, s, t, l2, idx, fv[c].x, fv[c].y, fv[c].z, fv[c].w, iv[c]);
 #pragma unroll
       for (int off = 16; off > 0; off >>= 1) {
         const float bm = __shfl_xor_sync(0xffffffffu, m, off);
@@ -378,22 +566,25 @@ __global__ void __cluster_dims__(kDecideCluster, 1, 1) __launch_bounds__(kDecide
     }
   }
   // the weight copy must have landed before any use (and before exit)
-  {
-    const bool ok = mbar_wait(&sm.bar, 0, 1000ull * 1000 * 1000, nullptr);
-    if (!ok && tid == 0) {
-      sm.wait_fail = 1;
-      atomicCAS(p.status, 0, EBD_ERR_TIMEOUT);
-    }
-  }
+  if (!mbar_wait(&sm.bar, 0, 1000ull * 1000 * 1000, nullptr) && tid == 0)
+    atomicCAS(p.status, 0, EBD_ERR_TIMEOUT);
   cluster.sync();
 
   // ---------------------------------------------------------------- 2. masked set
-  if (tid == 0) {
-    int nM = 0;
-    for (int j = 0; j < nr; ++j)
-      if (sm.f_mask[j]) sm.Mrows[nM++] = j;
-    sm.nM = nM;
-    sm.run_lbs = (sm.meta_s == 0 && nM > p.l_min) ? 1 : 0;
+  if (warp == 0) {
+    int base = 0;
+#pragma unroll 1
+    for (int j0 = 0; j0 < nr; j0 += 32) {
+      const int j = j0 + lane;
+      const bool m = j < nr && sm.f_mask[j];
+      const uint32_t bal = __ballot_sync(0xffffffffu, m);
+      if (m) sm.Mrows[base + __popc(bal & ((1u << lane) - 1u))] = j;
+      base += __popc(bal);
+    }
+    if (lane == 0) {
+      sm.nM = base;
+      sm.run_lbs = (sm.meta_s == 0 && base > p.l_min) ? 1 : 0;
+    }
   }
   __syncthreads();
   const int nM = sm.nM;
@@ -402,110 +593,145 @@ __global__ void __cluster_dims__(kDecideCluster, 1, 1) __launch_bounds__(kDecide
   if (sm.run_lbs) {
     const int n = nM;
     float* Z = P + P_Z;
-    float* X = P + P_X;
+    const HL Zh = hl_at(P + P_ZH, LDH);
+    const HL Xh = hl_at(P + P_XH, LDH);
+    float* Xin = P + P_XH;  // fp32 FFN partial inbox [8][64][16] (aliases Xh)
+    const HL Fh = hl_at(P + P_KV, 72);  // F_ent hidden (hi/lo)
+    const HL Hh = hl_at(P + P_KV, 40);  // FFN hidden slice (hi/lo)
     float* KV = P + P_KV;
     float* Q = P + P_Q;
-    float* S = P + P_S;
     const float* Vv = sm.v;
     // 3a. entropy branch F_ent and token branch, every rank for all rows
-    for (int it = tid; it < n * 64; it += blockDim.x) {
-      const int j = it >> 6, o = it & 63;
+#pragma unroll 1
+    for (int it = tid; it < n * 32; it += blockDim.x) {
+      const int j = it >> 5, o = 2 * (it & 31);
       const int row = sm.Mrows[j];
-      KV[j * LDKV + o] = gelu(fmaf(Vv[V_ENT1W + o], sm.f_ent[row], Vv[V_ENT1B + o]));
+      const float h = sm.f_ent[row];
+      hl_store2(Fh, j, o, gelu(fmaf(Vv[V_ENT1W + o], h, Vv[V_ENT1B + o])),
+                gelu(fmaf(Vv[V_ENT1W + o + 1], h, Vv[V_ENT1B + o + 1])));
       const int tok = sm.f_arg[row];
-      const float tv =
-          (tok >= 0 && tok < p.V) ? p.w.tok_table[static_cast<size_t>(tok) * 64 + o] : 0.f;
-      X[j * LDZ + 64 + o] = tv + Vv[V_TOKB + o];
+      float2 tv = make_float2(0.f, 0.f);
+      if (tok >= 0 && tok < p.V)
+        tv = *reinterpret_cast<const float2*>(p.w.tok_table + static_cast<size_t>(tok) * 64 + o);
+      hl_store2(Xh, j, 64 + o, tv.x + Vv[V_TOKB + o], tv.y + Vv[V_TOKB + o + 1]);
     }
     __syncthreads();
-    gemm_rows(KV, LDKV, n, 64, sm.w + W_ENT2, 64, 64, Vv + V_ENT2B,
-              [&](int j, int o, float v) { X[j * LDZ + o] = v; });
+    // the ent2 output goes to the z hi/lo region: z itself receives the
+    // other ranks' fusion outputs as soon as they get there
+    float* E2 = P + P_ZH;
+    gemm_hl(Fh, n, 64, sm.w + W_ENT2, 64, 64, [&](int j, int o, float a, float b) {
+      *reinterpret_cast<float2*>(E2 + j * LDZ + o) = make_float2(a + Vv[V_ENT2B + o], b + Vv[V_ENT2B + o + 1]);
+    });
     __syncthreads();
-    layer_norm_rows(X, LDZ, X, LDZ, n, 64, Vv + V_ENTLNG, Vv + V_ENTLNB);
+    ln_rows(E2, LDZ, nullptr, 0, &Xh, 0, n, 64, Vv + V_ENTLNG, Vv + V_ENTLNB);
     __syncthreads();
     // 3b. fusion W_combine [e; t] + E_pos[rank of the row]: this CTA's 16 outputs
     {
       const int o0 = kCombSlice * rank;
-      gemm_rows(X, LDZ, n, 128, sm.w + W_COMB, kCombSlice, kCombSlice, Vv + V_COMBB,
-                [&](int j, int o, float v) {
-                  const float val = v + __bfloat162float(sm.w[W_POS + j * kCombSlice + o]);
-                  for (int rr = 0; rr < kDecideCluster; ++rr)
-                    cluster.map_shared_rank(Z, rr)[j * LDZ + o0 + o] = val;
-                });
+      gemm_hl(Xh, n, 128, sm.w + W_COMB, kCombSlice, kCombSlice, [&](int j, int o, float a, float b) {
+        const float2 pe = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(sm.w + W_POS + j * kCombSlice + o));
+        const float2 val = make_float2(a + Vv[V_COMBB + o] + pe.x, b + Vv[V_COMBB + o + 1] + pe.y);
+#pragma unroll 1
+        for (int r = 0; r < kDecideCluster; ++r)
+          *reinterpret_cast<float2*>(cluster.map_shared_rank(Z, r) + j * LDZ + o0 + o) = val;
+      });
     }
     cluster.sync();
+    // z as the first QKV input (hi/lo), every rank for all rows
+#pragma unroll 1
+    for (int it = tid; it < n * 64; it += blockDim.x) {
+      const int j = it >> 6, o = 2 * (it & 63);
+      hl_store2(Zh, j, o, Z[j * LDZ + o], Z[j * LDZ + o + 1]);
+    }
+    __syncthreads();
     // 3c. two post-norm encoder layers
     const int hd = rank >> 1, half = rank & 1;
     const int nh = (n + 1) >> 1;
     const int qa = half == 0 ? 0 : nh, qb = half == 0 ? nh : n;
+#pragma unroll 1
     for (int l = 0; l < 2; ++l) {
       const __nv_bfloat16* Wl = sm.w + W_LAYER0 + l * W_LAYER_STRIDE;
       const float* Vl = Vv + V_LAYER0 + l * V_LAYER_STRIDE;
       // QKV: this CTA's 48 features for every row, scattered to the CTAs
       // that attend with them (head h lives in ranks 2h and 2h+1)
-      gemm_rows(Z, LDZ, n, 128, Wl + WL_QKV, kQkvSlice, kQkvSlice, Vl + VL_QKVB,
-                [&](int j, int o, float v) {
-                  const int f = kQkvSlice * rank + o;
-                  const int part = f >> 7, h = (f >> 5) & 3, dd = f & 31;
-                  if (part == 0) {
-                    const int dst = 2 * h + (j >= nh ? 1 : 0);
-                    const int jj = j >= nh ? j - nh : j;
-                    cluster.map_shared_rank(P, dst)[P_Q + jj * LDQ + dd] = v;
-                  } else {
-                    const int col = (part == 1 ? 0 : 32) + dd;
-                    cluster.map_shared_rank(P, 2 * h)[P_KV + j * LDKV + col] = v;
-                    cluster.map_shared_rank(P, 2 * h + 1)[P_KV + j * LDKV + col] = v;
-                  }
-                });
-      cluster.sync();
-      attend(Q, LDQ, KV, KV + 32, LDKV, qb - qa, n, 32, S, [&](int i, int d, float v) {
-        for (int rr = 0; rr < kDecideCluster; ++rr)
-          cluster.map_shared_rank(X, rr)[(qa + i) * LDZ + 32 * hd + d] = v;
+      gemm_hl(Zh, n, 128, Wl + WL_QKV, kQkvSlice, kQkvSlice, [&](int j, int o, float a, float b) {
+        const int f = kQkvSlice * rank + o;  // even; f and f+1 share part and head
+        const int part = f >> 7, h = (f >> 5) & 3, dd = f & 31;
+        const float2 val = make_float2(a + Vl[VL_QKVB + o], b + Vl[VL_QKVB + o + 1]);
+        if (part == 0) {
+          const int dst = 2 * h + (j >= nh ? 1 : 0);
+          const int jj = j >= nh ? j - nh : j;
+          *reinterpret_cast<float2*>(cluster.map_shared_rank(Q, dst) + jj * LDQ + dd) = val;
+        } else {
+          const int col = (part == 1 ? 0 : 32) + dd;
+          *reinterpret_cast<float2*>(cluster.map_shared_rank(KV, 2 * h) + j * LDKV + col) = val;
+          *reinterpret_cast<float2*>(cluster.map_shared_rank(KV, 2 * h + 1) + j * LDKV + col) = val;
+        }
       });
+      cluster.sync();
+      lbs_attention(cluster, P, qb - qa, n, qa, hd);
       cluster.sync();
       {  // output projection + residual, 16 outputs, written in place into z
         const int o0 = kOutSlice * rank;
-        gemm_rows(X, LDZ, n, 128, Wl + WL_OUT, kOutSlice, kOutSlice, Vl + VL_OUTB,
-                  [&](int j, int o, float v) {
-                    const float val = v + Z[j * LDZ + o0 + o];
-                    for (int rr = 0; rr < kDecideCluster; ++rr)
-                      cluster.map_shared_rank(Z, rr)[j * LDZ + o0 + o] = val;
-                  });
+        gemm_hl(Xh, n, 128, Wl + WL_OUT, kOutSlice, kOutSlice, [&](int j, int o, float a, float b) {
+          const float2 zz = *reinterpret_cast<const float2*>(Z + j * LDZ + o0 + o);
+          const float2 val = make_float2(zz.x + (a + Vl[VL_OUTB + o]), zz.y + (b + Vl[VL_OUTB + o + 1]));
+#pragma unroll 1
+          for (int r = 0; r < kDecideCluster; ++r)
+            *reinterpret_cast<float2*>(cluster.map_shared_rank(Z, r) + j * LDZ + o0 + o) = val;
+        });
       }
       cluster.sync();
-      layer_norm_rows(Z, LDZ, Z, LDZ, n, 128, Vl + VL_LN1G, Vl + VL_LN1B);
+      ln_rows(Z, LDZ, Z, LDZ, &Zh, 0, n, 128, Vl + VL_LN1G, Vl + VL_LN1B);
       __syncthreads();
       // FFN: hidden units [32r, 32r+32) locally, then the partial second
       // linear of those units sent to the owners of each 16-output slice
-      float* Hh = KV;  // [n][36]
-      gemm_rows(Z, LDZ, n, 128, Wl + WL_FF1, kFf1Slice, kFf1Slice, Vl + VL_FF1B,
-                [&](int j, int o, float v) { Hh[j * LDQ + o] = gelu(v); });
+      gemm_hl(Zh, n, 128, Wl + WL_FF1, kFf1Slice, kFf1Slice, [&](int j, int o, float a, float b) {
+        hl_store2(Hh, j, o, gelu(a + Vl[VL_FF1B + o]), gelu(b + Vl[VL_FF1B + o + 1]));
+      });
       __syncthreads();
-      gemm_rows(Hh, LDQ, n, kFf1Slice, Wl + WL_FF2, 128, 128, nullptr,
-                [&](int j, int o, float v) {
-                  const int owner = o >> 4;
-                  cluster.map_shared_rank(X, owner)[(rank * W + j) * 16 + (o & 15)] = v;
-                });
+      gemm_hl(Hh, n, kFf1Slice, Wl + WL_FF2, 128, 128, [&](int j, int o, float a, float b) {
+        *reinterpret_cast<float2*>(cluster.map_shared_rank(Xin, o >> 4) + (rank * W + j) * 16 + (o & 15)) =
+            make_float2(a, b);
+      });
       cluster.sync();
       {  // owner: sum the 8 partials + bias + residual, broadcast its slice
         const int o0 = kOutSlice * rank;
-        for (int it = tid; it < n * 16; it += blockDim.x) {
-          const int j = it >> 4, oo = it & 15;
-          float a = Vl[VL_FF2B + oo] + Z[j * LDZ + o0 + oo];
+#pragma unroll 1
+        for (int it = tid; it < n * 8; it += blockDim.x) {
+          const int j = it >> 3, oo = 2 * (it & 7);
+          float2 a = *reinterpret_cast<const float2*>(Z + j * LDZ + o0 + oo);
+          a.x += Vl[VL_FF2B + oo];
+          a.y += Vl[VL_FF2B + oo + 1];
 #pragma unroll
-          for (int src = 0; src < kDecideCluster; ++src) a += X[(src * W + j) * 16 + oo];
+          for (int src = 0; src < kDecideCluster; ++src) {
+            const float2 q = *reinterpret_cast<const float2*>(Xin + (src * W + j) * 16 + oo);
+            a.x += q.x;
+            a.y += q.y;
+          }
+#pragma unroll 1
           for (int rr = 0; rr < kDecideCluster; ++rr)
-            cluster.map_shared_rank(Z, rr)[j * LDZ + o0 + oo] = a;
+            *reinterpret_cast<float2*>(cluster.map_shared_rank(Z, rr) + j * LDZ + o0 + oo) = a;
         }
       }
       cluster.sync();
-      layer_norm_rows(Z, LDZ, Z, LDZ, n, 128, Vl + VL_LN2G, Vl + VL_LN2B);
+      ln_rows(Z, LDZ, Z, LDZ, &Zh, 0, n, 128, Vl + VL_LN2G, Vl + VL_LN2B);
       __syncthreads();
+      if (l == 0 && rank == 0 && tid == 0 && p.lps_enabled) {
+        // the first layer's weights (and everything before them) are dead:
+        // fetch the LPS weights into that region behind the second layer
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+        mbar_arrive_expect_tx(&sm.bar2, LPS_W_ELEMS * 2u);
+        bulk_copy(sm.w, p.w.lps_w, LPS_W_ELEMS * 2u, &sm.bar2);
+        sm.lps_loaded = 1;
+      }
     }
     // 3d. head Linear(128 -> 1), needed by rank 0
     if (rank == 0) {
+#pragma unroll 1
       for (int j = warp; j < n; j += (blockDim.x >> 5)) {
         float a = 0.f;
+#pragma unroll
         for (int c = 0; c < 4; ++c) a += Z[j * LDZ + lane + 32 * c] * Vv[V_HEADW + lane + 32 * c];
         a = warp_sum(a) + Vv[V_HEADB];
         if (lane == 0) sm.f_O[sm.Mrows[j]] = a;
@@ -516,85 +742,154 @@ __global__ void __cluster_dims__(kDecideCluster, 1, 1) __launch_bounds__(kDecide
   if (rank != 0) return;  // no distributed shared-memory access after this point
 
   // ---------------------------------------------------------------- 4. block selection
-  if (tid == 0) {
+  if (tid == 0 && !sm.lps_loaded && p.lps_enabled) {
+    // no LBS ran: the weight region is free now
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    mbar_arrive_expect_tx(&sm.bar2, LPS_W_ELEMS * 2u);
+    bulk_copy(sm.w, p.w.lps_w, LPS_W_ELEMS * 2u, &sm.bar2);
+    sm.lps_loaded = 1;
+  }
+  if (warp == 0) {
     if (sm.meta_s == 0) {
-      for (int j = 0; j < nr; ++j) sm.f_ib[j] = 0;
+      for (int j = lane; j < nr; j += 32) sm.f_ib[j] = 0;
+      __syncwarp();
       int nB = 0;
       if (nM <= p.l_min) {
-        for (int k = 0; k < nM; ++k) sm.Brows[nB++] = sm.Mrows[k];
+        for (int k = lane; k < nM; k += 32) sm.Brows[k] = sm.Mrows[k];
+        nB = nM;
       } else {
-        int last = 0;
-        for (int k = 0; k < nM; ++k) {
-          const int j = sm.Mrows[k];
-          const bool cand = sm.f_O[j] > 0.f && sm.f_arg[j] != p.eos_id && !sm.f_bad[j];
-          if (!cand) continue;
-          if (nB > 0 && sm.f_pos[j] - last > p.g_max) break;  // MaxGapFilter
-          sm.Brows[nB++] = j;
-          last = sm.f_pos[j];
+        // candidates (router O > 0, not EOS) compacted in ascending position
+        int nC = 0;
+        for (int k0 = 0; k0 < nM; k0 += 32) {
+          const int k = k0 + lane;
+          int j = -1;
+          bool c = false;
+          if (k < nM) {
+            j = sm.Mrows[k];
+            c = sm.f_O[j] > 0.f && sm.f_arg[j] != p.eos_id && !sm.f_bad[j];
+          }
+          const uint32_t bal = __ballot_sync(0xffffffffu, c);
+          if (c) sm.Brows[nC + __popc(bal & ((1u << lane) - 1u))] = j;
+          nC += __popc(bal);
         }
-        if (nB < p.l_min) {  // min-tokens fallback
-          nB = 0;
-          const int take = nM < p.l_b ? nM : p.l_b;
-          for (int k = 0; k < take; ++k) sm.Brows[nB++] = sm.Mrows[k];
+        __syncwarp();
+        // MaxGapFilter: cut at the first candidate farther than g_max from its predecessor
+        int cut = nC;
+        for (int c0 = 1; c0 < nC; c0 += 32) {
+          const int c = c0 + lane;
+          const bool gap = c < nC && sm.f_pos[sm.Brows[c]] - sm.f_pos[sm.Brows[c - 1]] > p.g_max;
+          const uint32_t bal = __ballot_sync(0xffffffffu, gap);
+          if (bal) {
+            cut = c0 + __ffs(bal) - 1;
+            break;
+          }
+        }
+        nB = cut;
+        if (nB < p.l_min) {  // min-tokens fallback: first min(L_B, |M|) masked rows
+          nB = nM < p.l_b ? nM : p.l_b;
+          __syncwarp();
+          for (int k = lane; k < nB; k += 32) sm.Brows[k] = sm.Mrows[k];
         }
       }
-      if (nB > 0) {
-        for (int k = 0; k < nB; ++k) sm.f_ib[sm.Brows[k]] = 1;
+      __syncwarp();
+      for (int k = lane; k < nB; k += 32) sm.f_ib[sm.Brows[k]] = 1;
+      if (lane == 0 && nB > 0) {
         sm.meta_b = sm.f_pos[sm.Brows[0]];
         sm.meta_s = nB;
       }
+      __syncwarp();
     }
-    int nBM = 0;
-    for (int j = 0; j < nr; ++j)
-      if (sm.f_ib[j] && sm.f_mask[j] && !sm.f_bad[j]) sm.BMrows[nBM++] = j;
-    sm.nBM = nBM;
+    int base = 0;
+    for (int j0 = 0; j0 < nr; j0 += 32) {
+      const int j = j0 + lane;
+      const bool m = j < nr && sm.f_ib[j] && sm.f_mask[j] && !sm.f_bad[j];
+      const uint32_t bal = __ballot_sync(0xffffffffu, m);
+      if (m) sm.BMrows[base + __popc(bal & ((1u << lane) - 1u))] = j;
+      base += __popc(bal);
+    }
+    if (lane == 0) sm.nBM = base;
   }
   __syncthreads();
 
   // ---------------------------------------------------------------- 5. LPS + accept + commit
+  // the LPS weight copy must have landed before use and before exit
+  if (sm.lps_loaded && !mbar_wait(&sm.bar2, 0, 1000ull * 1000 * 1000, nullptr))
+    atomicCAS(p.status, 0, EBD_ERR_TIMEOUT);
   const int nBM = sm.nBM;
-  if (nBM > 0) {
-    if (p.lps_enabled) lps_forward(sm, nBM);
-    if (tid == 0) {
-      int nacc = 0;
-      for (int i = 0; i < nBM; ++i) {
+  if (nBM > 0 && p.lps_enabled) {
+    float* feats = P + L_FEAT;
+    const float rho = static_cast<float>(nBM) / static_cast<float>(sm.meta_s);
+#pragma unroll 1
+    for (int i = tid; i < nBM; i += blockDim.x) {
+      const int r = sm.BMrows[i];
+      feats[i * 8 + 0] = sm.f_conf[r];
+      feats[i * 8 + 1] = sm.f_ent[r];
+      feats[i * 8 + 2] = sm.f_gap[r];
+      feats[i * 8 + 3] = rho;
+      feats[i * 8 + 4] = static_cast<float>(sm.f_pos[r] - sm.meta_b) / static_cast<float>(sm.meta_s);
+    }
+    __syncthreads();
+    const float* prob = P + L_PROB;
+    lps_forward(P, nBM, sm.w, sm.v + V_LPS);
+#pragma unroll 1
+    for (int i = tid; i < nBM; i += blockDim.x) sm.f_p[sm.BMrows[i]] = prob[i];
+    __syncthreads();
+  }
+  if (warp == 0) {
+    // union accept rule, anti-stall fallback, parallel commit, resolution
+    bool any = false;
+    for (int i0 = 0; i0 < nBM; i0 += 32) {
+      const int i = i0 + lane;
+      bool a = false;
+      if (i < nBM) {
         const int j = sm.BMrows[i];
-        const bool a = sm.f_conf[j] >= p.tau || (p.lps_enabled && sm.f_p[j] > p.tau_psi);
-        if (a) {
-          sm.f_acc[j] = 1;
-          ++nacc;
+        a = sm.f_conf[j] >= p.tau || (p.lps_enabled && sm.f_p[j] > p.tau_psi);
+        if (a) sm.f_acc[j] = 1;
+      }
+      any |= __ballot_sync(0xffffffffu, a) != 0;
+    }
+    if (!any && nBM > 0) {
+      // highest confidence; the lowest position among equal confidences
+      float best = -INFINITY;
+      int bj = INT_MAX;
+      for (int i = lane; i < nBM; i += 32) {
+        const int j = sm.BMrows[i];
+        const float c = sm.f_conf[j];
+        if (c > best || (c == best && j < bj)) {
+          best = c;
+          bj = j;
         }
       }
-      if (nacc == 0) {  // anti-stall: highest confidence, lowest position on ties
-        int best = sm.BMrows[0];
-        for (int i = 1; i < nBM; ++i) {
-          const int j = sm.BMrows[i];
-          if (sm.f_conf[j] > sm.f_conf[best]) best = j;
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) {
+        const float ob = __shfl_xor_sync(0xffffffffu, best, off);
+        const int oj = __shfl_xor_sync(0xffffffffu, bj, off);
+        if (ob > best || (ob == best && oj < bj)) {
+          best = ob;
+          bj = oj;
         }
-        sm.f_acc[best] = 1;
       }
-      bool open = false;
-      for (int j = 0; j < nr; ++j) {
+      if (lane == 0) sm.f_acc[bj] = 1;
+    }
+    __syncwarp();
+    bool open = false;
+    for (int j0 = 0; j0 < nr; j0 += 32) {
+      const int j = j0 + lane;
+      if (j < nr) {
         if (sm.f_acc[j]) {
           sm.f_tok[j] = sm.f_arg[j];
           sm.f_mask[j] = 0;
         }
-        if (sm.f_ib[j] && sm.f_mask[j]) open = true;
+        open |= sm.f_ib[j] && sm.f_mask[j];
       }
-      if (sm.meta_s > 0 && !open) {
-        for (int j = 0; j < nr; ++j) sm.f_ib[j] = 0;
+    }
+    open = __ballot_sync(0xffffffffu, open) != 0;
+    if (sm.meta_s > 0 && !open) {
+      for (int j = lane; j < nr; j += 32) sm.f_ib[j] = 0;
+      if (lane == 0) {
         sm.meta_b = 0;
         sm.meta_s = 0;
       }
-    }
-  } else if (tid == 0 && sm.meta_s > 0) {
-    bool open = false;
-    for (int j = 0; j < nr; ++j)
-      if (sm.f_ib[j] && sm.f_mask[j]) open = true;
-    if (!open) {
-      for (int j = 0; j < nr; ++j) sm.f_ib[j] = 0;
-      sm.meta_b = 0;
-      sm.meta_s = 0;
     }
   }
   __syncthreads();

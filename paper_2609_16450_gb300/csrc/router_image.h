@@ -26,12 +26,15 @@ constexpr int WL_FF1 = 8192;      // [128][32]  FFN first linear, hidden slice
 constexpr int WL_FF2 = 12288;     // [32][128]  FFN second linear, rows of the hidden slice
 constexpr int LBS_W_ELEMS = W_LAYER0 + 2 * W_LAYER_STRIDE;  // 39936
 
-// ---- LPS weights (one copy), bf16 elements, per layer
-constexpr int PL_QKV = 0;         // [32][96]
-constexpr int PL_OUT = 3072;      // [32][32]
-constexpr int PL_FF1 = 4096;      // [32][64]
-constexpr int PL_FF2 = 6144;      // [64][32]
-constexpr int PL_STRIDE = 8192;
+// ---- LPS weights (one copy), bf16, transposed [in][out] with each row padded
+// by 8 elements so that 8 consecutive rows hit distinct banks when ldmatrix
+// reads them as mma B fragments
+constexpr int PL_QKV = 0;         // [32][104]
+constexpr int PL_OUT = 3328;      // [32][40]
+constexpr int PL_FF1 = 4608;      // [32][72]
+constexpr int PL_FF2 = 6912;      // [64][40]
+constexpr int PL_STRIDE = 9472;
+constexpr int PL_LDQKV = 104, PL_LDOUT = 40, PL_LDFF1 = 72, PL_LDFF2 = 40;
 constexpr int LPS_W_ELEMS = 2 * PL_STRIDE;
 
 // ---- fp32 vectors of one rank
@@ -49,6 +52,7 @@ constexpr int V_ELEMS = 2800;
 
 static_assert(V_LAYER0 + 2 * V_LAYER_STRIDE <= V_LPS, "vector layout");
 static_assert(V_LPS + VP_LAYER0 + 2 * VP_LAYER_STRIDE <= V_ELEMS, "vector layout");
+static_assert(LPS_W_ELEMS <= LBS_W_ELEMS, "LPS weights reuse the LBS weight region");
 static_assert((LBS_W_ELEMS * 2) % 16 == 0 && (LPS_W_ELEMS * 2) % 16 == 0 &&
                   (V_ELEMS * 4) % 16 == 0,
               "bulk copies move multiples of 16 bytes");
