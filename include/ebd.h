@@ -236,6 +236,42 @@ const char* ebd_last_error(const ebd_handle* h);
 /* Library version string. */
 const char* ebd_version(void);
 
+/* ---- Allocation-free LM-head statistics ---------------------------------
+ * No counterpart in the paper.  ebd_lm_stats_noalloc computes what
+ * ebd_lm_stats computes (step 2: conf, entropy, ent_norm, gap, argmax of
+ * `rows` rows of `hidden`, any output may be NULL), but takes no handle and
+ * allocates no device memory, for callers that cannot allocate: a serving
+ * process whose weight and KV-cache pools reserved the free HBM up front
+ * (a further cudaMalloc fails or fragments them), or a decode loop that must
+ * not stall on the device-wide synchronisation of cudaFree.
+ *
+ *   hidden   device, bf16 [rows][d_model], 16-byte aligned
+ *   w_lm     device, bf16, 16-byte aligned: [vocab][d_model] row-major
+ *            (w_lm_layout 0) or the tiled copy of ebd_pack_lm_head (1)
+ *   rows     0 .. EBD_NOALLOC_MAX_ROWS; more returns EBD_ERR_UNSUPPORTED
+ *   status   device int32 owned by the caller; it must be 0 before the
+ *            call, and the kernels store the first device-side failure there
+ *            (EBD_ERR_TIMEOUT, EBD_ERR_NONFINITE), as ebd_sync_status reports
+ *            it for a handle
+ *   stream   cudaStream_t as void*; the call only enqueues
+ *
+ * Scratch: the LM-head partials live in a statically sized device array of
+ * EBD_NOALLOC_MAX_ROWS x EBD_NOALLOC_MAX_PARTS x 20 bytes (200 KiB), one per
+ * device; nothing in it has to start at zero.  Calls that overlap in time on
+ * one device (different streams or host threads) race on that array; calls
+ * on one stream are ordered and safe.  The first call on each device does a
+ * one-time setup (symbol address, kernel attributes) on the current device:
+ * make that first call before any stream capture begins.
+ * Returns EBD_ERR_INVALID_ARG for a null or misaligned pointer, a bad layout
+ * or a size below its range, EBD_ERR_UNSUPPORTED beyond the maximum or on a
+ * device other than sm_103, EBD_ERR_CUDA if a launch fails. */
+#define EBD_NOALLOC_MAX_ROWS 64
+#define EBD_NOALLOC_MAX_PARTS 160
+ebd_status ebd_lm_stats_noalloc(const uint16_t* hidden, const uint16_t* w_lm,
+                                int32_t w_lm_layout, int32_t rows, int32_t d_model,
+                                int32_t vocab, float* conf, float* entropy, float* ent_norm,
+                                float* gap, int32_t* argmax, int32_t* status, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -53,7 +53,7 @@ EXPORTS = ["ebd_create", "ebd_destroy", "ebd_bind_embedding", "ebd_step", "ebd_s
            "ebd_export_weights", "ebd_import_weights", "ebd_router_init_host",
            "ebd_weight_count", "ebd_lm_head_packed_bytes", "ebd_pack_lm_head",
            "ebd_profile_enable", "ebd_profile_read", "ebd_last_error",
-           "ebd_version"]
+           "ebd_version", "ebd_lm_stats_noalloc"]
 
 _lib = None
 
@@ -93,6 +93,10 @@ def load(path: str = LIB_PATH):
     lib.ebd_profile_enable.argtypes = [c_void_p, c_int32]
     lib.ebd_profile_read.argtypes = [c_void_p, P(c_float)]
     lib.ebd_version.argtypes = []
+    lib.ebd_lm_stats_noalloc.argtypes = [c_void_p, c_void_p, c_int32, c_int32, c_int32, c_int32,
+                                         c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
+                                         c_void_p, c_void_p]
+    lib.ebd_lm_stats_noalloc.restype = c_int32
     lib.ebd_version.restype = c_char_p
     for fn in EXPORTS:
         if getattr(lib, fn).restype is ctypes.c_int:
@@ -206,3 +210,19 @@ def ebd_last_error(h) -> str:
 
 def ebd_version() -> str:
     return load().ebd_version().decode()
+
+
+EBD_NOALLOC_MAX_ROWS = 64
+EBD_NOALLOC_MAX_PARTS = 160
+
+
+def ebd_lm_stats_noalloc(hidden_ptr: int, w_lm_ptr: int, w_lm_layout: int, rows: int,
+                         d_model: int, vocab: int, conf_ptr: int, entropy_ptr: int,
+                         ent_norm_ptr: int, gap_ptr: int, argmax_ptr: int, status_ptr: int,
+                         stream: int = 0) -> int:
+    """Allocation-free LM-head statistics; pointers are device addresses
+    (0 for an output that is not wanted)."""
+    return load().ebd_lm_stats_noalloc(hidden_ptr, w_lm_ptr, w_lm_layout, rows, d_model, vocab,
+                                       conf_ptr or None, entropy_ptr or None, ent_norm_ptr or None,
+                                       gap_ptr or None, argmax_ptr or None, status_ptr or None,
+                                       stream or None)

@@ -4,6 +4,7 @@
 #include <cmath>
 #include <cstdio>
 #include <cstring>
+#include <mutex>
 #include <string>
 #include <vector>
 
@@ -951,3 +952,121 @@ ebd_status ebd_sync_status(ebd_handle* h, void* stream) {
 }
 
 }  // extern "C"
+
+// ---------------------------------------------------------------------------
+// Allocation-free LM-head statistics (ebd_lm_stats_noalloc).
+//
+// The paper has no counterpart: this serves callers that must not allocate
+// device memory when they ask for the statistics of step 2.  Two kinds:
+//   - a serving process whose weight and KV-cache pools reserved the free HBM
+//     up front, where any further cudaMalloc fails or fragments the pool;
+//   - a decode loop that must not stall, where cudaFree (and cudaMalloc on
+//     some paths) synchronises the whole device.
+// The handle path allocates its workspace in ebd_create; this path needs no
+// handle: the LM-head partials live in the file-scope array below, sized for
+// EBD_NOALLOC_MAX_ROWS rows x EBD_NOALLOC_MAX_PARTS partials per row
+// (64 x 160 x 20 bytes = 200 KiB).  Nothing in it has to start at zero: every
+// LM-head CTA writes its partial of every row before the merge reads it.
+// There is one copy per device, so calls that overlap in time on one device
+// (two streams, or two host threads) race on it; calls on one stream are
+// ordered and safe.
+// ---------------------------------------------------------------------------
+static __device__ __align__(256) unsigned char
+    g_noalloc_scratch[static_cast<size_t>(EBD_NOALLOC_MAX_ROWS) * EBD_NOALLOC_MAX_PARTS *
+                      (sizeof(float4) + sizeof(int))];
+
+namespace {
+
+constexpr int kNoAllocMaxDevices = 64;
+struct NoAllocDevice {
+  bool ready = false;
+  int num_sms = 0;
+  float4* part_f = nullptr;  // [rows][grid], grid <= EBD_NOALLOC_MAX_PARTS
+  int* part_i = nullptr;     // [rows][grid]
+};
+NoAllocDevice g_noalloc_dev[kNoAllocMaxDevices];
+std::mutex g_noalloc_mu;
+
+// One-time setup of device `dev` (the current device): the scratch address
+// (cudaGetSymbolAddress), the LM-head kernel attributes and the SM count.
+// Allocates nothing.
+ebd_status noalloc_setup(int dev, NoAllocDevice** out) {
+  std::lock_guard<std::mutex> lock(g_noalloc_mu);
+  NoAllocDevice& d = g_noalloc_dev[dev];
+  if (!d.ready) {
+    int major = 0, minor = 0, sms = 0;
+    if (cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+      return EBD_ERR_CUDA;
+    if (major != 10 || minor != 3) return EBD_ERR_UNSUPPORTED;
+    void* base = nullptr;
+    if (cudaGetSymbolAddress(&base, g_noalloc_scratch) != cudaSuccess) return EBD_ERR_CUDA;
+    if (lm_configure() != cudaSuccess) return EBD_ERR_CUDA;
+    d.num_sms = sms;
+    d.part_f = static_cast<float4*>(base);
+    d.part_i = reinterpret_cast<int*>(static_cast<unsigned char*>(base) +
+                                      static_cast<size_t>(EBD_NOALLOC_MAX_ROWS) *
+                                          EBD_NOALLOC_MAX_PARTS * sizeof(float4));
+    d.ready = true;
+  }
+  *out = &d;
+  return EBD_OK;
+}
+
+}  // namespace
+
+extern "C" ebd_status ebd_lm_stats_noalloc(const uint16_t* hidden, const uint16_t* w_lm,
+                                           int32_t w_lm_layout, int32_t rows, int32_t d_model,
+                                           int32_t vocab, float* conf, float* entropy,
+                                           float* ent_norm, float* gap, int32_t* argmax,
+                                           int32_t* status, void* stream) {
+  if (rows < 0 || d_model <= 0 || d_model % 8 || vocab < 2 || (w_lm_layout != 0 && w_lm_layout != 1))
+    return EBD_ERR_INVALID_ARG;
+  if (rows > EBD_NOALLOC_MAX_ROWS) return EBD_ERR_UNSUPPORTED;
+  if (rows == 0) return EBD_OK;
+  if (hidden == nullptr || w_lm == nullptr || status == nullptr ||
+      reinterpret_cast<uintptr_t>(hidden) % 16 || reinterpret_cast<uintptr_t>(w_lm) % 16)
+    return EBD_ERR_INVALID_ARG;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return EBD_ERR_CUDA;
+  if (dev < 0 || dev >= kNoAllocMaxDevices) return EBD_ERR_UNSUPPORTED;
+  NoAllocDevice* nd = nullptr;
+  ebd_status s = noalloc_setup(dev, &nd);
+  if (s != EBD_OK) return s;
+  const bool packed = w_lm_layout == 1;
+  const uint64_t units = (static_cast<uint64_t>(vocab) + kUnit - 1) / kUnit;
+  const uint64_t nkb = (static_cast<uint64_t>(d_model) + 63) / 64;
+  CUtensorMap tw, th;
+  {
+    const uint64_t dims[2] = {packed ? 64ull : static_cast<uint64_t>(d_model),
+                              packed ? units * nkb * 64 : static_cast<uint64_t>(vocab)};
+    const uint64_t str[1] = {packed ? 128ull : static_cast<uint64_t>(d_model) * 2};
+    const uint32_t box[2] = {64, 64};
+    if (!encode_bf16(&tw, w_lm, 2, dims, str, box)) return EBD_ERR_CUDA;
+  }
+  LmParams p{};
+  lm_plan(p, rows, vocab, d_model,
+          nd->num_sms < EBD_NOALLOC_MAX_PARTS ? nd->num_sms : EBD_NOALLOC_MAX_PARTS);
+  if (p.stages < 2 || p.grid > EBD_NOALLOC_MAX_PARTS) return EBD_ERR_UNSUPPORTED;
+  p.row0 = 0;
+  p.packed = packed ? 1 : 0;
+  p.part_f = nd->part_f;
+  p.part_i = nd->part_i;
+  p.status = status;
+  p.limit_ns = kLimitNs;
+  p.force_timeout = 0;
+  {
+    const uint64_t dims[2] = {static_cast<uint64_t>(d_model), static_cast<uint64_t>(rows)};
+    const uint64_t str[1] = {static_cast<uint64_t>(d_model) * 2};
+    const uint32_t box[2] = {64, static_cast<uint32_t>(p.nb)};
+    if (!encode_bf16(&th, hidden, 2, dims, str, box)) return EBD_ERR_CUDA;
+  }
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  if (launch_lm_stats(tw, th, p, st) != cudaSuccess) return EBD_ERR_CUDA;
+  const float inv = static_cast<float>(1.0 / std::log(static_cast<double>(vocab)));
+  if (launch_merge_stats(nd->part_f, nd->part_i, rows, p.grid, vocab, inv, conf, entropy, ent_norm,
+                         gap, argmax, status, st) != cudaSuccess)
+    return EBD_ERR_CUDA;
+  return EBD_OK;
+}
