@@ -162,7 +162,10 @@ size_t ebd_lm_head_packed_bytes(const ebd_config* cfg);
 ebd_status ebd_pack_lm_head(ebd_handle* h, const uint16_t* w_lm, uint16_t* w_packed,
                             void* stream);
 
-/* One EB decoding step (see top of file).  Enqueue only. */
+/* One EB decoding step (see top of file).  Enqueue only.  The kernels run
+ * on `stream` in the order LM head, decision, window attention; the
+ * attention (needed by neither of the others) may start while the decision
+ * runs.  Later work on `stream` waits for all three. */
 ebd_status ebd_step(ebd_handle* h, const ebd_step_args* a, void* stream);
 
 /* Same step with the per-step tensors in HOST memory (pinned memory gives
@@ -222,12 +225,16 @@ ebd_status ebd_router_init_host(const ebd_config* cfg, void* host, size_t* bytes
 /* Number of bf16 elements of the weight blob for cfg. */
 size_t ebd_weight_count(const ebd_config* cfg);
 
-/* Per-kernel timing of ebd_step: with on != 0 every later ebd_step records
- * CUDA events on its stream before the first kernel and after the window
- * attention, the LM head and the decision (also inside a captured graph).
- * ebd_profile_read waits for the last recorded event and writes the three
- * durations in milliseconds to ms[0..2] (attention, LM head, decision). */
-ebd_status ebd_profile_enable(ebd_handle* h, int on);
+/* Timing of ebd_step.  mode 0: off.  mode 1: every later ebd_step records
+ * CUDA events on its stream around each kernel and runs them one after the
+ * other (LM head, decision, window attention); ebd_profile_read writes the
+ * durations in milliseconds to ms[0..2] = (attention, LM head, decision).
+ * mode 2: the step runs as in production, the window attention overlapping
+ * the decision; ms[1] = LM head, ms[2] = decision and attention together,
+ * ms[0] = -1.  Events are recorded inside a captured graph too.
+ * ebd_profile_read waits for the last recorded event; EBD_ERR_STATE if no
+ * profiled step was recorded. */
+ebd_status ebd_profile_enable(ebd_handle* h, int mode);
 ebd_status ebd_profile_read(ebd_handle* h, float* ms);
 
 /* Last error message of the handle (never NULL; "" if none). */

@@ -192,8 +192,9 @@ def ebd_pack_lm_head(h, w_lm_ptr: int, w_packed_ptr: int, stream: int = 0) -> in
     return load().ebd_pack_lm_head(h, c_void_p(w_lm_ptr), c_void_p(w_packed_ptr), c_void_p(stream))
 
 
-def ebd_profile_enable(h, on: bool) -> int:
-    return load().ebd_profile_enable(h, 1 if on else 0)
+def ebd_profile_enable(h, mode: int) -> int:
+    """mode 0 off, 1 every kernel timed on its own, 2 production overlap."""
+    return load().ebd_profile_enable(h, int(mode))
 
 
 def ebd_profile_read(h):

@@ -199,6 +199,7 @@ struct ebd_handle {
   size_t staging_bytes = 0;
   cudaEvent_t ev[4] = {nullptr, nullptr, nullptr, nullptr};
   int profile = 0;
+  int prof_mode = 0, prof_attn = 0;  // what the last ebd_step recorded
 };
 
 namespace {
@@ -424,7 +425,8 @@ ebd_status check_args(ebd_handle* h, const ebd_step_args* a, bool need_attn, boo
   return EBD_OK;
 }
 
-ebd_status run_attention(ebd_handle* h, const ebd_step_args* a, cudaStream_t st) {
+ebd_status run_attention(ebd_handle* h, const ebd_step_args* a, cudaStream_t st,
+                         bool pdl = false) {
   const ebd_config& c = h->cfg;
   const int D = c.head_dim, Hkv = c.n_heads_kv;
   CUtensorMap kc, vc, kw, vw;
@@ -466,7 +468,7 @@ ebd_status run_attention(ebd_handle* h, const ebd_step_args* a, cudaStream_t st)
   p.tickets = h->tickets;
   p.status = h->d_status;
   p.limit_ns = kLimitNs;
-  cudaError_t e = launch_attention(kc, vc, kw, vw, p, st);
+  cudaError_t e = launch_attention(kc, vc, kw, vw, p, st, pdl);
   if (e != cudaSuccess) return cuda_fail(h, e, "attention launch");
   return EBD_OK;
 }
@@ -762,20 +764,24 @@ ebd_status ebd_step(ebd_handle* h, const ebd_step_args* a, void* stream) {
   if (a->rows == 0 || a->batch == 0) return EBD_OK;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   (void)cudaGetLastError();  // a stale error of an earlier unrelated call is not ours
+  // Order on `st`: LM head, decision, window attention.  The attention feeds
+  // neither of the others, so unless every kernel is timed on its own
+  // (profile mode 1) it is launched as a programmatic dependent of the
+  // decision: it fills the SMs the decision's clusters leave idle.
+  const int prof = h->profile;
   cudaError_t e0 = cudaSuccess;
-  if (h->profile && (e0 = record(h->ev[0], st)) != cudaSuccess)
-    return cuda_fail(h, e0, "profile event");
-  if (attn && (s = run_attention(h, a, st)) != EBD_OK) return s;
-  if (h->profile && (e0 = record(h->ev[1], st)) != cudaSuccess)
-    return cuda_fail(h, e0, "profile event");
+  if (prof && (e0 = record(h->ev[0], st)) != cudaSuccess) return cuda_fail(h, e0, "profile event");
   if ((s = run_lm(h, a, st)) != EBD_OK) return s;
-  if (h->profile && (e0 = record(h->ev[2], st)) != cudaSuccess)
-    return cuda_fail(h, e0, "profile event");
+  if (prof && (e0 = record(h->ev[1], st)) != cudaSuccess) return cuda_fail(h, e0, "profile event");
   DecideParams p = decide_params(h, a, 0);
   cudaError_t e = launch_decide(p, st);
   if (e != cudaSuccess) return cuda_fail(h, e, "decision launch");
-  if (h->profile && (e0 = record(h->ev[3], st)) != cudaSuccess)
+  if (prof == 1 && (e0 = record(h->ev[2], st)) != cudaSuccess)
     return cuda_fail(h, e0, "profile event");
+  if (attn && (s = run_attention(h, a, st, prof != 1)) != EBD_OK) return s;
+  if (prof && (e0 = record(h->ev[3], st)) != cudaSuccess) return cuda_fail(h, e0, "profile event");
+  h->prof_mode = prof;
+  h->prof_attn = attn ? 1 : 0;
   return EBD_OK;
 }
 
@@ -914,19 +920,27 @@ ebd_status ebd_step_host(ebd_handle* h, const ebd_step_args* a, void* stream) {
   return EBD_OK;
 }
 
-ebd_status ebd_profile_enable(ebd_handle* h, int on) {
+ebd_status ebd_profile_enable(ebd_handle* h, int mode) {
   if (h == nullptr) return EBD_ERR_INVALID_ARG;
-  h->profile = on ? 1 : 0;
+  if (mode < 0 || mode > 2) return fail(h, EBD_ERR_INVALID_ARG, "profile mode must be 0, 1 or 2");
+  h->profile = mode;
   return EBD_OK;
 }
 
 ebd_status ebd_profile_read(ebd_handle* h, float* ms) {
   if (h == nullptr || ms == nullptr) return EBD_ERR_INVALID_ARG;
+  if (h->prof_mode == 0) return fail(h, EBD_ERR_STATE, "no profiled ebd_step recorded");
   cudaError_t e = cudaEventSynchronize(h->ev[3]);
   if (e != cudaSuccess) return cuda_fail(h, e, "cudaEventSynchronize");
-  for (int i = 0; i < 3; ++i) {
-    e = cudaEventElapsedTime(&ms[i], h->ev[i], h->ev[i + 1]);
-    if (e != cudaSuccess) return cuda_fail(h, e, "cudaEventElapsedTime");
+  auto span = [&](int i, int j, float* out) { return cudaEventElapsedTime(out, h->ev[i], h->ev[j]); };
+  if ((e = span(0, 1, &ms[1])) != cudaSuccess) return cuda_fail(h, e, "cudaEventElapsedTime");
+  if (h->prof_mode == 1) {
+    if ((e = span(1, 2, &ms[2])) != cudaSuccess) return cuda_fail(h, e, "cudaEventElapsedTime");
+    if ((e = span(2, 3, &ms[0])) != cudaSuccess) return cuda_fail(h, e, "cudaEventElapsedTime");
+    if (!h->prof_attn) ms[0] = 0.f;
+  } else {
+    if ((e = span(1, 3, &ms[2])) != cudaSuccess) return cuda_fail(h, e, "cudaEventElapsedTime");
+    ms[0] = -1.f;
   }
   return EBD_OK;
 }

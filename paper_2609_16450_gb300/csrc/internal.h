@@ -89,8 +89,12 @@ struct DecideParams {
 cudaError_t launch_lm_stats(const CUtensorMap& tmap_w, const CUtensorMap& tmap_h,
                             const LmParams& p, cudaStream_t st);
 void lm_plan(LmParams& p, int rows, int V, int d, int num_sms);
+// pdl: launched as a programmatic dependent of the kernel before it on
+// `st` (that kernel's CTAs release it early; the attention reads nothing the
+// earlier kernel writes)
 cudaError_t launch_attention(const CUtensorMap& kc, const CUtensorMap& vc, const CUtensorMap& kw,
-                             const CUtensorMap& vw, const AttnParams& p, cudaStream_t st);
+                             const CUtensorMap& vw, const AttnParams& p, cudaStream_t st,
+                             bool pdl = false);
 cudaError_t launch_decide(const DecideParams& p, cudaStream_t st);
 cudaError_t launch_pack_lm(const __nv_bfloat16* w, __nv_bfloat16* out, int V, int d,
                            cudaStream_t st);

@@ -311,14 +311,20 @@ cudaError_t attn_configure() {
 }
 
 cudaError_t launch_attention(const CUtensorMap& kc, const CUtensorMap& vc, const CUtensorMap& kw,
-                             const CUtensorMap& vw, const AttnParams& p, cudaStream_t st) {
-  const dim3 grid(p.splits, p.max_qtiles, p.B * p.Hkv);
-  const int bytes = kAttnStages * kStageBytes + 1024 + 64;
-  if (p.D == 64)
-    attn_kernel<64><<<grid, kAttnThreads, bytes, st>>>(kc, vc, kw, vw, p);
-  else
-    attn_kernel<128><<<grid, kAttnThreads, bytes, st>>>(kc, vc, kw, vw, p);
-  return cudaGetLastError();
+                             const CUtensorMap& vw, const AttnParams& p, cudaStream_t st,
+                             bool pdl) {
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = dim3(p.splits, p.max_qtiles, p.B * p.Hkv);
+  cfg.blockDim = dim3(kAttnThreads, 1, 1);
+  cfg.dynamicSmemBytes = kAttnStages * kStageBytes + 1024 + 64;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl ? 1 : 0;
+  if (p.D == 64) return cudaLaunchKernelEx(&cfg, attn_kernel<64>, kc, vc, kw, vw, p);
+  return cudaLaunchKernelEx(&cfg, attn_kernel<128>, kc, vc, kw, vw, p);
 }
 
 }  // namespace ebd

@@ -452,6 +452,10 @@ __global__ void __cluster_dims__(kDecideCluster, 1, 1) __launch_bounds__(kDecide
   const int seq = blockIdx.x / kDecideCluster;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   float* const P = sm.pool;
+  // a kernel launched after this one as a programmatic dependent (the window
+  // attention, which shares no data with the decision) may start on the SMs
+  // this grid leaves free once every CTA of it is resident
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 
   if (tid == 0) {
     // weights and vectors of this rank: bulk copies issued first, so they

@@ -202,3 +202,41 @@ def test_timeout_is_reported_and_context_survives():
     gpu = _run(sh, inp, w, h)
     res = _oracle(sh, inp)
     _check(sh, inp, gpu, res)
+
+
+def test_overlapped_and_serial_and_graph_steps_agree():
+    """The production order (attention as a programmatic dependent of the
+    decision), the fully serial order and a CUDA-graph replay give identical
+    bits."""
+    from paper_2609_16450_gb300 import _ebd as E
+    from paper_2609_16450_gb300 import runtime as rt
+    sh = synth.tiny
+    inp, w, h = _setup(sh)
+    outs = []
+    for mode in (0, 1, 2):
+        E.check(E.ebd_profile_enable(h.h, mode), h.h)
+        outs.append(_run(sh, inp, w, h))
+    E.check(E.ebd_profile_enable(h.h, 0), h.h)
+    ds = rt.DeviceStep(inp, w)
+    args = ds.args()
+    stream = torch.cuda.Stream()
+    with torch.cuda.stream(stream):
+        E.check(E.ebd_step(h.h, args, stream.cuda_stream), h.h)
+    torch.cuda.synchronize()
+    ds.restore_state()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=stream):
+        E.check(E.ebd_step(h.h, args, stream.cuda_stream), h.h)
+    torch.cuda.synchronize()
+    ds.restore_state()
+    for k in ("attn_out", "conf", "argmax"):
+        ds_val = getattr(ds, k)
+        ds_val.zero_()
+    torch.cuda.synchronize()
+    g.replay()
+    torch.cuda.synchronize()
+    assert h.sync_status() == 0
+    outs.append(ds.fetch())
+    for o2 in outs[1:]:
+        for k in outs[0]:
+            np.testing.assert_array_equal(outs[0][k], o2[k], err_msg=k)
