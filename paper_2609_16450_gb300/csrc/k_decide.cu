@@ -115,15 +115,12 @@ __device__ __forceinline__ void hl_store2(const HL& h, int j, int c, float x, fl
   *reinterpret_cast<uint32_t*>(h.p + j * h.ld + c) = hi;
   *reinterpret_cast<uint32_t*>(h.p + h.plane + j * h.ld + c) = lo;
 }
-__device__ __forceinline__ void hl_store1(const HL& h, int j, int c, float x) {
-  const __nv_bfloat16 hi = __float2bfloat16_rn(x);
-  h.p[j * h.ld + c] = hi;
-  h.p[h.plane + j * h.ld + c] = __float2bfloat16_rn(x - __bfloat162float(hi));
-}
 
 // out(j, o) = sum_k A[j][k] Wt[k][o] for j < n, o < Os, A = hi + lo in
 // shared memory, Wt bf16 [K][ldw].  Each warp owns 16-row x 16-output tiles;
-// epi(j, o, v0, v1) receives the outputs o and o + 1 of row j.
+// the high and low parts accumulate in separate chains (shorter dependency
+// chains), summed at the end.  epi(j, o, v0, v1) receives the outputs o and
+// o + 1 of row j.
 template <class Epi>
 __device__ __forceinline__ void gemm_hl(const HL& A, int n, int K, const __nv_bfloat16* Wt,
                                         int ldw, int Os, Epi epi) {
@@ -135,11 +132,12 @@ __device__ __forceinline__ void gemm_hl(const HL& A, int n, int K, const __nv_bf
   for (int unit = warp; unit < mt * np; unit += (blockDim.x >> 5)) {
     const int m0 = (unit / np) * 16, c0 = (unit % np) * 16;
     float acc[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
+    float acl[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
     const uint32_t ah_base =
         smem_u32(A.p + (m0 + (mi & 1) * 8 + rr) * A.ld + (mi >> 1) * 8);
     const uint32_t al_base = ah_base + static_cast<uint32_t>(A.plane * 2);
     const uint32_t w_base = smem_u32(Wt + ((mi & 1) * 8 + rr) * ldw + c0 + (mi >> 1) * 8);
-#pragma unroll 4
+#pragma unroll 2
     for (int k0 = 0; k0 < K; k0 += 16) {
       uint32_t ah[4], al[4], b0, b1, b2, b3;
       ldsm_x4(ah_base + k0 * 2, ah[0], ah[1], ah[2], ah[3]);
@@ -147,50 +145,75 @@ __device__ __forceinline__ void gemm_hl(const HL& A, int n, int K, const __nv_bf
       ldsm_x4_t(w_base + static_cast<uint32_t>(k0 * ldw * 2), b0, b1, b2, b3);
       mma_bf16(acc[0], ah, b0, b1);
       mma_bf16(acc[1], ah, b2, b3);
-      mma_bf16(acc[0], al, b0, b1);
-      mma_bf16(acc[1], al, b2, b3);
+      mma_bf16(acl[0], al, b0, b1);
+      mma_bf16(acl[1], al, b2, b3);
     }
     const int r_lo = m0 + g, r_hi = r_lo + 8;
 #pragma unroll
     for (int nt = 0; nt < 2; ++nt) {
       const int o = c0 + nt * 8 + 2 * t;
-      if (r_lo < n) epi(r_lo, o, acc[nt][0], acc[nt][1]);
-      if (r_hi < n) epi(r_hi, o, acc[nt][2], acc[nt][3]);
+      if (r_lo < n) epi(r_lo, o, acc[nt][0] + acl[nt][0], acc[nt][1] + acl[nt][1]);
+      if (r_hi < n) epi(r_hi, o, acc[nt][2] + acl[nt][2], acc[nt][3] + acl[nt][3]);
     }
   }
 }
 
-// LayerNorm (eps 1e-5) over `dim` (32, 64 or 128) of rows j < n, warp per
-// row; the result goes to an fp32 buffer (if dst) and/or a hi/lo buffer.
-__device__ __forceinline__ void ln_rows(const float* src, int lds, float* dst, int ldd,
-                                        const HL* hl, int hl_col, int n, int dim, const float* g,
-                                        const float* b) {
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+// Sum over the 8 lanes of an aligned lane group.
+__device__ __forceinline__ float group8_sum(float v) {
+  v += __shfl_xor_sync(0xffffffffu, v, 1);
+  v += __shfl_xor_sync(0xffffffffu, v, 2);
+  v += __shfl_xor_sync(0xffffffffu, v, 4);
+  return v;
+}
+
+// LayerNorm (eps 1e-5) over `dim` (32, 64 or 128) of rows j < n: 8 lanes per
+// row, lane q holding columns 4q + 32c (c < dim/32); the result goes to an
+// fp32 buffer (if dst) and/or a hi/lo buffer (if hl).  One copy of the code
+// serves every call.
+__device__ __noinline__ void ln_rows(const float* src, int lds, float* dst, int ldd, const HL* hl,
+                                     int n, int dim, const float* g, const float* b) {
+  const int q = threadIdx.x & 7;
   const int per = dim >> 5;
+  const float inv_dim = 1.0f / static_cast<float>(dim);
 #pragma unroll 1
-  for (int j = warp; j < n; j += (blockDim.x >> 5)) {
-    float v[4] = {0.f, 0.f, 0.f, 0.f};
+  for (int j0 = 0; j0 < n; j0 += (blockDim.x >> 3)) {
+    const int j = j0 + (threadIdx.x >> 3);
+    const bool ok = j < n;
+    float4 v[4];
     float s = 0.f;
 #pragma unroll
-    for (int c = 0; c < 4; ++c)
-      if (c < per) {
-        v[c] = src[j * lds + lane + 32 * c];
-        s += v[c];
-      }
-    const float mean = warp_sum(s) / dim;
-    float q = 0.f;
-#pragma unroll
-    for (int c = 0; c < 4; ++c)
-      if (c < per) q += (v[c] - mean) * (v[c] - mean);
-    const float inv = 1.0f / sqrtf(warp_sum(q) / dim + 1e-5f);
+    for (int c = 0; c < 4; ++c) {
+      v[c] = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (c < per && ok) v[c] = *reinterpret_cast<const float4*>(src + j * lds + 4 * q + 32 * c);
+      s += (v[c].x + v[c].y) + (v[c].z + v[c].w);
+    }
+    const float mean = group8_sum(s) * inv_dim;
+    float var = 0.f;
 #pragma unroll
     for (int c = 0; c < 4; ++c)
       if (c < per) {
-        const int o = lane + 32 * c;
-        const float y = (v[c] - mean) * inv * g[o] + b[o];
-        if (dst) dst[j * ldd + o] = y;
-        if (hl) hl_store1(*hl, j, hl_col + o, y);
+        const float a0 = v[c].x - mean, a1 = v[c].y - mean, a2 = v[c].z - mean, a3 = v[c].w - mean;
+        var += (a0 * a0 + a1 * a1) + (a2 * a2 + a3 * a3);
       }
+    const float inv = 1.0f / sqrtf(group8_sum(var) * inv_dim + 1e-5f);
+    if (ok) {
+#pragma unroll
+      for (int c = 0; c < 4; ++c)
+        if (c < per) {
+          const int o = 4 * q + 32 * c;
+          const float4 gg = *reinterpret_cast<const float4*>(g + o);
+          const float4 bb = *reinterpret_cast<const float4*>(b + o);
+          const float4 y = make_float4((v[c].x - mean) * inv * gg.x + bb.x,
+                                       (v[c].y - mean) * inv * gg.y + bb.y,
+                                       (v[c].z - mean) * inv * gg.z + bb.z,
+                                       (v[c].w - mean) * inv * gg.w + bb.w);
+          if (dst) *reinterpret_cast<float4*>(dst + j * ldd + o) = y;
+          if (hl) {
+            hl_store2(*hl, j, o, y.x, y.y);
+            hl_store2(*hl, j, o + 2, y.z, y.w);
+          }
+        }
+    }
   }
 }
 
@@ -285,7 +308,9 @@ __device__ __forceinline__ void lbs_attention(cg::cluster_group& cluster, float*
 
 // ------------------------------------------------------------------ LPS (rank 0)
 // One attention unit: 16 query rows [m0, m0+16) of head h (width 8) over the
-// n keys; qkv: [n][100] fp32 (q | k | v); the output goes to hi/lo columns
+// n keys, in blocks of 16 keys with a running max and sum (the result is
+// softmax(q k^T / sqrt(8)) v, the blocks only bound the live registers);
+// qkv: [n][100] fp32 (q | k | v); the output goes to hi/lo columns
 // 8h..8h+7 of `out`.
 __device__ __forceinline__ void lps_attention_unit(const float* qkv, int n, int m0, int h,
                                                    const HL& out) {
@@ -300,14 +325,15 @@ __device__ __forceinline__ void lps_attention_unit(const float* qkv, int n, int 
     split_bf16x2(q1.x, q1.y, qh[1], ql[1]);
     qh[2] = qh[3] = ql[2] = ql[3] = 0u;  // head width 8: upper k half is zero
   }
-  const int nkb = (n + 7) >> 3;
-  float s[8][4];
-  float mx0 = -INFINITY, mx1 = -INFINITY;
+  const float scale = 0.35355339059327373f;  // 1/sqrt(8)
+  float mx0 = -INFINITY, mx1 = -INFINITY, l0 = 0.f, l1 = 0.f;
+  float o[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll 1
+  for (int k0 = 0; k0 < n; k0 += 16) {
+    float s[2][4];
 #pragma unroll
-  for (int kb = 0; kb < 8; ++kb) {
-    s[kb][0] = s[kb][1] = s[kb][2] = s[kb][3] = -INFINITY;
-    if (kb < nkb) {
-      const int key = 8 * kb + g;
+    for (int hb = 0; hb < 2; ++hb) {
+      const int key = k0 + 8 * hb + g;
       const float2 kk = key < n ? *reinterpret_cast<const float2*>(qkv + key * 100 + 32 + 8 * h + 2 * t)
                                 : make_float2(0.f, 0.f);
       uint32_t bh, bl;
@@ -316,56 +342,57 @@ __device__ __forceinline__ void lps_attention_unit(const float* qkv, int n, int 
       mma_bf16(a, qh, bh, 0u);
       mma_bf16(a, qh, bl, 0u);
       mma_bf16(a, ql, bh, 0u);
-      const int c = 8 * kb + 2 * t;
-      s[kb][0] = c < n ? a[0] * 0.35355339059327373f : -INFINITY;  // 1/sqrt(8)
-      s[kb][1] = c + 1 < n ? a[1] * 0.35355339059327373f : -INFINITY;
-      s[kb][2] = c < n ? a[2] * 0.35355339059327373f : -INFINITY;
-      s[kb][3] = c + 1 < n ? a[3] * 0.35355339059327373f : -INFINITY;
-      mx0 = fmaxf(mx0, fmaxf(s[kb][0], s[kb][1]));
-      mx1 = fmaxf(mx1, fmaxf(s[kb][2], s[kb][3]));
+      const int c = k0 + 8 * hb + 2 * t;
+      s[hb][0] = c < n ? a[0] * scale : -INFINITY;
+      s[hb][1] = c + 1 < n ? a[1] * scale : -INFINITY;
+      s[hb][2] = c < n ? a[2] * scale : -INFINITY;
+      s[hb][3] = c + 1 < n ? a[3] * scale : -INFINITY;
     }
-  }
-  mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 1));
-  mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 2));
-  mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 1));
-  mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 2));
-  float l0 = 0.f, l1 = 0.f;
+    float b0 = fmaxf(fmaxf(s[0][0], s[0][1]), fmaxf(s[1][0], s[1][1]));
+    float b1 = fmaxf(fmaxf(s[0][2], s[0][3]), fmaxf(s[1][2], s[1][3]));
+    b0 = fmaxf(b0, __shfl_xor_sync(0xffffffffu, b0, 1));
+    b0 = fmaxf(b0, __shfl_xor_sync(0xffffffffu, b0, 2));
+    b1 = fmaxf(b1, __shfl_xor_sync(0xffffffffu, b1, 1));
+    b1 = fmaxf(b1, __shfl_xor_sync(0xffffffffu, b1, 2));
+    const float n0 = fmaxf(mx0, b0), n1 = fmaxf(mx1, b1);  // finite: key k0 is valid
+    const float c0 = expf(mx0 - n0), c1 = expf(mx1 - n1);
+    mx0 = n0;
+    mx1 = n1;
 #pragma unroll
-  for (int kb = 0; kb < 8; ++kb) {
-    s[kb][0] = expf(s[kb][0] - mx0);
-    s[kb][1] = expf(s[kb][1] - mx0);
-    s[kb][2] = expf(s[kb][2] - mx1);
-    s[kb][3] = expf(s[kb][3] - mx1);
-    l0 += s[kb][0] + s[kb][1];
-    l1 += s[kb][2] + s[kb][3];
+    for (int hb = 0; hb < 2; ++hb) {
+      s[hb][0] = expf(s[hb][0] - n0);
+      s[hb][1] = expf(s[hb][1] - n0);
+      s[hb][2] = expf(s[hb][2] - n1);
+      s[hb][3] = expf(s[hb][3] - n1);
+    }
+    l0 = l0 * c0 + ((s[0][0] + s[0][1]) + (s[1][0] + s[1][1]));
+    l1 = l1 * c1 + ((s[0][2] + s[0][3]) + (s[1][2] + s[1][3]));
+    o[0] *= c0;
+    o[1] *= c0;
+    o[2] *= c1;
+    o[3] *= c1;
+    uint32_t ph[4], pl[4];
+    split_bf16x2(s[0][0], s[0][1], ph[0], pl[0]);
+    split_bf16x2(s[0][2], s[0][3], ph[1], pl[1]);
+    split_bf16x2(s[1][0], s[1][1], ph[2], pl[2]);
+    split_bf16x2(s[1][2], s[1][3], ph[3], pl[3]);
+    float v[4];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      const int key = k0 + (e >> 1) * 8 + 2 * t + (e & 1);
+      v[e] = key < n ? qkv[key * 100 + 64 + 8 * h + g] : 0.f;
+    }
+    uint32_t v0h, v0l, v1h, v1l;
+    split_bf16x2(v[0], v[1], v0h, v0l);
+    split_bf16x2(v[2], v[3], v1h, v1l);
+    mma_bf16(o, ph, v0h, v1h);
+    mma_bf16(o, ph, v0l, v1l);
+    mma_bf16(o, pl, v0h, v1h);
   }
   l0 += __shfl_xor_sync(0xffffffffu, l0, 1);
   l0 += __shfl_xor_sync(0xffffffffu, l0, 2);
   l1 += __shfl_xor_sync(0xffffffffu, l1, 1);
   l1 += __shfl_xor_sync(0xffffffffu, l1, 2);
-  float o[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll
-  for (int j = 0; j < 4; ++j) {
-    if (16 * j < n) {
-      uint32_t ph[4], pl[4];
-      split_bf16x2(s[2 * j][0], s[2 * j][1], ph[0], pl[0]);
-      split_bf16x2(s[2 * j][2], s[2 * j][3], ph[1], pl[1]);
-      split_bf16x2(s[2 * j + 1][0], s[2 * j + 1][1], ph[2], pl[2]);
-      split_bf16x2(s[2 * j + 1][2], s[2 * j + 1][3], ph[3], pl[3]);
-      float v[4];
-#pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        const int key = 16 * j + (e >> 1) * 8 + 2 * t + (e & 1);
-        v[e] = key < n ? qkv[key * 100 + 64 + 8 * h + g] : 0.f;
-      }
-      uint32_t b0h, b0l, b1h, b1l;
-      split_bf16x2(v[0], v[1], b0h, b0l);
-      split_bf16x2(v[2], v[3], b1h, b1l);
-      mma_bf16(o, ph, b0h, b1h);
-      mma_bf16(o, ph, b0l, b1l);
-      mma_bf16(o, pl, b0h, b1h);
-    }
-  }
   const float i0 = 1.0f / l0, i1 = 1.0f / l1;
   if (r_lo < n) hl_store2(out, r_lo, 8 * h + 2 * t, o[0] * i0, o[1] * i0);
   if (r_hi < n) hl_store2(out, r_hi, 8 * h + 2 * t, o[2] * i1, o[3] * i1);
@@ -384,26 +411,44 @@ __device__ __noinline__ void lps_forward(float* P, int n, const __nv_bfloat16* W
   const HL Y = hl_at(P + L_YH, 40);
   const HL At = hl_at(P + L_AH, 40);
   const HL Hh = hl_at(P + L_HH, 72);
-  float* Yf = P + L_QKV;  // fp32 scratch for the input layer (before QKV is used)
+  {  // Linear(5 -> 32), LayerNorm, GELU: 8 lanes per row, 4 outputs each
+    const int q = lane & 7;
 #pragma unroll 1
-  for (int it = tid; it < n * 32; it += blockDim.x) {  // Linear(5 -> 32)
-    const int r = it >> 5, c = it & 31;
-    float a = V[VP_INB + c];
+    for (int j0 = 0; j0 < n; j0 += (blockDim.x >> 3)) {
+      const int j = j0 + (tid >> 3);
+      const bool ok = j < n;
+      float y[4];
+      float s = 0.f;
 #pragma unroll
-    for (int k = 0; k < 5; ++k) a = fmaf(feats[r * 8 + k], V[VP_INT + k * 32 + c], a);
-    Yf[r * LDQ + c] = a;
+      for (int e = 0; e < 4; ++e) {
+        const int c = 4 * q + e;
+        float a = V[VP_INB + c];
+#pragma unroll
+        for (int k = 0; k < 5; ++k) a = fmaf(ok ? feats[j * 8 + k] : 0.f, V[VP_INT + k * 32 + c], a);
+        y[e] = a;
+        s += a;
+      }
+      const float mean = group8_sum(s) * (1.0f / 32.0f);
+      float var = 0.f;
+#pragma unroll
+      for (int e = 0; e < 4; ++e) var += (y[e] - mean) * (y[e] - mean);
+      const float inv = 1.0f / sqrtf(group8_sum(var) * (1.0f / 32.0f) + 1e-5f);
+      if (ok) {
+        float4 z;
+        z.x = gelu((y[0] - mean) * inv * V[VP_INLNG + 4 * q + 0] + V[VP_INLNB + 4 * q + 0]);
+        z.y = gelu((y[1] - mean) * inv * V[VP_INLNG + 4 * q + 1] + V[VP_INLNB + 4 * q + 1]);
+        z.z = gelu((y[2] - mean) * inv * V[VP_INLNG + 4 * q + 2] + V[VP_INLNB + 4 * q + 2]);
+        z.w = gelu((y[3] - mean) * inv * V[VP_INLNG + 4 * q + 3] + V[VP_INLNB + 4 * q + 3]);
+        *reinterpret_cast<float4*>(Z + j * LDQ + 4 * q) = z;
+      }
+    }
   }
-  __syncthreads();
-  ln_rows(Yf, LDQ, Z, LDQ, nullptr, 0, n, 32, V + VP_INLNG, V + VP_INLNB);
-  __syncthreads();
-#pragma unroll 1
-  for (int it = tid; it < n * 32; it += blockDim.x) Z[(it >> 5) * LDQ + (it & 31)] = gelu(Z[(it >> 5) * LDQ + (it & 31)]);
   __syncthreads();
 #pragma unroll 1
   for (int l = 0; l < 2; ++l) {
     const __nv_bfloat16* Wl = Wlps + l * PL_STRIDE;
     const float* Vl = V + VP_LAYER0 + l * VP_LAYER_STRIDE;
-    ln_rows(Z, LDQ, nullptr, 0, &Y, 0, n, 32, Vl + VPL_LN1G, Vl + VPL_LN1B);
+    ln_rows(Z, LDQ, nullptr, 0, &Y, n, 32, Vl + VPL_LN1G, Vl + VPL_LN1B);
     __syncthreads();
     gemm_hl(Y, n, 32, Wl + PL_QKV, PL_LDQKV, 96, [&](int j, int o, float a, float b) {
       *reinterpret_cast<float2*>(QKV + j * 100 + o) = make_float2(a + Vl[VPL_QKVB + o], b + Vl[VPL_QKVB + o + 1]);
@@ -419,7 +464,7 @@ __device__ __noinline__ void lps_forward(float* P, int n, const __nv_bfloat16* W
       *z = make_float2(zz.x + (a + Vl[VPL_OUTB + o]), zz.y + (b + Vl[VPL_OUTB + o + 1]));
     });
     __syncthreads();
-    ln_rows(Z, LDQ, nullptr, 0, &Y, 0, n, 32, Vl + VPL_LN2G, Vl + VPL_LN2B);
+    ln_rows(Z, LDQ, nullptr, 0, &Y, n, 32, Vl + VPL_LN2G, Vl + VPL_LN2B);
     __syncthreads();
     gemm_hl(Y, n, 32, Wl + PL_FF1, PL_LDFF1, 64, [&](int j, int o, float a, float b) {
       hl_store2(Hh, j, o, gelu(a + Vl[VPL_FF1B + o]), gelu(b + Vl[VPL_FF1B + o + 1]));
@@ -627,7 +672,7 @@ __global__ void __cluster_dims__(kDecideCluster, 1, 1) __launch_bounds__(kDecide
       *reinterpret_cast<float2*>(E2 + j * LDZ + o) = make_float2(a + Vv[V_ENT2B + o], b + Vv[V_ENT2B + o + 1]);
     });
     __syncthreads();
-    ln_rows(E2, LDZ, nullptr, 0, &Xh, 0, n, 64, Vv + V_ENTLNG, Vv + V_ENTLNB);
+    ln_rows(E2, LDZ, nullptr, 0, &Xh, n, 64, Vv + V_ENTLNG, Vv + V_ENTLNB);
     __syncthreads();
     // 3b. fusion W_combine [e; t] + E_pos[rank of the row]: this CTA's 16 outputs
     {
@@ -686,7 +731,7 @@ __global__ void __cluster_dims__(kDecideCluster, 1, 1) __launch_bounds__(kDecide
         });
       }
       cluster.sync();
-      ln_rows(Z, LDZ, Z, LDZ, &Zh, 0, n, 128, Vl + VL_LN1G, Vl + VL_LN1B);
+      ln_rows(Z, LDZ, Z, LDZ, &Zh, n, 128, Vl + VL_LN1G, Vl + VL_LN1B);
       __syncthreads();
       // FFN: hidden units [32r, 32r+32) locally, then the partial second
       // linear of those units sent to the owners of each 16-output slice
@@ -719,7 +764,7 @@ __global__ void __cluster_dims__(kDecideCluster, 1, 1) __launch_bounds__(kDecide
         }
       }
       cluster.sync();
-      ln_rows(Z, LDZ, Z, LDZ, &Zh, 0, n, 128, Vl + VL_LN2G, Vl + VL_LN2B);
+      ln_rows(Z, LDZ, Z, LDZ, &Zh, n, 128, Vl + VL_LN2G, Vl + VL_LN2B);
       __syncthreads();
       if (l == 0 && rank == 0 && tid == 0 && p.lps_enabled) {
         // the first layer's weights (and everything before them) are dead:
