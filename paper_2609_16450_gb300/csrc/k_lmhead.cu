@@ -59,6 +59,37 @@ __device__ __forceinline__ bool named_barrier_and(uint32_t id, uint32_t n, bool 
   return r != 0;
 }
 
+// MMAs of one full pipeline stage: KBS k-boxes x 4 k16 steps into one
+// accumulator, descriptors advanced by immediates (k16 step = 32 bytes = 2 in
+// the descriptor's address field; k-box = kATile bytes of A, b_step of B).
+template <int KBS>
+__device__ __forceinline__ void mma_stage(uint32_t d, uint32_t a_lo, uint32_t b_lo,
+                                          uint32_t b_step, uint32_t hi, uint32_t idesc,
+                                          uint32_t acc0) {
+#pragma unroll
+  for (int j = 0; j < KBS; ++j)
+#pragma unroll
+    for (int kk = 0; kk < 4; ++kk)
+      umma_bf16_lo(d, a_lo + static_cast<uint32_t>(j * (kATile >> 4) + kk * 2),
+                   b_lo + static_cast<uint32_t>(j) * b_step + static_cast<uint32_t>(kk * 2), hi,
+                   idesc, (j | kk) != 0 ? 1u : acc0);
+}
+
+// Waits with a back-off between polls: for warps whose wait is long and not
+// latency-critical, so that they leave the issue slots of their SM
+// sub-partition to the producer and MMA threads.
+__device__ __forceinline__ bool mbar_wait_sleepy(uint64_t* bar, uint32_t parity, uint64_t limit_ns,
+                                                 volatile int* abort) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = global_timer_ns();
+  for (;;) {
+    __nanosleep(256);
+    if (mbar_try_wait(bar, parity)) return true;
+    if (abort != nullptr && *abort) return false;
+    if (global_timer_ns() - t0 > limit_ns) return false;
+  }
+}
+
 __device__ __forceinline__ void record_error(int* status, volatile int* abort, int code) {
   *abort = 1;
   atomicCAS(status, 0, code);
@@ -181,6 +212,7 @@ __global__ void __launch_bounds__(kLmThreads, 1)
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0) {
       const uint32_t idesc = umma_idesc_bf16(128, static_cast<uint32_t>(p.nb));
+      const uint32_t desc_hi = static_cast<uint32_t>(umma_desc_sw128(0) >> 32);
       int it = 0, c = 0;
       bool ok = true;
       for (int u = u0; u < u1 && ok; u += 2, ++c) {
@@ -203,6 +235,22 @@ __global__ void __launch_bounds__(kLmThreads, 1)
           const int nsubk = min(p.kbs, p.nkb - ks * p.kbs);
           const uint32_t a_addr = smem_u32(sA + static_cast<size_t>(s) * a_stage);
           const uint32_t b_addr = smem_u32(sB + static_cast<size_t>(s) * b_stage);
+          if (p.nsub == 1 && nsubk == p.kbs && p.kbs >= 2 && p.kbs <= 5) {
+            // full stage, one N sub-tile: the unrolled issue path
+            const uint32_t a_lo = static_cast<uint32_t>(umma_desc_sw128(a_addr));
+            const uint32_t b_lo = static_cast<uint32_t>(umma_desc_sw128(b_addr));
+            const uint32_t b_step = b_sub >> 4;
+            const uint32_t acc0 = ks != 0 ? 1u : 0u;
+            switch (p.kbs) {
+              case 2: mma_stage<2>(d0, a_lo, b_lo, b_step, desc_hi, idesc, acc0); break;
+              case 3: mma_stage<3>(d0, a_lo, b_lo, b_step, desc_hi, idesc, acc0); break;
+              case 4: mma_stage<4>(d0, a_lo, b_lo, b_step, desc_hi, idesc, acc0); break;
+              default: mma_stage<5>(d0, a_lo, b_lo, b_step, desc_hi, idesc, acc0); break;
+            }
+            umma_commit(&empty[s]);
+            ++it;
+            continue;
+          }
           for (int j = 0; j < nsubk; ++j) {
 #pragma unroll
             for (int kk = 0; kk < 4; ++kk) {
@@ -244,7 +292,7 @@ __global__ void __launch_bounds__(kLmThreads, 1)
       const int valid = min(nu * kUnit, p.V - u * kUnit);
       const int buf = c % p.nbuf;
       const uint32_t bph = static_cast<uint32_t>(c / p.nbuf) & 1u;
-      bool w = mbar_wait(&acc_full[buf], bph, p.limit_ns, abort);
+      bool w = mbar_wait_sleepy(&acc_full[buf], bph, p.limit_ns, abort);
       ok = named_barrier_and(1, 128, w);
       if (!ok) {
         if (et == 0 && !*abort) record_error(p.status, abort, EBD_ERR_TIMEOUT);
