@@ -235,13 +235,14 @@ __global__ void __launch_bounds__(kLmThreads, 1)
           const int nsubk = min(p.kbs, p.nkb - ks * p.kbs);
           const uint32_t a_addr = smem_u32(sA + static_cast<size_t>(s) * a_stage);
           const uint32_t b_addr = smem_u32(sB + static_cast<size_t>(s) * b_stage);
-          if (p.nsub == 1 && nsubk == p.kbs && p.kbs >= 2 && p.kbs <= 5) {
-            // full stage, one N sub-tile: the unrolled issue path
+          if (p.nsub == 1 && nsubk >= 1 && nsubk <= 5) {
+            // one N sub-tile: the unrolled issue path
             const uint32_t a_lo = static_cast<uint32_t>(umma_desc_sw128(a_addr));
             const uint32_t b_lo = static_cast<uint32_t>(umma_desc_sw128(b_addr));
             const uint32_t b_step = b_sub >> 4;
             const uint32_t acc0 = ks != 0 ? 1u : 0u;
-            switch (p.kbs) {
+            switch (nsubk) {
+              case 1: mma_stage<1>(d0, a_lo, b_lo, b_step, desc_hi, idesc, acc0); break;
               case 2: mma_stage<2>(d0, a_lo, b_lo, b_step, desc_hi, idesc, acc0); break;
               case 3: mma_stage<3>(d0, a_lo, b_lo, b_step, desc_hi, idesc, acc0); break;
               case 4: mma_stage<4>(d0, a_lo, b_lo, b_step, desc_hi, idesc, acc0); break;
@@ -406,7 +407,7 @@ void lm_plan(LmParams& p, int rows, int V, int d, int num_sms) {
   const uint32_t budget = 232448u - 1024u - tail;
   // k-boxes (64 columns each) per pipeline stage: longer contiguous runs of
   // each W row per request, while keeping at least two stages in flight
-  int kbs = 4;
+  int kbs = 5;
   if (const char* env = getenv("EBD_LM_KBS")) kbs = atoi(env);
   if (kbs < 1) kbs = 1;
   if (kbs > p.nkb) kbs = p.nkb;
