@@ -401,9 +401,12 @@ __device__ __forceinline__ void lps_attention_unit(const float* qkv, int n, int 
 // LPS (Sec. 5.2 / App. D.1): Linear(5->32) -> LayerNorm -> GELU, two pre-norm
 // blocks (4 heads of width 8, FFN 64, GELU), head Linear(32->1), p = sigmoid.
 // Over the n (<= 64) masked rows of the block (features at P + L_FEAT);
-// p_psi of row i -> P[L_PROB + i].  Called by the whole CTA.
+// p_psi of row i -> P[L_PROB + i].  Called by the whole CTA.  `from` > 0
+// skips the phases of the first block before phase `from` (1 LN1, 2 QKV,
+// 3 attention, 4 output projection, 5 LN2, 6 FF1, 7 FF2; 0 the input layer);
+// only the stand-in runs of the decision kernel use it.
 __device__ __noinline__ void lps_forward(float* P, int n, const __nv_bfloat16* Wlps,
-                                         const float* V) {
+                                         const float* V, int from) {
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const float* feats = P + L_FEAT;
   float* Z = P + L_Z;
@@ -411,7 +414,7 @@ __device__ __noinline__ void lps_forward(float* P, int n, const __nv_bfloat16* W
   const HL Y = hl_at(P + L_YH, 40);
   const HL At = hl_at(P + L_AH, 40);
   const HL Hh = hl_at(P + L_HH, 72);
-  {  // Linear(5 -> 32), LayerNorm, GELU: 8 lanes per row, 4 outputs each
+  if (from <= 0) {  // Linear(5 -> 32), LayerNorm, GELU: 8 lanes per row, 4 outputs each
     const int q = lane & 7;
 #pragma unroll 1
     for (int j0 = 0; j0 < n; j0 += (blockDim.x >> 3)) {
@@ -448,27 +451,33 @@ __device__ __noinline__ void lps_forward(float* P, int n, const __nv_bfloat16* W
   for (int l = 0; l < 2; ++l) {
     const __nv_bfloat16* Wl = Wlps + l * PL_STRIDE;
     const float* Vl = V + VP_LAYER0 + l * VP_LAYER_STRIDE;
-    ln_rows(Z, LDQ, nullptr, 0, &Y, n, 32, Vl + VPL_LN1G, Vl + VPL_LN1B);
+    const int f = l == 0 ? from : 0;
+    if (f <= 1) ln_rows(Z, LDQ, nullptr, 0, &Y, n, 32, Vl + VPL_LN1G, Vl + VPL_LN1B);
     __syncthreads();
-    gemm_hl(Y, n, 32, Wl + PL_QKV, PL_LDQKV, 96, [&](int j, int o, float a, float b) {
-      *reinterpret_cast<float2*>(QKV + j * 100 + o) = make_float2(a + Vl[VPL_QKVB + o], b + Vl[VPL_QKVB + o + 1]);
-    });
+    if (f <= 2)
+      gemm_hl(Y, n, 32, Wl + PL_QKV, PL_LDQKV, 96, [&](int j, int o, float a, float b) {
+        *reinterpret_cast<float2*>(QKV + j * 100 + o) = make_float2(a + Vl[VPL_QKVB + o], b + Vl[VPL_QKVB + o + 1]);
+      });
     __syncthreads();
     const int mt = (n + 15) >> 4;
+    if (f <= 3) {
 #pragma unroll 1
-    for (int u = warp; u < 4 * mt; u += (blockDim.x >> 5)) lps_attention_unit(QKV, n, 16 * (u >> 2), u & 3, At);
+      for (int u = warp; u < 4 * mt; u += (blockDim.x >> 5)) lps_attention_unit(QKV, n, 16 * (u >> 2), u & 3, At);
+    }
     __syncthreads();
-    gemm_hl(At, n, 32, Wl + PL_OUT, PL_LDOUT, 32, [&](int j, int o, float a, float b) {
-      float2* z = reinterpret_cast<float2*>(Z + j * LDQ + o);
-      const float2 zz = *z;
-      *z = make_float2(zz.x + (a + Vl[VPL_OUTB + o]), zz.y + (b + Vl[VPL_OUTB + o + 1]));
-    });
+    if (f <= 4)
+      gemm_hl(At, n, 32, Wl + PL_OUT, PL_LDOUT, 32, [&](int j, int o, float a, float b) {
+        float2* z = reinterpret_cast<float2*>(Z + j * LDQ + o);
+        const float2 zz = *z;
+        *z = make_float2(zz.x + (a + Vl[VPL_OUTB + o]), zz.y + (b + Vl[VPL_OUTB + o + 1]));
+      });
     __syncthreads();
-    ln_rows(Z, LDQ, nullptr, 0, &Y, n, 32, Vl + VPL_LN2G, Vl + VPL_LN2B);
+    if (f <= 5) ln_rows(Z, LDQ, nullptr, 0, &Y, n, 32, Vl + VPL_LN2G, Vl + VPL_LN2B);
     __syncthreads();
-    gemm_hl(Y, n, 32, Wl + PL_FF1, PL_LDFF1, 64, [&](int j, int o, float a, float b) {
-      hl_store2(Hh, j, o, gelu(a + Vl[VPL_FF1B + o]), gelu(b + Vl[VPL_FF1B + o + 1]));
-    });
+    if (f <= 6)
+      gemm_hl(Y, n, 32, Wl + PL_FF1, PL_LDFF1, 64, [&](int j, int o, float a, float b) {
+        hl_store2(Hh, j, o, gelu(a + Vl[VPL_FF1B + o]), gelu(b + Vl[VPL_FF1B + o + 1]));
+      });
     __syncthreads();
     gemm_hl(Hh, n, 64, Wl + PL_FF2, PL_LDFF2, 32, [&](int j, int o, float a, float b) {
       float2* z = reinterpret_cast<float2*>(Z + j * LDQ + o);
@@ -788,7 +797,13 @@ __global__ void __cluster_dims__(kDecideCluster, 1, 1) __launch_bounds__(kDecide
     }
     __syncthreads();
   }
-  if (rank != 0) return;  // no distributed shared-memory access after this point
+  // No distributed shared-memory access after this point.  Rank 0 makes the
+  // decision.  Ranks 1..7 make none: each runs a part of the LPS router, or
+  // the accept step, on a stand-in block of its own shared memory, skipping
+  // the block selection and writing nothing to global memory.  Every step
+  // starts with this kernel's code out of every cache; ahead of rank 0 and in
+  // parallel, those runs bring the code rank 0 is about to execute into L2.
+  const bool shadow = rank != 0;
 
   // ---------------------------------------------------------------- 4. block selection
   if (tid == 0 && !sm.lps_loaded && p.lps_enabled) {
@@ -799,7 +814,18 @@ __global__ void __cluster_dims__(kDecideCluster, 1, 1) __launch_bounds__(kDecide
     sm.lps_loaded = 1;
   }
   if (warp == 0) {
-    if (sm.meta_s == 0) {
+    if (shadow) {
+      // stand-in block: the first min(32, |M|) masked rows
+      const int nB = nM < 32 ? nM : 32;
+      for (int j = lane; j < nr; j += 32) sm.f_ib[j] = 0;
+      __syncwarp();
+      for (int k = lane; k < nB; k += 32) sm.f_ib[sm.Mrows[k]] = 1;
+      if (lane == 0 && nB > 0) {
+        sm.meta_b = sm.f_pos[sm.Mrows[0]];
+        sm.meta_s = nB;
+      }
+      __syncwarp();
+    } else if (sm.meta_s == 0) {
       for (int j = lane; j < nr; j += 32) sm.f_ib[j] = 0;
       __syncwarp();
       int nB = 0;
@@ -865,7 +891,9 @@ __global__ void __cluster_dims__(kDecideCluster, 1, 1) __launch_bounds__(kDecide
   if (sm.lps_loaded && !mbar_wait(&sm.bar2, 0, 1000ull * 1000 * 1000, nullptr))
     atomicCAS(p.status, 0, EBD_ERR_TIMEOUT);
   const int nBM = sm.nBM;
-  if (nBM > 0 && p.lps_enabled) {
+  // phase of the LPS router where a stand-in run starts (-1: accept only)
+  const int lps_from = !shadow ? 0 : (rank <= 4 ? rank - 1 : (rank == 5 ? 4 : (rank == 6 ? 6 : -1)));
+  if (nBM > 0 && p.lps_enabled && lps_from >= 0) {
     float* feats = P + L_FEAT;
     const float rho = static_cast<float>(nBM) / static_cast<float>(sm.meta_s);
 #pragma unroll 1
@@ -879,7 +907,7 @@ __global__ void __cluster_dims__(kDecideCluster, 1, 1) __launch_bounds__(kDecide
     }
     __syncthreads();
     const float* prob = P + L_PROB;
-    lps_forward(P, nBM, sm.w, sm.v + V_LPS);
+    lps_forward(P, nBM, sm.w, sm.v + V_LPS, lps_from);
 #pragma unroll 1
     for (int i = tid; i < nBM; i += blockDim.x) sm.f_p[sm.BMrows[i]] = prob[i];
     __syncthreads();
@@ -944,6 +972,7 @@ __global__ void __cluster_dims__(kDecideCluster, 1, 1) __launch_bounds__(kDecide
   __syncthreads();
 
   // ---------------------------------------------------------------- 6. write back
+  if (shadow) return;
   for (int j = tid; j < nr; j += blockDim.x) {
     const int r = r0 + j;
     p.tokens[r] = sm.f_tok[j];
