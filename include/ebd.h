@@ -243,6 +243,20 @@ const char* ebd_last_error(const ebd_handle* h);
 /* Library version string. */
 const char* ebd_version(void);
 
+/* Window of the next step of the generation loop (App. E algorithm in the
+ * block-forward setting of Sec. 6.4; a host function, no device work).
+ * Over the L response positions of one sequence with host arrays mask[L]
+ * and in_block[L] and the block state meta[2] = {b, |B|} (|B| = 0: no
+ * active block): f is the first masked position; with no active block the
+ * window is [f, min(f + max_window, L)), with an active block [f, max B + 1)
+ * where max B is the last position with in_block set.  Writes the window to
+ * *lo, *hi (relative positions); *lo = *hi = L when no position is masked.
+ * EBD_ERR_INVALID_ARG for a null pointer, L < 0 or max_window < 1;
+ * EBD_ERR_STATE for an active block with no in_block position, or a window
+ * longer than max_window. */
+ebd_status ebd_loop_window(const uint8_t* mask, const uint8_t* in_block, const int32_t* meta,
+                           int32_t L, int32_t max_window, int32_t* lo, int32_t* hi);
+
 /* ---- Allocation-free LM-head statistics ---------------------------------
  * No counterpart in the paper.  ebd_lm_stats_noalloc computes what
  * ebd_lm_stats computes (step 2: conf, entropy, ent_norm, gap, argmax of

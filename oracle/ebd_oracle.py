@@ -466,7 +466,8 @@ def generation_loop(shape, W, prm: DecisionParams, window_inputs, kv_rows,
             in_block[:] = 0
         commits.append(before - int(m.sum()))
         records.append(dict(step=steps, window=(lo, hi), accepted=d.accepted.copy(),
-                            flag=d.flag_accept, lbs_ran=d.lbs_ran, attn=attn))
+                            flag=d.flag_accept, flag_lbs=d.flag_lbs, lbs_ran=d.lbs_ran,
+                            attn=attn, stats=st))
         if on_step is not None:
             on_step(steps, records[-1])
         steps += 1

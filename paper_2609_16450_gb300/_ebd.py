@@ -53,7 +53,7 @@ EXPORTS = ["ebd_create", "ebd_destroy", "ebd_bind_embedding", "ebd_step", "ebd_s
            "ebd_export_weights", "ebd_import_weights", "ebd_router_init_host",
            "ebd_weight_count", "ebd_lm_head_packed_bytes", "ebd_pack_lm_head",
            "ebd_profile_enable", "ebd_profile_read", "ebd_last_error",
-           "ebd_version", "ebd_lm_stats_noalloc"]
+           "ebd_version", "ebd_lm_stats_noalloc", "ebd_loop_window"]
 
 _lib = None
 
@@ -97,6 +97,9 @@ def load(path: str = LIB_PATH):
                                          c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
                                          c_void_p, c_void_p]
     lib.ebd_lm_stats_noalloc.restype = c_int32
+    lib.ebd_loop_window.argtypes = [c_void_p, c_void_p, c_void_p, c_int32, c_int32, P(c_int32),
+                                    P(c_int32)]
+    lib.ebd_loop_window.restype = c_int32
     lib.ebd_version.restype = c_char_p
     for fn in EXPORTS:
         if getattr(lib, fn).restype is ctypes.c_int:
@@ -227,3 +230,16 @@ def ebd_lm_stats_noalloc(hidden_ptr: int, w_lm_ptr: int, w_lm_layout: int, rows:
                                        conf_ptr or None, entropy_ptr or None, ent_norm_ptr or None,
                                        gap_ptr or None, argmax_ptr or None, status_ptr or None,
                                        stream or None)
+
+
+def ebd_loop_window(mask, in_block, meta, max_window: int = 64):
+    """mask, in_block: host uint8 [L]; meta: host int32 [2].  Returns
+    (status, lo, hi)."""
+    import numpy as np
+    m = np.ascontiguousarray(mask, dtype=np.uint8)
+    ib = np.ascontiguousarray(in_block, dtype=np.uint8)
+    mt = np.ascontiguousarray(meta, dtype=np.int32)
+    lo, hi = c_int32(0), c_int32(0)
+    s = load().ebd_loop_window(m.ctypes.data, ib.ctypes.data, mt.ctypes.data, int(m.size),
+                               int(max_window), ctypes.byref(lo), ctypes.byref(hi))
+    return s, lo.value, hi.value

@@ -555,6 +555,40 @@ extern "C" {
 
 const char* ebd_version(void) { return "ebd 0.1 (sm_103a)"; }
 
+ebd_status ebd_loop_window(const uint8_t* mask, const uint8_t* in_block, const int32_t* meta,
+                           int32_t L, int32_t max_window, int32_t* lo, int32_t* hi) {
+  if (mask == nullptr || in_block == nullptr || meta == nullptr || lo == nullptr || hi == nullptr ||
+      L < 0 || max_window < 1)
+    return EBD_ERR_INVALID_ARG;
+  int32_t f = L;
+  for (int32_t i = 0; i < L; ++i)
+    if (mask[i]) {
+      f = i;
+      break;
+    }
+  if (f == L) {
+    *lo = *hi = L;
+    return EBD_OK;
+  }
+  int32_t end;
+  if (meta[1] == 0) {
+    end = f + max_window < L ? f + max_window : L;
+  } else {
+    int32_t last = -1;
+    for (int32_t i = L - 1; i >= 0; --i)
+      if (in_block[i]) {
+        last = i;
+        break;
+      }
+    if (last < 0) return EBD_ERR_STATE;
+    end = last + 1;
+    if (end <= f || end - f > max_window) return EBD_ERR_STATE;
+  }
+  *lo = f;
+  *hi = end;
+  return EBD_OK;
+}
+
 size_t ebd_weight_count(const ebd_config* cfg) {
   if (cfg == nullptr || cfg->d_base <= 0 || cfg->gen_len <= 0) return 0;
   return layout_count(router_layout(cfg->d_base, cfg->gen_len));

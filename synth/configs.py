@@ -78,7 +78,13 @@ loop_shape = Shape(name="loop_llada8b", batch=1, d_model=4096, vocab=126464,
                    windows=(64,), mask_frac=1.0, gen_len=256,
                    w_lm_std=1.0 / 64.0, seed=3)
 
-SHAPES = {s.name: s for s in (tiny, llada, dream, loop_shape)}
+# the generation loop at the tiny shape: prompt 64, gen 64 (the oracle runs the
+# whole loop in seconds)
+loop_tiny = Shape(name="loop_tiny", batch=1, d_model=256, vocab=4096, n_heads_q=4,
+                  n_heads_kv=4, head_dim=64, prefix=64, windows=(64,), mask_frac=1.0,
+                  gen_len=64, w_lm_std=0.02, seed=4)
+
+SHAPES = {s.name: s for s in (tiny, llada, dream, loop_shape, loop_tiny)}
 
 
 def sweep_points():
