@@ -81,15 +81,21 @@ def lm_kernel_hash():
 
 
 def profiled_traffic(workload):
-    """DRAM bytes per LM-head launch from a committed ncu summary, or None if
-    the kernel changed since the counters were taken."""
-    p = os.path.join(ROOT, "profiles", f"lm_head_{workload}.json")
+    """DRAM bytes per LM-head launch from the committed ncu summary
+    (profiles/lm_head_<workload>.md: lines "kernel_sha: ..." and
+    "dram_bytes_per_launch: ..."), or None if the kernel changed since the
+    counters were taken."""
+    p = os.path.join(ROOT, "profiles", f"lm_head_{workload}.md")
     try:
+        kv = {}
         with open(p) as f:
-            d = json.load(f)
-        if d.get("kernel_sha") != lm_kernel_hash():
+            for line in f:
+                if ":" in line and not line.startswith(("|", " ", "#")):
+                    k, v = line.split(":", 1)
+                    kv[k.strip()] = v.strip()
+        if kv.get("kernel_sha") != lm_kernel_hash():
             return None
-        return float(d["dram_bytes_per_launch"])
+        return float(kv["dram_bytes_per_launch"])
     except Exception:
         return None
 
