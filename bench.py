@@ -205,6 +205,24 @@ class L2Flush:
             self.r.sum()
 
 
+def max_over_ranks(x: float, world: int, device: str) -> float:
+    """The maximum of x over the ranks of the process group (x itself for one
+    rank): the step time of N independent replicas is the slowest one's."""
+    if world <= 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def replicas_value(rows_per_rank: int, world: int, t_step_s: float) -> float:
+    """Whole-job throughput of N replicas: positions of all ranks per second
+    of the slowest rank's step."""
+    return rows_per_rank * world / t_step_s
+
+
 def run_ours(args, rank, world, local_rank):
     import torch
     torch.cuda.set_device(local_rank)
@@ -293,11 +311,7 @@ def run_ours(args, rank, world, local_rank):
     if status != 0:
         raise SystemExit(f"device status {status}: {E.ebd_last_error(h.h)}")
     step_ms = [a.elapsed_time(b) for a, b in zip(ev0, ev1)]
-    mean_ms = float(np.mean(step_ms))
-    if world > 1:
-        t = torch.tensor([mean_ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        mean_ms = float(t.item())
+    mean_ms = max_over_ranks(float(np.mean(step_ms)), world, "cuda")
     kern = np.array(kern)
     k_lm, k_tail = float(np.mean(kern[:, 1])), float(np.mean(kern[:, 2]))
     # per-kernel breakdown outside the timed region: mode 1 runs the three
@@ -392,12 +406,7 @@ def run_e2e(args, h, ds, inp, sh, stream, world):
             times.append(e0.elapsed_time(e1))
     if h.sync_status(sid) != 0:
         raise SystemExit("device status after e2e")
-    mean_ms = float(np.mean(times))
-    if world > 1:
-        import torch.distributed as dist
-        t = torch.tensor([mean_ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        mean_ms = float(t.item())
+    mean_ms = max_over_ranks(float(np.mean(times)), world, "cuda")
     return dict(mean_ms=mean_ms, h2d=int(h2d), d2h=int(d2h))
 
 
@@ -534,7 +543,7 @@ def main():
     roof["peak_source"] = f"{peak_src} (MEASURED_PEAKS.json)" if peak_src == "measured" else "fallback"
     t_step = r["mean_ms"] / 1000.0
     t_roof = max(wk["step_bytes"] / (hbm * 1e9), wk["step_flops"] / (bf16 * 1e12))
-    value = r["rows"] * world / t_step
+    value = replicas_value(r["rows"], world, t_step)
     line = {
         "metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(r["mean_ms"], 5),
@@ -568,7 +577,7 @@ def main():
     }
     if r["e2e"] is not None:
         e = r["e2e"]
-        line["e2e"] = {"value": round(r["rows"] * world / (e["mean_ms"] / 1000.0), 1),
+        line["e2e"] = {"value": round(replicas_value(r["rows"], world, e["mean_ms"] / 1000.0), 1),
                        "unit": UNIT, "h2d_bytes_per_step": e["h2d"],
                        "d2h_bytes_per_step": e["d2h"], "ms_per_step": round(e["mean_ms"], 4),
                        "api": "ebd_step_host"}
