@@ -808,6 +808,7 @@ ebd_status ebd_step(ebd_handle* h, const ebd_step_args* a, void* stream) {
   if ((s = run_lm(h, a, st)) != EBD_OK) return s;
   if (prof && (e0 = record(h->ev[1], st)) != cudaSuccess) return cuda_fail(h, e0, "profile event");
   DecideParams p = decide_params(h, a, 0);
+  p.pdl = prof == 0 ? 1 : 0;  // no event between the LM head and the decision
   cudaError_t e = launch_decide(p, st);
   if (e != cudaSuccess) return cuda_fail(h, e, "decision launch");
   if (prof == 1 && (e0 = record(h->ev[2], st)) != cudaSuccess)

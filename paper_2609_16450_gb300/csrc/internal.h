@@ -67,6 +67,7 @@ struct RouterImage {
 struct DecideParams {
   int B, V, grid_lm;        // grid_lm: LM-head partials per row
   int features_in;          // 1: conf/ent_norm/gap/argmax are inputs
+  int pdl;                  // launched as a programmatic dependent of the LM head
   int gen_len, g_max, l_min, l_b, eos_id, lps_enabled;
   float tau, tau_psi, inv_log_v;
   const int* cu_rows;

@@ -560,6 +560,11 @@ __global__ void __cluster_dims__(kDecideCluster, 1, 1) __launch_bounds__(kDecide
   }
 
   // ---------------------------------------------------------------- 1. statistics
+  // Launched as a programmatic dependent of the LM head, the kernel may start
+  // while the LM head's last CTAs run: everything above (weights in flight,
+  // decode state loaded) overlaps them; the partial states are read only
+  // after the LM head's grid has completed and its writes are visible.
+  asm volatile("griddepcontrol.wait;" ::: "memory");
   if (p.features_in) {
 #pragma unroll 1
     for (int j = tid; j < nr; j += blockDim.x) {
@@ -1077,8 +1082,17 @@ cudaError_t decide_configure() {
 
 cudaError_t launch_decide(const DecideParams& p, cudaStream_t st) {
   if (p.B <= 0) return cudaSuccess;
-  decide_kernel<<<p.B * kDecideCluster, kDecideThreads, sizeof(Smem) + 16, st>>>(p);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = dim3(p.B * kDecideCluster, 1, 1);
+  cfg.blockDim = dim3(kDecideThreads, 1, 1);
+  cfg.dynamicSmemBytes = sizeof(Smem) + 16;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = p.pdl ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, decide_kernel, p);
 }
 
 cudaError_t launch_fold_tok(const __nv_bfloat16* w_tok, const __nv_bfloat16* w_emb, float* table,

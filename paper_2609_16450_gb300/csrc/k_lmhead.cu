@@ -122,6 +122,10 @@ __global__ void __launch_bounds__(kLmThreads, 1)
   volatile int* abort = reinterpret_cast<volatile int*>(tmem_holder + 1);
 
   const int tid = threadIdx.x;
+  // the decision kernel, launched after this one as a programmatic dependent,
+  // may be scheduled as soon as SMs free up; it waits for this grid's
+  // completion before it reads the partial states
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   const int warp = __shfl_sync(0xffffffffu, tid / 32, 0);
   const int lane = tid & 31;
   const int cta = blockIdx.x;
