@@ -59,20 +59,25 @@ __device__ __forceinline__ bool named_barrier_and(uint32_t id, uint32_t n, bool 
   return r != 0;
 }
 
-// MMAs of one full pipeline stage: KBS k-boxes x 4 k16 steps into one
-// accumulator, descriptors advanced by immediates (k16 step = 32 bytes = 2 in
-// the descriptor's address field; k-box = kATile bytes of A, b_step of B).
-template <int KBS>
+// MMAs of one pipeline stage: KBS k-boxes x 4 k16 steps x NSUB N sub-tiles,
+// descriptors advanced by immediates (k16 step = 32 bytes = 2 in the
+// descriptor's address field; k-box = kATile bytes of A, b_step of B; N
+// sub-tile sb at sb * sub_desc of B and sb * sub_cols TMEM columns).
+template <int KBS, int NSUB>
 __device__ __forceinline__ void mma_stage(uint32_t d, uint32_t a_lo, uint32_t b_lo,
-                                          uint32_t b_step, uint32_t hi, uint32_t idesc,
-                                          uint32_t acc0) {
+                                          uint32_t b_step, uint32_t sub_desc, uint32_t sub_cols,
+                                          uint32_t hi, uint32_t idesc, uint32_t acc0) {
 #pragma unroll
   for (int j = 0; j < KBS; ++j)
 #pragma unroll
     for (int kk = 0; kk < 4; ++kk)
-      umma_bf16_lo(d, a_lo + static_cast<uint32_t>(j * (kATile >> 4) + kk * 2),
-                   b_lo + static_cast<uint32_t>(j) * b_step + static_cast<uint32_t>(kk * 2), hi,
-                   idesc, (j | kk) != 0 ? 1u : acc0);
+#pragma unroll
+      for (int sb = 0; sb < NSUB; ++sb)
+        umma_bf16_lo(d + static_cast<uint32_t>(sb) * sub_cols,
+                     a_lo + static_cast<uint32_t>(j * (kATile >> 4) + kk * 2),
+                     b_lo + static_cast<uint32_t>(j) * b_step + static_cast<uint32_t>(sb) * sub_desc +
+                         static_cast<uint32_t>(kk * 2),
+                     hi, idesc, (j | kk) != 0 ? 1u : acc0);
 }
 
 // Waits with a back-off between polls: for warps whose wait is long and not
@@ -239,19 +244,33 @@ __global__ void __launch_bounds__(kLmThreads, 1)
           const int nsubk = min(p.kbs, p.nkb - ks * p.kbs);
           const uint32_t a_addr = smem_u32(sA + static_cast<size_t>(s) * a_stage);
           const uint32_t b_addr = smem_u32(sB + static_cast<size_t>(s) * b_stage);
-          if (p.nsub == 1 && nsubk >= 1 && nsubk <= 5) {
-            // one N sub-tile: the unrolled issue path
+          if (p.nsub <= 2 && nsubk >= 1 && nsubk <= 5) {
+            // the unrolled issue path
             const uint32_t a_lo = static_cast<uint32_t>(umma_desc_sw128(a_addr));
             const uint32_t b_lo = static_cast<uint32_t>(umma_desc_sw128(b_addr));
             const uint32_t b_step = b_sub >> 4;
+            const uint32_t sub_desc = static_cast<uint32_t>(p.nb) * 8u;  // nb rows x 128 B >> 4
+            const uint32_t sub_cols = static_cast<uint32_t>(p.nb);
             const uint32_t acc0 = ks != 0 ? 1u : 0u;
-            switch (nsubk) {
-              case 1: mma_stage<1>(d0, a_lo, b_lo, b_step, desc_hi, idesc, acc0); break;
-              case 2: mma_stage<2>(d0, a_lo, b_lo, b_step, desc_hi, idesc, acc0); break;
-              case 3: mma_stage<3>(d0, a_lo, b_lo, b_step, desc_hi, idesc, acc0); break;
-              case 4: mma_stage<4>(d0, a_lo, b_lo, b_step, desc_hi, idesc, acc0); break;
-              default: mma_stage<5>(d0, a_lo, b_lo, b_step, desc_hi, idesc, acc0); break;
+#define EBD_STAGE(K, S) mma_stage<K, S>(d0, a_lo, b_lo, b_step, sub_desc, sub_cols, desc_hi, idesc, acc0)
+            if (p.nsub == 1) {
+              switch (nsubk) {
+                case 1: EBD_STAGE(1, 1); break;
+                case 2: EBD_STAGE(2, 1); break;
+                case 3: EBD_STAGE(3, 1); break;
+                case 4: EBD_STAGE(4, 1); break;
+                default: EBD_STAGE(5, 1); break;
+              }
+            } else {
+              switch (nsubk) {
+                case 1: EBD_STAGE(1, 2); break;
+                case 2: EBD_STAGE(2, 2); break;
+                case 3: EBD_STAGE(3, 2); break;
+                case 4: EBD_STAGE(4, 2); break;
+                default: EBD_STAGE(5, 2); break;
+              }
             }
+#undef EBD_STAGE
             umma_commit(&empty[s]);
             ++it;
             continue;
@@ -326,18 +345,16 @@ __global__ void __launch_bounds__(kLmThreads, 1)
           float x[32];
 #pragma unroll
           for (int i = 0; i < 32; ++i) x[i] = sT[j * kTLd + q + 4 * i];
+          // branch-free scan: the threads of a warp see different data
           float m = -INFINITY, l2 = -INFINITY;
-          int idx = INT_MAX;
+          int ii = -1;
 #pragma unroll
           for (int i = 0; i < 32; ++i) {
-            if (x[i] > m) {
-              l2 = m;
-              m = x[i];
-              idx = vbase + q + 4 * i;
-            } else if (x[i] > l2) {
-              l2 = x[i];
-            }
+            l2 = fmaxf(l2, fminf(m, x[i]));
+            ii = x[i] > m ? i : ii;  // strict: the first (lowest) index of the maximum
+            m = fmaxf(m, x[i]);
           }
+          int idx = ii < 0 ? INT_MAX : vbase + q + 4 * ii;
           float s = 0.f, t = 0.f;
           if (m != -INFINITY) {
 #pragma unroll
@@ -345,7 +362,7 @@ __global__ void __launch_bounds__(kLmThreads, 1)
               const float dl = x[i] - m;
               const float e = __expf(dl);
               s += e;
-              if (e > 0.f) t = fmaf(e, dl, t);  // masked lanes: e = 0, dl = -inf
+              t = fmaf(e, e > 0.f ? dl : 0.f, t);  // masked lanes: e = 0, dl = -inf
             }
           }
 #pragma unroll
