@@ -11,7 +11,7 @@ namespace ebd {
 
 constexpr int kMaxWindow = 64;        // window rows per sequence
 constexpr int kUnit = 64;             // vocabulary rows per work unit of the LM head
-constexpr int kLmThreads = 192;       // TMA warp, MMA warp, 4 epilogue warps
+constexpr int kLmThreads = 320;  // TMA warp, MMA warp, two epilogue warpgroups of 4 warps
 constexpr int kMaxGroupRows = 512;    // rows per LM-head launch (TMEM: 512 columns)
 constexpr int kDecideCluster = 8;     // CTAs per sequence in the decision kernel
 constexpr int kDecideThreads = 256;
@@ -31,6 +31,7 @@ struct LmParams {
   int kbs, nks;             // k-blocks per pipeline stage, stages per vocabulary chunk
   int packed;               // W is tiled: tile (unit, k-block) at row (unit*nkb + kb)*64
   int stages, nbuf, acc_stride, tmem_cols;
+  int nwg;                  // epilogue warpgroups in use (1, or 2 for more than 32 rows)
   uint32_t off_a, off_b, off_t, off_st, off_bar, smem_bytes;
   float4* part_f;           // [R][grid] (max, sum exp, sum exp*(l-max), second logit)
   int* part_i;              // [R][grid] argmax

@@ -142,7 +142,7 @@ __global__ void __launch_bounds__(kLmThreads, 1)
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&acc_full[b], 1);
-      mbar_init(&acc_empty[b], 128);
+      mbar_init(&acc_empty[b], 128 * p.nwg);
     }
     mbar_init(drain, 1);
     mbar_init(dummy, 1);
@@ -153,7 +153,7 @@ __global__ void __launch_bounds__(kLmThreads, 1)
   }
   if (warp == 1) tmem_alloc(tmem_holder, p.tmem_cols);
   if (tid >= 64) {
-    for (int r = tid - 64; r < p.n_pad; r += 128) {
+    for (int r = tid - 64; r < p.n_pad; r += kLmThreads - 64) {
       st_m[r] = -INFINITY;
       st_s[r] = 0.f;
       st_t[r] = 0.f;
@@ -301,15 +301,22 @@ __global__ void __launch_bounds__(kLmThreads, 1)
     }
   } else {
     // ------------------------------------------------------------ epilogue
-    const int et = tid - 64;         // 0..127
-    const int quad = warp & 3;       // TMEM lane quadrant this warp may read
+    // p.nwg warpgroups of 4 warps (one per TMEM lane quadrant) take the
+    // 32-row column slices of the accumulator in turn; a second warpgroup is
+    // used when the accumulator is wider than one slice.
+    const int wg = (tid - 64) >> 7;
+    const int et = (tid - 64) & 127;  // thread within the warpgroup
+    const int quad = warp & 3;        // TMEM lane quadrant this warp may read
     const int lanev = quad * 32 + lane;
-    bool ok = true;
-    if (p.force_timeout) {
+    const uint32_t bar_id = 1u + static_cast<uint32_t>(wg);
+    float* const sTw = sT + wg * (kTBytes / 4);
+    bool ok = wg < p.nwg;
+    if (ok && p.force_timeout) {
       ok = mbar_wait(dummy, 0, 20ull * 1000 * 1000, nullptr);
-      ok = named_barrier_and(1, 128, ok);
-      if (!ok && et == 0) record_error(p.status, abort, EBD_ERR_TIMEOUT);
+      ok = named_barrier_and(bar_id, 128, ok);
+      if (!ok && et == 0 && wg == 0) record_error(p.status, abort, EBD_ERR_TIMEOUT);
     }
+    const bool active = ok;
     int c = 0;
     for (int u = u0; u < u1 && ok; u += 2, ++c) {
       const int nu = min(2, u1 - u);
@@ -317,14 +324,15 @@ __global__ void __launch_bounds__(kLmThreads, 1)
       const int buf = c % p.nbuf;
       const uint32_t bph = static_cast<uint32_t>(c / p.nbuf) & 1u;
       bool w = mbar_wait_sleepy(&acc_full[buf], bph, p.limit_ns, abort);
-      ok = named_barrier_and(1, 128, w);
+      ok = named_barrier_and(bar_id, 128, w);
       if (!ok) {
         if (et == 0 && !*abort) record_error(p.status, abort, EBD_ERR_TIMEOUT);
         break;
       }
       tc_fence_after();
       const int vbase = u * kUnit;
-      for (int cc = 0; cc < p.n_pad; cc += 32) {
+      bool released = false;
+      for (int cc = 32 * wg; cc < p.n_pad; cc += 32 * p.nwg) {
         float v[32];
         const uint32_t taddr = tmem_base + (static_cast<uint32_t>(quad * 32) << 16) +
                                static_cast<uint32_t>(buf * p.acc_stride + cc);
@@ -332,19 +340,20 @@ __global__ void __launch_bounds__(kLmThreads, 1)
           tmem_ld_32x32b_x32(taddr, v);
         else
           tmem_ld_32x32b_x16(taddr, v);
-        if (cc + 32 >= p.n_pad) {
+        if (cc + 32 * p.nwg >= p.n_pad) {  // this warpgroup's last slice is in registers
           tc_fence_before();
           mbar_arrive(&acc_empty[buf]);
+          released = true;
         }
         const bool lv = lanev < valid;
 #pragma unroll
-        for (int j = 0; j < 32; ++j) sT[j * kTLd + lanev] = lv ? v[j] : -INFINITY;
-        named_barrier(1, 128);
+        for (int j = 0; j < 32; ++j) sTw[j * kTLd + lanev] = lv ? v[j] : -INFINITY;
+        named_barrier(bar_id, 128);
         {
           const int j = et >> 2, q = et & 3;
           float x[32];
 #pragma unroll
-          for (int i = 0; i < 32; ++i) x[i] = sT[j * kTLd + q + 4 * i];
+          for (int i = 0; i < 32; ++i) x[i] = sTw[j * kTLd + q + 4 * i];
           // branch-free scan: the threads of a warp see different data
           float m = -INFINITY, l2 = -INFINITY;
           int ii = -1;
@@ -386,11 +395,17 @@ __global__ void __launch_bounds__(kLmThreads, 1)
             st_i[r] = I;
           }
         }
-        named_barrier(1, 128);
+        named_barrier(bar_id, 128);
+      }
+      if (!released) {  // no slice of this chunk for this warpgroup
+        tc_fence_before();
+        mbar_arrive(&acc_empty[buf]);
       }
     }
-    if (ok) {
+    if (ok && active) {
+      // the rows of this warpgroup's slices (its threads updated them last)
       for (int r = et; r < p.rows; r += 128) {
+        if (((r >> 5) % p.nwg) != wg) continue;
         const size_t o = static_cast<size_t>(p.row0 + r) * p.grid + cta;
         p.part_f[o] = make_float4(st_m[r], st_s[r], st_t[r], st_l2[r]);
         p.part_i[o] = st_i[r];
@@ -423,8 +438,10 @@ void lm_plan(LmParams& p, int rows, int V, int d, int num_sms) {
   p.n_units = (V + kUnit - 1) / kUnit;
   p.grid = num_sms < p.n_units ? num_sms : p.n_units;
   p.nkb = (d + 63) / 64;
+  p.nwg = p.n_pad > 32 ? 2 : 1;
   const uint32_t st_bytes = static_cast<uint32_t>(p.n_pad) * 20u;
-  const uint32_t tail = kTBytes + ((st_bytes + 7) / 8 * 8) + (2 * 8 + 6) * 8 + 16;
+  const uint32_t tail = kTBytes * static_cast<uint32_t>(p.nwg) + ((st_bytes + 7) / 8 * 8) +
+                        (2 * 8 + 6) * 8 + 16;
   const uint32_t budget = 232448u - 1024u - tail;
   // k-boxes (64 columns each) per pipeline stage: longer contiguous runs of
   // each W row per request, while keeping at least two stages in flight
@@ -442,7 +459,7 @@ void lm_plan(LmParams& p, int rows, int V, int d, int num_sms) {
   p.off_a = 0;
   p.off_b = p.off_a + static_cast<uint32_t>(stages) * kbs * kATile;
   p.off_t = p.off_b + static_cast<uint32_t>(stages) * kbs * static_cast<uint32_t>(p.n_pad) * 128u;
-  p.off_st = p.off_t + kTBytes;
+  p.off_st = p.off_t + kTBytes * static_cast<uint32_t>(p.nwg);
   p.off_bar = (p.off_st + st_bytes + 7) / 8 * 8;
   p.smem_bytes = p.off_bar + static_cast<uint32_t>(2 * stages + 6) * 8u + 16u + 1024u;
 }
