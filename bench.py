@@ -441,6 +441,50 @@ def oracle_step_sample(sh, inp, budget_s):
     return inp.rows * n / el, n, el
 
 
+def run_loop_bench(args):
+    """The generation loop (configs loop_*): one untimed loop, then
+    max(1, steps // 100) timed loops to completion; reports the number of
+    steps, the device time of all steps (CUDA events around every ebd_step)
+    and the wall time including the per-step host work (synthetic backbone
+    outputs, window rule, state read-back)."""
+    import torch
+    from paper_2609_16450_gb300 import build as B
+    B.build()
+    from paper_2609_16450_gb300 import loop as lp
+    from paper_2609_16450_gb300 import runtime as rt
+    import synth
+    sh = shape_for(args.config)
+    inp = synth.make_step_inputs(sh)
+    w = rt.upload_weights(inp)
+    h = rt.Handle(lp.config_for_loop(sh), w.w_emb)
+    if args.w_layout == "packed":
+        w = rt.pack_weights(h, w)
+    win = lambda s, p: synth.loop_window_inputs(sh, s, p)
+    kv = lambda p: synth.loop_kv(sh, p)
+    lp.run_loop(h, sh, w, win, kv, keep=False)  # warm-up loop
+    runs = []
+    for _ in range(max(1, args.steps // 100)):
+        t0 = time.perf_counter()
+        res = lp.run_loop(h, sh, w, win, kv, keep=False)
+        runs.append((res.steps, res.device_us, time.perf_counter() - t0))
+    steps = runs[0][0]
+    dev_us = float(np.mean([r[1] for r in runs]))
+    wall_s = float(np.mean([r[2] for r in runs]))
+    wk_rows = sh.gen_len
+    line = {"metric": "generation loop: steps and total time (LLaDA-8B shape)",
+            "value": round(wk_rows / (dev_us * 1e-6), 1), "unit": "positions/s",
+            "n_gpus": 1, "steps": len(runs), "warmup": 1, "ms_per_step": round(dev_us / steps / 1000, 5),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+            "data": "synthetic (seeded per step and position)",
+            "config": {"workload": f"{sh.name}: prompt {sh.prefix}, gen {sh.gen_len}, windows of "
+                                   f"at most 64 rows, attention over the committed prefix",
+                       "loop_steps": steps, "device_us_total": round(dev_us, 1),
+                       "wall_s_total": round(wall_s, 3),
+                       "l2": "not flushed between steps (consecutive steps of one loop)"}}
+    h.close()
+    print(json.dumps(line))
+
+
 def run_reference(args, rank, world):
     """The CPU oracle as the reference arm: rank 0 only."""
     if rank != 0:
@@ -521,6 +565,10 @@ def main():
     local_rank = int(os.environ.get("LOCAL_RANK", "0"))
     if args.impl == "reference":
         run_reference(args, rank, world)
+        return
+    if args.config.startswith("loop_"):
+        if rank == 0:
+            run_loop_bench(args)
         return
     import torch
     if world > 1:
