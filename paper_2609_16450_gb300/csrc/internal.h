@@ -32,6 +32,9 @@ struct LmParams {
   int packed;               // W is tiled: tile (unit, k-block) at row (unit*nkb + kb)*64
   int stages, nbuf, acc_stride, tmem_cols;
   int nwg;                  // epilogue warpgroups in use (1, or 2 for more than 32 rows)
+  int pair;                 // clusters of 2 CTAs: W multicast, rows split in halves
+  int rhalf;                // rows of one CTA of a pair (rows of the launch otherwise)
+  int ncols;                // partial states per row written (>= grid; extra ones neutral)
   uint32_t off_a, off_b, off_t, off_st, off_bar, smem_bytes;
   float4* part_f;           // [R][grid] (max, sum exp, sum exp*(l-max), second logit)
   int* part_i;              // [R][grid] argmax
@@ -90,7 +93,7 @@ struct DecideParams {
 // host launchers (defined next to their kernels)
 cudaError_t launch_lm_stats(const CUtensorMap& tmap_w, const CUtensorMap& tmap_h,
                             const LmParams& p, cudaStream_t st);
-void lm_plan(LmParams& p, int rows, int V, int d, int num_sms);
+void lm_plan(LmParams& p, int rows, int V, int d, int num_sms, bool pair = false);
 // pdl: launched as a programmatic dependent of the kernel before it on
 // `st` (that kernel's CTAs release it early; the attention reads nothing the
 // earlier kernel writes)

@@ -133,12 +133,18 @@ __global__ void __launch_bounds__(kLmThreads, 1)
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   const int warp = __shfl_sync(0xffffffffu, tid / 32, 0);
   const int lane = tid & 31;
-  const int cta = blockIdx.x;
+  // paired mode: the two CTAs of a cluster share a vocabulary range; each
+  // loads one of the two W units of a chunk and multicasts it to both, and
+  // accumulates half of the window rows
+  const uint32_t crank = p.pair ? cluster_ctarank() : 0u;
+  const int cta = p.pair ? static_cast<int>(blockIdx.x >> 1) : static_cast<int>(blockIdx.x);
+  const int rbase = p.row0 + static_cast<int>(crank) * p.rhalf;  // first row of this CTA
+  const int rows_c = min(p.rhalf, p.rows - static_cast<int>(crank) * p.rhalf);
 
   if (tid == 0) {
     for (int s = 0; s < p.stages; ++s) {
       mbar_init(&full[s], 1);
-      mbar_init(&empty[s], 1);
+      mbar_init(&empty[s], p.pair ? 2 : 1);  // paired: both CTAs' MMAs release a stage
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&acc_full[b], 1);
@@ -162,7 +168,10 @@ __global__ void __launch_bounds__(kLmThreads, 1)
     }
   }
   tc_fence_before();
-  __syncthreads();
+  if (p.pair)
+    cluster_sync_all();  // the peer's barriers exist before anything is multicast to them
+  else
+    __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_holder;
 
@@ -195,17 +204,23 @@ __global__ void __launch_bounds__(kLmThreads, 1)
           uint8_t* b_st = sB + static_cast<size_t>(s) * b_stage;
           // one row half at a time, its k-boxes back to back: each W row is
           // requested as one contiguous run of nsubk * 128 bytes
-          for (int ui = 0; ui < nu; ++ui)
-            for (int j = 0; j < nsubk; ++j)
-              tma_load_2d(a_st + j * kATile + ui * (kUnit * 128), &tmap_w, &full[s],
-                          p.packed ? 0 : (ks * p.kbs + j) * 64,
-                          p.packed ? ((u + ui) * p.nkb + ks * p.kbs + j) * kUnit
-                                   : (u + ui) * kUnit,
-                          pol_w);
+          for (int ui = 0; ui < nu; ++ui) {
+            if (p.pair && ui != static_cast<int>(crank)) continue;  // the peer loads it
+            for (int j = 0; j < nsubk; ++j) {
+              const int x = p.packed ? 0 : (ks * p.kbs + j) * 64;
+              const int y = p.packed ? ((u + ui) * p.nkb + ks * p.kbs + j) * kUnit
+                                     : (u + ui) * kUnit;
+              uint8_t* dst = a_st + j * kATile + ui * (kUnit * 128);
+              if (p.pair)
+                tma_load_2d_multicast(dst, &tmap_w, &full[s], x, y, 0x3, pol_w);
+              else
+                tma_load_2d(dst, &tmap_w, &full[s], x, y, pol_w);
+            }
+          }
           for (int j = 0; j < nsubk; ++j)
             for (int sb = 0; sb < p.nsub; ++sb)
               tma_load_2d(b_st + j * b_sub + sb * p.nb * 128, &tmap_h, &full[s],
-                          (ks * p.kbs + j) * 64, p.row0 + sb * p.nb, pol_h);
+                          (ks * p.kbs + j) * 64, rbase + sb * p.nb, pol_h);
           ++it;
         }
       }
@@ -271,7 +286,10 @@ __global__ void __launch_bounds__(kLmThreads, 1)
               }
             }
 #undef EBD_STAGE
-            umma_commit(&empty[s]);
+            if (p.pair)
+              umma_commit_multicast(&empty[s], 0x3);
+            else
+              umma_commit(&empty[s]);
             ++it;
             continue;
           }
@@ -287,7 +305,10 @@ __global__ void __launch_bounds__(kLmThreads, 1)
               }
             }
           }
-          umma_commit(&empty[s]);
+          if (p.pair)
+              umma_commit_multicast(&empty[s], 0x3);
+            else
+              umma_commit(&empty[s]);
           ++it;
         }
         if (!ok) break;
@@ -403,30 +424,40 @@ __global__ void __launch_bounds__(kLmThreads, 1)
       }
     }
     if (ok && active) {
-      // the rows of this warpgroup's slices (its threads updated them last)
-      for (int r = et; r < p.rows; r += 128) {
+      // the rows of this warpgroup's slices (its threads updated them last);
+      // in paired mode the pair's partial goes to column cta and a neutral
+      // state to column grid + cta, so that every row has ncols partials
+      for (int r = et; r < rows_c; r += 128) {
         if (((r >> 5) % p.nwg) != wg) continue;
-        const size_t o = static_cast<size_t>(p.row0 + r) * p.grid + cta;
+        const size_t o = static_cast<size_t>(rbase + r) * p.ncols + cta;
         p.part_f[o] = make_float4(st_m[r], st_s[r], st_t[r], st_l2[r]);
         p.part_i[o] = st_i[r];
+        for (int jc = p.grid + cta; jc < p.ncols; jc += p.grid) {  // neutral states
+          p.part_f[o - cta + jc] = make_float4(-INFINITY, 0.f, 0.f, -INFINITY);
+          p.part_i[o - cta + jc] = INT_MAX;
+        }
       }
     }
   }
 
   __syncthreads();
+  if (p.pair) cluster_sync_all();  // no multicast or remote arrival can target a CTA that left
   if (warp == 1) {
     tc_fence_after();
     tmem_dealloc(tmem_base, p.tmem_cols);
   }
 }
 
-void lm_plan(LmParams& p, int rows, int V, int d, int num_sms) {
+void lm_plan(LmParams& p, int rows, int V, int d, int num_sms, bool pair) {
   p.V = V;
   p.d = d;
   p.rows = rows;
-  p.nsub = (rows + 255) / 256;
+  p.pair = pair ? 1 : 0;
+  p.rhalf = pair ? (rows + 1) / 2 : rows;
+  const int rc = p.rhalf;  // rows one CTA accumulates
+  p.nsub = (rc + 255) / 256;
   if (p.nsub < 1) p.nsub = 1;
-  p.nb = ((rows + p.nsub - 1) / p.nsub + 15) / 16 * 16;
+  p.nb = ((rc + p.nsub - 1) / p.nsub + 15) / 16 * 16;
   if (p.nb < 16) p.nb = 16;
   p.n_pad = p.nb * p.nsub;
   p.acc_stride = (p.n_pad + 31) / 32 * 32;
@@ -437,6 +468,11 @@ void lm_plan(LmParams& p, int rows, int V, int d, int num_sms) {
   p.tmem_cols = tc;
   p.n_units = (V + kUnit - 1) / kUnit;
   p.grid = num_sms < p.n_units ? num_sms : p.n_units;
+  p.ncols = p.grid;  // partial states per row: the same in both modes
+  if (pair) {         // one pair per two SMs; each pair leaves one partial per row
+    p.grid = num_sms / 2 < p.n_units ? num_sms / 2 : p.n_units;
+    if (p.grid < 1) p.grid = 1;
+  }
   p.nkb = (d + 63) / 64;
   p.nwg = p.n_pad > 32 ? 2 : 1;
   const uint32_t st_bytes = static_cast<uint32_t>(p.n_pad) * 20u;
@@ -511,8 +547,19 @@ cudaError_t lm_configure() {
 
 cudaError_t launch_lm_stats(const CUtensorMap& tmap_w, const CUtensorMap& tmap_h,
                             const LmParams& p, cudaStream_t st) {
-  lm_stats_kernel<<<p.grid, kLmThreads, p.smem_bytes, st>>>(tmap_w, tmap_h, p);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = dim3(p.pair ? 2 * p.grid : p.grid, 1, 1);
+  cfg.blockDim = dim3(kLmThreads, 1, 1);
+  cfg.dynamicSmemBytes = p.smem_bytes;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = p.pair ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, lm_stats_kernel, tmap_w, tmap_h, p);
 }
 
 }  // namespace ebd
