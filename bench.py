@@ -456,16 +456,17 @@ def run_loop_bench(args):
     sh = shape_for(args.config)
     inp = synth.make_step_inputs(sh)
     w = rt.upload_weights(inp)
-    h = rt.Handle(lp.config_for_loop(sh), w.w_emb)
+    mode = {"eb": 0, "threshold": 1, "topm": 2}[args.decode]
+    h = rt.Handle(lp.config_for_loop(sh, decode_mode=mode, top_m=args.top_m), w.w_emb)
     if args.w_layout == "packed":
         w = rt.pack_weights(h, w)
     win = lambda s, p: synth.loop_window_inputs(sh, s, p)
     kv = lambda p: synth.loop_kv(sh, p)
-    lp.run_loop(h, sh, w, win, kv, keep=False)  # warm-up loop
+    lp.run_loop(h, sh, w, win, kv, keep=False, block=sh.l_b)  # warm-up loop
     runs = []
     for _ in range(max(1, args.steps // 100)):
         t0 = time.perf_counter()
-        res = lp.run_loop(h, sh, w, win, kv, keep=False)
+        res = lp.run_loop(h, sh, w, win, kv, keep=False, block=sh.l_b)
         runs.append((res.steps, res.device_us, time.perf_counter() - t0))
     steps = runs[0][0]
     dev_us = float(np.mean([r[1] for r in runs]))
@@ -478,6 +479,8 @@ def run_loop_bench(args):
             "data": "synthetic (seeded per step and position)",
             "config": {"workload": f"{sh.name}: prompt {sh.prefix}, gen {sh.gen_len}, windows of "
                                    f"at most 64 rows, attention over the committed prefix",
+                       "decode": args.decode + (f" (m={args.top_m})" if args.decode == "topm" else ""),
+                       "fixed_block": sh.l_b if args.decode != "eb" else None,
                        "loop_steps": steps, "device_us_total": round(dev_us, 1),
                        "wall_s_total": round(wall_s, 3),
                        "l2": "not flushed between steps (consecutive steps of one loop)"}}
@@ -555,6 +558,9 @@ def main():
     ap.add_argument("--skip-e2e", action="store_true", help="omit the end-to-end leg")
     ap.add_argument("--no-graph", action="store_true", help="launch ebd_step without a graph")
     ap.add_argument("--cpu-budget", type=float, default=12.0)
+    ap.add_argument("--decode", choices=["eb", "threshold", "topm"], default="eb",
+                    help="decision of the loop configs: EB, or a baseline's fixed-block rule")
+    ap.add_argument("--top-m", type=int, default=1, help="commits per step of --decode topm")
     ap.add_argument("--w-layout", choices=["packed", "rowmajor"], default="packed",
                     help="W_lm tiled once by ebd_pack_lm_head (default) or row-major")
     args = ap.parse_args()

@@ -64,6 +64,19 @@ typedef int32_t ebd_status;
 #define EBD_ERR_NONFINITE (-5)   /* NaN/Inf logit statistic; row not committed */
 #define EBD_ERR_STATE (-6)       /* call order: e.g. LBS needs a bound W_e   */
 
+/* decode_mode: which decision step 3 applies.  EBD_DECODE_EB is the EB
+ * decision (LBS + LPS, App. E).  The other two are the fixed-block update
+ * of the baselines (App. B, Eq. prelim-update) on the rows of the window,
+ * which the caller sets to the active fixed block (see
+ * ebd_loop_block_window); the routers do not run and the block state is
+ * left untouched.  THRESHOLD commits the masked rows with kappa >= tau, or
+ * the one with the highest kappa when none reaches tau (Fast-dLLM's rule).
+ * TOPM commits the min(top_m, |M|) masked rows with the highest kappa (the
+ * vanilla budget rule); ties go to the lower position in both. */
+#define EBD_DECODE_EB 0
+#define EBD_DECODE_THRESHOLD 1
+#define EBD_DECODE_TOPM 2
+
 /* debug_flags bits (tests only) */
 #define EBD_DEBUG_FORCE_TIMEOUT 1 /* LM-head kernel waits on a barrier that
                                      nothing completes, with a 20 ms limit */
@@ -92,6 +105,8 @@ typedef struct {
   float tau_psi;       /* LPS acceptance threshold (0.89 / 0.90 / 0.87)     */
   uint64_t seed;       /* seed of the routers' random init                  */
   int32_t debug_flags; /* EBD_DEBUG_* (tests); 0 in normal use              */
+  int32_t decode_mode; /* EBD_DECODE_*: EB decision or a baseline rule      */
+  int32_t top_m;       /* EBD_DECODE_TOPM: commits per step (>= 1)          */
   int32_t reserved;
 } ebd_config;
 
@@ -256,6 +271,14 @@ const char* ebd_version(void);
  * longer than max_window. */
 ebd_status ebd_loop_window(const uint8_t* mask, const uint8_t* in_block, const int32_t* meta,
                            int32_t L, int32_t max_window, int32_t* lo, int32_t* hi);
+
+/* Window of the next step under the baselines' fixed blocks (App. B): the
+ * first block [jB, jB + B) of the L response positions (host array mask[L])
+ * that still holds a masked position, clipped to L.  *lo = *hi = L when none
+ * does.  EBD_ERR_INVALID_ARG for a null pointer, L < 0 or block < 1.  A host
+ * function, no device work. */
+ebd_status ebd_loop_block_window(const uint8_t* mask, int32_t L, int32_t block, int32_t* lo,
+                                 int32_t* hi);
 
 /* ---- Allocation-free LM-head statistics ---------------------------------
  * No counterpart in the paper.  ebd_lm_stats_noalloc computes what

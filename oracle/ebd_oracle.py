@@ -51,6 +51,14 @@ where it is used):
   R14 kappa >= tau is inclusive; p_psi > tau_psi is strict; the anti-stall
       fallback takes the lowest position among equal kappa.
   R15 a router that does not run leaves NaN in its per-row output.
+  R20 the baselines' fixed-block rule (App. B, Eq. prelim-update) is read as
+      two modes on the rows of the active fixed block: 'threshold' commits
+      the masked rows with kappa >= tau, or, when none reaches tau, the one
+      with the highest kappa (the anti-stall fallback of the App. E
+      algorithm; Fast-dLLM's confidence rule); 'topm' commits the
+      min(m, |M|) masked rows with the highest kappa (Top-m), ties to the
+      lowest position.  The active block is the first block of B positions
+      that still holds a masked position.
 """
 from __future__ import annotations
 
@@ -360,6 +368,52 @@ def decide_sequence(pos, mask, tokens, in_block, meta, st: RowStats,
 
 
 # ----------------------------------------------------------------------------
+# (5b) the fixed-block rules of the baselines -- App. B, Eq. prelim-update
+# ----------------------------------------------------------------------------
+def decide_fixed_block(mask, tokens, st: RowStats, mode: str, tau: float,
+                       top_m: int) -> SeqDecision:
+    """One step of the standard block update on the rows of the active fixed
+    block (Reading R20).  mask and tokens are updated in place."""
+    n = len(mask)
+    out = SeqDecision(lbs_logit=np.full(n, np.nan), lps_prob=np.full(n, np.nan),
+                      accepted=np.zeros(n, np.uint8))
+    M = [i for i in range(n) if mask[i]]
+    if not M:
+        return out
+    by_conf = sorted(M, key=lambda i: (-st.conf[i], i))      # highest kappa first
+    if mode == "threshold":
+        A = [i for i in M if st.conf[i] >= tau]
+        flag = any(abs(st.conf[i] - tau) < NEAR_TIE for i in M)
+        if not A:
+            A = [by_conf[0]]
+            ks = [st.conf[i] for i in by_conf]
+            flag |= len(ks) > 1 and ks[0] - ks[1] < NEAR_TIE_STALL
+    elif mode == "topm":
+        k = min(top_m, len(M))
+        A = by_conf[:k]
+        ks = [st.conf[i] for i in by_conf]
+        flag = k < len(ks) and ks[k - 1] - ks[k] < NEAR_TIE_STALL
+    else:
+        raise ValueError(mode)
+    out.flag_accept = bool(flag or np.any(st.near_tie[A]))
+    for i in A:
+        tokens[i] = int(st.argmax[i])
+        mask[i] = 0
+        out.accepted[i] = 1
+    return out
+
+
+def fixed_block_window(mask, block: int):
+    """First fixed block [jB, jB + B) that holds a masked position (Reading
+    R16); (L, L) when none does."""
+    L = len(mask)
+    for j0 in range(0, L, block):
+        if any(mask[j0:j0 + block]):
+            return j0, min(j0 + block, L)
+    return L, L
+
+
+# ----------------------------------------------------------------------------
 # (6) one whole step over a batch of windows
 # ----------------------------------------------------------------------------
 @dataclass
@@ -433,12 +487,15 @@ def loop_window(frontier: int, end: int, meta, in_block_pos: List[int],
 
 def generation_loop(shape, W, prm: DecisionParams, window_inputs, kv_rows,
                     w_lm, w_emb, max_steps: Optional[int] = None,
-                    attention: bool = False, on_step=None):
+                    attention: bool = False, on_step=None, mode: str = "eb",
+                    block: int = 32, top_m: int = 1):
     """Run the App. E loop on the synthetic loop workload: a committed prompt
     of `shape.prefix` positions followed by `shape.gen_len` masked positions.
     window_inputs(step, positions) -> (hidden, q, k_win, v_win) and
     kv_rows(positions) -> (k, v) supply the per-step tensors.  Returns
-    (tokens, steps, per-step commit counts, per-step records)."""
+    (tokens, steps, per-step commit counts, per-step records).  mode 'eb'
+    runs the App. E algorithm; 'threshold' and 'topm' the fixed-block rules
+    of the baselines (Reading R20) with blocks of `block` positions."""
     P0, L = shape.prefix, shape.gen_len
     tokens = np.full(L, -1, np.int32)
     mask = np.ones(L, np.uint8)
@@ -448,9 +505,12 @@ def generation_loop(shape, W, prm: DecisionParams, window_inputs, kv_rows,
     while mask.any():
         if max_steps is not None and steps >= max_steps:
             break
-        f = int(np.argmax(mask))
-        blk = [i for i in range(L) if in_block[i]]
-        lo, hi = loop_window(f, L, meta, blk)
+        if mode == "eb":
+            f = int(np.argmax(mask))
+            blk = [i for i in range(L) if in_block[i]]
+            lo, hi = loop_window(f, L, meta, blk)
+        else:
+            lo, hi = fixed_block_window(mask, block)
         positions = P0 + np.arange(lo, hi, dtype=np.int32)
         hid, q, kw, vw = window_inputs(steps, positions)
         st = softmax_stats(lm_logits(hid, w_lm))
@@ -461,7 +521,10 @@ def generation_loop(shape, W, prm: DecisionParams, window_inputs, kv_rows,
                                     np.array([0, hi - lo]), np.array([P0 + lo]))
         t, m, ib = tokens[lo:hi], mask[lo:hi], in_block[lo:hi]
         before = int(m.sum())
-        d = decide_sequence(positions, m, t, ib, meta, st, w_emb, W, prm)
+        if mode == "eb":
+            d = decide_sequence(positions, m, t, ib, meta, st, w_emb, W, prm)
+        else:
+            d = decide_fixed_block(m, t, st, mode, prm.tau, top_m)
         if meta[1] == 0:
             in_block[:] = 0
         commits.append(before - int(m.sum()))

@@ -20,6 +20,9 @@ EBD_ERR_TIMEOUT = -4
 EBD_ERR_NONFINITE = -5
 EBD_ERR_STATE = -6
 EBD_DEBUG_FORCE_TIMEOUT = 1
+EBD_DECODE_EB = 0
+EBD_DECODE_THRESHOLD = 1
+EBD_DECODE_TOPM = 2
 
 STATUS_NAMES = {0: "EBD_OK", -1: "EBD_ERR_INVALID_ARG", -2: "EBD_ERR_UNSUPPORTED",
                 -3: "EBD_ERR_CUDA", -4: "EBD_ERR_TIMEOUT", -5: "EBD_ERR_NONFINITE",
@@ -33,7 +36,8 @@ class ebd_config(Structure):
                 ("max_prefix", c_int32), ("gen_len", c_int32), ("g_max", c_int32),
                 ("l_min", c_int32), ("l_b", c_int32), ("eos_id", c_int32),
                 ("lps_enabled", c_int32), ("tau", c_float), ("tau_psi", c_float),
-                ("seed", c_uint64), ("debug_flags", c_int32), ("reserved", c_int32)]
+                ("seed", c_uint64), ("debug_flags", c_int32), ("decode_mode", c_int32),
+                ("top_m", c_int32), ("reserved", c_int32)]
 
 
 class ebd_step_args(Structure):
@@ -53,7 +57,8 @@ EXPORTS = ["ebd_create", "ebd_destroy", "ebd_bind_embedding", "ebd_step", "ebd_s
            "ebd_export_weights", "ebd_import_weights", "ebd_router_init_host",
            "ebd_weight_count", "ebd_lm_head_packed_bytes", "ebd_pack_lm_head",
            "ebd_profile_enable", "ebd_profile_read", "ebd_last_error",
-           "ebd_version", "ebd_lm_stats_noalloc", "ebd_loop_window"]
+           "ebd_version", "ebd_lm_stats_noalloc", "ebd_loop_window",
+           "ebd_loop_block_window"]
 
 _lib = None
 
@@ -100,6 +105,8 @@ def load(path: str = LIB_PATH):
     lib.ebd_loop_window.argtypes = [c_void_p, c_void_p, c_void_p, c_int32, c_int32, P(c_int32),
                                     P(c_int32)]
     lib.ebd_loop_window.restype = c_int32
+    lib.ebd_loop_block_window.argtypes = [c_void_p, c_int32, c_int32, P(c_int32), P(c_int32)]
+    lib.ebd_loop_block_window.restype = c_int32
     lib.ebd_version.restype = c_char_p
     for fn in EXPORTS:
         if getattr(lib, fn).restype is ctypes.c_int:
@@ -242,4 +249,14 @@ def ebd_loop_window(mask, in_block, meta, max_window: int = 64):
     lo, hi = c_int32(0), c_int32(0)
     s = load().ebd_loop_window(m.ctypes.data, ib.ctypes.data, mt.ctypes.data, int(m.size),
                                int(max_window), ctypes.byref(lo), ctypes.byref(hi))
+    return s, lo.value, hi.value
+
+
+def ebd_loop_block_window(mask, block: int):
+    """mask: host uint8 [L].  Returns (status, lo, hi)."""
+    import numpy as np
+    m = np.ascontiguousarray(mask, dtype=np.uint8)
+    lo, hi = c_int32(0), c_int32(0)
+    s = load().ebd_loop_block_window(m.ctypes.data, int(m.size), int(block), ctypes.byref(lo),
+                                     ctypes.byref(hi))
     return s, lo.value, hi.value

@@ -231,6 +231,9 @@ ebd_status validate_config(const ebd_config* c, std::string& why) {
   if (c->gen_len < c->max_window) return bad("gen_len must be >= max_window");
   if (c->g_max < 0 || c->l_min < 0 || c->l_b < 0) return bad("g_max, l_min, l_b must be >= 0");
   if (!(c->tau == c->tau) || !(c->tau_psi == c->tau_psi)) return bad("tau/tau_psi is NaN");
+  if (c->decode_mode < EBD_DECODE_EB || c->decode_mode > EBD_DECODE_TOPM)
+    return bad("decode_mode must be EBD_DECODE_EB, _THRESHOLD or _TOPM");
+  if (c->decode_mode == EBD_DECODE_TOPM && c->top_m < 1) return bad("top_m must be >= 1");
   return EBD_OK;
 }
 
@@ -530,7 +533,9 @@ DecideParams decide_params(ebd_handle* h, const ebd_step_args* a, int features_i
   p.l_min = c.l_min;
   p.l_b = c.l_b;
   p.eos_id = c.eos_id;
-  p.lps_enabled = c.lps_enabled;
+  p.mode = c.decode_mode;
+  p.top_m = c.top_m;
+  p.lps_enabled = c.decode_mode == EBD_DECODE_EB ? c.lps_enabled : 0;
   p.tau = c.tau;
   p.tau_psi = c.tau_psi;
   p.inv_log_v = static_cast<float>(1.0 / std::log(static_cast<double>(c.vocab)));
@@ -561,6 +566,23 @@ DecideParams decide_params(ebd_handle* h, const ebd_step_args* a, int features_i
 extern "C" {
 
 const char* ebd_version(void) { return "ebd 0.1 (sm_103a)"; }
+
+ebd_status ebd_loop_block_window(const uint8_t* mask, int32_t L, int32_t block, int32_t* lo,
+                                 int32_t* hi) {
+  if (mask == nullptr || lo == nullptr || hi == nullptr || L < 0 || block < 1)
+    return EBD_ERR_INVALID_ARG;
+  for (int32_t j0 = 0; j0 < L; j0 += block) {
+    const int32_t j1 = j0 + block < L ? j0 + block : L;
+    for (int32_t i = j0; i < j1; ++i)
+      if (mask[i]) {
+        *lo = j0;
+        *hi = j1;
+        return EBD_OK;
+      }
+  }
+  *lo = *hi = L;
+  return EBD_OK;
+}
 
 ebd_status ebd_loop_window(const uint8_t* mask, const uint8_t* in_block, const int32_t* meta,
                            int32_t L, int32_t max_window, int32_t* lo, int32_t* hi) {

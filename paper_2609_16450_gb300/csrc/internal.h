@@ -72,6 +72,7 @@ struct DecideParams {
   int B, V, grid_lm;        // grid_lm: LM-head partials per row
   int features_in;          // 1: conf/ent_norm/gap/argmax are inputs
   int pdl;                  // launched as a programmatic dependent of the LM head
+  int mode, top_m;          // EBD_DECODE_*; commits per step of the Top-m rule
   int gen_len, g_max, l_min, l_b, eos_id, lps_enabled;
   float tau, tau_psi, inv_log_v;
   const int* cu_rows;

@@ -521,7 +521,7 @@ __global__ void __cluster_dims__(kDecideCluster, 1, 1) __launch_bounds__(kDecide
     fence_mbar_init();
     sm.meta_b = p.blk_meta[2 * seq];
     sm.meta_s = p.blk_meta[2 * seq + 1];
-    const bool lbs_possible = sm.meta_s == 0;
+    const bool lbs_possible = p.mode == EBD_DECODE_EB && sm.meta_s == 0;
     const uint32_t wb = LBS_W_ELEMS * 2u, vb = V_ELEMS * 4u;
     mbar_arrive_expect_tx(&sm.bar, vb + (lbs_possible ? wb : 0u));
     bulk_copy(sm.v, p.w.vec + static_cast<size_t>(rank) * V_ELEMS, vb, &sm.bar);
@@ -646,7 +646,7 @@ __global__ void __cluster_dims__(kDecideCluster, 1, 1) __launch_bounds__(kDecide
     }
     if (lane == 0) {
       sm.nM = base;
-      sm.run_lbs = (sm.meta_s == 0 && base > p.l_min) ? 1 : 0;
+      sm.run_lbs = (p.mode == EBD_DECODE_EB && sm.meta_s == 0 && base > p.l_min) ? 1 : 0;
     }
   }
   __syncthreads();
@@ -830,6 +830,8 @@ __global__ void __cluster_dims__(kDecideCluster, 1, 1) __launch_bounds__(kDecide
         sm.meta_s = nB;
       }
       __syncwarp();
+    } else if (p.mode != EBD_DECODE_EB) {
+      // baselines: the window is the active fixed block; no block state
     } else if (sm.meta_s == 0) {
       for (int j = lane; j < nr; j += 32) sm.f_ib[j] = 0;
       __syncwarp();
@@ -882,7 +884,8 @@ __global__ void __cluster_dims__(kDecideCluster, 1, 1) __launch_bounds__(kDecide
     int base = 0;
     for (int j0 = 0; j0 < nr; j0 += 32) {
       const int j = j0 + lane;
-      const bool m = j < nr && sm.f_ib[j] && sm.f_mask[j] && !sm.f_bad[j];
+      const bool inb = p.mode != EBD_DECODE_EB || sm.f_ib[j];
+      const bool m = j < nr && inb && sm.f_mask[j] && !sm.f_bad[j];
       const uint32_t bal = __ballot_sync(0xffffffffu, m);
       if (m) sm.BMrows[base + __popc(bal & ((1u << lane) - 1u))] = j;
       base += __popc(bal);
@@ -917,7 +920,27 @@ __global__ void __cluster_dims__(kDecideCluster, 1, 1) __launch_bounds__(kDecide
     for (int i = tid; i < nBM; i += blockDim.x) sm.f_p[sm.BMrows[i]] = prob[i];
     __syncthreads();
   }
-  if (warp == 0) {
+  if (warp == 0 && p.mode == EBD_DECODE_TOPM) {
+    // Top-m (App. B, Eq. prelim-update): the rank of a row is the number of
+    // rows ahead of it (higher kappa, or equal kappa and lower position)
+    for (int i = lane; i < nBM; i += 32) {
+      const int j = sm.BMrows[i];
+      const float c = sm.f_conf[j];
+      int rank = 0;
+      for (int k = 0; k < nBM; ++k) {
+        const int jk = sm.BMrows[k];
+        const float ck = sm.f_conf[jk];
+        rank += (ck > c || (ck == c && jk < j)) ? 1 : 0;
+      }
+      if (rank < p.top_m) sm.f_acc[j] = 1;
+    }
+    __syncwarp();
+    for (int j = lane; j < nr; j += 32)
+      if (sm.f_acc[j]) {
+        sm.f_tok[j] = sm.f_arg[j];
+        sm.f_mask[j] = 0;
+      }
+  } else if (warp == 0) {
     // union accept rule, anti-stall fallback, parallel commit, resolution
     bool any = false;
     for (int i0 = 0; i0 < nBM; i0 += 32) {
@@ -966,7 +989,7 @@ __global__ void __cluster_dims__(kDecideCluster, 1, 1) __launch_bounds__(kDecide
       }
     }
     open = __ballot_sync(0xffffffffu, open) != 0;
-    if (sm.meta_s > 0 && !open) {
+    if (p.mode == EBD_DECODE_EB && sm.meta_s > 0 && !open) {
       for (int j = lane; j < nr; j += 32) sm.f_ib[j] = 0;
       if (lane == 0) {
         sm.meta_b = 0;

@@ -52,17 +52,23 @@ class LoopResult:
     device_us: float = 0.0
 
 
-def config_for_loop(shape, max_window: int = 64) -> E.ebd_config:
+def config_for_loop(shape, max_window: int = 64, decode_mode: int = E.EBD_DECODE_EB,
+                    top_m: int = 1) -> E.ebd_config:
     return rt.config_for(shape, max_batch=1, max_window=max_window, max_rows=max_window,
-                         max_prefix=shape.prefix + shape.gen_len)
+                         max_prefix=shape.prefix + shape.gen_len, decode_mode=decode_mode,
+                         top_m=top_m)
 
 
 def run_loop(h: rt.Handle, shape, weights: rt.DeviceWeights,
              window_inputs: Callable, kv_rows: Callable, attention: bool = True,
              max_steps: Optional[int] = None, max_window: int = 64,
-             keep: bool = True, stream: Optional[torch.cuda.Stream] = None) -> LoopResult:
+             keep: bool = True, stream: Optional[torch.cuda.Stream] = None,
+             block: int = 32) -> LoopResult:
     """window_inputs(step, positions) -> (hidden, q, k_win, v_win) as bf16 bit
-    arrays; kv_rows(positions) -> (k, v).  Positions are absolute."""
+    arrays; kv_rows(positions) -> (k, v).  Positions are absolute.  Under the
+    handle's baseline decode modes the window is the active fixed block of
+    `block` positions (ebd_loop_block_window)."""
+    fixed = h.cfg.decode_mode != E.EBD_DECODE_EB
     dev = "cuda"
     P0, L = shape.prefix, shape.gen_len
     d, Hq, Hkv, D = shape.d_model, shape.n_heads_q, shape.n_heads_kv, shape.head_dim
@@ -103,9 +109,12 @@ def run_loop(h: rt.Handle, shape, weights: rt.DeviceWeights,
     while True:
         if max_steps is not None and step >= max_steps:
             break
-        s, lo, hi = E.ebd_loop_window(mask_h, ib_h, meta_h, W)
+        if fixed:
+            s, lo, hi = E.ebd_loop_block_window(mask_h, block)
+        else:
+            s, lo, hi = E.ebd_loop_window(mask_h, ib_h, meta_h, W)
         if s != E.EBD_OK:
-            raise E.EbdError(s, "ebd_loop_window")
+            raise E.EbdError(s, "loop window")
         if lo >= L:
             break
         R = hi - lo

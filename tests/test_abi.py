@@ -120,3 +120,24 @@ def test_loop_window_matches_oracle(lib):
     # invalid arguments and states
     assert E.ebd_loop_window(np.ones(4), np.zeros(4), np.array([0, 3]), 64)[0] == E.EBD_ERR_STATE
     assert E.ebd_loop_window(np.ones(4), np.zeros(4), np.zeros(2), 0)[0] == E.EBD_ERR_INVALID_ARG
+
+
+def test_loop_block_window_matches_oracle(lib):
+    from paper_2609_16450_gb300 import _ebd as E
+    rng = np.random.default_rng(11)
+    for _ in range(300):
+        L = int(rng.integers(0, 150))
+        mask = (rng.random(L) < rng.random() * 0.3).astype(np.uint8)
+        block = int(rng.integers(1, 40))
+        s, lo, hi = E.ebd_loop_block_window(mask, block)
+        assert s == E.EBD_OK
+        assert (lo, hi) == o.fixed_block_window(mask, block)
+    assert E.ebd_loop_block_window(np.ones(4, np.uint8), 0)[0] == E.EBD_ERR_INVALID_ARG
+
+
+def test_decode_mode_validation(lib):
+    from paper_2609_16450_gb300 import _ebd as E
+    from paper_2609_16450_gb300 import runtime as rt
+    for over in (dict(decode_mode=3), dict(decode_mode=E.EBD_DECODE_TOPM, top_m=0)):
+        s, h = E.ebd_create(rt.config_for(synth.tiny, **over))
+        assert s == E.EBD_ERR_UNSUPPORTED and not h.value
