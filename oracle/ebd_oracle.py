@@ -405,7 +405,7 @@ def decide_fixed_block(mask, tokens, st: RowStats, mode: str, tau: float,
 
 def fixed_block_window(mask, block: int):
     """First fixed block [jB, jB + B) that holds a masked position (Reading
-    R16); (L, L) when none does."""
+    R20); (L, L) when none does."""
     L = len(mask)
     for j0 in range(0, L, block):
         if any(mask[j0:j0 + block]):
