@@ -238,70 +238,135 @@ __device__ __forceinline__ void merge_state(float& m, float& s, float& t, float&
 
 // ------------------------------------------------------------------ LBS attention
 // This CTA's query rows [qa, qa + nq) of head hd (width 32) over the n rows'
-// keys/values; the output (hi/lo) goes to every rank's concat buffer.
+// keys/values: softmax(q k^T / sqrt(32)) v on the tensor cores, 16 query rows
+// per warp, keys in blocks of 16 with a running max and sum.  q, k, v and the
+// probabilities are split into bf16 high and low parts (three products per
+// pair).  The output goes, as hi/lo, to this CTA's concat buffer, and from
+// there, 16 bytes at a time by the whole CTA, to the other ranks'.
 __device__ __forceinline__ void lbs_attention(cg::cluster_group& cluster, float* P, int nq, int n,
                                               int qa, int hd) {
   const float* Q = P + P_Q;
   const float* KV = P + P_KV;
-  float* S = P + P_S;
+  __nv_bfloat16* X = reinterpret_cast<__nv_bfloat16*>(P + P_XH);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, g = lane >> 2, t = lane & 3;
   const float scale = 0.17677669529663687f;  // 1/sqrt(32)
-#pragma unroll 1
-  for (int it = threadIdx.x; it < nq * n; it += blockDim.x) {
-    const int i = it / n, k = it - i * n;
-    const float4* q4 = reinterpret_cast<const float4*>(Q + i * LDQ);
-    const float4* k4 = reinterpret_cast<const float4*>(KV + k * LDKV);
-    float a0 = 0.f, a1 = 0.f;
+  if (warp < ((nq + 15) >> 4)) {
+    const int r_lo = warp * 16 + g, r_hi = r_lo + 8;
+    uint32_t qh[2][4], ql[2][4];
 #pragma unroll
-    for (int d = 0; d < 8; d += 2) {
-      const float4 x0 = q4[d], y0 = k4[d], x1 = q4[d + 1], y1 = k4[d + 1];
-      a0 = fmaf(x0.x, y0.x, fmaf(x0.y, y0.y, fmaf(x0.z, y0.z, fmaf(x0.w, y0.w, a0))));
-      a1 = fmaf(x1.x, y1.x, fmaf(x1.y, y1.y, fmaf(x1.z, y1.z, fmaf(x1.w, y1.w, a1))));
+    for (int ks = 0; ks < 2; ++ks) {
+      const float2 z = make_float2(0.f, 0.f);
+      const float* ql0 = Q + r_lo * LDQ + 16 * ks + 2 * t;
+      const float* qh0 = Q + r_hi * LDQ + 16 * ks + 2 * t;
+      const float2 a0 = r_lo < nq ? *reinterpret_cast<const float2*>(ql0) : z;
+      const float2 a1 = r_hi < nq ? *reinterpret_cast<const float2*>(qh0) : z;
+      const float2 a2 = r_lo < nq ? *reinterpret_cast<const float2*>(ql0 + 8) : z;
+      const float2 a3 = r_hi < nq ? *reinterpret_cast<const float2*>(qh0 + 8) : z;
+      split_bf16x2(a0.x, a0.y, qh[ks][0], ql[ks][0]);
+      split_bf16x2(a1.x, a1.y, qh[ks][1], ql[ks][1]);
+      split_bf16x2(a2.x, a2.y, qh[ks][2], ql[ks][2]);
+      split_bf16x2(a3.x, a3.y, qh[ks][3], ql[ks][3]);
     }
-    S[i * LDS + k] = (a0 + a1) * scale;
+    float mx0 = -INFINITY, mx1 = -INFINITY, l0 = 0.f, l1 = 0.f;
+    float o[4][4];
+#pragma unroll
+    for (int nt = 0; nt < 4; ++nt) o[nt][0] = o[nt][1] = o[nt][2] = o[nt][3] = 0.f;
+#pragma unroll 1
+    for (int k0 = 0; k0 < n; k0 += 16) {
+      float s[2][4];
+#pragma unroll
+      for (int hb = 0; hb < 2; ++hb) {
+        const int key = k0 + 8 * hb + g;
+        float a[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+        for (int ks = 0; ks < 2; ++ks) {
+          const float2 z = make_float2(0.f, 0.f);
+          const float* kp = KV + key * LDKV + 16 * ks + 2 * t;
+          const float2 k0v = key < n ? *reinterpret_cast<const float2*>(kp) : z;
+          const float2 k1v = key < n ? *reinterpret_cast<const float2*>(kp + 8) : z;
+          uint32_t bh0, bl0, bh1, bl1;
+          split_bf16x2(k0v.x, k0v.y, bh0, bl0);
+          split_bf16x2(k1v.x, k1v.y, bh1, bl1);
+          mma_bf16(a, qh[ks], bh0, bh1);
+          mma_bf16(a, qh[ks], bl0, bl1);
+          mma_bf16(a, ql[ks], bh0, bh1);
+        }
+        const int c = k0 + 8 * hb + 2 * t;
+        s[hb][0] = c < n ? a[0] * scale : -INFINITY;
+        s[hb][1] = c + 1 < n ? a[1] * scale : -INFINITY;
+        s[hb][2] = c < n ? a[2] * scale : -INFINITY;
+        s[hb][3] = c + 1 < n ? a[3] * scale : -INFINITY;
+      }
+      float b0 = fmaxf(fmaxf(s[0][0], s[0][1]), fmaxf(s[1][0], s[1][1]));
+      float b1 = fmaxf(fmaxf(s[0][2], s[0][3]), fmaxf(s[1][2], s[1][3]));
+      b0 = fmaxf(b0, __shfl_xor_sync(0xffffffffu, b0, 1));
+      b0 = fmaxf(b0, __shfl_xor_sync(0xffffffffu, b0, 2));
+      b1 = fmaxf(b1, __shfl_xor_sync(0xffffffffu, b1, 1));
+      b1 = fmaxf(b1, __shfl_xor_sync(0xffffffffu, b1, 2));
+      const float n0 = fmaxf(mx0, b0), n1 = fmaxf(mx1, b1);  // finite: key k0 is valid
+      const float c0 = expf(mx0 - n0), c1 = expf(mx1 - n1);
+      mx0 = n0;
+      mx1 = n1;
+#pragma unroll
+      for (int hb = 0; hb < 2; ++hb) {
+        s[hb][0] = expf(s[hb][0] - n0);
+        s[hb][1] = expf(s[hb][1] - n0);
+        s[hb][2] = expf(s[hb][2] - n1);
+        s[hb][3] = expf(s[hb][3] - n1);
+      }
+      l0 = l0 * c0 + ((s[0][0] + s[0][1]) + (s[1][0] + s[1][1]));
+      l1 = l1 * c1 + ((s[0][2] + s[0][3]) + (s[1][2] + s[1][3]));
+      uint32_t ph[4], pl[4];
+      split_bf16x2(s[0][0], s[0][1], ph[0], pl[0]);
+      split_bf16x2(s[0][2], s[0][3], ph[1], pl[1]);
+      split_bf16x2(s[1][0], s[1][1], ph[2], pl[2]);
+      split_bf16x2(s[1][2], s[1][3], ph[3], pl[3]);
+#pragma unroll
+      for (int nt = 0; nt < 4; ++nt) {
+        o[nt][0] *= c0;
+        o[nt][1] *= c0;
+        o[nt][2] *= c1;
+        o[nt][3] *= c1;
+        float v[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const int key = k0 + (e >> 1) * 8 + 2 * t + (e & 1);
+          v[e] = key < n ? KV[key * LDKV + 32 + 8 * nt + g] : 0.f;
+        }
+        uint32_t v0h, v0l, v1h, v1l;
+        split_bf16x2(v[0], v[1], v0h, v0l);
+        split_bf16x2(v[2], v[3], v1h, v1l);
+        mma_bf16(o[nt], ph, v0h, v1h);
+        mma_bf16(o[nt], ph, v0l, v1l);
+        mma_bf16(o[nt], pl, v0h, v1h);
+      }
+    }
+    l0 += __shfl_xor_sync(0xffffffffu, l0, 1);
+    l0 += __shfl_xor_sync(0xffffffffu, l0, 2);
+    l1 += __shfl_xor_sync(0xffffffffu, l1, 1);
+    l1 += __shfl_xor_sync(0xffffffffu, l1, 2);
+    const float i0 = 1.0f / l0, i1 = 1.0f / l1;
+    const HL Xl{X, LDH, W * LDH};
+#pragma unroll
+    for (int nt = 0; nt < 4; ++nt) {
+      const int col = 32 * hd + 8 * nt + 2 * t;
+      if (r_lo < nq) hl_store2(Xl, qa + r_lo, col, o[nt][0] * i0, o[nt][1] * i0);
+      if (r_hi < nq) hl_store2(Xl, qa + r_hi, col, o[nt][2] * i1, o[nt][3] * i1);
+    }
   }
   __syncthreads();
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  // this CTA's slice of the concat buffer (rows [qa, qa+nq), columns of head
+  // hd, both planes) to the other ranks, 16 bytes per store
+  const int rank = static_cast<int>(cluster.block_rank());
 #pragma unroll 1
-  for (int i = warp; i < nq; i += (blockDim.x >> 5)) {
-    const float x0 = lane < n ? S[i * LDS + lane] : -INFINITY;
-    const float x1 = lane + 32 < n ? S[i * LDS + lane + 32] : -INFINITY;
-    const float m = warp_max(fmaxf(x0, x1));
-    const float e0 = lane < n ? expf(x0 - m) : 0.f;
-    const float e1 = lane + 32 < n ? expf(x1 - m) : 0.f;
-    const float inv = 1.0f / warp_sum(e0 + e1);
-    if (lane < n) S[i * LDS + lane] = e0 * inv;
-    if (lane + 32 < n) S[i * LDS + lane + 32] = e1 * inv;
-  }
-  __syncthreads();
-#pragma unroll 1
-  for (int it = threadIdx.x; it < nq * 16; it += blockDim.x) {
-    const int i = it >> 4, d = 2 * (it & 15);
-    float a0 = 0.f, a1 = 0.f, c0 = 0.f, c1 = 0.f;
-    int k = 0;
-#pragma unroll 2
-    for (; k + 1 < n; k += 2) {
-      const float p0 = S[i * LDS + k], p1 = S[i * LDS + k + 1];
-      const float2 v0 = *reinterpret_cast<const float2*>(KV + k * LDKV + 32 + d);
-      const float2 v1 = *reinterpret_cast<const float2*>(KV + (k + 1) * LDKV + 32 + d);
-      a0 = fmaf(p0, v0.x, a0);
-      a1 = fmaf(p0, v0.y, a1);
-      c0 = fmaf(p1, v1.x, c0);
-      c1 = fmaf(p1, v1.y, c1);
-    }
-    if (k < n) {
-      const float p0 = S[i * LDS + k];
-      const float2 v0 = *reinterpret_cast<const float2*>(KV + k * LDKV + 32 + d);
-      a0 = fmaf(p0, v0.x, a0);
-      a1 = fmaf(p0, v0.y, a1);
-    }
-    uint32_t hi, lo;
-    split_bf16x2(a0 + c0, a1 + c1, hi, lo);
-    const int off = (qa + i) * LDH + 32 * hd + d;
+  for (int it = threadIdx.x; it < nq * 8; it += blockDim.x) {
+    const int row = qa + (it >> 3), plane = (it >> 2) & 1, q4 = it & 3;
+    const int off = plane * W * LDH + row * LDH + 32 * hd + 8 * q4;
+    const uint4 val = *reinterpret_cast<const uint4*>(X + off);
 #pragma unroll 1
     for (int r = 0; r < kDecideCluster; ++r) {
-      __nv_bfloat16* X = reinterpret_cast<__nv_bfloat16*>(cluster.map_shared_rank(P + P_XH, r));
-      *reinterpret_cast<uint32_t*>(X + off) = hi;
-      *reinterpret_cast<uint32_t*>(X + W * LDH + off) = lo;
+      if (r == rank) continue;
+      *reinterpret_cast<uint4*>(cluster.map_shared_rank(X, r) + off) = val;
     }
   }
 }
@@ -664,19 +729,28 @@ __global__ void __cluster_dims__(kDecideCluster, 1, 1) __launch_bounds__(kDecide
     float* KV = P + P_KV;
     float* Q = P + P_Q;
     const float* Vv = sm.v;
-    // 3a. entropy branch F_ent and token branch, every rank for all rows
+    // 3a. entropy branch F_ent and token branch, every rank for all rows.
+    // The token branch's gathers from the folded table are issued first and
+    // stored only after the entropy branch, which hides their latency.
+    static_assert(kDecideThreads * 8 >= W * 32, "token-branch items per thread");
+    float2 tv[8];
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+      const int it = tid + k * kDecideThreads;
+      tv[k] = make_float2(0.f, 0.f);
+      if (it < n * 32) {
+        const int tok = sm.f_arg[sm.Mrows[it >> 5]];
+        if (tok >= 0 && tok < p.V)
+          tv[k] = __ldg(reinterpret_cast<const float2*>(p.w.tok_table + static_cast<size_t>(tok) * 64 +
+                                                       2 * (it & 31)));
+      }
+    }
 #pragma unroll 1
     for (int it = tid; it < n * 32; it += blockDim.x) {
       const int j = it >> 5, o = 2 * (it & 31);
-      const int row = sm.Mrows[j];
-      const float h = sm.f_ent[row];
+      const float h = sm.f_ent[sm.Mrows[j]];
       hl_store2(Fh, j, o, gelu(fmaf(Vv[V_ENT1W + o], h, Vv[V_ENT1B + o])),
                 gelu(fmaf(Vv[V_ENT1W + o + 1], h, Vv[V_ENT1B + o + 1])));
-      const int tok = sm.f_arg[row];
-      float2 tv = make_float2(0.f, 0.f);
-      if (tok >= 0 && tok < p.V)
-        tv = *reinterpret_cast<const float2*>(p.w.tok_table + static_cast<size_t>(tok) * 64 + o);
-      hl_store2(Xh, j, 64 + o, tv.x + Vv[V_TOKB + o], tv.y + Vv[V_TOKB + o + 1]);
     }
     __syncthreads();
     // the ent2 output goes to the z hi/lo region: z itself receives the
@@ -687,6 +761,14 @@ __global__ void __cluster_dims__(kDecideCluster, 1, 1) __launch_bounds__(kDecide
     });
     __syncthreads();
     ln_rows(E2, LDZ, nullptr, 0, &Xh, n, 64, Vv + V_ENTLNG, Vv + V_ENTLNB);
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {  // the token branch into columns 64..127
+      const int it = tid + k * kDecideThreads;
+      if (it < n * 32) {
+        const int o = 2 * (it & 31);
+        hl_store2(Xh, it >> 5, 64 + o, tv[k].x + Vv[V_TOKB + o], tv[k].y + Vv[V_TOKB + o + 1]);
+      }
+    }
     __syncthreads();
     // 3b. fusion W_combine [e; t] + E_pos[rank of the row]: this CTA's 16 outputs
     {
