@@ -102,6 +102,9 @@ __device__ __forceinline__ void record_error(int* status, volatile int* abort, i
 
 }  // namespace
 
+// PAIR: the paired mode (p.pair), a separate instantiation so that the
+// single-CTA path carries none of its code
+template <bool PAIR>
 __global__ void __launch_bounds__(kLmThreads, 1)
     lm_stats_kernel(const __grid_constant__ CUtensorMap tmap_w,
                     const __grid_constant__ CUtensorMap tmap_h, const LmParams p) {
@@ -136,15 +139,15 @@ __global__ void __launch_bounds__(kLmThreads, 1)
   // paired mode: the two CTAs of a cluster share a vocabulary range; each
   // loads one of the two W units of a chunk and multicasts it to both, and
   // accumulates half of the window rows
-  const uint32_t crank = p.pair ? cluster_ctarank() : 0u;
-  const int cta = p.pair ? static_cast<int>(blockIdx.x >> 1) : static_cast<int>(blockIdx.x);
+  const uint32_t crank = PAIR ? cluster_ctarank() : 0u;
+  const int cta = PAIR ? static_cast<int>(blockIdx.x >> 1) : static_cast<int>(blockIdx.x);
   const int rbase = p.row0 + static_cast<int>(crank) * p.rhalf;  // first row of this CTA
   const int rows_c = min(p.rhalf, p.rows - static_cast<int>(crank) * p.rhalf);
 
   if (tid == 0) {
     for (int s = 0; s < p.stages; ++s) {
       mbar_init(&full[s], 1);
-      mbar_init(&empty[s], p.pair ? 2 : 1);  // paired: both CTAs' MMAs release a stage
+      mbar_init(&empty[s], PAIR ? 2 : 1);  // paired: both CTAs' MMAs release a stage
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&acc_full[b], 1);
@@ -168,7 +171,7 @@ __global__ void __launch_bounds__(kLmThreads, 1)
     }
   }
   tc_fence_before();
-  if (p.pair)
+  if (PAIR)
     cluster_sync_all();  // the peer's barriers exist before anything is multicast to them
   else
     __syncthreads();
@@ -205,13 +208,13 @@ __global__ void __launch_bounds__(kLmThreads, 1)
           // one row half at a time, its k-boxes back to back: each W row is
           // requested as one contiguous run of nsubk * 128 bytes
           for (int ui = 0; ui < nu; ++ui) {
-            if (p.pair && ui != static_cast<int>(crank)) continue;  // the peer loads it
+            if (PAIR && ui != static_cast<int>(crank)) continue;  // the peer loads it
             for (int j = 0; j < nsubk; ++j) {
               const int x = p.packed ? 0 : (ks * p.kbs + j) * 64;
               const int y = p.packed ? ((u + ui) * p.nkb + ks * p.kbs + j) * kUnit
                                      : (u + ui) * kUnit;
               uint8_t* dst = a_st + j * kATile + ui * (kUnit * 128);
-              if (p.pair)
+              if (PAIR)
                 tma_load_2d_multicast(dst, &tmap_w, &full[s], x, y, 0x3, pol_w);
               else
                 tma_load_2d(dst, &tmap_w, &full[s], x, y, pol_w);
@@ -286,7 +289,7 @@ __global__ void __launch_bounds__(kLmThreads, 1)
               }
             }
 #undef EBD_STAGE
-            if (p.pair)
+            if (PAIR)
               umma_commit_multicast(&empty[s], 0x3);
             else
               umma_commit(&empty[s]);
@@ -305,7 +308,7 @@ __global__ void __launch_bounds__(kLmThreads, 1)
               }
             }
           }
-          if (p.pair)
+          if (PAIR)
               umma_commit_multicast(&empty[s], 0x3);
             else
               umma_commit(&empty[s]);
@@ -441,7 +444,7 @@ __global__ void __launch_bounds__(kLmThreads, 1)
   }
 
   __syncthreads();
-  if (p.pair) cluster_sync_all();  // no multicast or remote arrival can target a CTA that left
+  if (PAIR) cluster_sync_all();  // no multicast or remote arrival can target a CTA that left
   if (warp == 1) {
     tc_fence_after();
     tmem_dealloc(tmem_base, p.tmem_cols);
@@ -474,7 +477,10 @@ void lm_plan(LmParams& p, int rows, int V, int d, int num_sms, bool pair) {
     if (p.grid < 1) p.grid = 1;
   }
   p.nkb = (d + 63) / 64;
-  p.nwg = p.n_pad > 32 ? 2 : 1;
+  // a second epilogue warpgroup (and its transpose buffer) only pays when the
+  // accumulator is wide; below that the buffer is worth more as a larger
+  // pipeline stage (measured: 128 rows, 5 x 16 KB stages -> 183 us, 4 -> 246)
+  p.nwg = p.n_pad >= 192 ? 2 : 1;
   const uint32_t st_bytes = static_cast<uint32_t>(p.n_pad) * 20u;
   const uint32_t tail = kTBytes * static_cast<uint32_t>(p.nwg) + ((st_bytes + 7) / 8 * 8) +
                         (2 * 8 + 6) * 8 + 16;
@@ -541,7 +547,10 @@ cudaError_t launch_pack_lm(const __nv_bfloat16* w, __nv_bfloat16* out, int V, in
 }
 
 cudaError_t lm_configure() {
-  return cudaFuncSetAttribute(lm_stats_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  cudaError_t e = cudaFuncSetAttribute(lm_stats_kernel<true>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, 232448);
+  if (e != cudaSuccess) return e;
+  return cudaFuncSetAttribute(lm_stats_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                               232448);
 }
 
@@ -559,7 +568,8 @@ cudaError_t launch_lm_stats(const CUtensorMap& tmap_w, const CUtensorMap& tmap_h
   attr[0].val.clusterDim.z = 1;
   cfg.attrs = attr;
   cfg.numAttrs = p.pair ? 1 : 0;
-  return cudaLaunchKernelEx(&cfg, lm_stats_kernel, tmap_w, tmap_h, p);
+  if (p.pair) return cudaLaunchKernelEx(&cfg, lm_stats_kernel<true>, tmap_w, tmap_h, p);
+  return cudaLaunchKernelEx(&cfg, lm_stats_kernel<false>, tmap_w, tmap_h, p);
 }
 
 }  // namespace ebd
