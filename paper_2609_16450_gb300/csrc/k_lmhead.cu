@@ -102,9 +102,9 @@ __device__ __forceinline__ void record_error(int* status, volatile int* abort, i
 
 }  // namespace
 
-// PAIR: the paired mode (p.pair), a separate instantiation so that the
-// single-CTA path carries none of its code
-template <bool PAIR>
+// PAIR (p.pair) and PACKED (p.packed) are template parameters: a runtime
+// branch in the single-thread producer or MMA loop costs measurable time
+template <bool PAIR, bool PACKED>
 __global__ void __launch_bounds__(kLmThreads, 1)
     lm_stats_kernel(const __grid_constant__ CUtensorMap tmap_w,
                     const __grid_constant__ CUtensorMap tmap_h, const LmParams p) {
@@ -190,12 +190,12 @@ __global__ void __launch_bounds__(kLmThreads, 1)
       const uint64_t pol_w = l2_policy_evict_first();
       const uint64_t pol_h = l2_policy_evict_last();
       int it = 0;
+      int s = 0;        // stage of iteration it (it % stages, kept as a counter)
+      uint32_t ph = 0;  // its phase parity
       bool ok = true;
       for (int u = u0; u < u1 && ok; u += 2) {
         const int nu = min(2, u1 - u);
         for (int ks = 0; ks < p.nks; ++ks) {
-          const int s = it % p.stages;
-          const uint32_t ph = static_cast<uint32_t>(it / p.stages) & 1u;
           if (!mbar_wait(&empty[s], ph ^ 1u, p.limit_ns, abort)) {
             ok = false;
             break;
@@ -210,9 +210,9 @@ __global__ void __launch_bounds__(kLmThreads, 1)
           for (int ui = 0; ui < nu; ++ui) {
             if (PAIR && ui != static_cast<int>(crank)) continue;  // the peer loads it
             for (int j = 0; j < nsubk; ++j) {
-              const int x = p.packed ? 0 : (ks * p.kbs + j) * 64;
-              const int y = p.packed ? ((u + ui) * p.nkb + ks * p.kbs + j) * kUnit
-                                     : (u + ui) * kUnit;
+              const int x = PACKED ? 0 : (ks * p.kbs + j) * 64;
+              const int y = PACKED ? ((u + ui) * p.nkb + ks * p.kbs + j) * kUnit
+                                   : (u + ui) * kUnit;
               uint8_t* dst = a_st + j * kATile + ui * (kUnit * 128);
               if (PAIR)
                 tma_load_2d_multicast(dst, &tmap_w, &full[s], x, y, 0x3, pol_w);
@@ -225,6 +225,10 @@ __global__ void __launch_bounds__(kLmThreads, 1)
               tma_load_2d(b_st + j * b_sub + sb * p.nb * 128, &tmap_h, &full[s],
                           (ks * p.kbs + j) * 64, rbase + sb * p.nb, pol_h);
           ++it;
+          if (++s == p.stages) {
+            s = 0;
+            ph ^= 1u;
+          }
         }
       }
       if (!ok) {
@@ -241,6 +245,8 @@ __global__ void __launch_bounds__(kLmThreads, 1)
       const uint32_t idesc = umma_idesc_bf16(128, static_cast<uint32_t>(p.nb));
       const uint32_t desc_hi = static_cast<uint32_t>(umma_desc_sw128(0) >> 32);
       int it = 0, c = 0;
+      int s = 0;        // stage of iteration it, as in the producer
+      uint32_t ph = 0;
       bool ok = true;
       for (int u = u0; u < u1 && ok; u += 2, ++c) {
         const int buf = c % p.nbuf;
@@ -252,8 +258,6 @@ __global__ void __launch_bounds__(kLmThreads, 1)
         tc_fence_after();
         const uint32_t d0 = tmem_base + static_cast<uint32_t>(buf * p.acc_stride);
         for (int ks = 0; ks < p.nks; ++ks) {
-          const int s = it % p.stages;
-          const uint32_t ph = static_cast<uint32_t>(it / p.stages) & 1u;
           if (!mbar_wait(&full[s], ph, p.limit_ns, abort)) {
             ok = false;
             break;
@@ -294,6 +298,10 @@ __global__ void __launch_bounds__(kLmThreads, 1)
             else
               umma_commit(&empty[s]);
             ++it;
+            if (++s == p.stages) {
+              s = 0;
+              ph ^= 1u;
+            }
             continue;
           }
           for (int j = 0; j < nsubk; ++j) {
@@ -309,10 +317,14 @@ __global__ void __launch_bounds__(kLmThreads, 1)
             }
           }
           if (PAIR)
-              umma_commit_multicast(&empty[s], 0x3);
-            else
-              umma_commit(&empty[s]);
+            umma_commit_multicast(&empty[s], 0x3);
+          else
+            umma_commit(&empty[s]);
           ++it;
+          if (++s == p.stages) {
+            s = 0;
+            ph ^= 1u;
+          }
         }
         if (!ok) break;
         umma_commit(&acc_full[buf]);
@@ -547,11 +559,12 @@ cudaError_t launch_pack_lm(const __nv_bfloat16* w, __nv_bfloat16* out, int V, in
 }
 
 cudaError_t lm_configure() {
-  cudaError_t e = cudaFuncSetAttribute(lm_stats_kernel<true>,
-                                       cudaFuncAttributeMaxDynamicSharedMemorySize, 232448);
-  if (e != cudaSuccess) return e;
-  return cudaFuncSetAttribute(lm_stats_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              232448);
+  const cudaFuncAttribute a = cudaFuncAttributeMaxDynamicSharedMemorySize;
+  cudaError_t e;
+  if ((e = cudaFuncSetAttribute(lm_stats_kernel<true, true>, a, 232448)) != cudaSuccess) return e;
+  if ((e = cudaFuncSetAttribute(lm_stats_kernel<true, false>, a, 232448)) != cudaSuccess) return e;
+  if ((e = cudaFuncSetAttribute(lm_stats_kernel<false, true>, a, 232448)) != cudaSuccess) return e;
+  return cudaFuncSetAttribute(lm_stats_kernel<false, false>, a, 232448);
 }
 
 cudaError_t launch_lm_stats(const CUtensorMap& tmap_w, const CUtensorMap& tmap_h,
@@ -568,8 +581,11 @@ cudaError_t launch_lm_stats(const CUtensorMap& tmap_w, const CUtensorMap& tmap_h
   attr[0].val.clusterDim.z = 1;
   cfg.attrs = attr;
   cfg.numAttrs = p.pair ? 1 : 0;
-  if (p.pair) return cudaLaunchKernelEx(&cfg, lm_stats_kernel<true>, tmap_w, tmap_h, p);
-  return cudaLaunchKernelEx(&cfg, lm_stats_kernel<false>, tmap_w, tmap_h, p);
+  if (p.pair)
+    return p.packed ? cudaLaunchKernelEx(&cfg, lm_stats_kernel<true, true>, tmap_w, tmap_h, p)
+                    : cudaLaunchKernelEx(&cfg, lm_stats_kernel<true, false>, tmap_w, tmap_h, p);
+  return p.packed ? cudaLaunchKernelEx(&cfg, lm_stats_kernel<false, true>, tmap_w, tmap_h, p)
+                  : cudaLaunchKernelEx(&cfg, lm_stats_kernel<false, false>, tmap_w, tmap_h, p);
 }
 
 }  // namespace ebd
