@@ -282,10 +282,10 @@ ebd_status upload_router(ebd_handle* h) {
     uint16_t* w = lbs.data() + static_cast<size_t>(r) * LBS_W_ELEMS;
     float* v = vec.data() + static_cast<size_t>(r) * V_ELEMS;
     for (int k = 0; k < 64; ++k)
-      for (int o = 0; o < 64; ++o) w[W_ENT2 + k * 64 + o] = at("lbs.ent2.w", o, k);
+      for (int o = 0; o < 64; ++o) w[W_ENT2 + k * 64 + swz_col(k, o, 64)] = at("lbs.ent2.w", o, k);
     for (int k = 0; k < 128; ++k)
       for (int o = 0; o < kCombSlice; ++o)
-        w[W_COMB + k * kCombSlice + o] = at("lbs.comb.w", kCombSlice * r + o, k);
+        w[W_COMB + k * kCombSlice + swz_col(k, o, kCombSlice)] = at("lbs.comb.w", kCombSlice * r + o, k);
     for (int j = 0; j < kPosRows; ++j)
       for (int o = 0; o < kCombSlice; ++o)
         w[W_POS + j * kCombSlice + o] = j < gen_len ? at("lbs.pos", j, kCombSlice * r + o) : 0;
@@ -295,15 +295,15 @@ ebd_status upload_router(ebd_handle* h) {
       float* vl = v + V_LAYER0 + l * V_LAYER_STRIDE;
       for (int k = 0; k < 128; ++k) {
         for (int o = 0; o < kQkvSlice; ++o)
-          wl[WL_QKV + k * kQkvSlice + o] = at(pre + ".qkv.w", kQkvSlice * r + o, k);
+          wl[WL_QKV + k * kQkvSlice + swz_col(k, o, kQkvSlice)] = at(pre + ".qkv.w", kQkvSlice * r + o, k);
         for (int o = 0; o < kOutSlice; ++o)
-          wl[WL_OUT + k * kOutSlice + o] = at(pre + ".out.w", kOutSlice * r + o, k);
+          wl[WL_OUT + k * kOutSlice + swz_col(k, o, kOutSlice)] = at(pre + ".out.w", kOutSlice * r + o, k);
         for (int o = 0; o < kFf1Slice; ++o)
-          wl[WL_FF1 + k * kFf1Slice + o] = at(pre + ".ff1.w", kFf1Slice * r + o, k);
+          wl[WL_FF1 + k * kFf1Slice + swz_col(k, o, kFf1Slice)] = at(pre + ".ff1.w", kFf1Slice * r + o, k);
       }
       for (int hh = 0; hh < kFf1Slice; ++hh)
         for (int o = 0; o < 128; ++o)
-          wl[WL_FF2 + hh * 128 + o] = at(pre + ".ff2.w", o, kFf1Slice * r + hh);
+          wl[WL_FF2 + hh * 128 + swz_col(hh, o, 128)] = at(pre + ".ff2.w", o, kFf1Slice * r + hh);
       for (int o = 0; o < kQkvSlice; ++o) vl[VL_QKVB + o] = atf(pre + ".qkv.b", 0, kQkvSlice * r + o);
       for (int o = 0; o < kOutSlice; ++o) vl[VL_OUTB + o] = atf(pre + ".out.b", 0, kOutSlice * r + o);
       for (int o = 0; o < kFf1Slice; ++o) vl[VL_FF1B + o] = atf(pre + ".ff1.b", 0, kFf1Slice * r + o);

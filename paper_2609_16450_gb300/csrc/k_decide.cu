@@ -115,8 +115,8 @@ __device__ __forceinline__ void hl_store2(const HL& h, int j, int c, float x, fl
 // shared memory, Wt bf16 [K][ldw].  Each warp owns 16-row x 16-output tiles;
 // the high and low parts accumulate in separate chains (shorter dependency
 // chains), summed at the end.  epi(j, o, v0, v1) receives the outputs o and
-// o + 1 of row j.
-template <class Epi>
+// o + 1 of row j.  SWZ: Wt holds its 16-byte chunks permuted by swz_col.
+template <bool SWZ = false, class Epi>
 __device__ __forceinline__ void gemm_hl(const HL& A, int n, int K, const __nv_bfloat16* Wt,
                                         int ldw, int Os, Epi epi) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -131,7 +131,10 @@ __device__ __forceinline__ void gemm_hl(const HL& A, int n, int K, const __nv_bf
     const uint32_t ah_base =
         smem_u32(A.p + (m0 + (mi & 1) * 8 + rr) * A.ld + (mi >> 1) * 8);
     const uint32_t al_base = ah_base + static_cast<uint32_t>(A.plane * 2);
-    const uint32_t w_base = smem_u32(Wt + ((mi & 1) * 8 + rr) * ldw + c0 + (mi >> 1) * 8);
+    const int kr = (mi & 1) * 8 + rr;  // B row of this lane within a 16-row k step
+    const int ch = (c0 >> 3) + (mi >> 1);
+    const uint32_t w_base =
+        smem_u32(Wt + kr * ldw + 8 * (SWZ ? (ch ^ rimg::swz_mask(kr, ldw)) : ch));
 #pragma unroll 2
     for (int k0 = 0; k0 < K; k0 += 16) {
       uint32_t ah[4], al[4], b0, b1, b2, b3;
@@ -751,7 +754,7 @@ __global__ void __cluster_dims__(kDecideCluster, 1, 1) __launch_bounds__(kDecide
     // the ent2 output goes to the z hi/lo region: z itself receives the
     // other ranks' fusion outputs as soon as they get there
     float* E2 = P + P_ZH;
-    gemm_hl(Fh, n, 64, sm.w + W_ENT2, 64, 64, [&](int j, int o, float a, float b) {
+    gemm_hl<true>(Fh, n, 64, sm.w + W_ENT2, 64, 64, [&](int j, int o, float a, float b) {
       *reinterpret_cast<float2*>(E2 + j * LDZ + o) = make_float2(a + Vv[V_ENT2B + o], b + Vv[V_ENT2B + o + 1]);
     });
     __syncthreads();
@@ -768,7 +771,7 @@ __global__ void __cluster_dims__(kDecideCluster, 1, 1) __launch_bounds__(kDecide
     // 3b. fusion W_combine [e; t] + E_pos[rank of the row]: this CTA's 16 outputs
     {
       const int o0 = kCombSlice * rank;
-      gemm_hl(Xh, n, 128, sm.w + W_COMB, kCombSlice, kCombSlice, [&](int j, int o, float a, float b) {
+      gemm_hl<true>(Xh, n, 128, sm.w + W_COMB, kCombSlice, kCombSlice, [&](int j, int o, float a, float b) {
         const float2 pe = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(sm.w + W_POS + j * kCombSlice + o));
         const float2 val = make_float2(a + Vv[V_COMBB + o] + pe.x, b + Vv[V_COMBB + o + 1] + pe.y);
 #pragma unroll 1
@@ -794,7 +797,7 @@ __global__ void __cluster_dims__(kDecideCluster, 1, 1) __launch_bounds__(kDecide
       const float* Vl = Vv + V_LAYER0 + l * V_LAYER_STRIDE;
       // QKV: this CTA's 48 features for every row, scattered to the CTAs
       // that attend with them (head h lives in ranks 2h and 2h+1)
-      gemm_hl(Zh, n, 128, Wl + WL_QKV, kQkvSlice, kQkvSlice, [&](int j, int o, float a, float b) {
+      gemm_hl<true>(Zh, n, 128, Wl + WL_QKV, kQkvSlice, kQkvSlice, [&](int j, int o, float a, float b) {
         const int f = kQkvSlice * rank + o;  // even; f and f+1 share part and head
         const int part = f >> 7, h = (f >> 5) & 3, dd = f & 31;
         const float2 val = make_float2(a + Vl[VL_QKVB + o], b + Vl[VL_QKVB + o + 1]);
@@ -813,7 +816,7 @@ __global__ void __cluster_dims__(kDecideCluster, 1, 1) __launch_bounds__(kDecide
       cluster.sync();
       {  // output projection + residual, 16 outputs, written in place into z
         const int o0 = kOutSlice * rank;
-        gemm_hl(Xh, n, 128, Wl + WL_OUT, kOutSlice, kOutSlice, [&](int j, int o, float a, float b) {
+        gemm_hl<true>(Xh, n, 128, Wl + WL_OUT, kOutSlice, kOutSlice, [&](int j, int o, float a, float b) {
           const float2 zz = *reinterpret_cast<const float2*>(Z + j * LDZ + o0 + o);
           const float2 val = make_float2(zz.x + (a + Vl[VL_OUTB + o]), zz.y + (b + Vl[VL_OUTB + o + 1]));
 #pragma unroll 1
@@ -826,11 +829,11 @@ __global__ void __cluster_dims__(kDecideCluster, 1, 1) __launch_bounds__(kDecide
       __syncthreads();
       // FFN: hidden units [32r, 32r+32) locally, then the partial second
       // linear of those units sent to the owners of each 16-output slice
-      gemm_hl(Zh, n, 128, Wl + WL_FF1, kFf1Slice, kFf1Slice, [&](int j, int o, float a, float b) {
+      gemm_hl<true>(Zh, n, 128, Wl + WL_FF1, kFf1Slice, kFf1Slice, [&](int j, int o, float a, float b) {
         hl_store2(Hh, j, o, gelu(a + Vl[VL_FF1B + o]), gelu(b + Vl[VL_FF1B + o + 1]));
       });
       __syncthreads();
-      gemm_hl(Hh, n, kFf1Slice, Wl + WL_FF2, 128, 128, [&](int j, int o, float a, float b) {
+      gemm_hl<true>(Hh, n, kFf1Slice, Wl + WL_FF2, 128, 128, [&](int j, int o, float a, float b) {
         *reinterpret_cast<float2*>(cluster.map_shared_rank(Xin, o >> 4) + (rank * W + j) * 16 + (o & 15)) =
             make_float2(a, b);
       });

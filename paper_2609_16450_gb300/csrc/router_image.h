@@ -26,6 +26,20 @@ constexpr int WL_FF1 = 8192;      // [128][32]  FFN first linear, hidden slice
 constexpr int WL_FF2 = 12288;     // [32][128]  FFN second linear, rows of the hidden slice
 constexpr int LBS_W_ELEMS = W_LAYER0 + 2 * W_LAYER_STRIDE;  // 39936
 
+// The LBS matrices above except E_pos are stored with their 16-byte chunks
+// permuted within each row: element (k, c) of a [K][ld] matrix sits at
+// k * ld + swz_col(k, c, ld).  ldmatrix reads 8 consecutive rows of one
+// 8-column chunk as an mma B fragment; the XOR places those 8 row segments in
+// 8 distinct 16-byte bank groups for ld = 16, 32, 48, 64 and 128 (without it,
+// rows of 128 or 256 bytes put all 8 in one group).  K is a multiple of 16,
+// and the mask depends only on the low 3 bits of k.
+__host__ __device__ constexpr int swz_mask(int k, int ld) {
+  return ld >= 64 ? (k & 7) : ld == 32 ? ((k >> 1) & 3) : ((k >> 2) & 1);
+}
+__host__ __device__ constexpr int swz_col(int k, int c, int ld) {
+  return (((c >> 3) ^ swz_mask(k, ld)) << 3) | (c & 7);
+}
+
 // ---- LPS weights (one copy), bf16, transposed [in][out] with each row padded
 // by 8 elements so that 8 consecutive rows hit distinct banks when ldmatrix
 // reads them as mma B fragments
