@@ -164,53 +164,50 @@ __device__ __forceinline__ float group8_sum(float v) {
   return v;
 }
 
-// LayerNorm (eps 1e-5) over `dim` (32, 64 or 128) of rows j < n: 8 lanes per
-// row, lane q holding columns 4q + 32c (c < dim/32); the result goes to an
-// fp32 buffer (if dst) and/or a hi/lo buffer (if hl).  One copy of the code
-// serves every call.
-__device__ __noinline__ void ln_rows(const float* src, int lds, float* dst, int ldd, const HL* hl,
-                                     int n, int dim, const float* g, const float* b) {
+// LayerNorm (eps 1e-5) over DIM (32, 64 or 128) features of rows j < n:
+// 8 lanes per row, lane q holding columns 4q + 32c (c < DIM/32); the result
+// goes to the hi/lo buffer hl and, if DST, to an fp32 buffer (which may be
+// src itself: every lane reads its values before it writes them).
+template <int DIM, bool DST>
+__device__ __forceinline__ void ln_rows(const float* src, int lds, float* dst, int ldd, const HL hl,
+                                        int n, const float* g, const float* b) {
+  constexpr int PER = DIM / 32;
   const int q = threadIdx.x & 7;
-  const int per = dim >> 5;
-  const float inv_dim = 1.0f / static_cast<float>(dim);
 #pragma unroll 1
   for (int j0 = 0; j0 < n; j0 += (blockDim.x >> 3)) {
     const int j = j0 + (threadIdx.x >> 3);
     const bool ok = j < n;
-    float4 v[4];
+    float4 v[PER];
     float s = 0.f;
 #pragma unroll
-    for (int c = 0; c < 4; ++c) {
-      v[c] = make_float4(0.f, 0.f, 0.f, 0.f);
-      if (c < per && ok) v[c] = *reinterpret_cast<const float4*>(src + j * lds + 4 * q + 32 * c);
+    for (int c = 0; c < PER; ++c) {
+      v[c] = ok ? *reinterpret_cast<const float4*>(src + j * lds + 4 * q + 32 * c)
+                : make_float4(0.f, 0.f, 0.f, 0.f);
       s += (v[c].x + v[c].y) + (v[c].z + v[c].w);
     }
-    const float mean = group8_sum(s) * inv_dim;
+    const float mean = group8_sum(s) * (1.0f / DIM);
     float var = 0.f;
 #pragma unroll
-    for (int c = 0; c < 4; ++c)
-      if (c < per) {
-        const float a0 = v[c].x - mean, a1 = v[c].y - mean, a2 = v[c].z - mean, a3 = v[c].w - mean;
-        var += (a0 * a0 + a1 * a1) + (a2 * a2 + a3 * a3);
-      }
-    const float inv = 1.0f / sqrtf(group8_sum(var) * inv_dim + 1e-5f);
+    for (int c = 0; c < PER; ++c) {
+      const float a0 = v[c].x - mean, a1 = v[c].y - mean, a2 = v[c].z - mean, a3 = v[c].w - mean;
+      var += (a0 * a0 + a1 * a1) + (a2 * a2 + a3 * a3);
+    }
+    const float inv = rsqrtf(group8_sum(var) * (1.0f / DIM) + 1e-5f);
     if (ok) {
 #pragma unroll
-      for (int c = 0; c < 4; ++c)
-        if (c < per) {
-          const int o = 4 * q + 32 * c;
-          const float4 gg = *reinterpret_cast<const float4*>(g + o);
-          const float4 bb = *reinterpret_cast<const float4*>(b + o);
-          const float4 y = make_float4((v[c].x - mean) * inv * gg.x + bb.x,
-                                       (v[c].y - mean) * inv * gg.y + bb.y,
-                                       (v[c].z - mean) * inv * gg.z + bb.z,
-                                       (v[c].w - mean) * inv * gg.w + bb.w);
-          if (dst) *reinterpret_cast<float4*>(dst + j * ldd + o) = y;
-          if (hl) {
-            hl_store2(*hl, j, o, y.x, y.y);
-            hl_store2(*hl, j, o + 2, y.z, y.w);
-          }
-        }
+      for (int c = 0; c < PER; ++c) {
+        const int o = 4 * q + 32 * c;
+        const float4 gg = *reinterpret_cast<const float4*>(g + o);
+        const float4 bb = *reinterpret_cast<const float4*>(b + o);
+        const float4 y = make_float4((v[c].x - mean) * inv * gg.x + bb.x, (v[c].y - mean) * inv * gg.y + bb.y,
+                                     (v[c].z - mean) * inv * gg.z + bb.z, (v[c].w - mean) * inv * gg.w + bb.w);
+        if (DST) *reinterpret_cast<float4*>(dst + j * ldd + o) = y;
+        uint32_t h0, l0, h1, l1;
+        split_bf16x2(y.x, y.y, h0, l0);
+        split_bf16x2(y.z, y.w, h1, l1);
+        *reinterpret_cast<uint2*>(hl.p + j * hl.ld + o) = make_uint2(h0, h1);
+        *reinterpret_cast<uint2*>(hl.p + hl.plane + j * hl.ld + o) = make_uint2(l0, l1);
+      }
     }
   }
 }
@@ -515,7 +512,7 @@ __device__ __noinline__ void lps_forward(float* P, int n, const __nv_bfloat16* W
     const __nv_bfloat16* Wl = Wlps + l * PL_STRIDE;
     const float* Vl = V + VP_LAYER0 + l * VP_LAYER_STRIDE;
     const int f = l == 0 ? from : 0;
-    if (f <= 1) ln_rows(Z, LDQ, nullptr, 0, &Y, n, 32, Vl + VPL_LN1G, Vl + VPL_LN1B);
+    if (f <= 1) ln_rows<32, false>(Z, LDQ, nullptr, 0, Y, n, Vl + VPL_LN1G, Vl + VPL_LN1B);
     __syncthreads();
     if (f <= 2)
       gemm_hl(Y, n, 32, Wl + PL_QKV, PL_LDQKV, 96, [&](int j, int o, float a, float b) {
@@ -535,7 +532,7 @@ __device__ __noinline__ void lps_forward(float* P, int n, const __nv_bfloat16* W
         *z = make_float2(zz.x + (a + Vl[VPL_OUTB + o]), zz.y + (b + Vl[VPL_OUTB + o + 1]));
       });
     __syncthreads();
-    if (f <= 5) ln_rows(Z, LDQ, nullptr, 0, &Y, n, 32, Vl + VPL_LN2G, Vl + VPL_LN2B);
+    if (f <= 5) ln_rows<32, false>(Z, LDQ, nullptr, 0, Y, n, Vl + VPL_LN2G, Vl + VPL_LN2B);
     __syncthreads();
     if (f <= 6)
       gemm_hl(Y, n, 32, Wl + PL_FF1, PL_LDFF1, 64, [&](int j, int o, float a, float b) {
@@ -758,7 +755,7 @@ __global__ void __cluster_dims__(kDecideCluster, 1, 1) __launch_bounds__(kDecide
       *reinterpret_cast<float2*>(E2 + j * LDZ + o) = make_float2(a + Vv[V_ENT2B + o], b + Vv[V_ENT2B + o + 1]);
     });
     __syncthreads();
-    ln_rows(E2, LDZ, nullptr, 0, &Xh, n, 64, Vv + V_ENTLNG, Vv + V_ENTLNB);
+    ln_rows<64, false>(E2, LDZ, nullptr, 0, Xh, n, Vv + V_ENTLNG, Vv + V_ENTLNB);
 #pragma unroll
     for (int k = 0; k < 8; ++k) {  // the token branch into columns 64..127
       const int it = tid + k * kDecideThreads;
@@ -825,7 +822,7 @@ __global__ void __cluster_dims__(kDecideCluster, 1, 1) __launch_bounds__(kDecide
         });
       }
       cluster.sync();
-      ln_rows(Z, LDZ, Z, LDZ, &Zh, n, 128, Vl + VL_LN1G, Vl + VL_LN1B);
+      ln_rows<128, true>(Z, LDZ, Z, LDZ, Zh, n, Vl + VL_LN1G, Vl + VL_LN1B);
       __syncthreads();
       // FFN: hidden units [32r, 32r+32) locally, then the partial second
       // linear of those units sent to the owners of each 16-output slice
@@ -858,7 +855,7 @@ __global__ void __cluster_dims__(kDecideCluster, 1, 1) __launch_bounds__(kDecide
         }
       }
       cluster.sync();
-      ln_rows(Z, LDZ, Z, LDZ, &Zh, n, 128, Vl + VL_LN2G, Vl + VL_LN2B);
+      ln_rows<128, true>(Z, LDZ, Z, LDZ, Zh, n, Vl + VL_LN2G, Vl + VL_LN2B);
       __syncthreads();
       if (l == 0 && rank == 0 && tid == 0 && p.lps_enabled) {
         // the first layer's weights (and everything before them) are dead:
