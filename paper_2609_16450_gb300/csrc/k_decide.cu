@@ -111,48 +111,50 @@ __device__ __forceinline__ void hl_store2(const HL& h, int j, int c, float x, fl
   *reinterpret_cast<uint32_t*>(h.p + h.plane + j * h.ld + c) = lo;
 }
 
+__device__ __forceinline__ void ldsm_x2_t(uint32_t addr, uint32_t& r0, uint32_t& r1) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x2.trans.shared.b16 {%0,%1}, [%2];"
+               : "=r"(r0), "=r"(r1)
+               : "r"(addr));
+}
+
 // out(j, o) = sum_k A[j][k] Wt[k][o] for j < n, o < Os, A = hi + lo in
-// shared memory, Wt bf16 [K][ldw].  Each warp owns 16-row x 16-output tiles;
-// the high and low parts accumulate in separate chains (shorter dependency
-// chains), summed at the end.  epi(j, o, v0, v1) receives the outputs o and
-// o + 1 of row j.  SWZ: Wt holds its 16-byte chunks permuted by swz_col.
+// shared memory, Wt bf16 [K][ldw].  Each warp owns 16-row x 8-output tiles:
+// with the few rows of a window, narrow tiles spread a product over more
+// warps, and the tensor-core work per warp bounds a phase.  The high and low
+// parts accumulate in separate chains, summed at the end.  epi(j, o, v0, v1)
+// receives the outputs o and o + 1 of row j.  SWZ: Wt holds its 16-byte
+// chunks permuted by swz_col.
 template <bool SWZ = false, class Epi>
 __device__ __forceinline__ void gemm_hl(const HL& A, int n, int K, const __nv_bfloat16* Wt,
                                         int ldw, int Os, Epi epi) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int g = lane >> 2, t = lane & 3;
   const int mi = lane >> 3, rr = lane & 7;
-  const int mt = (n + 15) >> 4, np = Os >> 4;
+  const int mt = (n + 15) >> 4, np = Os >> 3;
+  const int kr = lane & 15;  // B row of this lane within a 16-row k step (lanes 16..31 unused)
 #pragma unroll 1
   for (int unit = warp; unit < mt * np; unit += (blockDim.x >> 5)) {
-    const int m0 = (unit / np) * 16, c0 = (unit % np) * 16;
-    float acc[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
-    float acl[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
+    const int m0 = (unit / np) * 16, c0 = (unit % np) * 8;
+    float acc[4] = {0.f, 0.f, 0.f, 0.f}, acl[4] = {0.f, 0.f, 0.f, 0.f};
     const uint32_t ah_base =
         smem_u32(A.p + (m0 + (mi & 1) * 8 + rr) * A.ld + (mi >> 1) * 8);
     const uint32_t al_base = ah_base + static_cast<uint32_t>(A.plane * 2);
-    const int kr = (mi & 1) * 8 + rr;  // B row of this lane within a 16-row k step
-    const int ch = (c0 >> 3) + (mi >> 1);
+    const int ch = c0 >> 3;
     const uint32_t w_base =
         smem_u32(Wt + kr * ldw + 8 * (SWZ ? (ch ^ rimg::swz_mask(kr, ldw)) : ch));
 #pragma unroll 2
     for (int k0 = 0; k0 < K; k0 += 16) {
-      uint32_t ah[4], al[4], b0, b1, b2, b3;
+      uint32_t ah[4], al[4], b0, b1;
       ldsm_x4(ah_base + k0 * 2, ah[0], ah[1], ah[2], ah[3]);
       ldsm_x4(al_base + k0 * 2, al[0], al[1], al[2], al[3]);
-      ldsm_x4_t(w_base + static_cast<uint32_t>(k0 * ldw * 2), b0, b1, b2, b3);
-      mma_bf16(acc[0], ah, b0, b1);
-      mma_bf16(acc[1], ah, b2, b3);
-      mma_bf16(acl[0], al, b0, b1);
-      mma_bf16(acl[1], al, b2, b3);
+      ldsm_x2_t(w_base + static_cast<uint32_t>(k0 * ldw * 2), b0, b1);
+      mma_bf16(acc, ah, b0, b1);
+      mma_bf16(acl, al, b0, b1);
     }
     const int r_lo = m0 + g, r_hi = r_lo + 8;
-#pragma unroll
-    for (int nt = 0; nt < 2; ++nt) {
-      const int o = c0 + nt * 8 + 2 * t;
-      if (r_lo < n) epi(r_lo, o, acc[nt][0] + acl[nt][0], acc[nt][1] + acl[nt][1]);
-      if (r_hi < n) epi(r_hi, o, acc[nt][2] + acl[nt][2], acc[nt][3] + acl[nt][3]);
-    }
+    const int o = c0 + 2 * t;
+    if (r_lo < n) epi(r_lo, o, acc[0] + acl[0], acc[1] + acl[1]);
+    if (r_hi < n) epi(r_hi, o, acc[2] + acl[2], acc[3] + acl[3]);
   }
 }
 
