@@ -235,20 +235,36 @@ __device__ __forceinline__ void merge_state(float& m, float& s, float& t, float&
 
 // ------------------------------------------------------------------ LBS attention
 // This CTA's query rows [qa, qa + nq) of head hd (width 32) over the n rows'
-// keys/values: softmax(q k^T / sqrt(32)) v on the tensor cores, 16 query rows
-// per warp, keys in blocks of 16 with a running max and sum.  q, k, v and the
-// probabilities are split into bf16 high and low parts (three products per
-// pair).  The output goes, as hi/lo, to this CTA's concat buffer, and from
-// there, 16 bytes at a time by the whole CTA, to the other ranks'.
+// keys/values: softmax(q k^T / sqrt(32)) v on the tensor cores.  q, k, v and
+// the probabilities are split into bf16 high and low parts (three products
+// per pair).  The work is spread over the warps: a warp takes one 16-query
+// tile, one block of 16 keys and (when tiles x blocks leave warps idle) a
+// group of the 8-column output tiles, and leaves its block's row max m, sum l
+// and unnormalised output o in shared memory (the z hi/lo region, free
+// between the QKV product and the next LayerNorm).  The whole CTA then
+// combines the blocks, out = sum_b e^(m_b - M) o_b / sum_b e^(m_b - M) l_b,
+// and writes the result as hi/lo, 16 bytes per store, into every rank's
+// concat buffer.
+constexpr int kAttLdp = 40;  // row stride of a partial output tile (floats)
+
 __device__ __forceinline__ void lbs_attention(cg::cluster_group& cluster, float* P, int nq, int n,
                                               int qa, int hd) {
   const float* Q = P + P_Q;
   const float* KV = P + P_KV;
+  float* part_o = P + P_ZH;                    // [unit][16][kAttLdp]
+  float* part_ml = part_o + 8 * 16 * kAttLdp;  // [unit][16][2]
+  static_assert(8 * 16 * (kAttLdp + 2) <= W * LDH, "attention partials fit the z hi/lo region");
   __nv_bfloat16* X = reinterpret_cast<__nv_bfloat16*>(P + P_XH);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, g = lane >> 2, t = lane & 3;
   const float scale = 0.17677669529663687f;  // 1/sqrt(32)
-  if (warp < ((nq + 15) >> 4)) {
-    const int r_lo = warp * 16 + g, r_hi = r_lo + 8;
+  const int mtq = (nq + 15) >> 4, nkb = (n + 15) >> 4;
+  const int units = mtq * nkb;  // <= 2 x 4
+  const int nsplit = units <= 2 ? 4 : (units <= 4 ? 2 : 1);
+  if (warp < units * nsplit) {
+    const int u = warp / nsplit, part = warp % nsplit;
+    const int qt = u / nkb, kb = u % nkb;
+    const int nt0 = part * (4 / nsplit), nt1 = nt0 + 4 / nsplit;
+    const int r_lo = qt * 16 + g, r_hi = r_lo + 8;
     uint32_t qh[2][4], ql[2][4];
 #pragma unroll
     for (int ks = 0; ks < 2; ++ks) {
@@ -264,106 +280,122 @@ __device__ __forceinline__ void lbs_attention(cg::cluster_group& cluster, float*
       split_bf16x2(a2.x, a2.y, qh[ks][2], ql[ks][2]);
       split_bf16x2(a3.x, a3.y, qh[ks][3], ql[ks][3]);
     }
-    float mx0 = -INFINITY, mx1 = -INFINITY, l0 = 0.f, l1 = 0.f;
-    float o[4][4];
+    const int k0 = 16 * kb;
+    float s[2][4];
 #pragma unroll
-    for (int nt = 0; nt < 4; ++nt) o[nt][0] = o[nt][1] = o[nt][2] = o[nt][3] = 0.f;
-#pragma unroll 1
-    for (int k0 = 0; k0 < n; k0 += 16) {
-      float s[2][4];
+    for (int hb = 0; hb < 2; ++hb) {
+      const int key = k0 + 8 * hb + g;
+      float a[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-      for (int hb = 0; hb < 2; ++hb) {
-        const int key = k0 + 8 * hb + g;
-        float a[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll
-        for (int ks = 0; ks < 2; ++ks) {
-          const float2 z = make_float2(0.f, 0.f);
-          const float* kp = KV + key * LDKV + 16 * ks + 2 * t;
-          const float2 k0v = key < n ? *reinterpret_cast<const float2*>(kp) : z;
-          const float2 k1v = key < n ? *reinterpret_cast<const float2*>(kp + 8) : z;
-          uint32_t bh0, bl0, bh1, bl1;
-          split_bf16x2(k0v.x, k0v.y, bh0, bl0);
-          split_bf16x2(k1v.x, k1v.y, bh1, bl1);
-          mma_bf16(a, qh[ks], bh0, bh1);
-          mma_bf16(a, qh[ks], bl0, bl1);
-          mma_bf16(a, ql[ks], bh0, bh1);
-        }
-        const int c = k0 + 8 * hb + 2 * t;
-        s[hb][0] = c < n ? a[0] * scale : -INFINITY;
-        s[hb][1] = c + 1 < n ? a[1] * scale : -INFINITY;
-        s[hb][2] = c < n ? a[2] * scale : -INFINITY;
-        s[hb][3] = c + 1 < n ? a[3] * scale : -INFINITY;
+      for (int ks = 0; ks < 2; ++ks) {
+        const float2 z = make_float2(0.f, 0.f);
+        const float* kp = KV + key * LDKV + 16 * ks + 2 * t;
+        const float2 k0v = key < n ? *reinterpret_cast<const float2*>(kp) : z;
+        const float2 k1v = key < n ? *reinterpret_cast<const float2*>(kp + 8) : z;
+        uint32_t bh0, bl0, bh1, bl1;
+        split_bf16x2(k0v.x, k0v.y, bh0, bl0);
+        split_bf16x2(k1v.x, k1v.y, bh1, bl1);
+        mma_bf16(a, qh[ks], bh0, bh1);
+        mma_bf16(a, qh[ks], bl0, bl1);
+        mma_bf16(a, ql[ks], bh0, bh1);
       }
-      float b0 = fmaxf(fmaxf(s[0][0], s[0][1]), fmaxf(s[1][0], s[1][1]));
-      float b1 = fmaxf(fmaxf(s[0][2], s[0][3]), fmaxf(s[1][2], s[1][3]));
-      b0 = fmaxf(b0, __shfl_xor_sync(0xffffffffu, b0, 1));
-      b0 = fmaxf(b0, __shfl_xor_sync(0xffffffffu, b0, 2));
-      b1 = fmaxf(b1, __shfl_xor_sync(0xffffffffu, b1, 1));
-      b1 = fmaxf(b1, __shfl_xor_sync(0xffffffffu, b1, 2));
-      const float n0 = fmaxf(mx0, b0), n1 = fmaxf(mx1, b1);  // finite: key k0 is valid
-      const float c0 = expf(mx0 - n0), c1 = expf(mx1 - n1);
-      mx0 = n0;
-      mx1 = n1;
-#pragma unroll
-      for (int hb = 0; hb < 2; ++hb) {
-        s[hb][0] = expf(s[hb][0] - n0);
-        s[hb][1] = expf(s[hb][1] - n0);
-        s[hb][2] = expf(s[hb][2] - n1);
-        s[hb][3] = expf(s[hb][3] - n1);
-      }
-      l0 = l0 * c0 + ((s[0][0] + s[0][1]) + (s[1][0] + s[1][1]));
-      l1 = l1 * c1 + ((s[0][2] + s[0][3]) + (s[1][2] + s[1][3]));
-      uint32_t ph[4], pl[4];
-      split_bf16x2(s[0][0], s[0][1], ph[0], pl[0]);
-      split_bf16x2(s[0][2], s[0][3], ph[1], pl[1]);
-      split_bf16x2(s[1][0], s[1][1], ph[2], pl[2]);
-      split_bf16x2(s[1][2], s[1][3], ph[3], pl[3]);
-#pragma unroll
-      for (int nt = 0; nt < 4; ++nt) {
-        o[nt][0] *= c0;
-        o[nt][1] *= c0;
-        o[nt][2] *= c1;
-        o[nt][3] *= c1;
-        float v[4];
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          const int key = k0 + (e >> 1) * 8 + 2 * t + (e & 1);
-          v[e] = key < n ? KV[key * LDKV + 32 + 8 * nt + g] : 0.f;
-        }
-        uint32_t v0h, v0l, v1h, v1l;
-        split_bf16x2(v[0], v[1], v0h, v0l);
-        split_bf16x2(v[2], v[3], v1h, v1l);
-        mma_bf16(o[nt], ph, v0h, v1h);
-        mma_bf16(o[nt], ph, v0l, v1l);
-        mma_bf16(o[nt], pl, v0h, v1h);
-      }
+      const int c = k0 + 8 * hb + 2 * t;
+      s[hb][0] = c < n ? a[0] * scale : -INFINITY;
+      s[hb][1] = c + 1 < n ? a[1] * scale : -INFINITY;
+      s[hb][2] = c < n ? a[2] * scale : -INFINITY;
+      s[hb][3] = c + 1 < n ? a[3] * scale : -INFINITY;
     }
-    l0 += __shfl_xor_sync(0xffffffffu, l0, 1);
-    l0 += __shfl_xor_sync(0xffffffffu, l0, 2);
-    l1 += __shfl_xor_sync(0xffffffffu, l1, 1);
-    l1 += __shfl_xor_sync(0xffffffffu, l1, 2);
-    const float i0 = 1.0f / l0, i1 = 1.0f / l1;
-    const HL Xl{X, LDH, W * LDH};
+    float m0 = fmaxf(fmaxf(s[0][0], s[0][1]), fmaxf(s[1][0], s[1][1]));
+    float m1 = fmaxf(fmaxf(s[0][2], s[0][3]), fmaxf(s[1][2], s[1][3]));
+    m0 = fmaxf(m0, __shfl_xor_sync(0xffffffffu, m0, 1));
+    m0 = fmaxf(m0, __shfl_xor_sync(0xffffffffu, m0, 2));
+    m1 = fmaxf(m1, __shfl_xor_sync(0xffffffffu, m1, 1));
+    m1 = fmaxf(m1, __shfl_xor_sync(0xffffffffu, m1, 2));  // finite: key k0 is valid
+#pragma unroll
+    for (int hb = 0; hb < 2; ++hb) {
+      s[hb][0] = expf(s[hb][0] - m0);
+      s[hb][1] = expf(s[hb][1] - m0);
+      s[hb][2] = expf(s[hb][2] - m1);
+      s[hb][3] = expf(s[hb][3] - m1);
+    }
+    uint32_t ph[4], pl[4];
+    split_bf16x2(s[0][0], s[0][1], ph[0], pl[0]);
+    split_bf16x2(s[0][2], s[0][3], ph[1], pl[1]);
+    split_bf16x2(s[1][0], s[1][1], ph[2], pl[2]);
+    split_bf16x2(s[1][2], s[1][3], ph[3], pl[3]);
+    float* po = part_o + u * 16 * kAttLdp;
 #pragma unroll
     for (int nt = 0; nt < 4; ++nt) {
-      const int col = 32 * hd + 8 * nt + 2 * t;
-      if (r_lo < nq) hl_store2(Xl, qa + r_lo, col, o[nt][0] * i0, o[nt][1] * i0);
-      if (r_hi < nq) hl_store2(Xl, qa + r_hi, col, o[nt][2] * i1, o[nt][3] * i1);
+      if (nt < nt0 || nt >= nt1) continue;
+      float o[4] = {0.f, 0.f, 0.f, 0.f};
+      float v[4];
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const int key = k0 + (e >> 1) * 8 + 2 * t + (e & 1);
+        v[e] = key < n ? KV[key * LDKV + 32 + 8 * nt + g] : 0.f;
+      }
+      uint32_t v0h, v0l, v1h, v1l;
+      split_bf16x2(v[0], v[1], v0h, v0l);
+      split_bf16x2(v[2], v[3], v1h, v1l);
+      mma_bf16(o, ph, v0h, v1h);
+      mma_bf16(o, ph, v0l, v1l);
+      mma_bf16(o, pl, v0h, v1h);
+      *reinterpret_cast<float2*>(po + g * kAttLdp + 8 * nt + 2 * t) = make_float2(o[0], o[1]);
+      *reinterpret_cast<float2*>(po + (g + 8) * kAttLdp + 8 * nt + 2 * t) = make_float2(o[2], o[3]);
+    }
+    if (part == 0) {
+      float l0 = (s[0][0] + s[0][1]) + (s[1][0] + s[1][1]);
+      float l1 = (s[0][2] + s[0][3]) + (s[1][2] + s[1][3]);
+      l0 += __shfl_xor_sync(0xffffffffu, l0, 1);
+      l0 += __shfl_xor_sync(0xffffffffu, l0, 2);
+      l1 += __shfl_xor_sync(0xffffffffu, l1, 1);
+      l1 += __shfl_xor_sync(0xffffffffu, l1, 2);
+      if (t == 0) {
+        float* pm = part_ml + u * 32;
+        *reinterpret_cast<float2*>(pm + 2 * g) = make_float2(m0, l0);
+        *reinterpret_cast<float2*>(pm + 2 * (g + 8)) = make_float2(m1, l1);
+      }
     }
   }
   __syncthreads();
-  // this CTA's slice of the concat buffer (rows [qa, qa+nq), columns of head
-  // hd, both planes) to the other ranks, 16 bytes per store
-  const int rank = static_cast<int>(cluster.block_rank());
+  // combine: one thread per (query row, 8 output columns), both planes to
+  // every rank (this one included)
 #pragma unroll 1
-  for (int it = threadIdx.x; it < nq * 8; it += blockDim.x) {
-    const int row = qa + (it >> 3), plane = (it >> 2) & 1, q4 = it & 3;
-    const int off = plane * W * LDH + row * LDH + 32 * hd + 8 * q4;
-    const uint4 val = *reinterpret_cast<const uint4*>(X + off);
+  for (int it = threadIdx.x; it < nq * 4; it += blockDim.x) {
+    const int r = it >> 2, c8 = it & 3, qt = r >> 4, rr = r & 15;
+    float M = -INFINITY;
 #pragma unroll 1
-    for (int r = 0; r < kDecideCluster; ++r) {
-      if (r == rank) continue;
-      *reinterpret_cast<uint4*>(cluster.map_shared_rank(X, r) + off) = val;
+    for (int kb = 0; kb < nkb; ++kb) M = fmaxf(M, part_ml[(qt * nkb + kb) * 32 + 2 * rr]);
+    float L = 0.f, acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+#pragma unroll 1
+    for (int kb = 0; kb < nkb; ++kb) {
+      const int u = qt * nkb + kb;
+      const float2 ml = *reinterpret_cast<const float2*>(part_ml + u * 32 + 2 * rr);
+      const float e = expf(ml.x - M);
+      L = fmaf(e, ml.y, L);
+      const float4* src = reinterpret_cast<const float4*>(part_o + (u * 16 + rr) * kAttLdp + 8 * c8);
+      const float4 x0 = src[0], x1 = src[1];
+      acc[0] = fmaf(e, x0.x, acc[0]);
+      acc[1] = fmaf(e, x0.y, acc[1]);
+      acc[2] = fmaf(e, x0.z, acc[2]);
+      acc[3] = fmaf(e, x0.w, acc[3]);
+      acc[4] = fmaf(e, x1.x, acc[4]);
+      acc[5] = fmaf(e, x1.y, acc[5]);
+      acc[6] = fmaf(e, x1.z, acc[6]);
+      acc[7] = fmaf(e, x1.w, acc[7]);
+    }
+    const float iL = 1.0f / L;
+    uint4 hi, lo;
+    split_bf16x2(acc[0] * iL, acc[1] * iL, hi.x, lo.x);
+    split_bf16x2(acc[2] * iL, acc[3] * iL, hi.y, lo.y);
+    split_bf16x2(acc[4] * iL, acc[5] * iL, hi.z, lo.z);
+    split_bf16x2(acc[6] * iL, acc[7] * iL, hi.w, lo.w);
+    const int off = (qa + r) * LDH + 32 * hd + 8 * c8;
+#pragma unroll 1
+    for (int rk = 0; rk < kDecideCluster; ++rk) {
+      __nv_bfloat16* dst = cluster.map_shared_rank(X, rk);
+      *reinterpret_cast<uint4*>(dst + off) = hi;
+      *reinterpret_cast<uint4*>(dst + W * LDH + off) = lo;
     }
   }
 }
