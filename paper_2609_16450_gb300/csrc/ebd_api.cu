@@ -663,7 +663,7 @@ ebd_status ebd_create(const ebd_config* cfg, ebd_handle** out) {
   cudaDeviceGetAttribute(&cc_major, cudaDevAttrComputeCapabilityMajor, h->device);
   cudaDeviceGetAttribute(&cc_minor, cudaDevAttrComputeCapabilityMinor, h->device);
   if (cc_major != 10 || cc_minor != 3)
-    return bail(fail(h, EBD_ERR_UNSUPPORTED, "this build targets sm_103a (GB300) only"));
+    return bail(fail(h, EBD_ERR_UNSUPPORTED, "the library is compiled for sm_103a (GB300) only"));
   if (get_encode() == nullptr)
     return bail(fail(h, EBD_ERR_CUDA, "cuTensorMapEncodeTiled is unavailable"));
   if ((e = lm_configure()) != cudaSuccess) return bail(cuda_fail(h, e, "LM-head attributes"));

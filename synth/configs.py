@@ -55,24 +55,24 @@ class Shape:
         return replace(self, **kw)
 
 
-# configs[0]: one small step the oracle finishes in seconds.
+# Tiny step: one small step the oracle finishes in seconds.
 tiny = Shape(name="tiny", batch=1, d_model=256, vocab=4096, n_heads_q=4,
              n_heads_kv=4, head_dim=64, prefix=128, windows=(32,),
              mask_frac=0.75, gen_len=512, w_lm_std=0.02, seed=0)
 
-# configs[1]: LLaDA-8B shaped step (hidden 4096, vocab 126464, 32x128 MHA).
+# LLaDA-8B shaped step (hidden 4096, vocab 126464, 32x128 MHA).
 llada = Shape(name="llada8b", batch=1, d_model=4096, vocab=126464,
               n_heads_q=32, n_heads_kv=32, head_dim=128, prefix=512,
               windows=(32,), mask_frac=0.75, gen_len=512,
               w_lm_std=1.0 / 64.0, seed=1)
 
-# configs[2]: Dream-7B shaped step (hidden 3584, vocab 152064, GQA 28/4).
+# Dream-7B shaped step (hidden 3584, vocab 152064, GQA 28/4).
 dream = Shape(name="dream7b", batch=8, d_model=3584, vocab=152064,
               n_heads_q=28, n_heads_kv=4, head_dim=128, prefix=1024,
               windows=None, mask_frac=0.75, gen_len=512,
               w_lm_std=1.0 / 64.0, tau_psi=0.90, seed=2)
 
-# configs[3]: the full decoding loop at LLaDA-8B shape, prompt 256, gen 256.
+# The full decoding loop at LLaDA-8B shape, prompt 256, gen 256.
 loop_shape = Shape(name="loop_llada8b", batch=1, d_model=4096, vocab=126464,
                    n_heads_q=32, n_heads_kv=32, head_dim=128, prefix=256,
                    windows=(64,), mask_frac=1.0, gen_len=256,
@@ -88,7 +88,7 @@ SHAPES = {s.name: s for s in (tiny, llada, dream, loop_shape, loop_tiny)}
 
 
 def sweep_points():
-    """configs[4]: batch x cached prefix x window at the LLaDA-8B head shape."""
+    """Throughput sweep: batch x cached prefix x window at the LLaDA-8B head shape."""
     pts = []
     k = 0
     for b in (1, 4, 16, 64):
