@@ -35,6 +35,8 @@ struct LmParams {
   int pair;                 // clusters of 2 CTAs: W multicast, rows split in halves
   int rhalf;                // rows of one CTA of a pair (rows of the launch otherwise)
   int ncols;                // partial states per row written (>= grid; extra ones neutral)
+  int mch;                  // 128-row vocabulary chunks per pipeline stage (1, or 2: one
+                            // hidden tile feeds two accumulators)
   uint32_t off_a, off_b, off_t, off_st, off_bar, smem_bytes;
   float4* part_f;           // [R][grid] (max, sum exp, sum exp*(l-max), second logit)
   int* part_i;              // [R][grid] argmax

@@ -102,9 +102,12 @@ __device__ __forceinline__ void record_error(int* status, volatile int* abort, i
 
 }  // namespace
 
-// PAIR (p.pair) and PACKED (p.packed) are template parameters: a runtime
-// branch in the single-thread producer or MMA loop costs measurable time
-template <bool PAIR, bool PACKED>
+// PAIR (p.pair), PACKED (p.packed) and MCH (p.mch) are template parameters:
+// a runtime branch in the single-thread producer or MMA loop costs
+// measurable time.  With MCH = 2 a pipeline stage holds two 128-row chunks of
+// W and one tile of hidden rows; the chunks accumulate into two TMEM regions,
+// which halves the hidden bytes per MMA where the tensor cores are the bound.
+template <bool PAIR, bool PACKED, int MCH>
 __global__ void __launch_bounds__(kLmThreads, 1)
     lm_stats_kernel(const __grid_constant__ CUtensorMap tmap_w,
                     const __grid_constant__ CUtensorMap tmap_h, const LmParams p) {
@@ -181,7 +184,8 @@ __global__ void __launch_bounds__(kLmThreads, 1)
   const int u0 = static_cast<int>((static_cast<long long>(cta) * p.n_units) / p.grid);
   const int u1 = static_cast<int>((static_cast<long long>(cta + 1) * p.n_units) / p.grid);
   const uint32_t b_sub = static_cast<uint32_t>(p.n_pad) * 128u;  // one k-box of hidden rows
-  const uint32_t a_stage = static_cast<uint32_t>(p.kbs) * kATile;
+  const uint32_t a_chunk = static_cast<uint32_t>(p.kbs) * kATile;  // one chunk's k-boxes
+  const uint32_t a_stage = static_cast<uint32_t>(MCH) * a_chunk;
   const uint32_t b_stage = static_cast<uint32_t>(p.kbs) * b_sub;
 
   if (warp == 0) {
@@ -193,8 +197,8 @@ __global__ void __launch_bounds__(kLmThreads, 1)
       int s = 0;        // stage of iteration it (it % stages, kept as a counter)
       uint32_t ph = 0;  // its phase parity
       bool ok = true;
-      for (int u = u0; u < u1 && ok; u += 2) {
-        const int nu = min(2, u1 - u);
+      for (int u = u0; u < u1 && ok; u += 2 * MCH) {
+        const int nu = min(2 * MCH, u1 - u);
         for (int ks = 0; ks < p.nks; ++ks) {
           if (!mbar_wait(&empty[s], ph ^ 1u, p.limit_ns, abort)) {
             ok = false;
@@ -208,12 +212,12 @@ __global__ void __launch_bounds__(kLmThreads, 1)
           // one row half at a time, its k-boxes back to back: each W row is
           // requested as one contiguous run of nsubk * 128 bytes
           for (int ui = 0; ui < nu; ++ui) {
-            if (PAIR && ui != static_cast<int>(crank)) continue;  // the peer loads it
+            if (PAIR && (ui & 1) != static_cast<int>(crank)) continue;  // the peer loads it
             for (int j = 0; j < nsubk; ++j) {
               const int x = PACKED ? 0 : (ks * p.kbs + j) * 64;
               const int y = PACKED ? ((u + ui) * p.nkb + ks * p.kbs + j) * kUnit
                                    : (u + ui) * kUnit;
-              uint8_t* dst = a_st + j * kATile + ui * (kUnit * 128);
+              uint8_t* dst = a_st + (ui >> 1) * a_chunk + j * kATile + (ui & 1) * (kUnit * 128);
               if (PAIR)
                 tma_load_2d_multicast(dst, &tmap_w, &full[s], x, y, 0x3, pol_w);
               else
@@ -248,7 +252,8 @@ __global__ void __launch_bounds__(kLmThreads, 1)
       int s = 0;        // stage of iteration it, as in the producer
       uint32_t ph = 0;
       bool ok = true;
-      for (int u = u0; u < u1 && ok; u += 2, ++c) {
+      for (int u = u0; u < u1 && ok; u += 2 * MCH, ++c) {
+        const int nch = MCH == 1 ? 1 : (min(2 * MCH, u1 - u) + 1) >> 1;  // chunks holding W
         const int buf = c % p.nbuf;
         const uint32_t bph = static_cast<uint32_t>(c / p.nbuf) & 1u;
         if (!mbar_wait(&acc_empty[buf], bph ^ 1u, p.limit_ns, abort)) {
@@ -256,7 +261,7 @@ __global__ void __launch_bounds__(kLmThreads, 1)
           break;
         }
         tc_fence_after();
-        const uint32_t d0 = tmem_base + static_cast<uint32_t>(buf * p.acc_stride);
+        const uint32_t d0 = tmem_base + static_cast<uint32_t>(buf * MCH * p.acc_stride);
         for (int ks = 0; ks < p.nks; ++ks) {
           if (!mbar_wait(&full[s], ph, p.limit_ns, abort)) {
             ok = false;
@@ -268,31 +273,36 @@ __global__ void __launch_bounds__(kLmThreads, 1)
           const uint32_t b_addr = smem_u32(sB + static_cast<size_t>(s) * b_stage);
           if (p.nsub <= 2 && nsubk >= 1 && nsubk <= 5) {
             // the unrolled issue path
-            const uint32_t a_lo = static_cast<uint32_t>(umma_desc_sw128(a_addr));
             const uint32_t b_lo = static_cast<uint32_t>(umma_desc_sw128(b_addr));
             const uint32_t b_step = b_sub >> 4;
             const uint32_t sub_desc = static_cast<uint32_t>(p.nb) * 8u;  // nb rows x 128 B >> 4
             const uint32_t sub_cols = static_cast<uint32_t>(p.nb);
             const uint32_t acc0 = ks != 0 ? 1u : 0u;
-#define EBD_STAGE(K, S) mma_stage<K, S>(d0, a_lo, b_lo, b_step, sub_desc, sub_cols, desc_hi, idesc, acc0)
-            if (p.nsub == 1) {
-              switch (nsubk) {
-                case 1: EBD_STAGE(1, 1); break;
-                case 2: EBD_STAGE(2, 1); break;
-                case 3: EBD_STAGE(3, 1); break;
-                case 4: EBD_STAGE(4, 1); break;
-                default: EBD_STAGE(5, 1); break;
+#pragma unroll
+            for (int ch = 0; ch < MCH; ++ch) {
+              if (ch >= nch) break;
+              const uint32_t a_lo = static_cast<uint32_t>(umma_desc_sw128(a_addr + ch * a_chunk));
+              const uint32_t dc = d0 + static_cast<uint32_t>(ch * p.acc_stride);
+#define EBD_STAGE(K, S) mma_stage<K, S>(dc, a_lo, b_lo, b_step, sub_desc, sub_cols, desc_hi, idesc, acc0)
+              if (p.nsub == 1) {
+                switch (nsubk) {
+                  case 1: EBD_STAGE(1, 1); break;
+                  case 2: EBD_STAGE(2, 1); break;
+                  case 3: EBD_STAGE(3, 1); break;
+                  case 4: EBD_STAGE(4, 1); break;
+                  default: EBD_STAGE(5, 1); break;
+                }
+              } else {
+                switch (nsubk) {
+                  case 1: EBD_STAGE(1, 2); break;
+                  case 2: EBD_STAGE(2, 2); break;
+                  case 3: EBD_STAGE(3, 2); break;
+                  case 4: EBD_STAGE(4, 2); break;
+                  default: EBD_STAGE(5, 2); break;
+                }
               }
-            } else {
-              switch (nsubk) {
-                case 1: EBD_STAGE(1, 2); break;
-                case 2: EBD_STAGE(2, 2); break;
-                case 3: EBD_STAGE(3, 2); break;
-                case 4: EBD_STAGE(4, 2); break;
-                default: EBD_STAGE(5, 2); break;
-              }
-            }
 #undef EBD_STAGE
+            }
             if (PAIR)
               umma_commit_multicast(&empty[s], 0x3);
             else
@@ -304,18 +314,19 @@ __global__ void __launch_bounds__(kLmThreads, 1)
             }
             continue;
           }
-          for (int j = 0; j < nsubk; ++j) {
+          for (int ch = 0; ch < nch; ++ch)
+            for (int j = 0; j < nsubk; ++j) {
 #pragma unroll
-            for (int kk = 0; kk < 4; ++kk) {
-              const uint64_t ad = umma_desc_sw128(a_addr + j * kATile + kk * 32);
-              for (int sb = 0; sb < p.nsub; ++sb) {
-                const uint64_t bd =
-                    umma_desc_sw128(b_addr + j * b_sub + sb * p.nb * 128 + kk * 32);
-                umma_bf16(d0 + static_cast<uint32_t>(sb * p.nb), ad, bd, idesc,
-                          (ks | j | kk) != 0 ? 1u : 0u);
+              for (int kk = 0; kk < 4; ++kk) {
+                const uint64_t ad = umma_desc_sw128(a_addr + ch * a_chunk + j * kATile + kk * 32);
+                for (int sb = 0; sb < p.nsub; ++sb) {
+                  const uint64_t bd =
+                      umma_desc_sw128(b_addr + j * b_sub + sb * p.nb * 128 + kk * 32);
+                  umma_bf16(d0 + static_cast<uint32_t>(ch * p.acc_stride + sb * p.nb), ad, bd, idesc,
+                            (ks | j | kk) != 0 ? 1u : 0u);
+                }
               }
             }
-          }
           if (PAIR)
             umma_commit_multicast(&empty[s], 0x3);
           else
@@ -354,9 +365,9 @@ __global__ void __launch_bounds__(kLmThreads, 1)
     }
     const bool active = ok;
     int c = 0;
-    for (int u = u0; u < u1 && ok; u += 2, ++c) {
-      const int nu = min(2, u1 - u);
-      const int valid = min(nu * kUnit, p.V - u * kUnit);
+    for (int u = u0; u < u1 && ok; u += 2 * MCH, ++c) {
+      const int nu = min(2 * MCH, u1 - u);
+      const int nch = MCH == 1 ? 1 : (nu + 1) >> 1;
       const int buf = c % p.nbuf;
       const uint32_t bph = static_cast<uint32_t>(c / p.nbuf) & 1u;
       bool w = mbar_wait_sleepy(&acc_full[buf], bph, p.limit_ns, abort);
@@ -366,17 +377,19 @@ __global__ void __launch_bounds__(kLmThreads, 1)
         break;
       }
       tc_fence_after();
-      const int vbase = u * kUnit;
       bool released = false;
+      for (int ch = 0; ch < nch; ++ch) {
+      const int vbase = (u + 2 * ch) * kUnit;
+      const int valid = min(min(2, nu - 2 * ch) * kUnit, p.V - vbase);
       for (int cc = 32 * wg; cc < p.n_pad; cc += 32 * p.nwg) {
         float v[32];
         const uint32_t taddr = tmem_base + (static_cast<uint32_t>(quad * 32) << 16) +
-                               static_cast<uint32_t>(buf * p.acc_stride + cc);
+                               static_cast<uint32_t>((buf * MCH + ch) * p.acc_stride + cc);
         if (p.n_pad - cc >= 32)
           tmem_ld_32x32b_x32(taddr, v);
         else
           tmem_ld_32x32b_x16(taddr, v);
-        if (cc + 32 * p.nwg >= p.n_pad) {  // this warpgroup's last slice is in registers
+        if (ch == nch - 1 && cc + 32 * p.nwg >= p.n_pad) {  // this warpgroup's last slice is in registers
           tc_fence_before();
           mbar_arrive(&acc_empty[buf]);
           released = true;
@@ -433,7 +446,8 @@ __global__ void __launch_bounds__(kLmThreads, 1)
         }
         named_barrier(bar_id, 128);
       }
-      if (!released) {  // no slice of this chunk for this warpgroup
+      }
+      if (!released) {  // no slice of these chunks for this warpgroup
         tc_fence_before();
         mbar_arrive(&acc_empty[buf]);
       }
@@ -476,8 +490,14 @@ void lm_plan(LmParams& p, int rows, int V, int d, int num_sms, bool pair) {
   if (p.nb < 16) p.nb = 16;
   p.n_pad = p.nb * p.nsub;
   p.acc_stride = (p.n_pad + 31) / 32 * 32;
-  p.nbuf = (2 * p.acc_stride <= 512) ? 2 : 1;
-  int cols = p.nbuf * p.acc_stride;
+  // two W chunks per stage in paired mode when both accumulators fit in
+  // TMEM below 256 columns each.  They lose the second accumulator buffer,
+  // so the epilogue no longer overlaps the MMAs; measured: 390 rows (208 per
+  // CTA) 408 -> 401 us, but 512 rows (256 per CTA) 444 -> 498 us.
+  p.mch = (pair && p.n_pad >= 128 && p.acc_stride < 256) ? 2 : 1;
+  if (const char* env = getenv("EBD_LM_MCH")) p.mch = (atoi(env) == 2 && pair && 2 * p.acc_stride <= 512) ? 2 : 1;
+  p.nbuf = (2 * p.mch * p.acc_stride <= 512) ? 2 : 1;
+  int cols = p.nbuf * p.mch * p.acc_stride;
   int tc = 32;
   while (tc < cols) tc <<= 1;
   p.tmem_cols = tc;
@@ -492,7 +512,7 @@ void lm_plan(LmParams& p, int rows, int V, int d, int num_sms, bool pair) {
   // a second epilogue warpgroup (and its transpose buffer) only pays when the
   // accumulator is wide; below that the buffer is worth more as a larger
   // pipeline stage (measured: 128 rows, 5 x 16 KB stages -> 183 us, 4 -> 246)
-  p.nwg = p.n_pad >= 192 ? 2 : 1;
+  p.nwg = (p.n_pad >= 192 || p.mch == 2) ? 2 : 1;
   const uint32_t st_bytes = static_cast<uint32_t>(p.n_pad) * 20u;
   const uint32_t tail = kTBytes * static_cast<uint32_t>(p.nwg) + ((st_bytes + 7) / 8 * 8) +
                         (2 * 8 + 6) * 8 + 16;
@@ -503,15 +523,16 @@ void lm_plan(LmParams& p, int rows, int V, int d, int num_sms, bool pair) {
   if (const char* env = getenv("EBD_LM_KBS")) kbs = atoi(env);
   if (kbs < 1) kbs = 1;
   if (kbs > p.nkb) kbs = p.nkb;
-  while (kbs > 1 && budget / (static_cast<uint32_t>(kbs) * (kATile + p.n_pad * 128u)) < 2) --kbs;
+  const uint32_t a_box = static_cast<uint32_t>(p.mch) * kATile;
+  while (kbs > 1 && budget / (static_cast<uint32_t>(kbs) * (a_box + p.n_pad * 128u)) < 2) --kbs;
   p.kbs = kbs;
   p.nks = (p.nkb + kbs - 1) / kbs;
-  const uint32_t stage = static_cast<uint32_t>(kbs) * (kATile + static_cast<uint32_t>(p.n_pad) * 128u);
+  const uint32_t stage = static_cast<uint32_t>(kbs) * (a_box + static_cast<uint32_t>(p.n_pad) * 128u);
   int stages = static_cast<int>(budget / stage);
   if (stages > 8) stages = 8;
   p.stages = stages;
   p.off_a = 0;
-  p.off_b = p.off_a + static_cast<uint32_t>(stages) * kbs * kATile;
+  p.off_b = p.off_a + static_cast<uint32_t>(stages) * kbs * a_box;
   p.off_t = p.off_b + static_cast<uint32_t>(stages) * kbs * static_cast<uint32_t>(p.n_pad) * 128u;
   p.off_st = p.off_t + kTBytes * static_cast<uint32_t>(p.nwg);
   p.off_bar = (p.off_st + st_bytes + 7) / 8 * 8;
@@ -561,10 +582,12 @@ cudaError_t launch_pack_lm(const __nv_bfloat16* w, __nv_bfloat16* out, int V, in
 cudaError_t lm_configure() {
   const cudaFuncAttribute a = cudaFuncAttributeMaxDynamicSharedMemorySize;
   cudaError_t e;
-  if ((e = cudaFuncSetAttribute(lm_stats_kernel<true, true>, a, 232448)) != cudaSuccess) return e;
-  if ((e = cudaFuncSetAttribute(lm_stats_kernel<true, false>, a, 232448)) != cudaSuccess) return e;
-  if ((e = cudaFuncSetAttribute(lm_stats_kernel<false, true>, a, 232448)) != cudaSuccess) return e;
-  return cudaFuncSetAttribute(lm_stats_kernel<false, false>, a, 232448);
+  if ((e = cudaFuncSetAttribute(lm_stats_kernel<true, true, 1>, a, 232448)) != cudaSuccess) return e;
+  if ((e = cudaFuncSetAttribute(lm_stats_kernel<true, false, 1>, a, 232448)) != cudaSuccess) return e;
+  if ((e = cudaFuncSetAttribute(lm_stats_kernel<true, true, 2>, a, 232448)) != cudaSuccess) return e;
+  if ((e = cudaFuncSetAttribute(lm_stats_kernel<true, false, 2>, a, 232448)) != cudaSuccess) return e;
+  if ((e = cudaFuncSetAttribute(lm_stats_kernel<false, true, 1>, a, 232448)) != cudaSuccess) return e;
+  return cudaFuncSetAttribute(lm_stats_kernel<false, false, 1>, a, 232448);
 }
 
 cudaError_t launch_lm_stats(const CUtensorMap& tmap_w, const CUtensorMap& tmap_h,
@@ -581,11 +604,14 @@ cudaError_t launch_lm_stats(const CUtensorMap& tmap_w, const CUtensorMap& tmap_h
   attr[0].val.clusterDim.z = 1;
   cfg.attrs = attr;
   cfg.numAttrs = p.pair ? 1 : 0;
+  if (p.pair && p.mch == 2)
+    return p.packed ? cudaLaunchKernelEx(&cfg, lm_stats_kernel<true, true, 2>, tmap_w, tmap_h, p)
+                    : cudaLaunchKernelEx(&cfg, lm_stats_kernel<true, false, 2>, tmap_w, tmap_h, p);
   if (p.pair)
-    return p.packed ? cudaLaunchKernelEx(&cfg, lm_stats_kernel<true, true>, tmap_w, tmap_h, p)
-                    : cudaLaunchKernelEx(&cfg, lm_stats_kernel<true, false>, tmap_w, tmap_h, p);
-  return p.packed ? cudaLaunchKernelEx(&cfg, lm_stats_kernel<false, true>, tmap_w, tmap_h, p)
-                  : cudaLaunchKernelEx(&cfg, lm_stats_kernel<false, false>, tmap_w, tmap_h, p);
+    return p.packed ? cudaLaunchKernelEx(&cfg, lm_stats_kernel<true, true, 1>, tmap_w, tmap_h, p)
+                    : cudaLaunchKernelEx(&cfg, lm_stats_kernel<true, false, 1>, tmap_w, tmap_h, p);
+  return p.packed ? cudaLaunchKernelEx(&cfg, lm_stats_kernel<false, true, 1>, tmap_w, tmap_h, p)
+                  : cudaLaunchKernelEx(&cfg, lm_stats_kernel<false, false, 1>, tmap_w, tmap_h, p);
 }
 
 }  // namespace ebd
