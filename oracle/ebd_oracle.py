@@ -7,8 +7,11 @@ nothing else.
 
 Everything is the plain definition, in float64, on bf16-decoded inputs:
   * window attention:   O = softmax(Q K^T / sqrt(D)) V, bidirectional, over the
-    cached prefix followed by the window (Sec. 3: bidirectional mask
-    predictor; Sec. 6.3 "Effect of KV-Cache Configuration": prefix cache);
+    cached prefix followed by the window and, with a dual cache, by a cached
+    suffix (Sec. 3: bidirectional mask predictor; Sec. 6.3 "Effect of
+    KV-Cache Configuration": prefix and dual cache);
+  * cache append:       the K/V of the rows committed in a step written into
+    the cache at their positions (Sec. 6.3);
   * LM head:            full logits row l = W h, materialised;
   * statistics:         softmax in two passes (max, then sum), then
     kappa = max_v p(v)  (App. B, Eq. app-confidence), x_hat = argmax_v p(v),
@@ -51,6 +54,11 @@ where it is used):
   R14 kappa >= tau is inclusive; p_psi > tau_psi is strict; the anti-stall
       fallback takes the lowest position among equal kappa.
   R15 a router that does not run leaves NaN in its per-row output.
+  R21 dual cache: the keys right of the active block are those of the
+      positions after the window; a step passes them as a range of cached
+      positions [s0, s0 + S).  Appending on commit writes a row's K/V at
+      its absolute position once its mask is 0 after the step; positions
+      outside the cache are skipped.
   R20 the baselines' fixed-block rule (App. B, Eq. prelim-update) is read as
       two modes on the rows of the active fixed block: 'threshold' commits
       the masked rows with kappa >= tau, or, when none reaches tau, the one
@@ -127,11 +135,13 @@ def sigmoid(x):
 # ----------------------------------------------------------------------------
 # (1) window attention -- Sec. 3 (bidirectional), Sec. 6.3 (prefix cache)
 # ----------------------------------------------------------------------------
-def window_attention(q, k_win, v_win, k_cache, v_cache, cu_rows, prefix_len):
+def window_attention(q, k_win, v_win, k_cache, v_cache, cu_rows, prefix_len, suffix=None):
     """q[R][Hq][D], k_win/v_win[R][Hkv][D], k_cache/v_cache[B][P][Hkv][D]
     (bf16 bits) -> O[R][Hq][D] float64.  Sequence b's window queries attend,
     without any mask, to its first prefix_len[b] cached keys followed by its
-    own window keys.  Query head h reads key/value head h // (Hq/Hkv)."""
+    own window keys and, if suffix is given (dual cache, Reading R21), by
+    the cached keys at positions [suffix[b][0], suffix[b][0] + suffix[b][1]).
+    Query head h reads key/value head h // (Hq/Hkv)."""
     R, Hq, D = q.shape
     Hkv = k_win.shape[1]
     group = Hq // Hkv
@@ -141,14 +151,33 @@ def window_attention(q, k_win, v_win, k_cache, v_cache, cu_rows, prefix_len):
         if r1 == r0:
             continue
         P = int(prefix_len[b])
+        s0, S = (int(suffix[b][0]), int(suffix[b][1])) if suffix is not None else (0, 0)
         for h in range(Hq):
             g = h // group
-            K = np.concatenate([bf16(k_cache[b, :P, g]), bf16(k_win[r0:r1, g])])
-            V = np.concatenate([bf16(v_cache[b, :P, g]), bf16(v_win[r0:r1, g])])
+            K = np.concatenate([bf16(k_cache[b, :P, g]), bf16(k_win[r0:r1, g]),
+                                bf16(k_cache[b, s0:s0 + S, g])])
+            V = np.concatenate([bf16(v_cache[b, :P, g]), bf16(v_win[r0:r1, g]),
+                                bf16(v_cache[b, s0:s0 + S, g])])
             Q = bf16(q[r0:r1, h])
             A = softmax_rows(Q @ K.T / math.sqrt(D))
             out[r0:r1, h] = A @ V
     return out
+
+
+def kv_append(k_cache, v_cache, k_win, v_win, cu_rows, row_pos, mask):
+    """Prefix-cache append on commit (Sec. 6.3; Reading R21): returns copies
+    of the caches in which every window row r of sequence b with mask[r] == 0
+    has its K/V (bit patterns) at position row_pos[r]; positions outside the
+    cache are skipped."""
+    kc, vc = np.array(k_cache, copy=True), np.array(v_cache, copy=True)
+    Pm = kc.shape[1]
+    for b in range(len(cu_rows) - 1):
+        for r in range(int(cu_rows[b]), int(cu_rows[b + 1])):
+            pos = int(row_pos[r])
+            if mask[r] == 0 and 0 <= pos < Pm:
+                kc[b, pos] = k_win[r]
+                vc[b, pos] = v_win[r]
+    return kc, vc
 
 
 # ----------------------------------------------------------------------------
@@ -488,14 +517,16 @@ def loop_window(frontier: int, end: int, meta, in_block_pos: List[int],
 def generation_loop(shape, W, prm: DecisionParams, window_inputs, kv_rows,
                     w_lm, w_emb, max_steps: Optional[int] = None,
                     attention: bool = False, on_step=None, mode: str = "eb",
-                    block: int = 32, top_m: int = 1):
+                    block: int = 32, top_m: int = 1, cache: str = "prefix"):
     """Run the App. E loop on the synthetic loop workload: a committed prompt
     of `shape.prefix` positions followed by `shape.gen_len` masked positions.
     window_inputs(step, positions) -> (hidden, q, k_win, v_win) and
     kv_rows(positions) -> (k, v) supply the per-step tensors.  Returns
     (tokens, steps, per-step commit counts, per-step records).  mode 'eb'
     runs the App. E algorithm; 'threshold' and 'topm' the fixed-block rules
-    of the baselines (Reading R20) with blocks of `block` positions."""
+    of the baselines (Reading R20) with blocks of `block` positions.  cache
+    'dual' adds the positions right of the window as cached keys (Reading
+    R21)."""
     P0, L = shape.prefix, shape.gen_len
     tokens = np.full(L, -1, np.int32)
     mask = np.ones(L, np.uint8)
@@ -516,9 +547,11 @@ def generation_loop(shape, W, prm: DecisionParams, window_inputs, kv_rows,
         st = softmax_stats(lm_logits(hid, w_lm))
         attn = None
         if attention:
-            kc, vc = kv_rows(np.arange(P0 + lo, dtype=np.int32))
+            dual = cache == "dual"
+            kc, vc = kv_rows(np.arange(P0 + (L if dual else lo), dtype=np.int32))
+            suffix = np.array([[P0 + hi, L - hi]]) if dual else None
             attn = window_attention(q, kw, vw, kc[None], vc[None],
-                                    np.array([0, hi - lo]), np.array([P0 + lo]))
+                                    np.array([0, hi - lo]), np.array([P0 + lo]), suffix)
         t, m, ib = tokens[lo:hi], mask[lo:hi], in_block[lo:hi]
         before = int(m.sum())
         if mode == "eb":
