@@ -121,8 +121,11 @@ typedef struct {
   const uint16_t* q;          /* [R][Hq][D] bf16 window queries                  */
   const uint16_t* k_win;      /* [R][Hkv][D] bf16 window keys                    */
   const uint16_t* v_win;      /* [R][Hkv][D] bf16 window values                  */
-  const uint16_t* k_cache;    /* [B][max_prefix][Hkv][D] bf16 cached prefix keys */
-  const uint16_t* v_cache;    /* [B][max_prefix][Hkv][D] bf16 cached values      */
+  uint16_t* k_cache;          /* [B][max_prefix][Hkv][D] bf16 K/V cache, indexed by
+                                 absolute position: the prefix [0, prefix_len),
+                                 the suffix range (dual cache); written only
+                                 when kv_append is set                         */
+  uint16_t* v_cache;          /* [B][max_prefix][Hkv][D] bf16 cached values      */
   const uint16_t* w_lm;       /* [vocab][d_model] bf16 LM-head weight            */
   /* decode state, read and updated in place */
   int32_t* tokens;            /* [R] token ids; committed rows get x_hat         */
@@ -143,7 +146,23 @@ typedef struct {
   int32_t w_lm_layout;        /* 0: w_lm is [vocab][d_model] row-major;
                                  1: w_lm is the tiled copy written by
                                  ebd_pack_lm_head()                           */
-  int32_t reserved;
+  /* KV-cache integration (Sec. 6.3, prefix and dual cache) */
+  int32_t kv_append;          /* 1: after the decision, every window row that is
+                                 committed (mask 0 after the step) has its
+                                 k_win/v_win row written into k_cache/v_cache
+                                 at row_pos (the prefix-cache append on
+                                 commit); rows at positions >= max_prefix are
+                                 skipped.  The window attention of the same
+                                 step then runs after it instead of
+                                 overlapping the decision.  0: the cache is
+                                 only read.                                   */
+  const int32_t* suffix;      /* [B][2] {s0, S}, device (host in
+                                 ebd_step_host): the window also attends to
+                                 the cached keys/values at positions
+                                 [s0, s0 + S) after its own (dual cache).  The
+                                 range is clamped to [0, max_prefix) and must
+                                 not overlap the window's positions.  NULL:
+                                 prefix cache only.                           */
 } ebd_step_args;
 
 /* Creates a handle on the current CUDA device: validates *cfg, allocates the

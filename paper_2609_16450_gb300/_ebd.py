@@ -49,7 +49,8 @@ class ebd_step_args(Structure):
                 ("blk_meta", c_void_p), ("attn_out", c_void_p), ("conf", c_void_p),
                 ("entropy", c_void_p), ("ent_norm", c_void_p), ("gap", c_void_p),
                 ("argmax", c_void_p), ("lbs_logit", c_void_p), ("lps_prob", c_void_p),
-                ("accepted", c_void_p), ("w_lm_layout", c_int32), ("reserved", c_int32)]
+                ("accepted", c_void_p), ("w_lm_layout", c_int32), ("kv_append", c_int32),
+                ("suffix", c_void_p)]
 
 
 EXPORTS = ["ebd_create", "ebd_destroy", "ebd_bind_embedding", "ebd_step", "ebd_step_host",

@@ -426,6 +426,18 @@ ebd_status check_args(ebd_handle* h, const ebd_step_args* a, bool need_attn, boo
         (c.max_prefix > 0 && (!aligned(a->k_cache, 16) || !aligned(a->v_cache, 16))))
       return fail(h, EBD_ERR_INVALID_ARG, "q/k/v/attn_out must be 16-byte aligned");
   }
+  if (a->suffix != nullptr && c.max_prefix <= 0)
+    return fail(h, EBD_ERR_INVALID_ARG, "a suffix range needs a K/V cache (max_prefix > 0)");
+  if (a->kv_append != 0 && a->kv_append != 1)
+    return fail(h, EBD_ERR_INVALID_ARG, "kv_append must be 0 or 1");
+  if (a->kv_append) {
+    if (c.max_prefix <= 0 || !a->k_cache || !a->v_cache || !a->k_win || !a->v_win ||
+        !a->row_pos || !a->cu_rows || !a->mask)
+      return fail(h, EBD_ERR_INVALID_ARG, "kv_append needs the K/V cache, k_win/v_win, row_pos and mask");
+    if (!aligned(a->k_cache, 16) || !aligned(a->v_cache, 16) || !aligned(a->k_win, 16) ||
+        !aligned(a->v_win, 16))
+      return fail(h, EBD_ERR_INVALID_ARG, "K/V cache and window K/V must be 16-byte aligned");
+  }
   return EBD_OK;
 }
 
@@ -465,6 +477,7 @@ ebd_status run_attention(ebd_handle* h, const ebd_step_args* a, cudaStream_t st,
   p.splits = h->attn_splits;
   p.cu_rows = a->cu_rows;
   p.prefix_len = a->prefix_len;
+  p.suffix = c.max_prefix > 0 ? a->suffix : nullptr;
   p.q = reinterpret_cast<const __nv_bfloat16*>(a->q);
   p.out = a->attn_out;
   p.part = h->attn_part;
@@ -721,6 +734,7 @@ ebd_status ebd_create(const ebd_config* cfg, ebd_handle** out) {
     add((B + 1) * 4); add(B * 4); add(R * 4); add(R * d * 2); add(R * Hq * D * 2);
     add(R * Hkv * D * 2); add(R * Hkv * D * 2); add(R * 4); add(R); add(R); add(B * 8);
     add(R * Hq * D * 4); for (int i = 0; i < 6; ++i) add(R * 4); add(R * 4); add(R);
+    add(B * 8);  // suffix ranges
     h->staging_bytes = bytes;
     if ((e = cudaMalloc(&h->staging, bytes)) != cudaSuccess)
       return bail(cuda_fail(h, e, "cudaMalloc(staging)"));
@@ -826,10 +840,12 @@ ebd_status ebd_step(ebd_handle* h, const ebd_step_args* a, void* stream) {
   if (a->rows == 0 || a->batch == 0) return EBD_OK;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   (void)cudaGetLastError();  // a stale error of an earlier unrelated call is not ours
-  // Order on `st`: LM head, decision, window attention.  The attention feeds
-  // neither of the others, so unless every kernel is timed on its own
-  // (profile mode 1) it is launched as a programmatic dependent of the
-  // decision: it fills the SMs the decision's clusters leave idle.
+  // Order on `st`: LM head, decision, (cache append), window attention.  The
+  // attention feeds neither of the others, so unless every kernel is timed
+  // on its own (profile mode 1) it is launched as a programmatic dependent
+  // of the kernel before it: it fills the SMs the decision's clusters leave
+  // idle.  The append reads the mask the decision writes, so it is an
+  // ordinary launch after it; the attention reads no position it writes.
   const int prof = h->profile;
   cudaError_t e0 = cudaSuccess;
   if (prof && (e0 = record(h->ev[0], st)) != cudaSuccess) return cuda_fail(h, e0, "profile event");
@@ -841,6 +857,12 @@ ebd_status ebd_step(ebd_handle* h, const ebd_step_args* a, void* stream) {
   if (e != cudaSuccess) return cuda_fail(h, e, "decision launch");
   if (prof == 1 && (e0 = record(h->ev[2], st)) != cudaSuccess)
     return cuda_fail(h, e0, "profile event");
+  if (a->kv_append) {
+    const ebd_config& c = h->cfg;
+    e = launch_kv_append(a->k_cache, a->v_cache, a->k_win, a->v_win, a->cu_rows, a->row_pos, a->mask,
+                         a->batch, a->rows, c.max_prefix, c.n_heads_kv * c.head_dim, st);
+    if (e != cudaSuccess) return cuda_fail(h, e, "cache append launch");
+  }
   if (attn && (s = run_attention(h, a, st, prof != 1)) != EBD_OK) return s;
   if (prof && (e0 = record(h->ev[3], st)) != cudaSuccess) return cuda_fail(h, e0, "profile event");
   h->prof_mode = prof;
@@ -926,6 +948,7 @@ ebd_status ebd_step_host(ebd_handle* h, const ebd_step_args* a, void* stream) {
   for (int i = 0; i < 6; ++i) f[i] = reinterpret_cast<float*>(take(RM * 4));
   int32_t* am = reinterpret_cast<int32_t*>(take(RM * 4));
   uint8_t* acc = take(RM);
+  int32_t* sfx = reinterpret_cast<int32_t*>(take(BM * 8));
   auto h2d = [&](void* dst, const void* src, size_t n) {
     return n == 0 || src == nullptr ? cudaSuccess
                                     : cudaMemcpyAsync(dst, src, n, cudaMemcpyHostToDevice, st);
@@ -943,8 +966,9 @@ ebd_status ebd_step_host(ebd_handle* h, const ebd_step_args* a, void* stream) {
   chk(h2d(pl, a->prefix_len, B * 4));
   chk(h2d(rp, a->row_pos, R * 4));
   chk(h2d(hid, a->hidden, R * d * 2));
-  if (attn) {
-    chk(h2d(q, a->q, R * Hq * D * 2));
+  const bool kv = attn || a->kv_append;  // the window K/V feed the attention and the append
+  if (attn) chk(h2d(q, a->q, R * Hq * D * 2));
+  if (kv) {
     chk(h2d(kw, a->k_win, R * Hkv * D * 2));
     chk(h2d(vw, a->v_win, R * Hkv * D * 2));
   }
@@ -952,10 +976,12 @@ ebd_status ebd_step_host(ebd_handle* h, const ebd_step_args* a, void* stream) {
   chk(h2d(msk, a->mask, R));
   chk(h2d(ib, a->in_block, R));
   chk(h2d(meta, a->blk_meta, B * 8));
+  if (a->suffix) chk(h2d(sfx, a->suffix, B * 8));
   if (e != cudaSuccess) return cuda_fail(h, e, "host-to-device copy");
   g.cu_rows = cu; g.prefix_len = pl; g.row_pos = rp; g.hidden = hid;
-  g.q = attn ? q : nullptr; g.k_win = attn ? kw : nullptr; g.v_win = attn ? vw : nullptr;
+  g.q = attn ? q : nullptr; g.k_win = kv ? kw : nullptr; g.v_win = kv ? vw : nullptr;
   g.tokens = tok; g.mask = msk; g.in_block = ib; g.blk_meta = meta;
+  g.suffix = a->suffix ? sfx : nullptr;
   g.attn_out = attn ? ao : nullptr;
   g.conf = a->conf ? f[0] : nullptr;
   g.entropy = a->entropy ? f[1] : nullptr;

@@ -52,6 +52,7 @@ struct AttnParams {
   int max_qtiles, splits;
   const int* cu_rows;
   const int* prefix_len;
+  const int* suffix;        // [B][2] {s0, S} cached keys after the window, or null
   const __nv_bfloat16* q;   // [R][Hq][D]
   float* out;               // [R][Hq][D]
   float* part;              // [B*Hkv*max_qtiles*splits][64][D] unnormalised O
@@ -104,6 +105,12 @@ cudaError_t launch_attention(const CUtensorMap& kc, const CUtensorMap& vc, const
                              const CUtensorMap& vw, const AttnParams& p, cudaStream_t st,
                              bool pdl = false);
 cudaError_t launch_decide(const DecideParams& p, cudaStream_t st);
+// prefix-cache append on commit: window row r of sequence b with mask[r] == 0
+// is copied (K and V, Hkv * D bf16 each) to cache position row_pos[r] < Pmax
+cudaError_t launch_kv_append(uint16_t* k_cache, uint16_t* v_cache, const uint16_t* k_win,
+                             const uint16_t* v_win, const int* cu_rows, const int* row_pos,
+                             const uint8_t* mask, int B, int rows, int Pmax, int hkvd,
+                             cudaStream_t st);
 cudaError_t launch_pack_lm(const __nv_bfloat16* w, __nv_bfloat16* out, int V, int d,
                            cudaStream_t st);
 cudaError_t launch_fold_tok(const __nv_bfloat16* w_tok, const __nv_bfloat16* w_emb, float* table,

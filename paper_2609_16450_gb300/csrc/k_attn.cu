@@ -1,7 +1,10 @@
 // Window attention: the active window's queries attend, without a mask, to
-// the sequence's cached prefix keys followed by the window's own keys
-// (bidirectional dLLM, Sec. 3; prefix cache at the block boundary, Sec. 6.3).
+// the sequence's cached prefix keys, the window's own keys and, with a dual
+// cache, a cached suffix range (bidirectional dLLM, Sec. 3; prefix and dual
+// cache at the block boundaries, Sec. 6.3).
 //   O = softmax(Q K^T / sqrt(D)) V, fp32 output.
+// The key range is a list of 64-key chunks: prefix tiles of the cache, one
+// tile of window rows, then suffix tiles of the cache.
 //
 // Grid: (key split, query tile, sequence x kv head).  A query tile is 64 rows
 // of (query head of the kv group, window row); each of the 4 warps owns 16
@@ -48,8 +51,13 @@ __global__ void __launch_bounds__(kAttnThreads)
   if (wb <= 0 || wb > kMaxWindow || qt * 64 >= m_total) return;
   int P = p.prefix_len[b];
   P = P < 0 ? 0 : (P > p.max_prefix ? p.max_prefix : P);
+  int S0 = 0, S = 0;  // suffix range of the cache (dual cache)
+  if (p.suffix != nullptr) {
+    S0 = min(max(p.suffix[2 * b], 0), p.max_prefix);
+    S = min(max(p.suffix[2 * b + 1], 0), p.max_prefix - S0);
+  }
   const int ncc = (P + kAttnChunk - 1) / kAttnChunk;
-  const int nch = ncc + 1;
+  const int nch = ncc + 1 + (S + kAttnChunk - 1) / kAttnChunk;
   const int c0 = static_cast<int>((static_cast<long long>(split) * nch) / p.splits);
   const int c1 = static_cast<int>((static_cast<long long>(split + 1) * nch) / p.splits);
   const int nmy = c1 - c0;
@@ -73,9 +81,13 @@ __global__ void __launch_bounds__(kAttnThreads)
       if (c < ncc) {
         tma_load_4d(kd + hf * 8192, &tm_kc, &full[s], hf * 64, g, c * kAttnChunk, b);
         tma_load_4d(vd + hf * 8192, &tm_vc, &full[s], hf * 64, g, c * kAttnChunk, b);
-      } else {
+      } else if (c == ncc) {
         tma_load_3d(kd + hf * 8192, &tm_kw, &full[s], hf * 64, g, r0);
         tma_load_3d(vd + hf * 8192, &tm_vw, &full[s], hf * 64, g, r0);
+      } else {
+        const int y = S0 + (c - ncc - 1) * kAttnChunk;
+        tma_load_4d(kd + hf * 8192, &tm_kc, &full[s], hf * 64, g, y, b);
+        tma_load_4d(vd + hf * 8192, &tm_vc, &full[s], hf * 64, g, y, b);
       }
     }
   };
@@ -125,7 +137,8 @@ __global__ void __launch_bounds__(kAttnThreads)
       break;
     }
     const int c = c0 + i;
-    const int nvalid = c < ncc ? min(kAttnChunk, P - c * kAttnChunk) : wb;
+    const int nvalid = c < ncc ? min(kAttnChunk, P - c * kAttnChunk)
+                       : (c == ncc ? wb : min(kAttnChunk, S - (c - ncc - 1) * kAttnChunk));
     const uint32_t kbase = smem_u32(smem + s * kStageBytes);
     const uint32_t vbase = kbase + 2 * 8192;
     if (warp_active) {
@@ -301,6 +314,42 @@ __global__ void __launch_bounds__(kAttnThreads)
     *reinterpret_cast<float4*>(out_row(qt * 64 + r) + d) = acc;
   }
   if (tid == 0) p.tickets[slot] = 0;
+}
+
+// ------------------------------------------------------------------ cache append
+// Prefix-cache append on commit (Sec. 6.3): window row r (blockIdx.x) of its
+// sequence, if committed after the step (mask 0), is copied 16 bytes per
+// thread into the cache at its absolute position; positions outside the
+// cache are skipped.
+__global__ void __launch_bounds__(256)
+    kv_append_kernel(uint4* __restrict__ k_cache, uint4* __restrict__ v_cache,
+                     const uint4* __restrict__ k_win, const uint4* __restrict__ v_win,
+                     const int* __restrict__ cu_rows, const int* __restrict__ row_pos,
+                     const uint8_t* __restrict__ mask, int B, int Pmax, int vec_per_row) {
+  const int r = blockIdx.x;
+  if (mask[r] != 0) return;
+  const int pos = row_pos[r];
+  if (pos < 0 || pos >= Pmax) return;
+  int b = 0;
+  while (b + 1 < B && cu_rows[b + 1] <= r) ++b;
+  const size_t dst = (static_cast<size_t>(b) * Pmax + pos) * vec_per_row;
+  const size_t src = static_cast<size_t>(r) * vec_per_row;
+  for (int i = threadIdx.x; i < vec_per_row; i += blockDim.x) {
+    k_cache[dst + i] = k_win[src + i];
+    v_cache[dst + i] = v_win[src + i];
+  }
+}
+
+cudaError_t launch_kv_append(uint16_t* k_cache, uint16_t* v_cache, const uint16_t* k_win,
+                             const uint16_t* v_win, const int* cu_rows, const int* row_pos,
+                             const uint8_t* mask, int B, int rows, int Pmax, int hkvd,
+                             cudaStream_t st) {
+  if (rows <= 0) return cudaSuccess;
+  kv_append_kernel<<<rows, 256, 0, st>>>(
+      reinterpret_cast<uint4*>(k_cache), reinterpret_cast<uint4*>(v_cache),
+      reinterpret_cast<const uint4*>(k_win), reinterpret_cast<const uint4*>(v_win), cu_rows,
+      row_pos, mask, B, Pmax, hkvd / 8);
+  return cudaGetLastError();
 }
 
 cudaError_t attn_configure() {

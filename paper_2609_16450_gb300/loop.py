@@ -6,10 +6,13 @@ Each step asks the library for the next window (ebd_loop_window), has the
 caller supply that window's backbone outputs (hidden states, q, k, v) and
 runs ebd_step on it.  The decode state (tokens, mask, block flags, block
 meta) of the whole response stays on the device; a step's window is a slice
-of it.  The K/V cache holds every position once (K/V of a position do not
-change), and a step attends to its first prefix + frontier rows.  This
-module only marshals buffers; the window rule and every step of the method
-run in the library."""
+of it.  The K/V cache is indexed by absolute position; a step attends to its
+first prefix + frontier rows (prefix cache) and, with cache='dual', also to
+the positions right of the window (dual cache, Sec. 6.3).  With append=True
+each step writes the K/V of the rows it commits into the cache
+(ebd_step_args.kv_append); the cache then starts with the prompt only.
+This module only marshals buffers; the window rule and every step of the
+method run in the library."""
 from __future__ import annotations
 
 from dataclasses import dataclass, field
@@ -50,6 +53,8 @@ class LoopResult:
     commits: List[int] = field(default_factory=list)
     records: List[LoopStep] = field(default_factory=list)
     device_us: float = 0.0
+    k_cache: Optional[np.ndarray] = None  # [P0 + L][Hkv][D] int16 bits after the loop
+    v_cache: Optional[np.ndarray] = None
 
 
 def config_for_loop(shape, max_window: int = 64, decode_mode: int = E.EBD_DECODE_EB,
@@ -63,11 +68,16 @@ def run_loop(h: rt.Handle, shape, weights: rt.DeviceWeights,
              window_inputs: Callable, kv_rows: Callable, attention: bool = True,
              max_steps: Optional[int] = None, max_window: int = 64,
              keep: bool = True, stream: Optional[torch.cuda.Stream] = None,
-             block: int = 32) -> LoopResult:
+             block: int = 32, cache: str = "prefix", append: bool = False) -> LoopResult:
     """window_inputs(step, positions) -> (hidden, q, k_win, v_win) as bf16 bit
     arrays; kv_rows(positions) -> (k, v).  Positions are absolute.  Under the
     handle's baseline decode modes the window is the active fixed block of
-    `block` positions (ebd_loop_block_window)."""
+    `block` positions (ebd_loop_block_window).  cache: 'prefix' or 'dual';
+    append: the step appends committed rows' K/V to the cache, which starts
+    with the prompt's K/V only (with 'dual', with every position's, the
+    positions right of the window standing for the K/V a dual cache holds)."""
+    if cache not in ("prefix", "dual"):
+        raise ValueError("cache must be 'prefix' or 'dual'")
     fixed = h.cfg.decode_mode != E.EBD_DECODE_EB
     dev = "cuda"
     P0, L = shape.prefix, shape.gen_len
@@ -99,10 +109,14 @@ def run_loop(h: rt.Handle, shape, weights: rt.DeviceWeights,
     accepted = torch.empty((W,), **u8)
     attn_out = torch.empty((W, Hq, D), **f32) if attention else None
     kc = vc = None
-    if attention:
-        kk, vv = kv_rows(np.arange(P0 + L, dtype=np.int32))
-        kc = rt._dev(kk, dev).reshape(1, P0 + L, Hkv, D)
-        vc = rt._dev(vv, dev).reshape(1, P0 + L, Hkv, D)
+    sfx = torch.zeros((2,), **i32)
+    if attention or append:
+        n0 = P0 if (append and cache == "prefix") else P0 + L
+        kk, vv = kv_rows(np.arange(n0, dtype=np.int32))
+        kc = torch.zeros((1, P0 + L, Hkv, D), dtype=torch.int16, device=dev)
+        vc = torch.zeros((1, P0 + L, Hkv, D), dtype=torch.int16, device=dev)
+        kc[0, :n0] = rt._dev(kk, dev).reshape(n0, Hkv, D)
+        vc[0, :n0] = rt._dev(vv, dev).reshape(n0, Hkv, D)
     ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     res = LoopResult(tokens=None, steps=0)
     step = 0
@@ -128,13 +142,18 @@ def run_loop(h: rt.Handle, shape, weights: rt.DeviceWeights,
             cu.copy_(torch.tensor([0, R], dtype=torch.int32))
             pl.copy_(torch.tensor([P0 + lo], dtype=torch.int32))
             rp[:R].copy_(torch.from_numpy(positions))
+            sfx.copy_(torch.tensor([P0 + hi, L - hi], dtype=torch.int32))
         a = E.ebd_step_args()
         a.batch, a.rows = 1, R
         a.cu_rows, a.prefix_len, a.row_pos = cu.data_ptr(), pl.data_ptr(), rp.data_ptr()
         a.hidden, a.q, a.k_win, a.v_win = hid.data_ptr(), q.data_ptr(), kw.data_ptr(), vw.data_ptr()
-        if attention:
+        if attention or append:
             a.k_cache, a.v_cache = kc.data_ptr(), vc.data_ptr()
+        if attention:
             a.attn_out = attn_out.data_ptr()
+            if cache == "dual":
+                a.suffix = sfx.data_ptr()
+        a.kv_append = 1 if append else 0
         a.w_lm, a.w_lm_layout = weights.w_lm.data_ptr(), weights.layout
         a.tokens = tokens.data_ptr() + 4 * lo
         a.mask = mask.data_ptr() + lo
@@ -178,4 +197,6 @@ def run_loop(h: rt.Handle, shape, weights: rt.DeviceWeights,
         step += 1
     res.tokens = tokens.cpu().numpy()
     res.steps = step
+    if kc is not None:
+        res.k_cache, res.v_cache = kc[0].cpu().numpy(), vc[0].cpu().numpy()
     return res
