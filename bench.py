@@ -167,16 +167,27 @@ class ClockSampler:
 
 
 # ----------------------------------------------------------------------------- work model
-def step_work(sh, rows, masked, grid_lm, lbs_runs):
-    """Algorithmic bytes and flops of one step (each input read once)."""
+def suffix_len(sh):
+    """Cached positions after the window in dual-cache mode: the rest of a
+    gen_len response whose first positions form the largest window."""
+    import synth
+    return int(sh.gen_len - int(np.max(synth.window_sizes(sh))))
+
+
+def step_work(sh, rows, masked, grid_lm, lbs_runs, suffix=0, append=False):
+    """Algorithmic bytes and flops of one step (each input read once); suffix:
+    cached keys after each window (dual cache); append: committed rows'
+    K/V written to the cache (counted for every row, an upper bound)."""
     d, V, Hq, Hkv, D = sh.d_model, sh.vocab, sh.n_heads_q, sh.n_heads_kv, sh.head_dim
     import synth
     w = synth.window_sizes(sh)
-    keys = int(sum(sh.prefix + int(x) for x in w))
+    keys = int(sum(sh.prefix + int(x) + suffix for x in w))
     lm_bytes = V * d * 2 + rows * d * 2 + rows * grid_lm * 20
     lm_flops = 2 * rows * d * V
     attn_bytes = keys * Hkv * D * 2 * 2 + rows * Hq * D * 2 + rows * Hq * D * 4
-    attn_flops = 4 * sum(int(x) * (sh.prefix + int(x)) for x in w) * Hq * D
+    attn_flops = 4 * sum(int(x) * (sh.prefix + int(x) + suffix) for x in w) * Hq * D
+    if append:
+        attn_bytes += rows * Hkv * D * 2 * 2 * 2
     dec_bytes = rows * grid_lm * 20 + rows * 40
     if lbs_runs:
         dec_bytes += 2 * (613761 - 262208) + masked * 64 * 4
@@ -241,14 +252,22 @@ def run_ours(args, rank, world, local_rank):
     inp = synth.make_step_inputs(sh)
     if args.state == "inblock":
         synth.preset_in_block(inp, 20)
+    sfx = None
+    if args.cache == "dual":  # the rest of a gen_len response after the window
+        inp, sfx = synth.with_suffix_cache(inp, suffix_len(sh))
     w = rt.upload_weights(inp)
-    h = rt.Handle(rt.config_for(sh), w.w_emb)
+    h = rt.Handle(rt.config_for(sh, max_prefix=inp.k_cache.shape[1]), w.w_emb)
     if args.w_layout == "packed":
         w = rt.pack_weights(h, w)  # one-time tiling of W_lm (model load)
     ds = rt.DeviceStep(inp, w, attention=True)
     stream = torch.cuda.Stream()
     sid = stream.cuda_stream
     args_c = ds.args()
+    sfx_d = None
+    if sfx is not None:
+        sfx_d = torch.from_numpy(sfx).cuda()
+        args_c.suffix = sfx_d.data_ptr()
+    args_c.kv_append = 1 if args.append else 0
     flush = L2Flush(torch)
     torch.cuda.synchronize()
 
@@ -346,13 +365,14 @@ def run_ours(args, rank, world, local_rank):
     # end to end through ebd_step_host: pinned host inputs in, results out
     e2e = None
     if not args.skip_e2e:
-        e2e = run_e2e(args, h, ds, inp, sh, stream, world)
+        e2e = run_e2e(args, h, ds, inp, sh, stream, world, sfx)
     out = dict(sh=sh, inp=inp, rows=inp.rows, masked=int(inp.mask.sum()), mean_ms=mean_ms,
                step_ms=step_ms, k_attn=k_attn, k_lm=k_lm, k_dec=k_dec, k_tail=k_tail,
                grid_lm=None,
                clocks=sampler.summary(), e2e=e2e, t_wall=t_wall,
                lbs_runs=args.state == "select")
-    out["launches_per_step"] = 2 + (inp.rows + 511) // 512
+    out["launches_per_step"] = 2 + (inp.rows + 511) // 512 + (1 if args.append else 0)
+    out["suffix"] = None if sfx is None else sfx
     out["fetch"] = ds.fetch()
     h_sms = torch.cuda.get_device_properties(local_rank).multi_processor_count
     out["grid_lm"] = min(h_sms, (sh.vocab + 63) // 64)
@@ -361,7 +381,7 @@ def run_ours(args, rank, world, local_rank):
     return out
 
 
-def run_e2e(args, h, ds, inp, sh, stream, world):
+def run_e2e(args, h, ds, inp, sh, stream, world, sfx=None):
     """Same step through ebd_step_host: every step copies its inputs from
     pinned host memory and its results back inside the timed interval."""
     import torch
@@ -388,6 +408,10 @@ def run_e2e(args, h, ds, inp, sh, stream, world):
     a.k_cache, a.v_cache, a.w_lm = ds.k_cache.data_ptr(), ds.v_cache.data_ptr(), \
         ds.weights.w_lm.data_ptr()
     a.w_lm_layout = ds.weights.layout
+    if sfx is not None:
+        host_in["suffix"] = pin(sfx)
+        a.suffix = host_in["suffix"].data_ptr()
+    a.kv_append = 1 if args.append else 0
     h2d = sum(t.numel() * t.element_size() for t in host_in.values()) + \
         sum(t.numel() * t.element_size() for t in host_state.values())
     d2h = sum(t.numel() * t.element_size() for t in host_state.values()) + \
@@ -423,7 +447,7 @@ def run_e2e(args, h, ds, inp, sh, stream, world):
 
 
 # ----------------------------------------------------------------------------- oracle arm
-def oracle_step_sample(sh, inp, budget_s):
+def oracle_step_sample(sh, inp, budget_s, suffix=None):
     """Times the CPU oracle on the step's inputs: full steps until budget_s
     has passed (at least one).  Returns (positions/s, steps, seconds)."""
     from oracle import ebd_oracle as o
@@ -433,7 +457,7 @@ def oracle_step_sample(sh, inp, budget_s):
                            g_max=sh.g_max, eos_id=sh.eos_id, lps_enabled=bool(sh.lps_enabled))
     n, t0 = 0, time.perf_counter()
     while True:
-        o.step(inp, W, prm)
+        o.step(inp, W, prm, suffix=suffix)
         n += 1
         el = time.perf_counter() - t0
         if el >= budget_s:
@@ -462,11 +486,12 @@ def run_loop_bench(args):
         w = rt.pack_weights(h, w)
     win = lambda s, p: synth.loop_window_inputs(sh, s, p)
     kv = lambda p: synth.loop_kv(sh, p)
-    lp.run_loop(h, sh, w, win, kv, keep=False, block=sh.l_b)  # warm-up loop
+    opts = dict(keep=False, block=sh.l_b, cache=args.cache, append=args.append)
+    lp.run_loop(h, sh, w, win, kv, **opts)  # warm-up loop
     runs = []
     for _ in range(max(1, args.steps // 100)):
         t0 = time.perf_counter()
-        res = lp.run_loop(h, sh, w, win, kv, keep=False, block=sh.l_b)
+        res = lp.run_loop(h, sh, w, win, kv, **opts)
         runs.append((res.steps, res.device_us, time.perf_counter() - t0))
     steps = runs[0][0]
     dev_us = float(np.mean([r[1] for r in runs]))
@@ -481,6 +506,11 @@ def run_loop_bench(args):
                                    f"at most 64 rows, attention over the committed prefix",
                        "decode": args.decode + (f" (m={args.top_m})" if args.decode == "topm" else ""),
                        "fixed_block": sh.l_b if args.decode != "eb" else None,
+                       "kv_cache": ("dual: the window also attends to the positions after it"
+                                    if args.cache == "dual" else "prefix") +
+                                   ("; committed rows appended to the cache by each step, which "
+                                    "starts with the prompt only" if args.append and args.cache == "prefix"
+                                    else "; committed rows appended by each step" if args.append else ""),
                        "loop_steps": steps, "device_us_total": round(dev_us, 1),
                        "wall_s_total": round(wall_s, 3),
                        "l2": "not flushed between steps (consecutive steps of one loop)"}}
@@ -561,6 +591,10 @@ def main():
     ap.add_argument("--decode", choices=["eb", "threshold", "topm"], default="eb",
                     help="decision of the loop configs: EB, or a baseline's fixed-block rule")
     ap.add_argument("--top-m", type=int, default=1, help="commits per step of --decode topm")
+    ap.add_argument("--cache", choices=["prefix", "dual"], default="prefix",
+                    help="dual: each window also attends to the cached rest of its response")
+    ap.add_argument("--append", action="store_true",
+                    help="write committed rows' K/V into the cache every step")
     ap.add_argument("--w-layout", choices=["packed", "rowmajor"], default="packed",
                     help="W_lm tiled once by ebd_pack_lm_head (default) or row-major")
     args = ap.parse_args()
@@ -592,7 +626,8 @@ def main():
 
     sh = r["sh"]
     hbm, bf16, bf16_sus, peak_src = load_peaks()
-    wk = step_work(sh, r["rows"], r["masked"], r["grid_lm"], r["lbs_runs"])
+    wk = step_work(sh, r["rows"], r["masked"], r["grid_lm"], r["lbs_runs"],
+                   suffix=suffix_len(sh) if args.cache == "dual" else 0, append=args.append)
     t_lm = r["k_lm"] / 1000.0
     lm_hbm_t = wk["lm_bytes"] / (hbm * 1e9)
     lm_tc_t = wk["lm_flops"] / (bf16 * 1e12)
@@ -624,6 +659,9 @@ def main():
                    "l2": "flushed before every timed step: 256 MB write, then 256 MB read (write-back "
                          "done outside the timed region); W_lm (1 GB) > L2",
                    "launch": "cuda_graph" if not args.no_graph else "stream",
+                   "kv_cache": (f"dual: prefix + window + {suffix_len(sh)} cached positions after "
+                                f"the window" if args.cache == "dual" else "prefix") +
+                               ("; committed rows appended every step" if args.append else ""),
                    "w_lm": ("64x64 tiles, unit-major (ebd_pack_lm_head, once at load)"
                             if args.w_layout == "packed" else "row-major [V][d]")},
         "roofline": roof,
@@ -649,7 +687,7 @@ def main():
                        "d2h_bytes_per_step": e["d2h"], "ms_per_step": round(e["mean_ms"], 4),
                        "api": "ebd_step_host"}
     if not args.skip_cpu and world == 1:
-        v, n, el = oracle_step_sample(sh, r["inp"], args.cpu_budget)
+        v, n, el = oracle_step_sample(sh, r["inp"], args.cpu_budget, r["suffix"])
         line["cpu_baseline"] = {"value": round(v, 3), "unit": UNIT, "cores": os.cpu_count(),
                                 "kind": "oracle",
                                 "sample": f"{n} full oracle steps of {sh.name} "

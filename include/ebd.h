@@ -152,10 +152,9 @@ typedef struct {
                                  k_win/v_win row written into k_cache/v_cache
                                  at row_pos (the prefix-cache append on
                                  commit); rows at positions >= max_prefix are
-                                 skipped.  The window attention of the same
-                                 step then runs after it instead of
-                                 overlapping the decision.  0: the cache is
-                                 only read.                                   */
+                                 skipped.  It runs after the step's window
+                                 attention, which reads the cache as it was
+                                 before.  0: the cache is only read.          */
   const int32_t* suffix;      /* [B][2] {s0, S}, device (host in
                                  ebd_step_host): the window also attends to
                                  the cached keys/values at positions

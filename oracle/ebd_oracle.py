@@ -484,11 +484,12 @@ def decide(cu_rows, row_pos, tokens, mask, in_block, blk_meta, st: RowStats,
 
 
 def step(inp, W, prm: DecisionParams, rows: Optional[np.ndarray] = None,
-         attention: bool = True) -> StepResult:
+         attention: bool = True, suffix=None) -> StepResult:
     """One EB decoding step (window attention, LM head + statistics, decision)
-    on a synthetic StepInputs-like object `inp`."""
+    on a synthetic StepInputs-like object `inp`; suffix: the dual cache's
+    ranges (window_attention)."""
     attn = (window_attention(inp.q, inp.k_win, inp.v_win, inp.k_cache,
-                             inp.v_cache, inp.cu_rows, inp.prefix_len)
+                             inp.v_cache, inp.cu_rows, inp.prefix_len, suffix)
             if attention else None)
     st = softmax_stats(lm_logits(inp.hidden, inp.w_lm))
     res = decide(inp.cu_rows, inp.row_pos, inp.tokens, inp.mask, inp.in_block,

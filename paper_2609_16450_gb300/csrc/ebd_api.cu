@@ -442,7 +442,7 @@ ebd_status check_args(ebd_handle* h, const ebd_step_args* a, bool need_attn, boo
 }
 
 ebd_status run_attention(ebd_handle* h, const ebd_step_args* a, cudaStream_t st,
-                         bool pdl = false) {
+                         bool pdl = false, bool wait_prior = false) {
   const ebd_config& c = h->cfg;
   const int D = c.head_dim, Hkv = c.n_heads_kv;
   CUtensorMap kc, vc, kw, vw;
@@ -485,6 +485,7 @@ ebd_status run_attention(ebd_handle* h, const ebd_step_args* a, cudaStream_t st,
   p.tickets = h->tickets;
   p.status = h->d_status;
   p.limit_ns = kLimitNs;
+  p.wait_prior = wait_prior ? 1 : 0;
   cudaError_t e = launch_attention(kc, vc, kw, vw, p, st, pdl);
   if (e != cudaSuccess) return cuda_fail(h, e, "attention launch");
   return EBD_OK;
@@ -840,12 +841,14 @@ ebd_status ebd_step(ebd_handle* h, const ebd_step_args* a, void* stream) {
   if (a->rows == 0 || a->batch == 0) return EBD_OK;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   (void)cudaGetLastError();  // a stale error of an earlier unrelated call is not ours
-  // Order on `st`: LM head, decision, (cache append), window attention.  The
+  // Order on `st`: LM head, decision, window attention, (cache append).  The
   // attention feeds neither of the others, so unless every kernel is timed
   // on its own (profile mode 1) it is launched as a programmatic dependent
-  // of the kernel before it: it fills the SMs the decision's clusters leave
-  // idle.  The append reads the mask the decision writes, so it is an
-  // ordinary launch after it; the attention reads no position it writes.
+  // of the decision: it fills the SMs the decision's clusters leave idle.
+  // The append reads the mask the decision writes: it is a programmatic
+  // dependent of the attention and waits for it, and the attention, in that
+  // case, waits for the decision before it exits.  The attention reads no
+  // cache position the append writes.
   const int prof = h->profile;
   cudaError_t e0 = cudaSuccess;
   if (prof && (e0 = record(h->ev[0], st)) != cudaSuccess) return cuda_fail(h, e0, "profile event");
@@ -857,13 +860,16 @@ ebd_status ebd_step(ebd_handle* h, const ebd_step_args* a, void* stream) {
   if (e != cudaSuccess) return cuda_fail(h, e, "decision launch");
   if (prof == 1 && (e0 = record(h->ev[2], st)) != cudaSuccess)
     return cuda_fail(h, e0, "profile event");
+  const bool pdl_attn = prof != 1;
+  if (attn && (s = run_attention(h, a, st, pdl_attn, a->kv_append != 0)) != EBD_OK) return s;
   if (a->kv_append) {
     const ebd_config& c = h->cfg;
+    // a programmatic dependent only of a kernel that waits for the decision
     e = launch_kv_append(a->k_cache, a->v_cache, a->k_win, a->v_win, a->cu_rows, a->row_pos, a->mask,
-                         a->batch, a->rows, c.max_prefix, c.n_heads_kv * c.head_dim, st);
+                         a->batch, a->rows, c.max_prefix, c.n_heads_kv * c.head_dim, st,
+                         attn && pdl_attn);
     if (e != cudaSuccess) return cuda_fail(h, e, "cache append launch");
   }
-  if (attn && (s = run_attention(h, a, st, prof != 1)) != EBD_OK) return s;
   if (prof && (e0 = record(h->ev[3], st)) != cudaSuccess) return cuda_fail(h, e0, "profile event");
   h->prof_mode = prof;
   h->prof_attn = attn ? 1 : 0;

@@ -60,6 +60,7 @@ struct AttnParams {
   int* tickets;             // [B*Hkv*max_qtiles]
   int* status;
   uint64_t limit_ns;
+  int wait_prior;           // every CTA waits for the grid it depends on before exiting
 };
 
 // ------------------------------------------------------------------ routers
@@ -110,7 +111,7 @@ cudaError_t launch_decide(const DecideParams& p, cudaStream_t st);
 cudaError_t launch_kv_append(uint16_t* k_cache, uint16_t* v_cache, const uint16_t* k_win,
                              const uint16_t* v_win, const int* cu_rows, const int* row_pos,
                              const uint8_t* mask, int B, int rows, int Pmax, int hkvd,
-                             cudaStream_t st);
+                             cudaStream_t st, bool pdl);
 cudaError_t launch_pack_lm(const __nv_bfloat16* w, __nv_bfloat16* out, int V, int d,
                            cudaStream_t st);
 cudaError_t launch_fold_tok(const __nv_bfloat16* w_tok, const __nv_bfloat16* w_emb, float* table,

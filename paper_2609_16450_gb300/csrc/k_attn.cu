@@ -30,10 +30,9 @@ __device__ __forceinline__ uint32_t swz(int r, int c) {
 }  // namespace
 
 template <int D>
-__global__ void __launch_bounds__(kAttnThreads)
-    attn_kernel(const __grid_constant__ CUtensorMap tm_kc, const __grid_constant__ CUtensorMap tm_vc,
-                const __grid_constant__ CUtensorMap tm_kw, const __grid_constant__ CUtensorMap tm_vw,
-                const AttnParams p) {
+__device__ __forceinline__ void attn_body(const CUtensorMap& tm_kc, const CUtensorMap& tm_vc,
+                                          const CUtensorMap& tm_kw, const CUtensorMap& tm_vw,
+                                          const AttnParams& p) {
   constexpr int NH = D / 64;   // 64-dim halves
   constexpr int KS = D / 16;   // k-steps of Q K^T
   constexpr int NT = D / 8;    // n-tiles of the output
@@ -326,6 +325,9 @@ __global__ void __launch_bounds__(256)
                      const uint4* __restrict__ k_win, const uint4* __restrict__ v_win,
                      const int* __restrict__ cu_rows, const int* __restrict__ row_pos,
                      const uint8_t* __restrict__ mask, int B, int Pmax, int vec_per_row) {
+  // launched as a programmatic dependent of the attention, which completes
+  // only after the decision: the mask read below is final
+  asm volatile("griddepcontrol.wait;" ::: "memory");
   const int r = blockIdx.x;
   if (mask[r] != 0) return;
   const int pos = row_pos[r];
@@ -343,13 +345,34 @@ __global__ void __launch_bounds__(256)
 cudaError_t launch_kv_append(uint16_t* k_cache, uint16_t* v_cache, const uint16_t* k_win,
                              const uint16_t* v_win, const int* cu_rows, const int* row_pos,
                              const uint8_t* mask, int B, int rows, int Pmax, int hkvd,
-                             cudaStream_t st) {
+                             cudaStream_t st, bool pdl) {
   if (rows <= 0) return cudaSuccess;
-  kv_append_kernel<<<rows, 256, 0, st>>>(
-      reinterpret_cast<uint4*>(k_cache), reinterpret_cast<uint4*>(v_cache),
-      reinterpret_cast<const uint4*>(k_win), reinterpret_cast<const uint4*>(v_win), cu_rows,
-      row_pos, mask, B, Pmax, hkvd / 8);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = dim3(rows, 1, 1);
+  cfg.blockDim = dim3(256, 1, 1);
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, kv_append_kernel, reinterpret_cast<uint4*>(k_cache),
+                            reinterpret_cast<uint4*>(v_cache), reinterpret_cast<const uint4*>(k_win),
+                            reinterpret_cast<const uint4*>(v_win), cu_rows, row_pos, mask, B, Pmax,
+                            hkvd / 8);
+}
+
+// The whole kernel; with p.wait_prior every CTA, whichever way it finishes,
+// waits for the grid it is a programmatic dependent of (the decision) before
+// it exits, so that a kernel launched after this one as its dependent sees
+// that grid complete as well.
+template <int D>
+__global__ void __launch_bounds__(kAttnThreads)
+    attn_kernel(const __grid_constant__ CUtensorMap tm_kc, const __grid_constant__ CUtensorMap tm_vc,
+                const __grid_constant__ CUtensorMap tm_kw, const __grid_constant__ CUtensorMap tm_vw,
+                const AttnParams p) {
+  attn_body<D>(tm_kc, tm_vc, tm_kw, tm_vw, p);
+  if (p.wait_prior) asm volatile("griddepcontrol.wait;" ::: "memory");
 }
 
 cudaError_t attn_configure() {

@@ -10,7 +10,7 @@ from .configs import (Shape, SHAPES, tiny, llada, dream, loop_shape, loop_tiny,
 from .gen import (StepInputs, make_step_inputs, normal_f32, normal_bf16,
                   uniform01, bf16_round, bf16_to_f32, f32_to_bf16_bits,
                   preset_in_block, loop_window_inputs, loop_kv, window_sizes,
-                  MASK_TOKEN)
+                  with_suffix_cache, MASK_TOKEN)
 from .router_init import (RouterLayout, router_layout, router_weights,
                           splitmix64_uniform, pack_blob, unpack_blob)
 
@@ -19,7 +19,7 @@ __all__ = [
     "sweep_points", "sweep_point", "StepInputs", "make_step_inputs",
     "normal_f32", "normal_bf16", "uniform01", "bf16_round", "bf16_to_f32",
     "f32_to_bf16_bits", "preset_in_block", "loop_window_inputs", "loop_kv",
-    "window_sizes",
+    "window_sizes", "with_suffix_cache",
     "MASK_TOKEN", "RouterLayout", "router_layout", "router_weights",
     "splitmix64_uniform", "pack_blob", "unpack_blob",
 ]

@@ -15,6 +15,7 @@ Value recipe (stand-ins for the paper's LLaDA-8B / Dream-7B decoding runs):
 """
 from __future__ import annotations
 
+import dataclasses
 import math
 import os
 from concurrent.futures import ThreadPoolExecutor
@@ -32,6 +33,7 @@ _CHUNK = 1 << 22
 # tensor ids of the step inputs
 T_WLM, T_WEMB, T_HID, T_HSCALE, T_Q, T_KWIN, T_VWIN, T_KC, T_VC = range(1, 10)
 T_PERM, T_TOK, T_WIN, T_LOOPHID, T_LOOPQ, T_LOOPKV = range(10, 16)
+T_KSUF, T_VSUF = range(16, 18)
 
 
 def _gen(seed: int, tid: int, chunk: int) -> np.random.Generator:
@@ -232,6 +234,23 @@ def preset_in_block(inp: StepInputs, span: int = 20) -> StepInputs:
 def _row(seed: int, tid: int, key: int, n: int) -> np.ndarray:
     """n standard normals keyed by (seed, tid, key); for small rows."""
     return _gen(seed, tid, key).standard_normal(n, dtype=np.float32)
+
+
+def with_suffix_cache(inp: StepInputs, suffix: int):
+    """A copy of `inp` whose K/V cache also holds the positions after each
+    window: capacity prefix + max window + suffix, the new positions drawn
+    N(0,1) like the prefix.  Returns (inputs, suffix ranges [B][2] =
+    {first position after the window, suffix})."""
+    sh = inp.shape
+    B, P, Hkv, D = inp.k_cache.shape
+    w = np.diff(inp.cu_rows).astype(np.int64)
+    extra = int(w.max()) + suffix
+    k_ext = normal_bf16(sh.seed, T_KSUF, (B, extra, Hkv, D))
+    v_ext = normal_bf16(sh.seed, T_VSUF, (B, extra, Hkv, D))
+    out = dataclasses.replace(inp, k_cache=np.concatenate([inp.k_cache, k_ext], axis=1),
+                              v_cache=np.concatenate([inp.v_cache, v_ext], axis=1))
+    rng = np.stack([inp.prefix_len.astype(np.int64) + w, np.full(B, suffix)], axis=1)
+    return out, rng.astype(np.int32)
 
 
 def loop_window_inputs(shape: Shape, step: int, positions: np.ndarray):
