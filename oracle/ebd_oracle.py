@@ -518,7 +518,8 @@ def loop_window(frontier: int, end: int, meta, in_block_pos: List[int],
 def generation_loop(shape, W, prm: DecisionParams, window_inputs, kv_rows,
                     w_lm, w_emb, max_steps: Optional[int] = None,
                     attention: bool = False, on_step=None, mode: str = "eb",
-                    block: int = 32, top_m: int = 1, cache: str = "prefix"):
+                    block: int = 32, top_m: int = 1, cache: str = "prefix",
+                    window: str = "block"):
     """Run the App. E loop on the synthetic loop workload: a committed prompt
     of `shape.prefix` positions followed by `shape.gen_len` masked positions.
     window_inputs(step, positions) -> (hidden, q, k_win, v_win) and
@@ -527,7 +528,8 @@ def generation_loop(shape, W, prm: DecisionParams, window_inputs, kv_rows,
     runs the App. E algorithm; 'threshold' and 'topm' the fixed-block rules
     of the baselines (Reading R20) with blocks of `block` positions.  cache
     'dual' adds the positions right of the window as cached keys (Reading
-    R21)."""
+    R21).  window 'full': every step's window is the whole response (the
+    full-sequence setting: M is every masked position)."""
     P0, L = shape.prefix, shape.gen_len
     tokens = np.full(L, -1, np.int32)
     mask = np.ones(L, np.uint8)
@@ -537,7 +539,9 @@ def generation_loop(shape, W, prm: DecisionParams, window_inputs, kv_rows,
     while mask.any():
         if max_steps is not None and steps >= max_steps:
             break
-        if mode == "eb":
+        if window == "full":
+            lo, hi = 0, L
+        elif mode == "eb":
             f = int(np.argmax(mask))
             blk = [i for i in range(L) if in_block[i]]
             lo, hi = loop_window(f, L, meta, blk)

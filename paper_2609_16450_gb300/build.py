@@ -18,7 +18,7 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libebd.so")
-SOURCES = ["ebd_api.cu", "k_lmhead.cu", "k_attn.cu", "k_decide.cu"]
+SOURCES = ["ebd_api.cu", "k_lmhead.cu", "k_attn.cu", "k_decide.cu", "k_decide_seq.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

@@ -198,6 +198,11 @@ struct ebd_handle {
   int* d_status = nullptr;
   uint8_t* staging = nullptr;
   size_t staging_bytes = 0;
+  // the grid-wide decision (max_window > kMaxWindow)
+  float* d_seqw = nullptr;   // SeqWeights image
+  SeqWeights seqw{};
+  uint8_t* seq_scratch = nullptr;
+  SeqParams seqp{};          // scratch pointers, filled at create
   cudaEvent_t ev[4] = {nullptr, nullptr, nullptr, nullptr};
   int profile = 0;
   int prof_mode = 0, prof_attn = 0;  // what the last ebd_step recorded
@@ -225,7 +230,7 @@ ebd_status validate_config(const ebd_config* c, std::string& why) {
   if (c->n_heads_kv <= 0 || c->n_heads_q <= 0 || c->n_heads_q % c->n_heads_kv)
     return bad("n_heads_q must be a positive multiple of n_heads_kv");
   if (c->max_batch <= 0 || c->max_batch > 65535) return bad("max_batch out of range");
-  if (c->max_window <= 0 || c->max_window > kMaxWindow) return bad("max_window must be 1..64");
+  if (c->max_window <= 0 || c->max_window > kMaxSeqRows) return bad("max_window must be 1..512");
   if (c->max_rows <= 0 || c->max_rows > 4096) return bad("max_rows must be 1..4096");
   if (c->max_prefix < 0) return bad("max_prefix must be >= 0");
   if (c->gen_len < c->max_window) return bad("gen_len must be >= max_window");
@@ -242,6 +247,113 @@ ebd_status check_device(ebd_handle* h) {
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return cuda_fail(h, e, "cudaGetDevice");
   if (dev != h->device) return fail(h, EBD_ERR_INVALID_ARG, "current device differs from the handle's");
+  return EBD_OK;
+}
+
+// fp32 image of the router weights for the grid-wide decision: matrices
+// [in][out], vectors as they are (SeqWeights).
+ebd_status upload_seq_weights(ebd_handle* h) {
+  // element (r, c) of a blob tensor, its offset resolved once per name
+  std::string last;
+  size_t last_off = 0, last_cols = 0;
+  auto atf = [&](const std::string& name, int r, int c) -> float {
+    if (name != last) {
+      size_t off = 0;
+      bool found = false;
+      for (const auto& t : h->layout) {
+        if (t.name == name) {
+          last_cols = static_cast<size_t>(t.cols);
+          found = true;
+          break;
+        }
+        off += static_cast<size_t>(t.rows) * t.cols;
+      }
+      last = name;
+      last_off = found ? off : 0;
+    }
+    return bf16_to_f32(h->h_blob[last_off + static_cast<size_t>(r) * last_cols + c]);
+  };
+  SeqWeights& o = h->seqw;
+  int n = 0;
+  auto take = [&](int count) {
+    const int at = n;
+    n += (count + 3) / 4 * 4;
+    return at;
+  };
+  const int L = h->cfg.gen_len;
+  o.ent1_w = take(64); o.ent1_b = take(64); o.ent2_t = take(64 * 64); o.ent2_b = take(64);
+  o.entln_g = take(64); o.entln_b = take(64); o.tok_b = take(64);
+  o.comb_t = take(128 * 128); o.comb_b = take(128); o.pos = take(L * 128);
+  for (int l = 0; l < 2; ++l) {
+    SeqLayer& q = o.l[l];
+    q.qkv_t = take(128 * 384); q.qkv_b = take(384); q.out_t = take(128 * 128); q.out_b = take(128);
+    q.ln1_g = take(128); q.ln1_b = take(128); q.ff1_t = take(128 * 256); q.ff1_b = take(256);
+    q.ff2_t = take(256 * 128); q.ff2_b = take(128); q.ln2_g = take(128); q.ln2_b = take(128);
+  }
+  o.head_w = take(128); o.head_b = take(1);
+  o.in_t = take(5 * 32); o.in_b = take(32); o.inln_g = take(32); o.inln_b = take(32);
+  for (int l = 0; l < 2; ++l) {
+    SeqBlock& q = o.p[l];
+    q.ln1_g = take(32); q.ln1_b = take(32); q.qkv_t = take(32 * 96); q.qkv_b = take(96);
+    q.out_t = take(32 * 32); q.out_b = take(32); q.ln2_g = take(32); q.ln2_b = take(32);
+    q.ff1_t = take(32 * 64); q.ff1_b = take(64); q.ff2_t = take(64 * 32); q.ff2_b = take(32);
+  }
+  o.phead_w = take(32); o.phead_b = take(1);
+  o.total = n;
+  std::vector<float> w(static_cast<size_t>(n), 0.f);
+  // [in][out] copy of a [out][in] matrix, and a vector
+  auto mat = [&](int at, const std::string& name, int nin, int nout) {
+    for (int k = 0; k < nin; ++k)
+      for (int c = 0; c < nout; ++c) w[at + static_cast<size_t>(k) * nout + c] = atf(name, c, k);
+  };
+  auto vec = [&](int at, const std::string& name, int count) {
+    for (int c = 0; c < count; ++c) w[at + c] = atf(name, 0, c);
+  };
+  for (int c = 0; c < 64; ++c) w[o.ent1_w + c] = atf("lbs.ent1.w", c, 0);
+  vec(o.ent1_b, "lbs.ent1.b", 64);
+  mat(o.ent2_t, "lbs.ent2.w", 64, 64);
+  vec(o.ent2_b, "lbs.ent2.b", 64);
+  vec(o.entln_g, "lbs.ent_ln.g", 64);
+  vec(o.entln_b, "lbs.ent_ln.b", 64);
+  vec(o.tok_b, "lbs.tok.b", 64);
+  mat(o.comb_t, "lbs.comb.w", 128, 128);
+  vec(o.comb_b, "lbs.comb.b", 128);
+  for (int j = 0; j < L; ++j)
+    for (int c = 0; c < 128; ++c) w[o.pos + static_cast<size_t>(j) * 128 + c] = atf("lbs.pos", j, c);
+  for (int l = 0; l < 2; ++l) {
+    const std::string pre = "lbs.l" + std::to_string(l);
+    const SeqLayer& q = o.l[l];
+    mat(q.qkv_t, pre + ".qkv.w", 128, 384); vec(q.qkv_b, pre + ".qkv.b", 384);
+    mat(q.out_t, pre + ".out.w", 128, 128); vec(q.out_b, pre + ".out.b", 128);
+    vec(q.ln1_g, pre + ".ln1.g", 128); vec(q.ln1_b, pre + ".ln1.b", 128);
+    mat(q.ff1_t, pre + ".ff1.w", 128, 256); vec(q.ff1_b, pre + ".ff1.b", 256);
+    mat(q.ff2_t, pre + ".ff2.w", 256, 128); vec(q.ff2_b, pre + ".ff2.b", 128);
+    vec(q.ln2_g, pre + ".ln2.g", 128); vec(q.ln2_b, pre + ".ln2.b", 128);
+  }
+  vec(o.head_w, "lbs.head.w", 128);
+  vec(o.head_b, "lbs.head.b", 1);
+  mat(o.in_t, "lps.in.w", 5, 32);
+  vec(o.in_b, "lps.in.b", 32);
+  vec(o.inln_g, "lps.in_ln.g", 32);
+  vec(o.inln_b, "lps.in_ln.b", 32);
+  for (int l = 0; l < 2; ++l) {
+    const std::string pre = "lps.l" + std::to_string(l);
+    const SeqBlock& q = o.p[l];
+    vec(q.ln1_g, pre + ".ln1.g", 32); vec(q.ln1_b, pre + ".ln1.b", 32);
+    mat(q.qkv_t, pre + ".qkv.w", 32, 96); vec(q.qkv_b, pre + ".qkv.b", 96);
+    mat(q.out_t, pre + ".out.w", 32, 32); vec(q.out_b, pre + ".out.b", 32);
+    vec(q.ln2_g, pre + ".ln2.g", 32); vec(q.ln2_b, pre + ".ln2.b", 32);
+    mat(q.ff1_t, pre + ".ff1.w", 32, 64); vec(q.ff1_b, pre + ".ff1.b", 64);
+    mat(q.ff2_t, pre + ".ff2.w", 64, 32); vec(q.ff2_b, pre + ".ff2.b", 32);
+  }
+  vec(o.phead_w, "lps.head.w", 32);
+  vec(o.phead_b, "lps.head.b", 1);
+  if (h->d_seqw == nullptr) {
+    cudaError_t e = cudaMalloc(&h->d_seqw, w.size() * sizeof(float));
+    if (e != cudaSuccess) return cuda_fail(h, e, "cudaMalloc(router fp32 image)");
+  }
+  cudaError_t e = cudaMemcpy(h->d_seqw, w.data(), w.size() * sizeof(float), cudaMemcpyHostToDevice);
+  if (e != cudaSuccess) return cuda_fail(h, e, "cudaMemcpy(router fp32 image)");
   return EBD_OK;
 }
 
@@ -381,7 +493,7 @@ ebd_status upload_router(ebd_handle* h) {
   h->img.lps_w = reinterpret_cast<const __nv_bfloat16*>(h->d_image + o_lps);
   h->img.vec = reinterpret_cast<const float*>(h->d_image + o_vec);
   h->img.tok_table = h->d_tok;
-  return EBD_OK;
+  return upload_seq_weights(h);
 }
 
 ebd_status fold(ebd_handle* h, cudaStream_t st) {
@@ -703,7 +815,8 @@ ebd_status ebd_create(const ebd_config* cfg, ebd_handle** out) {
   // attention split-KV workspace
   {
     const int group = cfg->n_heads_q / cfg->n_heads_kv;
-    h->attn_max_qtiles = (cfg->max_window * group + 63) / 64;
+    const int aw = cfg->max_window < kMaxWindow ? cfg->max_window : kMaxWindow;
+    h->attn_max_qtiles = (aw * group + 63) / 64;
     const int slots = cfg->max_batch * cfg->n_heads_kv * h->attn_max_qtiles;
     const int nch = (cfg->max_prefix + kAttnChunk - 1) / kAttnChunk + 1;
     int splits = (2 * h->num_sms + slots - 1) / slots;
@@ -740,6 +853,46 @@ ebd_status ebd_create(const ebd_config* cfg, ebd_handle** out) {
     if ((e = cudaMalloc(&h->staging, bytes)) != cudaSuccess)
       return bail(cuda_fail(h, e, "cudaMalloc(staging)"));
   }
+  if (cfg->max_window > kMaxWindow) {  // scratch of the grid-wide decision
+    const size_t R = cfg->max_rows, B = cfg->max_batch;
+    size_t bytes = 0;
+    auto add = [&](size_t n) {
+      const size_t at = bytes;
+      bytes += (n + 255) / 256 * 256;
+      return at;
+    };
+    const size_t o_conf = add(R * 4), o_entn = add(R * 4), o_gap = add(R * 4), o_arg = add(R * 4);
+    const size_t o_seq = add(R * 4), o_mr = add(R * 4), o_mrows = add(R * 4), o_bmr = add(R * 4),
+                 o_bmrows = add(R * 4), o_bad = add(R), o_ib = add(R), o_sq = add(B * 8 * 4),
+                 o_O = add(R * 4), o_P = add(R * 4), o_f = add(R * 8 * 4), o_Z = add(R * 128 * 4),
+                 o_QKV = add(R * 384 * 4), o_A = add(R * 128 * 4), o_Zp = add(R * 32 * 4),
+                 o_QKVp = add(R * 96 * 4), o_Ap = add(R * 32 * 4);
+    if ((e = cudaMalloc(&h->seq_scratch, bytes)) != cudaSuccess)
+      return bail(cuda_fail(h, e, "cudaMalloc(decision scratch)"));
+    uint8_t* b0 = h->seq_scratch;
+    SeqParams& q = h->seqp;
+    q.conf = reinterpret_cast<float*>(b0 + o_conf);
+    q.ent_norm = reinterpret_cast<float*>(b0 + o_entn);
+    q.gap = reinterpret_cast<float*>(b0 + o_gap);
+    q.argmax = reinterpret_cast<int*>(b0 + o_arg);
+    q.seq_of = reinterpret_cast<int*>(b0 + o_seq);
+    q.mrank = reinterpret_cast<int*>(b0 + o_mr);
+    q.mrows = reinterpret_cast<int*>(b0 + o_mrows);
+    q.bmrank = reinterpret_cast<int*>(b0 + o_bmr);
+    q.bmrows = reinterpret_cast<int*>(b0 + o_bmrows);
+    q.bad = b0 + o_bad;
+    q.ib = b0 + o_ib;
+    q.sq = reinterpret_cast<int*>(b0 + o_sq);
+    q.O = reinterpret_cast<float*>(b0 + o_O);
+    q.P = reinterpret_cast<float*>(b0 + o_P);
+    q.feats = reinterpret_cast<float*>(b0 + o_f);
+    q.Z = reinterpret_cast<float*>(b0 + o_Z);
+    q.QKV = reinterpret_cast<float*>(b0 + o_QKV);
+    q.A = reinterpret_cast<float*>(b0 + o_A);
+    q.Zp = reinterpret_cast<float*>(b0 + o_Zp);
+    q.QKVp = reinterpret_cast<float*>(b0 + o_QKVp);
+    q.Ap = reinterpret_cast<float*>(b0 + o_Ap);
+  }
   for (int i = 0; i < 4; ++i)
     if ((e = cudaEventCreate(&h->ev[i])) != cudaSuccess)
       return bail(cuda_fail(h, e, "cudaEventCreate"));
@@ -763,6 +916,8 @@ void ebd_destroy(ebd_handle* h) {
   cudaFree(h->tickets);
   cudaFree(h->d_status);
   cudaFree(h->staging);
+  cudaFree(h->d_seqw);
+  cudaFree(h->seq_scratch);
   for (int i = 0; i < 4; ++i)
     if (h->ev[i]) cudaEventDestroy(h->ev[i]);
   if (prev >= 0 && prev != h->device) cudaSetDevice(prev);
@@ -831,6 +986,77 @@ ebd_status ebd_pack_lm_head(ebd_handle* h, const uint16_t* w_lm, uint16_t* w_pac
   return EBD_OK;
 }
 
+namespace {
+// windows of more than kMaxWindow rows per sequence: the grid-wide decision
+bool seq_mode(const ebd_handle* h) { return h->cfg.max_window > kMaxWindow; }
+
+SeqParams seq_params(ebd_handle* h, const ebd_step_args* a, const float* conf,
+                     const float* ent_norm, const float* gap, const int* argmax) {
+  const ebd_config& c = h->cfg;
+  SeqParams p = h->seqp;  // scratch
+  p.B = a->batch;
+  p.R = a->rows;
+  p.V = c.vocab;
+  p.gen_len = c.gen_len;
+  p.g_max = c.g_max;
+  p.l_min = c.l_min;
+  p.l_b = c.l_b;
+  p.eos_id = c.eos_id;
+  p.mode = c.decode_mode;
+  p.top_m = c.top_m;
+  p.lps_enabled = c.decode_mode == EBD_DECODE_EB ? c.lps_enabled : 0;
+  p.tau = c.tau;
+  p.tau_psi = c.tau_psi;
+  p.cu_rows = a->cu_rows;
+  p.row_pos = a->row_pos;
+  p.tokens = a->tokens;
+  p.mask = a->mask;
+  p.in_block = a->in_block;
+  p.blk_meta = a->blk_meta;
+  p.conf = conf;
+  p.ent_norm = ent_norm;
+  p.gap = gap;
+  p.argmax = argmax;
+  p.accepted = a->accepted;
+  p.lbs_logit = a->lbs_logit;
+  p.lps_prob = a->lps_prob;
+  p.w = h->d_seqw;
+  p.o = h->seqw;
+  p.tok_table = h->d_tok;
+  p.status = h->d_status;
+  return p;
+}
+
+// LM head, merge into the statistics, grid-wide decision
+ebd_status step_seq(ebd_handle* h, const ebd_step_args* a, cudaStream_t st) {
+  if (a->attn_out != nullptr || a->kv_append)
+    return fail(h, EBD_ERR_UNSUPPORTED,
+                "the window attention and the cache append need windows of at most 64 rows "
+                "(this handle has max_window > 64)");
+  const int prof = h->profile;
+  cudaError_t e;
+  if (prof && (e = record(h->ev[0], st)) != cudaSuccess) return cuda_fail(h, e, "profile event");
+  ebd_status s = run_lm(h, a, st);
+  if (s != EBD_OK) return s;
+  if (prof && (e = record(h->ev[1], st)) != cudaSuccess) return cuda_fail(h, e, "profile event");
+  float* conf = a->conf ? a->conf : const_cast<float*>(h->seqp.conf);
+  float* entn = a->ent_norm ? a->ent_norm : const_cast<float*>(h->seqp.ent_norm);
+  float* gap = a->gap ? a->gap : const_cast<float*>(h->seqp.gap);
+  int* arg = a->argmax ? a->argmax : const_cast<int*>(h->seqp.argmax);
+  const float inv = static_cast<float>(1.0 / std::log(static_cast<double>(h->cfg.vocab)));
+  if ((e = launch_merge_stats(h->part_f, h->part_i, a->rows, h->grid_lm, h->cfg.vocab, inv, conf,
+                              a->entropy, entn, gap, arg, h->d_status, st)) != cudaSuccess)
+    return cuda_fail(h, e, "merge launch");
+  if ((e = launch_decide_seq(seq_params(h, a, conf, entn, gap, arg), st)) != cudaSuccess)
+    return cuda_fail(h, e, "decision launch");
+  if (prof && (e = record(h->ev[2], st)) != cudaSuccess) return cuda_fail(h, e, "profile event");
+  if (prof && (e = record(h->ev[3], st)) != cudaSuccess) return cuda_fail(h, e, "profile event");
+  h->prof_mode = prof;
+  h->prof_attn = 0;
+  return EBD_OK;
+}
+}  // namespace
+
 ebd_status ebd_step(ebd_handle* h, const ebd_step_args* a, void* stream) {
   if (h == nullptr) return EBD_ERR_INVALID_ARG;
   ebd_status s = check_device(h);
@@ -841,6 +1067,7 @@ ebd_status ebd_step(ebd_handle* h, const ebd_step_args* a, void* stream) {
   if (a->rows == 0 || a->batch == 0) return EBD_OK;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   (void)cudaGetLastError();  // a stale error of an earlier unrelated call is not ours
+  if (seq_mode(h)) return step_seq(h, a, st);
   // Order on `st`: LM head, decision, window attention, (cache append).  The
   // attention feeds neither of the others, so unless every kernel is timed
   // on its own (profile mode 1) it is launched as a programmatic dependent
@@ -885,6 +1112,12 @@ ebd_status ebd_decide(ebd_handle* h, const ebd_step_args* a, void* stream) {
     return fail(h, EBD_ERR_INVALID_ARG, "conf/ent_norm/gap/argmax inputs must be set");
   if (h->w_emb == nullptr) return fail(h, EBD_ERR_STATE, "bind the token embedding first");
   if (a->rows == 0 || a->batch == 0) return EBD_OK;
+  if (seq_mode(h)) {
+    cudaError_t e = launch_decide_seq(seq_params(h, a, a->conf, a->ent_norm, a->gap, a->argmax),
+                                      static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(h, e, "decision launch");
+    return EBD_OK;
+  }
   DecideParams p = decide_params(h, a, 1);
   p.entropy = nullptr;
   cudaError_t e = launch_decide(p, static_cast<cudaStream_t>(stream));
@@ -1051,9 +1284,8 @@ ebd_status ebd_sync_status(ebd_handle* h, void* stream) {
     return cuda_fail(h, e, "status read");
   if (v != 0) {
     cudaMemset(h->d_status, 0, sizeof(int));
-    const int group = h->cfg.n_heads_q / h->cfg.n_heads_kv;
-    const int slots = h->cfg.max_batch * h->cfg.n_heads_kv * ((h->cfg.max_window * group + 63) / 64);
-    cudaMemset(h->tickets, 0, static_cast<size_t>(slots) * sizeof(int));
+    const int slots = h->cfg.max_batch * h->cfg.n_heads_kv * h->attn_max_qtiles;
+    if (h->tickets) cudaMemset(h->tickets, 0, static_cast<size_t>(slots) * sizeof(int));
     cudaDeviceSynchronize();
     h->err = "device reported status " + std::to_string(v);
   }

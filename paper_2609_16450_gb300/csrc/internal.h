@@ -9,7 +9,8 @@
 
 namespace ebd {
 
-constexpr int kMaxWindow = 64;        // window rows per sequence
+constexpr int kMaxWindow = 64;        // window rows per sequence of the cluster decision
+constexpr int kMaxSeqRows = 512;      // window rows per sequence of the grid-wide decision
 constexpr int kUnit = 64;             // vocabulary rows per work unit of the LM head
 constexpr int kLmThreads = 320;  // TMA warp, MMA warp, two epilogue warpgroups of 4 warps
 constexpr int kMaxGroupRows = 512;    // rows per LM-head launch (TMEM: 512 columns)
@@ -95,6 +96,66 @@ struct DecideParams {
   RouterImage w;
 };
 
+// ------------------------------------------------------------------ grid-wide decision
+// fp32 copy of the router weights for the grid-wide decision (windows of up
+// to kMaxSeqRows rows per sequence): float offsets into one allocation;
+// matrices are stored [in][out] (consecutive outputs contiguous).
+struct SeqLayer {                // one LBS encoder layer
+  int qkv_t, qkv_b, out_t, out_b, ln1_g, ln1_b, ff1_t, ff1_b, ff2_t, ff2_b, ln2_g, ln2_b;
+};
+struct SeqBlock {                // one LPS block
+  int ln1_g, ln1_b, qkv_t, qkv_b, out_t, out_b, ln2_g, ln2_b, ff1_t, ff1_b, ff2_t, ff2_b;
+};
+struct SeqWeights {
+  int ent1_w, ent1_b, ent2_t, ent2_b, entln_g, entln_b, tok_b, comb_t, comb_b, pos;
+  SeqLayer l[2];
+  int head_w, head_b;
+  int in_t, in_b, inln_g, inln_b;  // LPS input layer
+  SeqBlock p[2];
+  int phead_w, phead_b;
+  int total;
+};
+
+struct SeqParams {
+  int B, R, V, gen_len, g_max, l_min, l_b, eos_id, lps_enabled, mode, top_m;
+  float tau, tau_psi;
+  const int* cu_rows;
+  const int* row_pos;
+  int* tokens;
+  uint8_t* mask;
+  uint8_t* in_block;
+  int* blk_meta;
+  const float* conf;        // statistics of every row (inputs)
+  const float* ent_norm;
+  const float* gap;
+  const int* argmax;
+  uint8_t* accepted;        // outputs, may be null
+  float* lbs_logit;
+  float* lps_prob;
+  const float* w;           // SeqWeights image
+  SeqWeights o;
+  const float* tok_table;   // [V][64]
+  // scratch, [R] or [R][k] unless noted
+  int* seq_of;
+  int* mrank;               // rank of a masked row within its sequence's M, else -1
+  int* mrows;               // sequence b's masked rows at [cu_rows[b], cu_rows[b] + |M|)
+  int* bmrank;              // rank within B n M (rows the LPS scores), else -1
+  int* bmrows;
+  uint8_t* bad;
+  uint8_t* ib;              // block membership after the selection
+  int* sq;                  // [B][8] per-sequence state (kSq* indices)
+  float* O;                 // LBS logit
+  float* P;                 // LPS probability
+  float* feats;             // [R][8]
+  float* Z;                 // [R][128]
+  float* QKV;               // [R][384]
+  float* A;                 // [R][128]
+  float* Zp;                // [R][32]
+  float* QKVp;              // [R][96]
+  float* Ap;                // [R][32]
+  int* status;
+};
+
 // host launchers (defined next to their kernels)
 cudaError_t launch_lm_stats(const CUtensorMap& tmap_w, const CUtensorMap& tmap_h,
                             const LmParams& p, cudaStream_t st);
@@ -106,6 +167,8 @@ cudaError_t launch_attention(const CUtensorMap& kc, const CUtensorMap& vc, const
                              const CUtensorMap& vw, const AttnParams& p, cudaStream_t st,
                              bool pdl = false);
 cudaError_t launch_decide(const DecideParams& p, cudaStream_t st);
+// the grid-wide decision: a chain of kernels on `st` (k_decide_seq.cu)
+cudaError_t launch_decide_seq(const SeqParams& p, cudaStream_t st);
 // prefix-cache append on commit: window row r of sequence b with mask[r] == 0
 // is copied (K and V, Hkv * D bf16 each) to cache position row_pos[r] < Pmax
 cudaError_t launch_kv_append(uint16_t* k_cache, uint16_t* v_cache, const uint16_t* k_win,

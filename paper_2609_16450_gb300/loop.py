@@ -68,7 +68,8 @@ def run_loop(h: rt.Handle, shape, weights: rt.DeviceWeights,
              window_inputs: Callable, kv_rows: Callable, attention: bool = True,
              max_steps: Optional[int] = None, max_window: int = 64,
              keep: bool = True, stream: Optional[torch.cuda.Stream] = None,
-             block: int = 32, cache: str = "prefix", append: bool = False) -> LoopResult:
+             block: int = 32, cache: str = "prefix", append: bool = False,
+             window: str = "block") -> LoopResult:
     """window_inputs(step, positions) -> (hidden, q, k_win, v_win) as bf16 bit
     arrays; kv_rows(positions) -> (k, v).  Positions are absolute.  Under the
     handle's baseline decode modes the window is the active fixed block of
@@ -78,11 +79,16 @@ def run_loop(h: rt.Handle, shape, weights: rt.DeviceWeights,
     positions right of the window standing for the K/V a dual cache holds)."""
     if cache not in ("prefix", "dual"):
         raise ValueError("cache must be 'prefix' or 'dual'")
+    if window not in ("block", "full"):
+        raise ValueError("window must be 'block' or 'full'")
+    full = window == "full"  # the full-sequence setting: the window is the whole response
+    if full and (attention or append):
+        raise ValueError("the full-sequence window runs without the window attention")
     fixed = h.cfg.decode_mode != E.EBD_DECODE_EB
     dev = "cuda"
     P0, L = shape.prefix, shape.gen_len
     d, Hq, Hkv, D = shape.d_model, shape.n_heads_q, shape.n_heads_kv, shape.head_dim
-    W = max_window
+    W = L if full else max_window
     stream = stream or torch.cuda.current_stream()
     sid = stream.cuda_stream
     i32 = dict(dtype=torch.int32, device=dev)
@@ -123,7 +129,9 @@ def run_loop(h: rt.Handle, shape, weights: rt.DeviceWeights,
     while True:
         if max_steps is not None and step >= max_steps:
             break
-        if fixed:
+        if full:
+            s, lo, hi = E.EBD_OK, (0 if mask_h.any() else L), L
+        elif fixed:
             s, lo, hi = E.ebd_loop_block_window(mask_h, block)
         else:
             s, lo, hi = E.ebd_loop_window(mask_h, ib_h, meta_h, W)

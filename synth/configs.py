@@ -84,7 +84,25 @@ loop_tiny = Shape(name="loop_tiny", batch=1, d_model=256, vocab=4096, n_heads_q=
                   n_heads_kv=4, head_dim=64, prefix=64, windows=(64,), mask_frac=1.0,
                   gen_len=64, w_lm_std=0.02, seed=4)
 
-SHAPES = {s.name: s for s in (tiny, llada, dream, loop_shape, loop_tiny)}
+# The full-sequence setting (every position of the response is a row of the
+# step; the LBS sees all masked positions; no KV cache): LLaDA-8B shapes with
+# a 512-token response, and a tiny one the oracle finishes in seconds.
+llada_full = Shape(name="llada8b_full", batch=1, d_model=4096, vocab=126464,
+                   n_heads_q=32, n_heads_kv=32, head_dim=128, prefix=0,
+                   windows=(512,), mask_frac=0.75, gen_len=512,
+                   w_lm_std=1.0 / 64.0, seed=5)
+tiny_full = Shape(name="tiny_full", batch=3, d_model=256, vocab=4096, n_heads_q=4,
+                  n_heads_kv=4, head_dim=64, prefix=0, windows=(256, 100, 40),
+                  mask_frac=0.75, gen_len=256, w_lm_std=0.02, seed=6)
+# the generation loop in the full-sequence setting at the tiny shape (gen 96)
+loop_full_tiny = Shape(name="loop_full_tiny", batch=1, d_model=256, vocab=4096, n_heads_q=4,
+                       n_heads_kv=4, head_dim=64, prefix=64, windows=(96,), mask_frac=1.0,
+                       gen_len=96, w_lm_std=0.02, seed=23)
+# ... and at the LLaDA-8B loop shape (prompt 256, gen 256)
+loop_full = loop_shape.with_(name="loop_full_llada8b", windows=(256,), seed=8)
+
+SHAPES = {s.name: s for s in (tiny, llada, dream, loop_shape, loop_tiny, llada_full, tiny_full,
+                              loop_full_tiny, loop_full)}
 
 
 def sweep_points():

@@ -196,3 +196,32 @@ def test_small_generation_loop_terminates_within_L():
     assert (tokens >= 0).all() and steps <= sh.gen_len
     assert all(c >= 1 for c in commits) and sum(commits) == sh.gen_len
     assert all(r["window"][1] - r["window"][0] <= 64 for r in recs)
+
+
+def test_full_sequence_loop_invariants():
+    """The full-sequence setting: every step's window is the whole response,
+    M is every masked position.  The loop ends within L steps, commits at
+    least one position per step, commits only masked positions of the
+    window, and never unmasks anything else."""
+    sh = synth.tiny.with_(name="loop_full", prefix=16, gen_len=80, d_model=64,
+                          vocab=512, n_heads_q=2, n_heads_kv=2, head_dim=16, seed=3)
+    W = o.weights_f64(synth.router_weights(sh.seed, sh.d_base, sh.gen_len))
+    wl = synth.normal_bf16(3, 1, (sh.vocab, sh.d_model), 0.1)
+    we = synth.normal_bf16(3, 2, (sh.vocab, sh.d_base), 1.0)
+    prm = o.DecisionParams(tau=sh.tau, tau_psi=sh.tau_psi, l_min=sh.l_min, l_b=sh.l_b,
+                           g_max=sh.g_max, eos_id=sh.eos_id)
+    seen = []
+    tokens, steps, commits, recs = o.generation_loop(
+        sh, W, prm, lambda s, p: synth.loop_window_inputs(sh, s, p),
+        lambda p: synth.loop_kv(sh, p), wl, we, window="full",
+        on_step=lambda s, r: seen.append(r["accepted"].copy()))
+    assert (tokens >= 0).all() and steps <= sh.gen_len
+    assert all(c >= 1 for c in commits) and sum(commits) == sh.gen_len
+    assert all(r["window"] == (0, sh.gen_len) for r in recs)
+    committed = np.zeros(sh.gen_len, bool)
+    for acc in seen:
+        acc = acc.astype(bool)
+        assert not np.any(committed & acc), "a position was committed twice"
+        committed |= acc
+    assert committed.all()
+    assert any(r["lbs_ran"] for r in recs), "the LBS never ran on the whole response"
