@@ -64,9 +64,22 @@ def shape_for(name):
     raise SystemExit(f"unknown config {name}")
 
 
+def full_sequence(sh):
+    """The full-sequence setting: windows of more than 64 rows (every
+    position of the response), decided by the grid-wide kernels, without
+    the window attention."""
+    import synth
+    return int(np.max(synth.window_sizes(sh))) > 64
+
+
 def workload_text(sh, state):
     import synth
     w = synth.window_sizes(sh)
+    if full_sequence(sh):
+        return (f"{sh.name} full-sequence step: batch {sh.batch}, hidden {sh.d_model}, vocab {sh.vocab}, "
+                f"every position of a {int(w.max())}-token response is a row ({int(w.sum())} rows), "
+                f"LBS over all masked positions ({'no active block: LBS runs' if state == 'select' else 'active block'}); "
+                f"no window attention")
     return (f"{sh.name} decoding step: batch {sh.batch}, hidden {sh.d_model}, vocab {sh.vocab}, "
             f"{sh.n_heads_q}q/{sh.n_heads_kv}kv heads x {sh.head_dim}, cached prefix {sh.prefix}, "
             f"window rows {int(w.sum())} ({'no active block: LBS runs' if state == 'select' else 'active block'})")
@@ -182,12 +195,15 @@ def step_work(sh, rows, masked, grid_lm, lbs_runs, suffix=0, append=False):
     import synth
     w = synth.window_sizes(sh)
     keys = int(sum(sh.prefix + int(x) + suffix for x in w))
+    attn = not full_sequence(sh)
     lm_bytes = V * d * 2 + rows * d * 2 + rows * grid_lm * 20
     lm_flops = 2 * rows * d * V
     attn_bytes = keys * Hkv * D * 2 * 2 + rows * Hq * D * 2 + rows * Hq * D * 4
     attn_flops = 4 * sum(int(x) * (sh.prefix + int(x) + suffix) for x in w) * Hq * D
     if append:
         attn_bytes += rows * Hkv * D * 2 * 2 * 2
+    if not attn:
+        attn_bytes = attn_flops = 0
     dec_bytes = rows * grid_lm * 20 + rows * 40
     if lbs_runs:
         dec_bytes += 2 * (613761 - 262208) + masked * 64 * 4
@@ -259,7 +275,7 @@ def run_ours(args, rank, world, local_rank):
     h = rt.Handle(rt.config_for(sh, max_prefix=inp.k_cache.shape[1]), w.w_emb)
     if args.w_layout == "packed":
         w = rt.pack_weights(h, w)  # one-time tiling of W_lm (model load)
-    ds = rt.DeviceStep(inp, w, attention=True)
+    ds = rt.DeviceStep(inp, w, attention=not full_sequence(sh))
     stream = torch.cuda.Stream()
     sid = stream.cuda_stream
     args_c = ds.args()
@@ -372,6 +388,8 @@ def run_ours(args, rank, world, local_rank):
                clocks=sampler.summary(), e2e=e2e, t_wall=t_wall,
                lbs_runs=args.state == "select")
     out["launches_per_step"] = 2 + (inp.rows + 511) // 512 + (1 if args.append else 0)
+    if full_sequence(sh):  # LM head groups, merge, memsets and the decision chain
+        out["launches_per_step"] = (inp.rows + 511) // 512 + 1 + (2 + 12 + 8 if args.state == "select" else 2 + 12)
     out["suffix"] = None if sfx is None else sfx
     out["fetch"] = ds.fetch()
     h_sms = torch.cuda.get_device_properties(local_rank).multi_processor_count
@@ -393,10 +411,14 @@ def run_e2e(args, h, ds, inp, sh, stream, world, sfx=None):
                    row_pos=pin(inp.row_pos.astype(np.int32)),
                    hidden=pin(inp.hidden.view(np.int16)), q=pin(inp.q.view(np.int16)),
                    k_win=pin(inp.k_win.view(np.int16)), v_win=pin(inp.v_win.view(np.int16)))
+    if ds.attn_out is None:  # no window attention: its inputs are not copied
+        for k in ("q", "k_win", "v_win"):
+            del host_in[k]
     st0 = dict(tokens=inp.tokens.astype(np.int32), mask=inp.mask.astype(np.uint8),
                in_block=inp.in_block.astype(np.uint8), blk_meta=inp.blk_meta.astype(np.int32))
     host_state = {k: pin(v) for k, v in st0.items()}
-    host_out = dict(attn_out=torch.empty((R, Hq, D), dtype=torch.float32).pin_memory())
+    host_out = dict(attn_out=torch.empty((R, Hq, D), dtype=torch.float32).pin_memory()) \
+        if ds.attn_out is not None else {}
     for k in ("conf", "entropy", "ent_norm", "gap", "lbs_logit", "lps_prob"):
         host_out[k] = torch.empty(R, dtype=torch.float32).pin_memory()
     host_out["argmax"] = torch.empty(R, dtype=torch.int32).pin_memory()
@@ -481,12 +503,16 @@ def run_loop_bench(args):
     inp = synth.make_step_inputs(sh)
     w = rt.upload_weights(inp)
     mode = {"eb": 0, "threshold": 1, "topm": 2}[args.decode]
-    h = rt.Handle(lp.config_for_loop(sh, decode_mode=mode, top_m=args.top_m), w.w_emb)
+    full = full_sequence(sh)
+    h = rt.Handle(lp.config_for_loop(sh, max_window=sh.gen_len if full else 64, decode_mode=mode,
+                                     top_m=args.top_m), w.w_emb)
     if args.w_layout == "packed":
         w = rt.pack_weights(h, w)
     win = lambda s, p: synth.loop_window_inputs(sh, s, p)
     kv = lambda p: synth.loop_kv(sh, p)
     opts = dict(keep=False, block=sh.l_b, cache=args.cache, append=args.append)
+    if full:
+        opts.update(window="full", attention=False)
     lp.run_loop(h, sh, w, win, kv, **opts)  # warm-up loop
     runs = []
     for _ in range(max(1, args.steps // 100)):
@@ -502,8 +528,11 @@ def run_loop_bench(args):
             "n_gpus": 1, "steps": len(runs), "warmup": 1, "ms_per_step": round(dev_us / steps / 1000, 5),
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
             "data": "synthetic (seeded per step and position)",
-            "config": {"workload": f"{sh.name}: prompt {sh.prefix}, gen {sh.gen_len}, windows of "
-                                   f"at most 64 rows, attention over the committed prefix",
+            "config": {"workload": (f"{sh.name}: prompt {sh.prefix}, gen {sh.gen_len}, every step's "
+                                    f"window is the whole response (full-sequence setting), no "
+                                    f"window attention") if full else
+                                   (f"{sh.name}: prompt {sh.prefix}, gen {sh.gen_len}, windows of "
+                                    f"at most 64 rows, attention over the committed prefix"),
                        "decode": args.decode + (f" (m={args.top_m})" if args.decode == "topm" else ""),
                        "fixed_block": sh.l_b if args.decode != "eb" else None,
                        "kv_cache": ("dual: the window also attends to the positions after it"

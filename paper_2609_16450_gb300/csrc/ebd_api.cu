@@ -863,7 +863,7 @@ ebd_status ebd_create(const ebd_config* cfg, ebd_handle** out) {
     };
     const size_t o_conf = add(R * 4), o_entn = add(R * 4), o_gap = add(R * 4), o_arg = add(R * 4);
     const size_t o_seq = add(R * 4), o_mr = add(R * 4), o_mrows = add(R * 4), o_bmr = add(R * 4),
-                 o_bmrows = add(R * 4), o_bad = add(R), o_ib = add(R), o_sq = add(B * 8 * 4),
+                 o_bmrows = add(R * 4), o_bad = add(R), o_ib = add(R), o_sq = add((B + 1) * 8 * 4),
                  o_O = add(R * 4), o_P = add(R * 4), o_f = add(R * 8 * 4), o_Z = add(R * 128 * 4),
                  o_QKV = add(R * 384 * 4), o_A = add(R * 128 * 4), o_Zp = add(R * 32 * 4),
                  o_QKVp = add(R * 96 * 4), o_Ap = add(R * 32 * 4);

@@ -143,7 +143,7 @@ struct SeqParams {
   int* bmrows;
   uint8_t* bad;
   uint8_t* ib;              // block membership after the selection
-  int* sq;                  // [B][8] per-sequence state (kSq* indices)
+  int* sq;                  // [B + 1][8] per-sequence state (kSq* indices), then step flags
   float* O;                 // LBS logit
   float* P;                 // LPS probability
   float* feats;             // [R][8]

@@ -9,17 +9,25 @@
 // which holds 64 rows.  Here every phase is a grid-wide kernel over the rows
 // of all sequences, with the activations in an L2-resident scratch:
 //   prep      masked set M of each sequence (compaction), LBS on/off
-//   embed     F_ent and the token branch, fusion + E_pos      (warp per row)
-//   2 layers  QKV; attention (warp per row and head); output projection,
-//             LayerNorm, FFN, LayerNorm (warp per row); LBS head
+//   embed     F_ent hidden and the token branch (warp per row); ent2 +
+//             LayerNorm, fusion + E_pos (GEMMs)
+//   2 layers  QKV (GEMM); attention (CTA per query block and head, keys
+//             staged in shared memory); output projection + LayerNorm, FF1 +
+//             GELU, FF2 + LayerNorm (GEMMs); LBS head
 //   select    candidates, MaxGapFilter, min-tokens fallback; B n M; LPS
 //             features                                        (CTA per sequence)
 //   LPS       input layer; 2 blocks as above (d 32, 4 heads); head, sigmoid
 //   accept    union accept, anti-stall, commit, block resolution
 // Products are fp32 FMAs on an fp32 copy of the (bf16-valued) weights stored
-// [in][out]: a warp holds a row's vector spread over its lanes (element
-// lane + 32 i in register i) and broadcasts one input at a time.
+// [in][out].  The LBS products are CTA-tiled GEMMs over all window rows (32
+// rows x 32*CPT columns per CTA, operands staged in shared memory) with the
+// bias, residual, LayerNorm, GELU or head fused into the epilogue: a warp
+// holds 4 whole rows of the tile.  Rows outside the LBS compute garbage in
+// their own scratch rows, which nothing reads.  The small LPS products run
+// one warp per row (a row's vector spread over the lanes, element lane + 32 i
+// in register i, one input broadcast at a time).
 #include <climits>
+#include <cstdlib>
 
 #include "internal.h"
 
@@ -32,6 +40,8 @@ constexpr int kWarpsPerCta = 8;
 // per-sequence state, sq[b * 8 + k]
 constexpr int kSqNM = 0, kSqRunLbs = 1, kSqNBM = 2, kSqMetaB = 3, kSqMetaS = 4, kSqRunLps = 5,
               kSqN = 6;
+// step-wide flags after the per-sequence state: sq[8 * B + kFlagAnyLbs]
+constexpr int kFlagAnyLbs = 0;
 
 __device__ __forceinline__ float gelu_f(float x) {
   return 0.5f * x * (1.0f + erff(x * 0.70710678118654752f));
@@ -39,11 +49,6 @@ __device__ __forceinline__ float gelu_f(float x) {
 __device__ __forceinline__ float wsum(float v) {
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-  return v;
-}
-__device__ __forceinline__ float wmax(float v) {
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
   return v;
 }
 
@@ -135,6 +140,7 @@ __global__ void __launch_bounds__(kSeqThreads) seq_prep_kernel(const SeqParams p
     const int meta_s = p.blk_meta[2 * b + 1];
     sq[kSqNM] = nM;
     sq[kSqRunLbs] = (p.mode == EBD_DECODE_EB && meta_s == 0 && nM > p.l_min) ? 1 : 0;
+    if (sq[kSqRunLbs]) atomicOr(p.sq + 8 * p.B + kFlagAnyLbs, 1);
     sq[kSqNBM] = 0;
     sq[kSqMetaB] = p.blk_meta[2 * b];
     sq[kSqMetaS] = meta_s;
@@ -155,134 +161,353 @@ __device__ __forceinline__ int lps_row(const SeqParams& p, int r) {
 }
 
 // ------------------------------------------------------------------ LBS
-// F_ent (Linear 1->64, GELU, Linear 64->64, LayerNorm) of H~, the token
-// branch W_tok W_e[x_hat] + b (folded table), fusion W_combine [e; t] + b +
-// E_pos[rank]  (Eq. lbs_feat)
-__global__ void __launch_bounds__(256) lbs_embed_kernel(const SeqParams p) {
+// Multi-head attention of NQ query rows and one head over the rows
+// `rows[0..n)`: softmax(q k^T / sqrt(DH)) v, qkv rows of stride LD with q at
+// qo, k at ko, v at vo; query i is row qrows[i] (-1: none).  G = DH / 4 lanes
+// share a key (4 dimensions each, one float4 of k and of v, loaded once for
+// the NQ queries), so 32 / G keys are in flight per warp, each lane group
+// with a running max and sum per query; the groups merge at the end.  Lanes
+// [0, G) return, per query, the output dimensions 4 * lane .. 4 * lane + 3.
+template <int DH, int NQ>
+__device__ __forceinline__ void attend_rows(const float* __restrict__ qkv, int LD, const int (&qrows)[NQ],
+                                            int qo, int ko, int vo, const int* __restrict__ rows,
+                                            int n, float4 (&out)[NQ]) {
+  constexpr int G = DH / 4, KP = 32 / G;
+  const int lane = threadIdx.x & 31, grp = lane / G, sub = lane % G;
+  const float scale = rsqrtf(static_cast<float>(DH));
+  float4 q[NQ], o[NQ];
+  float m[NQ], l[NQ];
+#pragma unroll
+  for (int i = 0; i < NQ; ++i) {
+    q[i] = qrows[i] >= 0 ? *reinterpret_cast<const float4*>(qkv + static_cast<size_t>(qrows[i]) * LD + qo + 4 * sub)
+                         : make_float4(0.f, 0.f, 0.f, 0.f);
+    o[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+    m[i] = -INFINITY;
+    l[i] = 0.f;
+  }
+#pragma unroll 4
+  for (int k0 = 0; k0 < n; k0 += KP) {
+    const int k = k0 + grp;
+    const bool ok = k < n;
+    const float* kr = qkv + static_cast<size_t>(__ldg(rows + (ok ? k : 0))) * LD;
+    const float4 kv = *reinterpret_cast<const float4*>(kr + ko + 4 * sub);
+    const float4 vv = *reinterpret_cast<const float4*>(kr + vo + 4 * sub);
+    float s[NQ];
+#pragma unroll
+    for (int i = 0; i < NQ; ++i) s[i] = q[i].x * kv.x + q[i].y * kv.y + q[i].z * kv.z + q[i].w * kv.w;
+#pragma unroll
+    for (int off = 1; off < G; off <<= 1)
+#pragma unroll
+      for (int i = 0; i < NQ; ++i) s[i] += __shfl_xor_sync(0xffffffffu, s[i], off);
+#pragma unroll
+    for (int i = 0; i < NQ; ++i) {
+      const float si = ok ? s[i] * scale : -INFINITY;
+      const float mn = fmaxf(m[i], si);
+      const float c = mn == -INFINITY ? 1.f : expf(m[i] - mn), e = mn == -INFINITY ? 0.f : expf(si - mn);
+      l[i] = l[i] * c + e;
+      o[i].x = fmaf(e, vv.x, o[i].x * c);
+      o[i].y = fmaf(e, vv.y, o[i].y * c);
+      o[i].z = fmaf(e, vv.z, o[i].z * c);
+      o[i].w = fmaf(e, vv.w, o[i].w * c);
+      m[i] = mn;
+    }
+  }
+#pragma unroll
+  for (int i = 0; i < NQ; ++i) {
+    float M = m[i];
+#pragma unroll
+    for (int off = G; off < 32; off <<= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
+    const float c = m[i] == -INFINITY ? 0.f : expf(m[i] - M);
+    float li = l[i] * c;
+    float4 oi = make_float4(o[i].x * c, o[i].y * c, o[i].z * c, o[i].w * c);
+#pragma unroll
+    for (int off = G; off < 32; off <<= 1) {
+      li += __shfl_xor_sync(0xffffffffu, li, off);
+      oi.x += __shfl_xor_sync(0xffffffffu, oi.x, off);
+      oi.y += __shfl_xor_sync(0xffffffffu, oi.y, off);
+      oi.z += __shfl_xor_sync(0xffffffffu, oi.z, off);
+      oi.w += __shfl_xor_sync(0xffffffffu, oi.w, off);
+    }
+    const float il = 1.0f / li;
+    out[i] = make_float4(oi.x * il, oi.y * il, oi.z * il, oi.w * il);
+  }
+}
+
+// Tiled fp32 GEMM over the window rows: CTA (blockIdx.x, blockIdx.y)
+// computes rows [8 bx, 8 bx + 8) x columns [32 CPT by, +32 CPT) of
+// A[R][lda] (first K columns) times W[K][ldw]; warp w owns row 8 bx + w,
+// lane l columns l + 32 j (j < CPT).  K is staged in chunks of kGemmK rows,
+// double-buffered: the next chunk's global loads are in flight while the
+// current one is multiplied.  epi(row, acc[CPT], col0) gets a warp's row
+// (rows >= R included: their A rows read as zero).
+constexpr int kGemmK = 32;  // k-chunk staged per step
+constexpr int kGemmRows = 8;
+template <int CPT, class Epi>
+__device__ __forceinline__ void gemm_rows(const float* __restrict__ A, int lda, int K,
+                                          const float* __restrict__ W, int ldw, int R, Epi epi) {
+  constexpr int NC = 32 * CPT;
+  constexpr int NB4 = kGemmK * NC / 4 / 256;  // float4 of a B chunk per thread
+  static_assert(NB4 * 256 * 4 == kGemmK * NC, "B chunk split");
+  static_assert(kGemmRows * kGemmK == 256, "one A element per thread");
+  __shared__ __align__(16) float As[2][kGemmRows][kGemmK];
+  __shared__ __align__(16) float Bs[2][kGemmK][NC];
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int row0 = blockIdx.x * kGemmRows, col0 = blockIdx.y * NC;
+  const int ar = tid / kGemmK, ak = tid % kGemmK;  // this thread's A element of a chunk
+  const bool arow = row0 + ar < R;
+  float acc[CPT];
+#pragma unroll
+  for (int j = 0; j < CPT; ++j) acc[j] = 0.f;
+  float ra;
+  float4 rb[NB4];
+  auto load = [&](int k0) {
+    ra = arow ? A[static_cast<size_t>(row0 + ar) * lda + k0 + ak] : 0.f;
+#pragma unroll
+    for (int u = 0; u < NB4; ++u) {
+      const int it = tid + 256 * u, kk = it / (NC / 4), c4 = it % (NC / 4);
+      rb[u] = __ldg(reinterpret_cast<const float4*>(W + static_cast<size_t>(k0 + kk) * ldw + col0 + 4 * c4));
+    }
+  };
+  auto store = [&](int buf) {
+    As[buf][ar][ak] = ra;
+#pragma unroll
+    for (int u = 0; u < NB4; ++u) {
+      const int it = tid + 256 * u, kk = it / (NC / 4), c4 = it % (NC / 4);
+      *reinterpret_cast<float4*>(&Bs[buf][kk][4 * c4]) = rb[u];
+    }
+  };
+  load(0);
+  store(0);
+  __syncthreads();
+  const int nch = K / kGemmK;
+  for (int c = 0; c < nch; ++c) {
+    const int buf = c & 1;
+    if (c + 1 < nch) load((c + 1) * kGemmK);
+#pragma unroll 8
+    for (int kk = 0; kk < kGemmK; ++kk) {
+      const float a = As[buf][warp][kk];
+#pragma unroll
+      for (int j = 0; j < CPT; ++j) acc[j] = fmaf(a, Bs[buf][kk][lane + 32 * j], acc[j]);
+    }
+    if (c + 1 < nch) store(buf ^ 1);
+    __syncthreads();
+  }
+  epi(row0 + warp, acc, col0);
+}
+
+__device__ __forceinline__ bool any_lbs(const SeqParams& p) {
+  return p.sq[8 * p.B + kFlagAnyLbs] != 0;
+}
+
+// F_ent hidden (Linear 1 -> 64, GELU) of H~ -> U[r][0..64), and the token
+// branch W_tok W_e[x_hat] + b (folded table) -> X[r][64..128)  (Eq. lbs_feat)
+__global__ void __launch_bounds__(256) lbs_pre_kernel(const SeqParams p) {
   const int lane = threadIdx.x & 31;
   const int r = lbs_row(p, blockIdx.x * kWarpsPerCta + (threadIdx.x >> 5));
   if (r < 0) return;
   const float* w = p.w;
   const float h = p.ent_norm[r];
-  float u[2], e[2];
-#pragma unroll
-  for (int i = 0; i < 2; ++i)
-    u[i] = gelu_f(fmaf(w[p.o.ent1_w + lane + 32 * i], h, w[p.o.ent1_b + lane + 32 * i]));
-  matvec<2, 2>(u, w + p.o.ent2_t, w + p.o.ent2_b, e);
-  layer_norm_w<2>(e, w + p.o.entln_g, w + p.o.entln_b);
   const int tok = p.argmax[r];
-  float x[4] = {e[0], e[1], 0.f, 0.f};
 #pragma unroll
-  for (int i = 0; i < 2; ++i)
-    x[2 + i] = (tok >= 0 && tok < p.V ? __ldg(p.tok_table + static_cast<size_t>(tok) * 64 + lane + 32 * i) : 0.f) +
-               w[p.o.tok_b + lane + 32 * i];
-  float z[4];
-  matvec<4, 4>(x, w + p.o.comb_t, w + p.o.comb_b, z);
-  const float* pos = w + p.o.pos + static_cast<size_t>(p.mrank[r]) * 128;
+  for (int i = 0; i < 2; ++i) {
+    const int c = lane + 32 * i;
+    p.A[static_cast<size_t>(r) * 128 + c] = gelu_f(fmaf(w[p.o.ent1_w + c], h, w[p.o.ent1_b + c]));
+    p.Z[static_cast<size_t>(r) * 128 + 64 + c] =
+        (tok >= 0 && tok < p.V ? __ldg(p.tok_table + static_cast<size_t>(tok) * 64 + c) : 0.f) +
+        w[p.o.tok_b + c];
+  }
+}
+
+// e = LN(W_ent2 u + b) -> X[r][0..64)  (X lives in Z; U in A)
+__global__ void __launch_bounds__(256) lbs_ent2_kernel(const SeqParams p) {
+  if (!any_lbs(p)) return;
+  const float* w = p.w;
+  gemm_rows<2>(p.A, 128, 64, w + p.o.ent2_t, 64, p.R, [&](int r, float (&acc)[2], int) {
+    const int lane = threadIdx.x & 31;
 #pragma unroll
-  for (int i = 0; i < 4; ++i) p.Z[static_cast<size_t>(r) * 128 + lane + 32 * i] = z[i] + pos[lane + 32 * i];
+    for (int j = 0; j < 2; ++j) acc[j] += w[p.o.ent2_b + lane + 32 * j];
+    layer_norm_w<2>(acc, w + p.o.entln_g, w + p.o.entln_b);
+    if (r < p.R)
+#pragma unroll
+      for (int j = 0; j < 2; ++j) p.Z[static_cast<size_t>(r) * 128 + lane + 32 * j] = acc[j];
+  });
+}
+
+// z = W_combine [e; t] + b + E_pos[rank], in place in Z: a CTA owns all 128
+// columns of its rows and has read them before its epilogue
+__global__ void __launch_bounds__(256) lbs_comb_kernel(const SeqParams p) {
+  if (!any_lbs(p)) return;
+  const float* w = p.w;
+  gemm_rows<4>(p.Z, 128, 128, w + p.o.comb_t, 128, p.R, [&](int r, float (&acc)[4], int) {
+    const int lane = threadIdx.x & 31;
+    if (r >= p.R) return;
+    const int k = p.mrank[r];
+    const float* pos = w + p.o.pos + static_cast<size_t>(k < 0 ? 0 : k) * 128;
+#pragma unroll
+    for (int j = 0; j < 4; ++j)
+      p.Z[static_cast<size_t>(r) * 128 + lane + 32 * j] =
+          acc[j] + w[p.o.comb_b + lane + 32 * j] + pos[lane + 32 * j];
+  });
 }
 
 __global__ void __launch_bounds__(256) lbs_qkv_kernel(const SeqParams p, int l) {
-  const int lane = threadIdx.x & 31;
-  const int r = lbs_row(p, blockIdx.x * kWarpsPerCta + (threadIdx.x >> 5));
-  if (r < 0) return;
+  if (!any_lbs(p)) return;
   const SeqLayer& L = p.o.l[l];
-  float z[4], y[12];
-#pragma unroll
-  for (int i = 0; i < 4; ++i) z[i] = p.Z[static_cast<size_t>(r) * 128 + lane + 32 * i];
-  matvec<4, 12>(z, p.w + L.qkv_t, p.w + L.qkv_b, y);
-#pragma unroll
-  for (int i = 0; i < 12; ++i) p.QKV[static_cast<size_t>(r) * 384 + lane + 32 * i] = y[i];
+  const float* bq = p.w + L.qkv_b;
+  gemm_rows<1>(p.Z, 128, 128, p.w + L.qkv_t, 384, p.R, [&](int r, float (&acc)[1], int col0) {
+    const int lane = threadIdx.x & 31;
+    if (r < p.R) p.QKV[static_cast<size_t>(r) * 384 + col0 + lane] = acc[0] + bq[col0 + lane];
+  });
 }
 
-// softmax(q k^T / sqrt(DH)) v of one row and one head over the rows of
-// `rows[0..n)`; qkv rows of stride LD with q at qo, k at ko, v at vo.  The
-// lanes split the keys (running max and sum each), then merge.  Returns the
-// output element `lane` (lanes >= DH return 0).
-template <int DH>
-__device__ __forceinline__ float attend_row(const float* __restrict__ qkv, int LD, int r, int qo,
-                                            int ko, int vo, const int* __restrict__ rows, int n) {
-  const int lane = threadIdx.x & 31;
-  float q[DH], o[DH];
-  const float* qp = qkv + static_cast<size_t>(r) * LD + qo;
-#pragma unroll
-  for (int d = 0; d < DH; ++d) {
-    q[d] = qp[d];
-    o[d] = 0.f;
-  }
-  const float scale = rsqrtf(static_cast<float>(DH));
-  float m = -INFINITY, l = 0.f;
-  for (int k = lane; k < n; k += 32) {
-    const float* kr = qkv + static_cast<size_t>(rows[k]) * LD;
-    float s = 0.f;
-#pragma unroll
-    for (int d = 0; d < DH; ++d) s = fmaf(q[d], kr[ko + d], s);
-    s *= scale;
-    const float mn = fmaxf(m, s);
-    const float c = expf(m - mn), e = expf(s - mn);
-    l = l * c + e;
-#pragma unroll
-    for (int d = 0; d < DH; ++d) o[d] = fmaf(e, kr[vo + d], o[d] * c);
-    m = mn;
-  }
-  const float M = wmax(m);
-  const float c = m == -INFINITY ? 0.f : expf(m - M);
-  const float L = wsum(l * c);
-  float mine = 0.f;
-#pragma unroll
-  for (int d = 0; d < DH; ++d) {
-    const float t = wsum(o[d] * c);
-    if (d == lane) mine = t;
-  }
-  return mine / L;
-}
-
+// LBS attention: CTA (x, h, b) takes 8 NQ queries of sequence b's M
+// (rank 8 NQ x + NQ w + i for warp w, i < NQ) and head h.  Blocks of 64
+// keys (k and v of head h) are staged in shared memory once for the 8
+// warps; 8 lanes share a key (4 dimensions each), 4 keys per step, with a
+// running max and sum per (query, lane group), merged at the end.
+constexpr int kAttnKB = 64;
+template <int NQ>
 __global__ void __launch_bounds__(256) lbs_attn_kernel(const SeqParams p) {
-  const int lane = threadIdx.x & 31;
-  const int wid = blockIdx.x * kWarpsPerCta + (threadIdx.x >> 5);
-  const int r = lbs_row(p, wid >> 2), h = wid & 3;
-  if (r < 0) return;
-  const int b = p.seq_of[r];
-  const float v = attend_row<32>(p.QKV, 384, r, 32 * h, 128 + 32 * h, 256 + 32 * h,
-                                 p.mrows + p.cu_rows[b], p.sq[8 * b + kSqNM]);
-  p.A[static_cast<size_t>(r) * 128 + 32 * h + lane] = v;
+  constexpr int kAttnQB = 8 * NQ;
+  __shared__ __align__(16) float Ks[kAttnKB][32];
+  __shared__ __align__(16) float Vs[kAttnKB][32];
+  const int b = blockIdx.z, h = blockIdx.y, qb = blockIdx.x;
+  const int* sq = p.sq + 8 * b;
+  const int nM = sq[kSqNM];
+  if (!sq[kSqRunLbs] || qb * kAttnQB >= nM) return;  // uniform over the CTA
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31, grp = lane >> 3, sub = lane & 7;
+  const int* rows = p.mrows + p.cu_rows[b];
+  int qr[NQ];
+  float4 q[NQ], o[NQ];
+  float m[NQ], l[NQ];
+#pragma unroll
+  for (int i = 0; i < NQ; ++i) {
+    const int qi = qb * kAttnQB + warp * NQ + i;
+    qr[i] = qi < nM ? rows[qi] : -1;
+    q[i] = qr[i] >= 0 ? *reinterpret_cast<const float4*>(p.QKV + static_cast<size_t>(qr[i]) * 384 + 32 * h + 4 * sub)
+                      : make_float4(0.f, 0.f, 0.f, 0.f);
+    o[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+    m[i] = -INFINITY;
+    l[i] = 0.f;
+  }
+  const float scale = rsqrtf(32.0f);
+  for (int kb = 0; kb < nM; kb += kAttnKB) {
+    __syncthreads();
+    for (int it = tid; it < kAttnKB * 16; it += 256) {
+      const int key = it >> 4, part = it & 15, c4 = part & 7;
+      const int kidx = kb + key;
+      float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (kidx < nM)
+        v = *reinterpret_cast<const float4*>(p.QKV + static_cast<size_t>(rows[kidx]) * 384 +
+                                             (part < 8 ? 128 : 256) + 32 * h + 4 * c4);
+      *reinterpret_cast<float4*>(part < 8 ? &Ks[key][4 * c4] : &Vs[key][4 * c4]) = v;
+    }
+    __syncthreads();
+    const int nk = min(kAttnKB, nM - kb);
+    for (int k0 = 0; k0 < nk; k0 += 4) {
+      const int k = k0 + grp;
+      const bool ok = k < nk;
+      const float4 kv = *reinterpret_cast<const float4*>(&Ks[k][4 * sub]);
+      const float4 vv = *reinterpret_cast<const float4*>(&Vs[k][4 * sub]);
+      float s[NQ];
+#pragma unroll
+      for (int i = 0; i < NQ; ++i) s[i] = q[i].x * kv.x + q[i].y * kv.y + q[i].z * kv.z + q[i].w * kv.w;
+#pragma unroll
+      for (int off = 1; off < 8; off <<= 1)
+#pragma unroll
+        for (int i = 0; i < NQ; ++i) s[i] += __shfl_xor_sync(0xffffffffu, s[i], off);
+#pragma unroll
+      for (int i = 0; i < NQ; ++i) {
+        const float si = ok ? s[i] * scale : -INFINITY;
+        const float mn = fmaxf(m[i], si);
+        const float c = mn == -INFINITY ? 1.f : expf(m[i] - mn), e = mn == -INFINITY ? 0.f : expf(si - mn);
+        l[i] = l[i] * c + e;
+        o[i].x = fmaf(e, vv.x, o[i].x * c);
+        o[i].y = fmaf(e, vv.y, o[i].y * c);
+        o[i].z = fmaf(e, vv.z, o[i].z * c);
+        o[i].w = fmaf(e, vv.w, o[i].w * c);
+        m[i] = mn;
+      }
+    }
+  }
+#pragma unroll
+  for (int i = 0; i < NQ; ++i) {
+    float M = m[i];
+#pragma unroll
+    for (int off = 8; off < 32; off <<= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
+    const float c = m[i] == -INFINITY ? 0.f : expf(m[i] - M);
+    float li = l[i] * c;
+    float4 oi = make_float4(o[i].x * c, o[i].y * c, o[i].z * c, o[i].w * c);
+#pragma unroll
+    for (int off = 8; off < 32; off <<= 1) {
+      li += __shfl_xor_sync(0xffffffffu, li, off);
+      oi.x += __shfl_xor_sync(0xffffffffu, oi.x, off);
+      oi.y += __shfl_xor_sync(0xffffffffu, oi.y, off);
+      oi.z += __shfl_xor_sync(0xffffffffu, oi.z, off);
+      oi.w += __shfl_xor_sync(0xffffffffu, oi.w, off);
+    }
+    if (lane < 8 && qr[i] >= 0) {
+      const float il = 1.0f / li;
+      *reinterpret_cast<float4*>(p.A + static_cast<size_t>(qr[i]) * 128 + 32 * h + 4 * lane) =
+          make_float4(oi.x * il, oi.y * il, oi.z * il, oi.w * il);
+    }
+  }
 }
 
-// output projection + residual + LN1, FFN + residual + LN2 (post-norm
-// layer); after the last layer, the LBS head O = w . z + b
-__global__ void __launch_bounds__(256) lbs_out_ffn_kernel(const SeqParams p, int l) {
-  const int lane = threadIdx.x & 31;
-  const int r = lbs_row(p, blockIdx.x * kWarpsPerCta + (threadIdx.x >> 5));
-  if (r < 0) return;
+// z = LN1(z + W_out a + b), in place (post-norm layer)
+__global__ void __launch_bounds__(256) lbs_out_kernel(const SeqParams p, int l) {
+  if (!any_lbs(p)) return;
   const SeqLayer& L = p.o.l[l];
   const float* w = p.w;
-  float a[4], z[4], y[4], hdn[8], f[4];
+  gemm_rows<4>(p.A, 128, 128, w + L.out_t, 128, p.R, [&](int r, float (&acc)[4], int) {
+    const int lane = threadIdx.x & 31;
+    const int rr = r < p.R ? r : 0;
 #pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    a[i] = p.A[static_cast<size_t>(r) * 128 + lane + 32 * i];
-    z[i] = p.Z[static_cast<size_t>(r) * 128 + lane + 32 * i];
-  }
-  matvec<4, 4>(a, w + L.out_t, w + L.out_b, y);
+    for (int j = 0; j < 4; ++j)
+      acc[j] += w[L.out_b + lane + 32 * j] + p.Z[static_cast<size_t>(rr) * 128 + lane + 32 * j];
+    layer_norm_w<4>(acc, w + L.ln1_g, w + L.ln1_b);
+    if (r < p.R)
 #pragma unroll
-  for (int i = 0; i < 4; ++i) z[i] += y[i];
-  layer_norm_w<4>(z, w + L.ln1_g, w + L.ln1_b);
-  matvec<4, 8>(z, w + L.ff1_t, w + L.ff1_b, hdn);
+      for (int j = 0; j < 4; ++j) p.Z[static_cast<size_t>(r) * 128 + lane + 32 * j] = acc[j];
+  });
+}
+
+// h = GELU(W_1 z + b_1) -> the QKV scratch (256 of its 384 columns)
+__global__ void __launch_bounds__(256) lbs_ff1_kernel(const SeqParams p, int l) {
+  if (!any_lbs(p)) return;
+  const SeqLayer& L = p.o.l[l];
+  const float* b1 = p.w + L.ff1_b;
+  gemm_rows<1>(p.Z, 128, 128, p.w + L.ff1_t, 256, p.R, [&](int r, float (&acc)[1], int col0) {
+    const int lane = threadIdx.x & 31;
+    if (r < p.R) p.QKV[static_cast<size_t>(r) * 384 + col0 + lane] = gelu_f(acc[0] + b1[col0 + lane]);
+  });
+}
+
+// z = LN2(z + W_2 h + b_2), in place; after the last layer the LBS head
+// O = w . z + b
+__global__ void __launch_bounds__(256) lbs_ff2_kernel(const SeqParams p, int l) {
+  if (!any_lbs(p)) return;
+  const SeqLayer& L = p.o.l[l];
+  const float* w = p.w;
+  gemm_rows<4>(p.QKV, 384, 256, w + L.ff2_t, 128, p.R, [&](int r, float (&acc)[4], int) {
+    const int lane = threadIdx.x & 31;
+    const int rr = r < p.R ? r : 0;
 #pragma unroll
-  for (int i = 0; i < 8; ++i) hdn[i] = gelu_f(hdn[i]);
-  matvec<8, 4>(hdn, w + L.ff2_t, w + L.ff2_b, f);
-#pragma unroll
-  for (int i = 0; i < 4; ++i) z[i] += f[i];
-  layer_norm_w<4>(z, w + L.ln2_g, w + L.ln2_b);
-#pragma unroll
-  for (int i = 0; i < 4; ++i) p.Z[static_cast<size_t>(r) * 128 + lane + 32 * i] = z[i];
-  if (l == 1) {
+    for (int j = 0; j < 4; ++j)
+      acc[j] += w[L.ff2_b + lane + 32 * j] + p.Z[static_cast<size_t>(rr) * 128 + lane + 32 * j];
+    layer_norm_w<4>(acc, w + L.ln2_g, w + L.ln2_b);
+    if (r >= p.R) return;
     float s = 0.f;
 #pragma unroll
-    for (int i = 0; i < 4; ++i) s = fmaf(z[i], w[p.o.head_w + lane + 32 * i], s);
-    s = wsum(s) + w[p.o.head_b];
-    if (lane == 0) p.O[r] = s;
-  }
+    for (int j = 0; j < 4; ++j) {
+      p.Z[static_cast<size_t>(r) * 128 + lane + 32 * j] = acc[j];
+      s = fmaf(acc[j], w[p.o.head_w + lane + 32 * j], s);
+    }
+    if (l == 1) {
+      s = wsum(s) + w[p.o.head_b];
+      if (lane == 0 && lbs_row(p, r) >= 0) p.O[r] = s;
+    }
+  });
 }
 
 // ------------------------------------------------------------------ selection
@@ -395,9 +620,11 @@ __global__ void __launch_bounds__(256) lps_attn_kernel(const SeqParams p) {
   const int r = lps_row(p, wid >> 2), h = wid & 3;
   if (r < 0) return;
   const int b = p.seq_of[r];
-  const float v = attend_row<8>(p.QKVp, 96, r, 8 * h, 32 + 8 * h, 64 + 8 * h,
-                                p.bmrows + p.cu_rows[b], p.sq[8 * b + kSqNBM]);
-  if (lane < 8) p.Ap[static_cast<size_t>(r) * 32 + 8 * h + lane] = v;
+  const int q[1] = {r};
+  float4 v[1];
+  attend_rows<8, 1>(p.QKVp, 96, q, 8 * h, 32 + 8 * h, 64 + 8 * h, p.bmrows + p.cu_rows[b],
+                    p.sq[8 * b + kSqNBM], v);
+  if (lane < 2) *reinterpret_cast<float4*>(p.Ap + static_cast<size_t>(r) * 32 + 8 * h + 4 * lane) = v[0];
 }
 
 // output projection + residual, LN2, FFN + residual; after the last block
@@ -506,15 +733,32 @@ cudaError_t launch_decide_seq(const SeqParams& p, cudaStream_t st) {
   cudaError_t e;
   if ((e = cudaMemsetAsync(p.mrank, 0xff, static_cast<size_t>(p.R) * sizeof(int), st)) != cudaSuccess) return e;
   if ((e = cudaMemsetAsync(p.bmrank, 0xff, static_cast<size_t>(p.R) * sizeof(int), st)) != cudaSuccess) return e;
+  if ((e = cudaMemsetAsync(p.sq + 8 * p.B, 0, 8 * sizeof(int), st)) != cudaSuccess) return e;
   const unsigned rows_grid = static_cast<unsigned>((p.R + kWarpsPerCta - 1) / kWarpsPerCta);
   const unsigned head_grid = static_cast<unsigned>((4 * p.R + kWarpsPerCta - 1) / kWarpsPerCta);
   seq_prep_kernel<<<p.B, kSeqThreads, 0, st>>>(p);
   if (p.mode == EBD_DECODE_EB) {
-    lbs_embed_kernel<<<rows_grid, 256, 0, st>>>(p);
+    const unsigned tiles = static_cast<unsigned>((p.R + kGemmRows - 1) / kGemmRows);
+    // queries per warp; measured at 512 rows (384 masked): 1 -> 656 us per
+    // step, 2 -> 664, 4 -> 693 (more CTAs beat more reuse of a staged block)
+    int nq = 1;
+    if (const char* env = getenv("EBD_SEQ_ATTN_NQ")) nq = atoi(env);
+    nq = nq == 2 || nq == 4 ? nq : 1;
+    const dim3 attn_grid(kMaxSeqRows / (8 * nq), 4, static_cast<unsigned>(p.B));
+    lbs_pre_kernel<<<rows_grid, 256, 0, st>>>(p);
+    lbs_ent2_kernel<<<dim3(tiles, 1), 256, 0, st>>>(p);
+    lbs_comb_kernel<<<dim3(tiles, 1), 256, 0, st>>>(p);
     for (int l = 0; l < 2; ++l) {
-      lbs_qkv_kernel<<<rows_grid, 256, 0, st>>>(p, l);
-      lbs_attn_kernel<<<head_grid, 256, 0, st>>>(p);
-      lbs_out_ffn_kernel<<<rows_grid, 256, 0, st>>>(p, l);
+      lbs_qkv_kernel<<<dim3(tiles, 12), 256, 0, st>>>(p, l);
+      if (nq == 1)
+        lbs_attn_kernel<1><<<attn_grid, 256, 0, st>>>(p);
+      else if (nq == 4)
+        lbs_attn_kernel<4><<<attn_grid, 256, 0, st>>>(p);
+      else
+        lbs_attn_kernel<2><<<attn_grid, 256, 0, st>>>(p);
+      lbs_out_kernel<<<dim3(tiles, 1), 256, 0, st>>>(p, l);
+      lbs_ff1_kernel<<<dim3(tiles, 8), 256, 0, st>>>(p, l);
+      lbs_ff2_kernel<<<dim3(tiles, 1), 256, 0, st>>>(p, l);
     }
   }
   seq_select_kernel<<<p.B, kSeqThreads, 0, st>>>(p);
