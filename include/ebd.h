@@ -37,9 +37,15 @@
  *     by ebd_sync_status().
  *   - Supported shapes: d_model % 8 == 0, d_base % 8 == 0, head_dim in
  *     {64, 128}, n_heads_q % n_heads_kv == 0, 1 <= window rows of a
- *     sequence <= max_window <= 64, gen_len >= max_window, vocab >= 2,
+ *     sequence <= max_window <= 512, gen_len >= max_window, vocab >= 2,
  *     rows of a step <= max_rows <= 4096.  Anything else returns
  *     EBD_ERR_UNSUPPORTED.
+ *   - max_window <= 64: the decision runs as one thread-block cluster per
+ *     sequence.  max_window > 64 (the full-sequence setting, where every
+ *     position of the response is a row, App. E with M = all masked
+ *     positions): the decision runs as a chain of grid-wide kernels, and a
+ *     step takes no window attention (attn_out and kv_append must be unset:
+ *     EBD_ERR_UNSUPPORTED otherwise).
  *   - stream arguments are cudaStream_t values passed as void* (NULL = the
  *     legacy default stream).
  */
@@ -91,7 +97,8 @@ typedef struct {
   int32_t d_base;      /* width of the frozen token embedding W_e           */
   /* capacity of the handle */
   int32_t max_batch;   /* sequences per step                                */
-  int32_t max_window;  /* window rows per sequence (<= 64)                  */
+  int32_t max_window;  /* window rows per sequence (<= 512; > 64: the
+                          full-sequence setting, see above)                 */
   int32_t max_rows;    /* window rows per step, all sequences (<= 4096)     */
   int32_t max_prefix;  /* P_max: second dimension of the K/V cache          */
   /* EB hyper-parameters (App. F) */
