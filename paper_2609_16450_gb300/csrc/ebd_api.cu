@@ -1150,6 +1150,83 @@ ebd_status ebd_attention(ebd_handle* h, const ebd_step_args* a, void* stream) {
   return run_attention(h, a, static_cast<cudaStream_t>(stream));
 }
 
+namespace {
+// ebd_step_host moves its inputs in and its results out with one kernel
+// each way where the host buffers are pinned and mapped into the device's
+// address space (cudaHostAlloc / cudaHostRegister memory): one launch
+// instead of a dozen small copies.  Other host buffers are copied with
+// cudaMemcpyAsync.
+struct CopyItem {
+  const uint8_t* src;
+  uint8_t* dst;
+  uint32_t bytes;
+};
+constexpr int kMaxCopyItems = 16;
+struct CopyList {
+  CopyItem it[kMaxCopyItems];
+  int n;
+};
+
+__global__ void __launch_bounds__(256) copy_list_kernel(const CopyList cl) {
+  const int i = blockIdx.y;
+  if (i >= cl.n) return;
+  const CopyItem c = cl.it[i];
+  const size_t stride = static_cast<size_t>(gridDim.x) * blockDim.x;
+  const size_t t0 = static_cast<size_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+  const bool vec = ((reinterpret_cast<uintptr_t>(c.src) | reinterpret_cast<uintptr_t>(c.dst) | c.bytes) & 15u) == 0;
+  if (vec) {
+    const size_t n = c.bytes / 16;
+    for (size_t k = t0; k < n; k += stride)
+      reinterpret_cast<uint4*>(c.dst)[k] = reinterpret_cast<const uint4*>(c.src)[k];
+  } else {
+    for (size_t k = t0; k < c.bytes; k += stride) c.dst[k] = c.src[k];
+  }
+}
+
+// the device address of a pinned, mapped host buffer, else null
+const void* mapped_host(const void* host) {
+  if (host == nullptr) return nullptr;
+  cudaPointerAttributes at{};
+  if (cudaPointerGetAttributes(&at, host) != cudaSuccess) {
+    (void)cudaGetLastError();
+    return nullptr;
+  }
+  return at.type == cudaMemoryTypeHost ? at.devicePointer : nullptr;
+}
+
+// copies (dst, src, bytes): mapped host buffers go to one copy_list_kernel,
+// the others to cudaMemcpyAsync
+struct HostMover {
+  cudaStream_t st;
+  bool to_device;
+  CopyList list{};
+  cudaError_t err = cudaSuccess;
+  void add(void* dst, const void* src, size_t bytes) {
+    if (bytes == 0 || dst == nullptr || src == nullptr || err != cudaSuccess) return;
+    const void* host = to_device ? src : dst;
+    const void* dev = mapped_host(host);
+    if (dev != nullptr && list.n < kMaxCopyItems && bytes < (1ull << 31)) {
+      CopyItem& c = list.it[list.n++];
+      c.src = static_cast<const uint8_t*>(to_device ? dev : src);
+      c.dst = static_cast<uint8_t*>(to_device ? dst : const_cast<void*>(dev));
+      c.bytes = static_cast<uint32_t>(bytes);
+      return;
+    }
+    err = cudaMemcpyAsync(dst, src, bytes, to_device ? cudaMemcpyHostToDevice : cudaMemcpyDeviceToHost, st);
+  }
+  cudaError_t flush() {
+    if (err != cudaSuccess || list.n == 0) return err;
+    uint32_t most = 0;
+    for (int i = 0; i < list.n; ++i) most = list.it[i].bytes > most ? list.it[i].bytes : most;
+    unsigned bx = (most + 16 * 256 - 1) / (16 * 256);
+    bx = bx < 1 ? 1 : (bx > 64 ? 64 : bx);
+    copy_list_kernel<<<dim3(bx, static_cast<unsigned>(list.n)), 256, 0, st>>>(list);
+    list.n = 0;
+    return cudaGetLastError();
+  }
+};
+}  // namespace
+
 ebd_status ebd_step_host(ebd_handle* h, const ebd_step_args* a, void* stream) {
   if (h == nullptr) return EBD_ERR_INVALID_ARG;
   ebd_status s = check_device(h);
@@ -1188,34 +1265,24 @@ ebd_status ebd_step_host(ebd_handle* h, const ebd_step_args* a, void* stream) {
   int32_t* am = reinterpret_cast<int32_t*>(take(RM * 4));
   uint8_t* acc = take(RM);
   int32_t* sfx = reinterpret_cast<int32_t*>(take(BM * 8));
-  auto h2d = [&](void* dst, const void* src, size_t n) {
-    return n == 0 || src == nullptr ? cudaSuccess
-                                    : cudaMemcpyAsync(dst, src, n, cudaMemcpyHostToDevice, st);
-  };
-  auto d2h = [&](void* dst, const void* src, size_t n) {
-    return n == 0 || dst == nullptr ? cudaSuccess
-                                    : cudaMemcpyAsync(dst, src, n, cudaMemcpyDeviceToHost, st);
-  };
-  cudaError_t e = cudaSuccess;
   const bool attn = a->attn_out != nullptr;
-  auto chk = [&](cudaError_t x) {
-    if (e == cudaSuccess) e = x;
-  };
-  chk(h2d(cu, a->cu_rows, (B + 1) * 4));
-  chk(h2d(pl, a->prefix_len, B * 4));
-  chk(h2d(rp, a->row_pos, R * 4));
-  chk(h2d(hid, a->hidden, R * d * 2));
+  HostMover in{st, true};
+  in.add(cu, a->cu_rows, (B + 1) * 4);
+  in.add(pl, a->prefix_len, B * 4);
+  in.add(rp, a->row_pos, R * 4);
+  in.add(hid, a->hidden, R * d * 2);
   const bool kv = attn || a->kv_append;  // the window K/V feed the attention and the append
-  if (attn) chk(h2d(q, a->q, R * Hq * D * 2));
+  if (attn) in.add(q, a->q, R * Hq * D * 2);
   if (kv) {
-    chk(h2d(kw, a->k_win, R * Hkv * D * 2));
-    chk(h2d(vw, a->v_win, R * Hkv * D * 2));
+    in.add(kw, a->k_win, R * Hkv * D * 2);
+    in.add(vw, a->v_win, R * Hkv * D * 2);
   }
-  chk(h2d(tok, a->tokens, R * 4));
-  chk(h2d(msk, a->mask, R));
-  chk(h2d(ib, a->in_block, R));
-  chk(h2d(meta, a->blk_meta, B * 8));
-  if (a->suffix) chk(h2d(sfx, a->suffix, B * 8));
+  in.add(tok, a->tokens, R * 4);
+  in.add(msk, a->mask, R);
+  in.add(ib, a->in_block, R);
+  in.add(meta, a->blk_meta, B * 8);
+  if (a->suffix) in.add(sfx, a->suffix, B * 8);
+  cudaError_t e = in.flush();
   if (e != cudaSuccess) return cuda_fail(h, e, "host-to-device copy");
   g.cu_rows = cu; g.prefix_len = pl; g.row_pos = rp; g.hidden = hid;
   g.q = attn ? q : nullptr; g.k_win = kv ? kw : nullptr; g.v_win = kv ? vw : nullptr;
@@ -1231,20 +1298,21 @@ ebd_status ebd_step_host(ebd_handle* h, const ebd_step_args* a, void* stream) {
   g.argmax = a->argmax ? am : nullptr;
   g.accepted = a->accepted ? acc : nullptr;
   if ((s = ebd_step(h, &g, stream)) != EBD_OK) return s;
-  chk(d2h(a->tokens, tok, R * 4));
-  chk(d2h(a->mask, msk, R));
-  chk(d2h(a->in_block, ib, R));
-  chk(d2h(a->blk_meta, meta, B * 8));
-  if (attn) chk(d2h(a->attn_out, ao, R * Hq * D * 4));
-  chk(d2h(a->conf, f[0], R * 4));
-  chk(d2h(a->entropy, f[1], R * 4));
-  chk(d2h(a->ent_norm, f[2], R * 4));
-  chk(d2h(a->gap, f[3], R * 4));
-  chk(d2h(a->lbs_logit, f[4], R * 4));
-  chk(d2h(a->lps_prob, f[5], R * 4));
-  chk(d2h(a->argmax, am, R * 4));
-  chk(d2h(a->accepted, acc, R));
-  if (e != cudaSuccess) return cuda_fail(h, e, "device-to-host copy");
+  HostMover out{st, false};
+  out.add(a->tokens, tok, R * 4);
+  out.add(a->mask, msk, R);
+  out.add(a->in_block, ib, R);
+  out.add(a->blk_meta, meta, B * 8);
+  if (attn) out.add(a->attn_out, ao, R * Hq * D * 4);
+  out.add(a->conf, f[0], R * 4);
+  out.add(a->entropy, f[1], R * 4);
+  out.add(a->ent_norm, f[2], R * 4);
+  out.add(a->gap, f[3], R * 4);
+  out.add(a->lbs_logit, f[4], R * 4);
+  out.add(a->lps_prob, f[5], R * 4);
+  out.add(a->argmax, am, R * 4);
+  out.add(a->accepted, acc, R);
+  if ((e = out.flush()) != cudaSuccess) return cuda_fail(h, e, "device-to-host copy");
   return EBD_OK;
 }
 

@@ -117,6 +117,43 @@ def test_host_step_matches_device_step():
         np.testing.assert_array_equal(st[k], dev[k], err_msg=k)
 
 
+def test_host_step_pinned_matches_device_step():
+    """The same with pinned (device-mapped) host buffers, which ebd_step_host
+    moves with one kernel each way instead of copies."""
+    from paper_2609_16450_gb300 import _ebd as E
+    from paper_2609_16450_gb300 import runtime as rt
+    sh = synth.tiny
+    inp, w, h = _setup(sh)
+    dev = _run(sh, inp, w, h)
+    R, Hq, D = inp.rows, sh.n_heads_q, sh.head_dim
+    pin = lambda x: torch.from_numpy(np.ascontiguousarray(x)).pin_memory()  # noqa: E731
+    host = {k: pin(np.zeros(R, np.float32)) for k in ("conf", "entropy", "ent_norm", "gap",
+                                                       "lbs_logit", "lps_prob")}
+    host["argmax"] = pin(np.zeros(R, np.int32))
+    host["accepted"] = pin(np.zeros(R, np.uint8))
+    host["attn_out"] = pin(np.zeros((R, Hq, D), np.float32))
+    st = {"tokens": pin(inp.tokens), "mask": pin(inp.mask), "in_block": pin(inp.in_block),
+          "blk_meta": pin(inp.blk_meta)}
+    ins = {"cu_rows": pin(inp.cu_rows.astype(np.int32)), "prefix_len": pin(inp.prefix_len.astype(np.int32)),
+           "row_pos": pin(inp.row_pos.astype(np.int32)), "hidden": pin(inp.hidden.view(np.int16)),
+           "q": pin(inp.q.view(np.int16)), "k_win": pin(inp.k_win.view(np.int16)),
+           "v_win": pin(inp.v_win.view(np.int16))}
+    a = E.ebd_step_args()
+    a.batch, a.rows = sh.batch, R
+    for k, v in {**ins, **st, **host}.items():
+        setattr(a, k, v.data_ptr())
+    kc = torch.from_numpy(inp.k_cache.view(np.int16)).cuda()
+    vc = torch.from_numpy(inp.v_cache.view(np.int16)).cuda()
+    a.k_cache, a.v_cache, a.w_lm = kc.data_ptr(), vc.data_ptr(), w.w_lm.data_ptr()
+    E.check(E.ebd_step_host(h.h, a, rt.stream_handle(None)), h.h)
+    assert h.sync_status() == 0
+    for k in ("conf", "entropy", "gap", "argmax", "accepted", "lbs_logit", "lps_prob"):
+        np.testing.assert_array_equal(host[k].numpy(), dev[k], err_msg=k)
+    np.testing.assert_array_equal(host["attn_out"].numpy(), dev["attn_out"])
+    for k in ("tokens", "mask", "in_block", "blk_meta"):
+        np.testing.assert_array_equal(st[k].numpy(), dev[k], err_msg=k)
+
+
 def test_weights_init_and_roundtrip():
     from paper_2609_16450_gb300 import _ebd as E
     sh = synth.tiny
