@@ -111,7 +111,7 @@ def test_dream_step(state):
             assert gpu["accepted"][r0:r1].sum() >= 1
 
 
-@pytest.mark.parametrize("point", [(4, 1024, 32), (16, 256, 64), (1, 4096, 8)])
+@pytest.mark.parametrize("point", [(4, 1024, 32), (16, 256, 64), (1, 4096, 8), (64, 1024, 64), (64, 4096, 64)])
 def test_sweep_point(point):
     sh = synth.sweep_point(*point)
     inp, w, h = _setup(sh)
