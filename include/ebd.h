@@ -215,7 +215,13 @@ ebd_status ebd_step(ebd_handle* h, const ebd_step_args* a, void* stream);
  * model weights and cache).  The handle copies the inputs to its own device
  * staging, runs the step and copies state and outputs back, all on
  * `stream`; the host buffers must stay valid until the stream reaches that
- * point (e.g. ebd_sync_status).  Enqueue only. */
+ * point (e.g. ebd_sync_status).  Enqueue only.
+ * Pinned, mapped buffers (cudaHostAlloc / cudaHostRegister) move by kernel
+ * instead of cudaMemcpyAsync.  With max_window <= 64 the kernels also write
+ * the decode state and the outputs straight into such buffers (attn_out
+ * when 16-byte aligned), and q, k_win and v_win are copied while the
+ * decision runs; the state and outputs then hold the step's results only
+ * once the stream has passed the step, as in every other case. */
 ebd_status ebd_step_host(ebd_handle* h, const ebd_step_args* a, void* stream);
 
 /* Only the decision (step 3) on caller-provided statistics: reads

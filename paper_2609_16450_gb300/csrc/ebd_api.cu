@@ -206,6 +206,12 @@ struct ebd_handle {
   cudaEvent_t ev[4] = {nullptr, nullptr, nullptr, nullptr};
   int profile = 0;
   int prof_mode = 0, prof_attn = 0;  // what the last ebd_step recorded
+  // ebd_step_host: the attention's inputs on a copy engine (created at first use)
+  int copy_route = -1;               // -1 not set up yet, 0 unavailable, 1 ready
+  cudaStream_t s_copy = nullptr;
+  cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
+  unsigned* d_ready = nullptr;
+  unsigned ticket = 0;
 };
 
 namespace {
@@ -554,7 +560,8 @@ ebd_status check_args(ebd_handle* h, const ebd_step_args* a, bool need_attn, boo
 }
 
 ebd_status run_attention(ebd_handle* h, const ebd_step_args* a, cudaStream_t st,
-                         bool pdl = false, bool wait_prior = false) {
+                         bool pdl = false, bool wait_prior = false, const unsigned* ready = nullptr,
+                         unsigned ready_ticket = 0) {
   const ebd_config& c = h->cfg;
   const int D = c.head_dim, Hkv = c.n_heads_kv;
   CUtensorMap kc, vc, kw, vw;
@@ -598,6 +605,8 @@ ebd_status run_attention(ebd_handle* h, const ebd_step_args* a, cudaStream_t st,
   p.status = h->d_status;
   p.limit_ns = kLimitNs;
   p.wait_prior = wait_prior ? 1 : 0;
+  p.ready = ready;
+  p.ready_ticket = ready_ticket;
   cudaError_t e = launch_attention(kc, vc, kw, vw, p, st, pdl);
   if (e != cudaSuccess) return cuda_fail(h, e, "attention launch");
   return EBD_OK;
@@ -672,6 +681,10 @@ DecideParams decide_params(ebd_handle* h, const ebd_step_args* a, int features_i
   p.mask = a->mask;
   p.in_block = a->in_block;
   p.blk_meta = a->blk_meta;
+  p.tokens_out = a->tokens;
+  p.mask_out = a->mask;
+  p.in_block_out = a->in_block;
+  p.blk_meta_out = a->blk_meta;
   p.conf = a->conf;
   p.entropy = a->entropy;
   p.ent_norm = a->ent_norm;
@@ -907,6 +920,10 @@ void ebd_destroy(ebd_handle* h) {
   cudaGetDevice(&prev);
   if (prev != h->device) cudaSetDevice(h->device);
   cudaDeviceSynchronize();
+  if (h->s_copy) cudaStreamDestroy(h->s_copy);
+  if (h->ev_fork) cudaEventDestroy(h->ev_fork);
+  if (h->ev_join) cudaEventDestroy(h->ev_join);
+  cudaFree(h->d_ready);
   cudaFree(h->d_blob);
   cudaFree(h->d_image);
   cudaFree(h->d_tok);
@@ -987,170 +1004,6 @@ ebd_status ebd_pack_lm_head(ebd_handle* h, const uint16_t* w_lm, uint16_t* w_pac
 }
 
 namespace {
-// windows of more than kMaxWindow rows per sequence: the grid-wide decision
-bool seq_mode(const ebd_handle* h) { return h->cfg.max_window > kMaxWindow; }
-
-SeqParams seq_params(ebd_handle* h, const ebd_step_args* a, const float* conf,
-                     const float* ent_norm, const float* gap, const int* argmax) {
-  const ebd_config& c = h->cfg;
-  SeqParams p = h->seqp;  // scratch
-  p.B = a->batch;
-  p.R = a->rows;
-  p.V = c.vocab;
-  p.gen_len = c.gen_len;
-  p.g_max = c.g_max;
-  p.l_min = c.l_min;
-  p.l_b = c.l_b;
-  p.eos_id = c.eos_id;
-  p.mode = c.decode_mode;
-  p.top_m = c.top_m;
-  p.lps_enabled = c.decode_mode == EBD_DECODE_EB ? c.lps_enabled : 0;
-  p.tau = c.tau;
-  p.tau_psi = c.tau_psi;
-  p.cu_rows = a->cu_rows;
-  p.row_pos = a->row_pos;
-  p.tokens = a->tokens;
-  p.mask = a->mask;
-  p.in_block = a->in_block;
-  p.blk_meta = a->blk_meta;
-  p.conf = conf;
-  p.ent_norm = ent_norm;
-  p.gap = gap;
-  p.argmax = argmax;
-  p.accepted = a->accepted;
-  p.lbs_logit = a->lbs_logit;
-  p.lps_prob = a->lps_prob;
-  p.w = h->d_seqw;
-  p.o = h->seqw;
-  p.tok_table = h->d_tok;
-  p.status = h->d_status;
-  return p;
-}
-
-// LM head, merge into the statistics, grid-wide decision
-ebd_status step_seq(ebd_handle* h, const ebd_step_args* a, cudaStream_t st) {
-  if (a->attn_out != nullptr || a->kv_append)
-    return fail(h, EBD_ERR_UNSUPPORTED,
-                "the window attention and the cache append need windows of at most 64 rows "
-                "(this handle has max_window > 64)");
-  const int prof = h->profile;
-  cudaError_t e;
-  if (prof && (e = record(h->ev[0], st)) != cudaSuccess) return cuda_fail(h, e, "profile event");
-  ebd_status s = run_lm(h, a, st);
-  if (s != EBD_OK) return s;
-  if (prof && (e = record(h->ev[1], st)) != cudaSuccess) return cuda_fail(h, e, "profile event");
-  float* conf = a->conf ? a->conf : const_cast<float*>(h->seqp.conf);
-  float* entn = a->ent_norm ? a->ent_norm : const_cast<float*>(h->seqp.ent_norm);
-  float* gap = a->gap ? a->gap : const_cast<float*>(h->seqp.gap);
-  int* arg = a->argmax ? a->argmax : const_cast<int*>(h->seqp.argmax);
-  const float inv = static_cast<float>(1.0 / std::log(static_cast<double>(h->cfg.vocab)));
-  if ((e = launch_merge_stats(h->part_f, h->part_i, a->rows, h->grid_lm, h->cfg.vocab, inv, conf,
-                              a->entropy, entn, gap, arg, h->d_status, st)) != cudaSuccess)
-    return cuda_fail(h, e, "merge launch");
-  if ((e = launch_decide_seq(seq_params(h, a, conf, entn, gap, arg), st)) != cudaSuccess)
-    return cuda_fail(h, e, "decision launch");
-  if (prof && (e = record(h->ev[2], st)) != cudaSuccess) return cuda_fail(h, e, "profile event");
-  if (prof && (e = record(h->ev[3], st)) != cudaSuccess) return cuda_fail(h, e, "profile event");
-  h->prof_mode = prof;
-  h->prof_attn = 0;
-  return EBD_OK;
-}
-}  // namespace
-
-ebd_status ebd_step(ebd_handle* h, const ebd_step_args* a, void* stream) {
-  if (h == nullptr) return EBD_ERR_INVALID_ARG;
-  ebd_status s = check_device(h);
-  if (s != EBD_OK) return s;
-  const bool attn = a != nullptr && a->attn_out != nullptr;
-  if ((s = check_args(h, a, attn, true, true)) != EBD_OK) return s;
-  if (h->w_emb == nullptr) return fail(h, EBD_ERR_STATE, "bind the token embedding first");
-  if (a->rows == 0 || a->batch == 0) return EBD_OK;
-  cudaStream_t st = static_cast<cudaStream_t>(stream);
-  (void)cudaGetLastError();  // a stale error of an earlier unrelated call is not ours
-  if (seq_mode(h)) return step_seq(h, a, st);
-  // Order on `st`: LM head, decision, window attention, (cache append).  The
-  // attention feeds neither of the others, so unless every kernel is timed
-  // on its own (profile mode 1) it is launched as a programmatic dependent
-  // of the decision: it fills the SMs the decision's clusters leave idle.
-  // The append reads the mask the decision writes: it is a programmatic
-  // dependent of the attention and waits for it, and the attention, in that
-  // case, waits for the decision before it exits.  The attention reads no
-  // cache position the append writes.
-  const int prof = h->profile;
-  cudaError_t e0 = cudaSuccess;
-  if (prof && (e0 = record(h->ev[0], st)) != cudaSuccess) return cuda_fail(h, e0, "profile event");
-  if ((s = run_lm(h, a, st)) != EBD_OK) return s;
-  if (prof && (e0 = record(h->ev[1], st)) != cudaSuccess) return cuda_fail(h, e0, "profile event");
-  DecideParams p = decide_params(h, a, 0);
-  p.pdl = prof == 0 ? 1 : 0;  // no event between the LM head and the decision
-  cudaError_t e = launch_decide(p, st);
-  if (e != cudaSuccess) return cuda_fail(h, e, "decision launch");
-  if (prof == 1 && (e0 = record(h->ev[2], st)) != cudaSuccess)
-    return cuda_fail(h, e0, "profile event");
-  const bool pdl_attn = prof != 1;
-  if (attn && (s = run_attention(h, a, st, pdl_attn, a->kv_append != 0)) != EBD_OK) return s;
-  if (a->kv_append) {
-    const ebd_config& c = h->cfg;
-    // a programmatic dependent only of a kernel that waits for the decision
-    e = launch_kv_append(a->k_cache, a->v_cache, a->k_win, a->v_win, a->cu_rows, a->row_pos, a->mask,
-                         a->batch, a->rows, c.max_prefix, c.n_heads_kv * c.head_dim, st,
-                         attn && pdl_attn);
-    if (e != cudaSuccess) return cuda_fail(h, e, "cache append launch");
-  }
-  if (prof && (e0 = record(h->ev[3], st)) != cudaSuccess) return cuda_fail(h, e0, "profile event");
-  h->prof_mode = prof;
-  h->prof_attn = attn ? 1 : 0;
-  return EBD_OK;
-}
-
-ebd_status ebd_decide(ebd_handle* h, const ebd_step_args* a, void* stream) {
-  if (h == nullptr) return EBD_ERR_INVALID_ARG;
-  ebd_status s = check_device(h);
-  if (s != EBD_OK) return s;
-  if ((s = check_args(h, a, false, false, true)) != EBD_OK) return s;
-  if (!a->conf || !a->ent_norm || !a->gap || !a->argmax)
-    return fail(h, EBD_ERR_INVALID_ARG, "conf/ent_norm/gap/argmax inputs must be set");
-  if (h->w_emb == nullptr) return fail(h, EBD_ERR_STATE, "bind the token embedding first");
-  if (a->rows == 0 || a->batch == 0) return EBD_OK;
-  if (seq_mode(h)) {
-    cudaError_t e = launch_decide_seq(seq_params(h, a, a->conf, a->ent_norm, a->gap, a->argmax),
-                                      static_cast<cudaStream_t>(stream));
-    if (e != cudaSuccess) return cuda_fail(h, e, "decision launch");
-    return EBD_OK;
-  }
-  DecideParams p = decide_params(h, a, 1);
-  p.entropy = nullptr;
-  cudaError_t e = launch_decide(p, static_cast<cudaStream_t>(stream));
-  if (e != cudaSuccess) return cuda_fail(h, e, "decision launch");
-  return EBD_OK;
-}
-
-ebd_status ebd_lm_stats(ebd_handle* h, const ebd_step_args* a, void* stream) {
-  if (h == nullptr) return EBD_ERR_INVALID_ARG;
-  ebd_status s = check_device(h);
-  if (s != EBD_OK) return s;
-  if ((s = check_args(h, a, false, true, false)) != EBD_OK) return s;
-  if (a->rows == 0) return EBD_OK;
-  cudaStream_t st = static_cast<cudaStream_t>(stream);
-  if ((s = run_lm(h, a, st)) != EBD_OK) return s;
-  const float inv = static_cast<float>(1.0 / std::log(static_cast<double>(h->cfg.vocab)));
-  cudaError_t e = launch_merge_stats(h->part_f, h->part_i, a->rows, h->grid_lm, h->cfg.vocab, inv,
-                                     a->conf, a->entropy, a->ent_norm, a->gap, a->argmax,
-                                     h->d_status, st);
-  if (e != cudaSuccess) return cuda_fail(h, e, "merge launch");
-  return EBD_OK;
-}
-
-ebd_status ebd_attention(ebd_handle* h, const ebd_step_args* a, void* stream) {
-  if (h == nullptr) return EBD_ERR_INVALID_ARG;
-  ebd_status s = check_device(h);
-  if (s != EBD_OK) return s;
-  if ((s = check_args(h, a, true, false, false)) != EBD_OK) return s;
-  if (a->rows == 0 || a->batch == 0) return EBD_OK;
-  return run_attention(h, a, static_cast<cudaStream_t>(stream));
-}
-
-namespace {
 // ebd_step_host moves its inputs in and its results out with one kernel
 // each way where the host buffers are pinned and mapped into the device's
 // address space (cudaHostAlloc / cudaHostRegister memory): one launch
@@ -1225,8 +1078,244 @@ struct HostMover {
     return cudaGetLastError();
   }
 };
+
+// What ebd_step_host changes in a step: the ticket the attention waits for
+// (its inputs come in on the copy stream) and where the decision writes the
+// decode state (the caller's buffers, when it read a staged copy).
+struct StepRoute {
+  const unsigned* ready;
+  unsigned ready_ticket;
+  int* tokens_out;
+  uint8_t* mask_out;
+  uint8_t* in_block_out;
+  int* blk_meta_out;
+};
+
+typedef CUresult (*WriteValue32Fn)(CUstream, CUdeviceptr, cuuint32_t, unsigned int);
+WriteValue32Fn get_write_value() {
+  static WriteValue32Fn fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* ptr = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuStreamWriteValue32", &ptr, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<WriteValue32Fn>(ptr);
+  });
+  return fn;
+}
+
+// The copy stream, its two events and the ticket word; false where the
+// driver offers no stream write (the inputs then go with the others).
+bool copy_route_ready(ebd_handle* h) {
+  if (h->copy_route >= 0) return h->copy_route == 1;
+  h->copy_route = 0;
+  if (get_write_value() == nullptr) return false;
+  if (cudaStreamCreateWithFlags(&h->s_copy, cudaStreamNonBlocking) != cudaSuccess ||
+      cudaEventCreateWithFlags(&h->ev_fork, cudaEventDisableTiming) != cudaSuccess ||
+      cudaEventCreateWithFlags(&h->ev_join, cudaEventDisableTiming) != cudaSuccess ||
+      cudaMalloc(&h->d_ready, sizeof(unsigned)) != cudaSuccess ||
+      cudaMemsetAsync(h->d_ready, 0, sizeof(unsigned), h->s_copy) != cudaSuccess ||
+      cudaStreamSynchronize(h->s_copy) != cudaSuccess) {
+    (void)cudaGetLastError();
+    return false;
+  }
+  h->copy_route = 1;
+  return true;
+}
 }  // namespace
 
+namespace {
+// windows of more than kMaxWindow rows per sequence: the grid-wide decision
+bool seq_mode(const ebd_handle* h) { return h->cfg.max_window > kMaxWindow; }
+
+SeqParams seq_params(ebd_handle* h, const ebd_step_args* a, const float* conf,
+                     const float* ent_norm, const float* gap, const int* argmax) {
+  const ebd_config& c = h->cfg;
+  SeqParams p = h->seqp;  // scratch
+  p.B = a->batch;
+  p.R = a->rows;
+  p.V = c.vocab;
+  p.gen_len = c.gen_len;
+  p.g_max = c.g_max;
+  p.l_min = c.l_min;
+  p.l_b = c.l_b;
+  p.eos_id = c.eos_id;
+  p.mode = c.decode_mode;
+  p.top_m = c.top_m;
+  p.lps_enabled = c.decode_mode == EBD_DECODE_EB ? c.lps_enabled : 0;
+  p.tau = c.tau;
+  p.tau_psi = c.tau_psi;
+  p.cu_rows = a->cu_rows;
+  p.row_pos = a->row_pos;
+  p.tokens = a->tokens;
+  p.mask = a->mask;
+  p.in_block = a->in_block;
+  p.blk_meta = a->blk_meta;
+  p.conf = conf;
+  p.ent_norm = ent_norm;
+  p.gap = gap;
+  p.argmax = argmax;
+  p.accepted = a->accepted;
+  p.lbs_logit = a->lbs_logit;
+  p.lps_prob = a->lps_prob;
+  p.w = h->d_seqw;
+  p.o = h->seqw;
+  p.tok_table = h->d_tok;
+  p.status = h->d_status;
+  return p;
+}
+
+// LM head, merge into the statistics, grid-wide decision
+ebd_status step_seq(ebd_handle* h, const ebd_step_args* a, cudaStream_t st) {
+  if (a->attn_out != nullptr || a->kv_append)
+    return fail(h, EBD_ERR_UNSUPPORTED,
+                "the window attention and the cache append need windows of at most 64 rows "
+                "(this handle has max_window > 64)");
+  const int prof = h->profile;
+  cudaError_t e;
+  if (prof && (e = record(h->ev[0], st)) != cudaSuccess) return cuda_fail(h, e, "profile event");
+  ebd_status s = run_lm(h, a, st);
+  if (s != EBD_OK) return s;
+  if (prof && (e = record(h->ev[1], st)) != cudaSuccess) return cuda_fail(h, e, "profile event");
+  float* conf = a->conf ? a->conf : const_cast<float*>(h->seqp.conf);
+  float* entn = a->ent_norm ? a->ent_norm : const_cast<float*>(h->seqp.ent_norm);
+  float* gap = a->gap ? a->gap : const_cast<float*>(h->seqp.gap);
+  int* arg = a->argmax ? a->argmax : const_cast<int*>(h->seqp.argmax);
+  const float inv = static_cast<float>(1.0 / std::log(static_cast<double>(h->cfg.vocab)));
+  if ((e = launch_merge_stats(h->part_f, h->part_i, a->rows, h->grid_lm, h->cfg.vocab, inv, conf,
+                              a->entropy, entn, gap, arg, h->d_status, st)) != cudaSuccess)
+    return cuda_fail(h, e, "merge launch");
+  if ((e = launch_decide_seq(seq_params(h, a, conf, entn, gap, arg), st)) != cudaSuccess)
+    return cuda_fail(h, e, "decision launch");
+  if (prof && (e = record(h->ev[2], st)) != cudaSuccess) return cuda_fail(h, e, "profile event");
+  if (prof && (e = record(h->ev[3], st)) != cudaSuccess) return cuda_fail(h, e, "profile event");
+  h->prof_mode = prof;
+  h->prof_attn = 0;
+  return EBD_OK;
+}
+}  // namespace
+
+namespace {
+// One step of the block-window setting (windows of at most kMaxWindow rows).
+// Order on `st`: LM head, decision, window attention, (cache append).  The
+// attention feeds neither of the others, so unless every kernel is timed on
+// its own (profile mode 1) it is launched as a programmatic dependent of the
+// decision: it fills the SMs the decision's clusters leave idle.  The append
+// reads the mask the decision writes: it is a programmatic dependent of the
+// attention and waits for it, and the attention, in that case, waits for the
+// decision before it exits.  The attention reads no cache position the
+// append writes.
+ebd_status step_run(ebd_handle* h, const ebd_step_args* a, cudaStream_t st, const StepRoute* rt) {
+  const bool attn = a->attn_out != nullptr;
+  ebd_status s;
+  const int prof = h->profile;
+  cudaError_t e0 = cudaSuccess;
+  if (prof && (e0 = record(h->ev[0], st)) != cudaSuccess) return cuda_fail(h, e0, "profile event");
+  if ((s = run_lm(h, a, st)) != EBD_OK) return s;
+  if (prof && (e0 = record(h->ev[1], st)) != cudaSuccess) return cuda_fail(h, e0, "profile event");
+  DecideParams p = decide_params(h, a, 0);
+  p.pdl = prof == 0 ? 1 : 0;  // no event between the LM head and the decision
+  if (rt != nullptr) {
+    p.tokens_out = rt->tokens_out;
+    p.mask_out = rt->mask_out;
+    p.in_block_out = rt->in_block_out;
+    p.blk_meta_out = rt->blk_meta_out;
+  }
+  cudaError_t e = launch_decide(p, st);
+  if (e != cudaSuccess) return cuda_fail(h, e, "decision launch");
+  if (prof == 1 && (e0 = record(h->ev[2], st)) != cudaSuccess)
+    return cuda_fail(h, e0, "profile event");
+  const bool pdl_attn = prof != 1;
+  if (attn && (s = run_attention(h, a, st, pdl_attn, a->kv_append != 0, rt ? rt->ready : nullptr,
+                                 rt ? rt->ready_ticket : 0u)) != EBD_OK)
+    return s;
+  if (a->kv_append) {
+    const ebd_config& c = h->cfg;
+    // a programmatic dependent only of a kernel that waits for the decision
+    e = launch_kv_append(a->k_cache, a->v_cache, a->k_win, a->v_win, a->cu_rows, a->row_pos,
+                         rt != nullptr ? rt->mask_out : a->mask, a->batch, a->rows, c.max_prefix,
+                         c.n_heads_kv * c.head_dim, st, attn && pdl_attn);
+    if (e != cudaSuccess) return cuda_fail(h, e, "cache append launch");
+  }
+  if (prof && (e0 = record(h->ev[3], st)) != cudaSuccess) return cuda_fail(h, e0, "profile event");
+  h->prof_mode = prof;
+  h->prof_attn = attn ? 1 : 0;
+  return EBD_OK;
+}
+}  // namespace
+
+ebd_status ebd_step(ebd_handle* h, const ebd_step_args* a, void* stream) {
+  if (h == nullptr) return EBD_ERR_INVALID_ARG;
+  ebd_status s = check_device(h);
+  if (s != EBD_OK) return s;
+  const bool attn = a != nullptr && a->attn_out != nullptr;
+  if ((s = check_args(h, a, attn, true, true)) != EBD_OK) return s;
+  if (h->w_emb == nullptr) return fail(h, EBD_ERR_STATE, "bind the token embedding first");
+  if (a->rows == 0 || a->batch == 0) return EBD_OK;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  (void)cudaGetLastError();  // a stale error of an earlier unrelated call is not ours
+  if (seq_mode(h)) return step_seq(h, a, st);
+  return step_run(h, a, st, nullptr);
+}
+
+ebd_status ebd_decide(ebd_handle* h, const ebd_step_args* a, void* stream) {
+  if (h == nullptr) return EBD_ERR_INVALID_ARG;
+  ebd_status s = check_device(h);
+  if (s != EBD_OK) return s;
+  if ((s = check_args(h, a, false, false, true)) != EBD_OK) return s;
+  if (!a->conf || !a->ent_norm || !a->gap || !a->argmax)
+    return fail(h, EBD_ERR_INVALID_ARG, "conf/ent_norm/gap/argmax inputs must be set");
+  if (h->w_emb == nullptr) return fail(h, EBD_ERR_STATE, "bind the token embedding first");
+  if (a->rows == 0 || a->batch == 0) return EBD_OK;
+  if (seq_mode(h)) {
+    cudaError_t e = launch_decide_seq(seq_params(h, a, a->conf, a->ent_norm, a->gap, a->argmax),
+                                      static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(h, e, "decision launch");
+    return EBD_OK;
+  }
+  DecideParams p = decide_params(h, a, 1);
+  p.entropy = nullptr;
+  cudaError_t e = launch_decide(p, static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(h, e, "decision launch");
+  return EBD_OK;
+}
+
+ebd_status ebd_lm_stats(ebd_handle* h, const ebd_step_args* a, void* stream) {
+  if (h == nullptr) return EBD_ERR_INVALID_ARG;
+  ebd_status s = check_device(h);
+  if (s != EBD_OK) return s;
+  if ((s = check_args(h, a, false, true, false)) != EBD_OK) return s;
+  if (a->rows == 0) return EBD_OK;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  if ((s = run_lm(h, a, st)) != EBD_OK) return s;
+  const float inv = static_cast<float>(1.0 / std::log(static_cast<double>(h->cfg.vocab)));
+  cudaError_t e = launch_merge_stats(h->part_f, h->part_i, a->rows, h->grid_lm, h->cfg.vocab, inv,
+                                     a->conf, a->entropy, a->ent_norm, a->gap, a->argmax,
+                                     h->d_status, st);
+  if (e != cudaSuccess) return cuda_fail(h, e, "merge launch");
+  return EBD_OK;
+}
+
+ebd_status ebd_attention(ebd_handle* h, const ebd_step_args* a, void* stream) {
+  if (h == nullptr) return EBD_ERR_INVALID_ARG;
+  ebd_status s = check_device(h);
+  if (s != EBD_OK) return s;
+  if ((s = check_args(h, a, true, false, false)) != EBD_OK) return s;
+  if (a->rows == 0 || a->batch == 0) return EBD_OK;
+  return run_attention(h, a, static_cast<cudaStream_t>(stream));
+}
+
+
+// In the block-window setting the results go straight into the caller's
+// mapped host buffers (the kernels' stores cross the host link; nothing is
+// copied back after the step), and with the attention, its own inputs (q and
+// the window K/V, which nothing else before it reads) come in on a copy
+// engine while the LM head runs: a second stream, forked after the copy of
+// what the LM head and the decision read, copies them and then writes the
+// step's ticket, which the attention waits for; `stream` waits for that
+// stream at the end of the step.
 ebd_status ebd_step_host(ebd_handle* h, const ebd_step_args* a, void* stream) {
   if (h == nullptr) return EBD_ERR_INVALID_ARG;
   ebd_status s = check_device(h);
@@ -1237,6 +1326,12 @@ ebd_status ebd_step_host(ebd_handle* h, const ebd_step_args* a, void* stream) {
   if (!a->cu_rows || !a->prefix_len || !a->row_pos || !a->hidden || !a->tokens || !a->mask ||
       !a->in_block || !a->blk_meta || !a->w_lm)
     return fail(h, EBD_ERR_INVALID_ARG, "missing host input");
+  const bool attn = a->attn_out != nullptr;
+  const bool kv = attn || a->kv_append;  // the window K/V feed the attention and the append
+  if ((attn && !a->q) || (kv && (!a->k_win || !a->v_win)))
+    return fail(h, EBD_ERR_INVALID_ARG, "missing host input (q / window K/V)");
+  if (h->w_emb == nullptr) return fail(h, EBD_ERR_STATE, "bind the token embedding first");
+  if (a->rows == 0 || a->batch == 0) return EBD_OK;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   const ebd_config& c = h->cfg;
   const size_t R = a->rows, B = a->batch, RM = c.max_rows, BM = c.max_batch;
@@ -1265,53 +1360,94 @@ ebd_status ebd_step_host(ebd_handle* h, const ebd_step_args* a, void* stream) {
   int32_t* am = reinterpret_cast<int32_t*>(take(RM * 4));
   uint8_t* acc = take(RM);
   int32_t* sfx = reinterpret_cast<int32_t*>(take(BM * 8));
-  const bool attn = a->attn_out != nullptr;
+  const bool route = !seq_mode(h);
+  const bool dma = route && attn && copy_route_ready(h);
   HostMover in{st, true};
+  in.add(hid, a->hidden, R * d * 2);
   in.add(cu, a->cu_rows, (B + 1) * 4);
   in.add(pl, a->prefix_len, B * 4);
   in.add(rp, a->row_pos, R * 4);
-  in.add(hid, a->hidden, R * d * 2);
-  const bool kv = attn || a->kv_append;  // the window K/V feed the attention and the append
-  if (attn) in.add(q, a->q, R * Hq * D * 2);
-  if (kv) {
-    in.add(kw, a->k_win, R * Hkv * D * 2);
-    in.add(vw, a->v_win, R * Hkv * D * 2);
-  }
   in.add(tok, a->tokens, R * 4);
   in.add(msk, a->mask, R);
   in.add(ib, a->in_block, R);
   in.add(meta, a->blk_meta, B * 8);
   if (a->suffix) in.add(sfx, a->suffix, B * 8);
+  if (!dma) {
+    if (attn) in.add(q, a->q, R * Hq * D * 2);
+    if (kv) {
+      in.add(kw, a->k_win, R * Hkv * D * 2);
+      in.add(vw, a->v_win, R * Hkv * D * 2);
+    }
+  }
   cudaError_t e = in.flush();
   if (e != cudaSuccess) return cuda_fail(h, e, "host-to-device copy");
+  unsigned ticket = 0;
+  if (dma) {
+    if (++h->ticket == 0) h->ticket = 1;  // 0 is the word's initial value
+    ticket = h->ticket;
+    const cudaMemcpyKind k = cudaMemcpyHostToDevice;
+    if ((e = cudaEventRecord(h->ev_fork, st)) != cudaSuccess ||
+        (e = cudaStreamWaitEvent(h->s_copy, h->ev_fork, 0)) != cudaSuccess ||
+        (e = cudaMemcpyAsync(q, a->q, R * Hq * D * 2, k, h->s_copy)) != cudaSuccess ||
+        (e = cudaMemcpyAsync(kw, a->k_win, R * Hkv * D * 2, k, h->s_copy)) != cudaSuccess ||
+        (e = cudaMemcpyAsync(vw, a->v_win, R * Hkv * D * 2, k, h->s_copy)) != cudaSuccess)
+      return cuda_fail(h, e, "host-to-device copy (copy stream)");
+    if (get_write_value()(reinterpret_cast<CUstream>(h->s_copy), reinterpret_cast<CUdeviceptr>(h->d_ready),
+                          ticket, 0) != CUDA_SUCCESS)
+      return fail(h, EBD_ERR_CUDA, "cuStreamWriteValue32 failed");
+    if ((e = cudaEventRecord(h->ev_join, h->s_copy)) != cudaSuccess)
+      return cuda_fail(h, e, "copy stream event");
+  }
   g.cu_rows = cu; g.prefix_len = pl; g.row_pos = rp; g.hidden = hid;
   g.q = attn ? q : nullptr; g.k_win = kv ? kw : nullptr; g.v_win = kv ? vw : nullptr;
   g.tokens = tok; g.mask = msk; g.in_block = ib; g.blk_meta = meta;
   g.suffix = a->suffix ? sfx : nullptr;
-  g.attn_out = attn ? ao : nullptr;
-  g.conf = a->conf ? f[0] : nullptr;
-  g.entropy = a->entropy ? f[1] : nullptr;
-  g.ent_norm = a->ent_norm ? f[2] : nullptr;
-  g.gap = a->gap ? f[3] : nullptr;
-  g.lbs_logit = a->lbs_logit ? f[4] : nullptr;
-  g.lps_prob = a->lps_prob ? f[5] : nullptr;
-  g.argmax = a->argmax ? am : nullptr;
-  g.accepted = a->accepted ? acc : nullptr;
-  if ((s = ebd_step(h, &g, stream)) != EBD_OK) return s;
+  // A result buffer: the caller's own (its device address) where it is
+  // mapped and aligned as the kernel's stores need, else the staging buffer,
+  // copied back after the step.
+  struct Back {
+    void* host;
+    const void* stage;
+    size_t bytes;
+  } back[16];
+  int nback = 0;
+  auto result = [&](void* host, void* stage, size_t bytes, uintptr_t align) -> void* {
+    if (host == nullptr) return nullptr;
+    if (route) {
+      const void* dev = mapped_host(host);
+      if (dev != nullptr && (reinterpret_cast<uintptr_t>(dev) & (align - 1)) == 0) return const_cast<void*>(dev);
+    }
+    back[nback++] = Back{host, stage, bytes};
+    return stage;
+  };
+  StepRoute rt{dma ? h->d_ready : nullptr, ticket, nullptr, nullptr, nullptr, nullptr};
+  rt.tokens_out = static_cast<int32_t*>(result(a->tokens, tok, R * 4, 4));
+  rt.mask_out = static_cast<uint8_t*>(result(a->mask, msk, R, 1));
+  rt.in_block_out = static_cast<uint8_t*>(result(a->in_block, ib, R, 1));
+  rt.blk_meta_out = static_cast<int32_t*>(result(a->blk_meta, meta, B * 8, 4));
+  g.attn_out = attn ? static_cast<float*>(result(a->attn_out, ao, R * Hq * D * 4, 16)) : nullptr;
+  g.conf = static_cast<float*>(result(a->conf, f[0], R * 4, 4));
+  g.entropy = static_cast<float*>(result(a->entropy, f[1], R * 4, 4));
+  g.ent_norm = static_cast<float*>(result(a->ent_norm, f[2], R * 4, 4));
+  g.gap = static_cast<float*>(result(a->gap, f[3], R * 4, 4));
+  g.lbs_logit = static_cast<float*>(result(a->lbs_logit, f[4], R * 4, 4));
+  g.lps_prob = static_cast<float*>(result(a->lps_prob, f[5], R * 4, 4));
+  g.argmax = static_cast<int32_t*>(result(a->argmax, am, R * 4, 4));
+  g.accepted = static_cast<uint8_t*>(result(a->accepted, acc, R, 1));
+  if (route) {
+    if ((s = check_args(h, &g, attn, true, true)) != EBD_OK) return s;
+    (void)cudaGetLastError();  // a stale error of an earlier unrelated call is not ours
+    s = step_run(h, &g, st, &rt);
+  } else {
+    s = ebd_step(h, &g, stream);  // in place on the staged decode state
+  }
+  if (dma) {  // later work on `stream` follows the copy stream too (also after a failed launch)
+    if ((e = cudaStreamWaitEvent(st, h->ev_join, 0)) != cudaSuccess && s == EBD_OK)
+      return cuda_fail(h, e, "copy stream join");
+  }
+  if (s != EBD_OK) return s;
   HostMover out{st, false};
-  out.add(a->tokens, tok, R * 4);
-  out.add(a->mask, msk, R);
-  out.add(a->in_block, ib, R);
-  out.add(a->blk_meta, meta, B * 8);
-  if (attn) out.add(a->attn_out, ao, R * Hq * D * 4);
-  out.add(a->conf, f[0], R * 4);
-  out.add(a->entropy, f[1], R * 4);
-  out.add(a->ent_norm, f[2], R * 4);
-  out.add(a->gap, f[3], R * 4);
-  out.add(a->lbs_logit, f[4], R * 4);
-  out.add(a->lps_prob, f[5], R * 4);
-  out.add(a->argmax, am, R * 4);
-  out.add(a->accepted, acc, R);
+  for (int i = 0; i < nback; ++i) out.add(back[i].host, back[i].stage, back[i].bytes);
   if ((e = out.flush()) != cudaSuccess) return cuda_fail(h, e, "device-to-host copy");
   return EBD_OK;
 }

@@ -62,6 +62,8 @@ struct AttnParams {
   int* status;
   uint64_t limit_ns;
   int wait_prior;           // every CTA waits for the grid it depends on before exiting
+  const unsigned* ready;     // non-null: q and the window K/V are being copied in by
+  unsigned ready_ticket;    // another stream, which then writes ready_ticket to *ready
 };
 
 // ------------------------------------------------------------------ routers
@@ -84,10 +86,14 @@ struct DecideParams {
   const int* row_pos;
   const float4* part_f;
   const int* part_i;
-  int* tokens;
-  uint8_t* mask;
-  uint8_t* in_block;
-  int* blk_meta;
+  const int* tokens;         // decode state in: read before the LM head's grid completes
+  const uint8_t* mask;
+  const uint8_t* in_block;
+  const int* blk_meta;
+  int* tokens_out;           // decode state out: the same buffers as the state in,
+  uint8_t* mask_out;         // unless the state in is a staged copy of the caller's
+  uint8_t* in_block_out;
+  int* blk_meta_out;
   float *conf, *entropy, *ent_norm, *gap, *lbs_logit, *lps_prob;
   int* argmax;
   uint8_t* accepted;

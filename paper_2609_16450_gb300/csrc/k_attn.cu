@@ -362,6 +362,33 @@ cudaError_t launch_kv_append(uint16_t* k_cache, uint16_t* v_cache, const uint16_
                             hkvd / 8);
 }
 
+// q and the window K/V copied in by another stream (a copy engine), which
+// then writes the step's ticket to *p.ready: thread 0 polls it with an
+// acquire at system scope, with a time limit; on timeout the CTA records
+// EBD_ERR_TIMEOUT and does no work.
+__device__ __forceinline__ bool wait_ready(const AttnParams& p) {
+  __shared__ int s_ok;
+  if (threadIdx.x == 0) {
+    auto seen = [&]() {
+      unsigned v;
+      asm volatile("ld.acquire.sys.global.u32 %0, [%1];" : "=r"(v) : "l"(p.ready) : "memory");
+      return v == p.ready_ticket;
+    };
+    bool ok = seen();
+    if (!ok) {
+      const uint64_t t0 = global_timer_ns();
+      while (!(ok = seen()) && global_timer_ns() - t0 <= p.limit_ns) __nanosleep(200);
+    }
+    if (ok)
+      asm volatile("fence.proxy.async.global;" ::: "memory");  // the TMA reads of the window K/V
+    else
+      atomicCAS(p.status, 0, EBD_ERR_TIMEOUT);
+    s_ok = ok ? 1 : 0;
+  }
+  __syncthreads();
+  return s_ok != 0;
+}
+
 // The whole kernel; with p.wait_prior every CTA, whichever way it finishes,
 // waits for the grid it is a programmatic dependent of (the decision) before
 // it exits, so that a kernel launched after this one as its dependent sees
@@ -371,7 +398,7 @@ __global__ void __launch_bounds__(kAttnThreads)
     attn_kernel(const __grid_constant__ CUtensorMap tm_kc, const __grid_constant__ CUtensorMap tm_vc,
                 const __grid_constant__ CUtensorMap tm_kw, const __grid_constant__ CUtensorMap tm_vw,
                 const AttnParams p) {
-  attn_body<D>(tm_kc, tm_vc, tm_kw, tm_vw, p);
+  if (p.ready == nullptr || wait_ready(p)) attn_body<D>(tm_kc, tm_vc, tm_kw, tm_vw, p);
   if (p.wait_prior) asm volatile("griddepcontrol.wait;" ::: "memory");
 }
 

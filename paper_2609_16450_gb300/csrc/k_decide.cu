@@ -1114,16 +1114,16 @@ __global__ void __cluster_dims__(kDecideCluster, 1, 1) __launch_bounds__(kDecide
   if (shadow) return;
   for (int j = tid; j < nr; j += blockDim.x) {
     const int r = r0 + j;
-    p.tokens[r] = sm.f_tok[j];
-    p.mask[r] = sm.f_mask[j];
-    p.in_block[r] = sm.f_ib[j];
+    p.tokens_out[r] = sm.f_tok[j];
+    p.mask_out[r] = sm.f_mask[j];
+    p.in_block_out[r] = sm.f_ib[j];
     if (p.accepted) p.accepted[r] = sm.f_acc[j];
     if (p.lbs_logit) p.lbs_logit[r] = sm.f_O[j];
     if (p.lps_prob) p.lps_prob[r] = sm.f_p[j];
   }
   if (tid == 0 && !sm.bad_seq) {
-    p.blk_meta[2 * seq] = sm.meta_b;
-    p.blk_meta[2 * seq + 1] = sm.meta_s;
+    p.blk_meta_out[2 * seq] = sm.meta_b;
+    p.blk_meta_out[2 * seq + 1] = sm.meta_s;
   }
 }
 
