@@ -187,6 +187,19 @@ def suffix_len(sh):
     return int(sh.gen_len - int(np.max(synth.window_sizes(sh))))
 
 
+def lm_grid(num_sms, n_units):
+    """CTAs of the library's unpaired LM-head launch, hence partial states
+    per row (the same rule as the library's lm_grid): the fewest CTAs that
+    take at most one 64-row vocabulary unit more each than an even split over
+    every SM, if that keeps 90 % of the SMs."""
+    num_sms = max(1, num_sms)
+    if n_units <= num_sms:
+        return max(1, n_units)
+    per = -(-n_units // num_sms) + 1
+    g = -(-n_units // per)
+    return g if 10 * g >= 9 * num_sms else num_sms
+
+
 def step_work(sh, rows, masked, grid_lm, lbs_runs, suffix=0, append=False):
     """Algorithmic bytes and flops of one step (each input read once); suffix:
     cached keys after each window (dual cache); append: committed rows'
@@ -393,7 +406,7 @@ def run_ours(args, rank, world, local_rank):
     out["suffix"] = None if sfx is None else sfx
     out["fetch"] = ds.fetch()
     h_sms = torch.cuda.get_device_properties(local_rank).multi_processor_count
-    out["grid_lm"] = min(h_sms, (sh.vocab + 63) // 64)
+    out["grid_lm"] = lm_grid(h_sms, (sh.vocab + 63) // 64)
     out["num_sms"] = h_sms
     h.close()
     return out

@@ -818,8 +818,7 @@ ebd_status ebd_create(const ebd_config* cfg, ebd_handle** out) {
   if ((s = upload_router(h)) != EBD_OK) return bail(s);
 
   // LM-head partials: one state per (row, CTA)
-  h->grid_lm = h->num_sms < (cfg->vocab + kUnit - 1) / kUnit ? h->num_sms
-                                                             : (cfg->vocab + kUnit - 1) / kUnit;
+  h->grid_lm = lm_grid(h->num_sms, (cfg->vocab + kUnit - 1) / kUnit);
   const size_t np = static_cast<size_t>(cfg->max_rows) * h->grid_lm;
   if ((e = cudaMalloc(&h->part_f, np * sizeof(float4))) != cudaSuccess)
     return bail(cuda_fail(h, e, "cudaMalloc(partials)"));

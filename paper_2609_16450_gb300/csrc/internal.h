@@ -165,6 +165,7 @@ struct SeqParams {
 // host launchers (defined next to their kernels)
 cudaError_t launch_lm_stats(const CUtensorMap& tmap_w, const CUtensorMap& tmap_h,
                             const LmParams& p, cudaStream_t st);
+int lm_grid(int num_sms, int n_units);  // partial states per row of the LM head
 void lm_plan(LmParams& p, int rows, int V, int d, int num_sms, bool pair = false);
 // pdl: launched as a programmatic dependent of the kernel before it on
 // `st` (that kernel's CTAs release it early; the attention reads nothing the

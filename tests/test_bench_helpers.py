@@ -49,3 +49,17 @@ def test_full_sequence_has_no_window_attention():
     assert wk["attn_bytes"] == 0 and wk["attn_flops"] == 0
     assert wk["lm_flops"] == 2 * 512 * 4096 * 126464
     assert np.isclose(wk["lm_flops"] / 1897.5e12 * 1e6, 279.5, atol=0.5)  # tensor roofline, us
+
+
+def test_lm_grid_rule():
+    """The LM-head grid: LLaDA-8B's 1976 units on 152 SMs go to 142 CTAs of at
+    most 14 units; few units take one CTA each; a split that would drop
+    below 90 % of the SMs keeps every SM."""
+    b = _bench()
+    assert b.lm_grid(152, 1976) == 142
+    assert b.lm_grid(152, 2376) == 140
+    assert b.lm_grid(152, 64) == 64
+    assert b.lm_grid(152, 200) == 152  # 2 per CTA -> 3 per CTA would need only 67 CTAs
+    for units in (153, 1000, 1976, 2376, 5000):
+        g = b.lm_grid(152, units)
+        assert -(-units // g) <= -(-units // 152) + 1
