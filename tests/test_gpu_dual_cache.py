@@ -121,6 +121,10 @@ def _step_with_append(inp, host=False):
                       attn_out=np.zeros((R, sh.n_heads_q, sh.head_dim), np.float32),
                       accepted=np.zeros(R, np.uint8))
             hb = {k: np.ascontiguousarray(v) for k, v in hb.items()}
+            if host == "pinned":  # mapped buffers: results stored by the kernels themselves
+                pinned = {k: torch.from_numpy(v.view(np.int16) if v.dtype == np.uint16 else v).pin_memory()
+                          for k, v in hb.items()}
+                hb = {k: t.numpy().view(hb[k].dtype) for k, t in pinned.items()}
             for k, v in hb.items():
                 setattr(a, k, v.ctypes.data)
             for k in ("conf", "entropy", "ent_norm", "gap", "argmax", "lbs_logit", "lps_prob"):
@@ -136,7 +140,7 @@ def _step_with_append(inp, host=False):
         h.close()
 
 
-@pytest.mark.parametrize("host", [False, True])
+@pytest.mark.parametrize("host", [False, True, "pinned"])
 def test_append_tiny_matches_oracle(host):
     sh = synth.tiny
     inp = _with_suffix_cache(synth.make_step_inputs(sh), 64, seed=21)
