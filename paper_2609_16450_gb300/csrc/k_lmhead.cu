@@ -523,10 +523,13 @@ void lm_plan(LmParams& p, int rows, int V, int d, int num_sms, bool pair) {
     if (p.grid < 1) p.grid = 1;
   }
   p.nkb = (d + 63) / 64;
-  // a second epilogue warpgroup (and its transpose buffer) only pays when the
-  // accumulator is wide; below that the buffer is worth more as a larger
-  // pipeline stage (measured: 128 rows, 5 x 16 KB stages -> 183 us, 4 -> 246)
-  p.nwg = (p.n_pad >= 192 || p.mch == 2) ? 2 : 1;
+  // a second epilogue warpgroup (and its transpose buffer) only pays where
+  // the epilogue is exposed, i.e. with a single accumulator buffer; with two,
+  // one warpgroup keeps up with the MMAs and its buffer is worth more as
+  // pipeline stages (measured: 256 rows 270.7 -> 247.2 us, 512 rows in CTA
+  // pairs 445 -> 408.5 us; two chunks per stage (one buffer) 405 -> 432 us
+  // with one warpgroup)
+  p.nwg = p.mch == 2 ? 2 : 1;
   const uint32_t st_bytes = static_cast<uint32_t>(p.n_pad) * 20u;
   const uint32_t tail = kTBytes * static_cast<uint32_t>(p.nwg) + ((st_bytes + 7) / 8 * 8) +
                         (2 * 8 + 6) * 8 + 16;
