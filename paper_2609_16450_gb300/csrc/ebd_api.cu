@@ -20,7 +20,7 @@ cudaError_t lm_configure();
 cudaError_t launch_merge_stats(const float4* part_f, const int* part_i, int rows, int grid,
                                int V, float inv_log_v, float* conf, float* entropy,
                                float* ent_norm, float* gap, int* argmax, int* status,
-                               cudaStream_t st);
+                               cudaStream_t st, bool pdl = false);
 }  // namespace ebd
 
 using namespace ebd;
@@ -1174,20 +1174,23 @@ ebd_status step_seq(ebd_handle* h, const ebd_step_args* a, cudaStream_t st) {
                 "(this handle has max_window > 64)");
   const int prof = h->profile;
   cudaError_t e;
-  if (prof && (e = record(h->ev[0], st)) != cudaSuccess) return cuda_fail(h, e, "profile event");
-  ebd_status s = run_lm(h, a, st);
-  if (s != EBD_OK) return s;
-  if (prof && (e = record(h->ev[1], st)) != cudaSuccess) return cuda_fail(h, e, "profile event");
   float* conf = a->conf ? a->conf : const_cast<float*>(h->seqp.conf);
   float* entn = a->ent_norm ? a->ent_norm : const_cast<float*>(h->seqp.ent_norm);
   float* gap = a->gap ? a->gap : const_cast<float*>(h->seqp.gap);
   int* arg = a->argmax ? a->argmax : const_cast<int*>(h->seqp.argmax);
+  const SeqParams sp = seq_params(h, a, conf, entn, gap, arg);
+  // the decision's scratch reset first: from the LM head on, every kernel is
+  // a programmatic dependent of the one before it (unless profiled)
+  if ((e = launch_decide_seq_init(sp, st)) != cudaSuccess) return cuda_fail(h, e, "decision reset");
+  if (prof && (e = record(h->ev[0], st)) != cudaSuccess) return cuda_fail(h, e, "profile event");
+  ebd_status s = run_lm(h, a, st);
+  if (s != EBD_OK) return s;
+  if (prof && (e = record(h->ev[1], st)) != cudaSuccess) return cuda_fail(h, e, "profile event");
   const float inv = static_cast<float>(1.0 / std::log(static_cast<double>(h->cfg.vocab)));
   if ((e = launch_merge_stats(h->part_f, h->part_i, a->rows, h->grid_lm, h->cfg.vocab, inv, conf,
-                              a->entropy, entn, gap, arg, h->d_status, st)) != cudaSuccess)
+                              a->entropy, entn, gap, arg, h->d_status, st, prof == 0)) != cudaSuccess)
     return cuda_fail(h, e, "merge launch");
-  if ((e = launch_decide_seq(seq_params(h, a, conf, entn, gap, arg), st)) != cudaSuccess)
-    return cuda_fail(h, e, "decision launch");
+  if ((e = launch_decide_seq(sp, st, true)) != cudaSuccess) return cuda_fail(h, e, "decision launch");
   if (prof && (e = record(h->ev[2], st)) != cudaSuccess) return cuda_fail(h, e, "profile event");
   if (prof && (e = record(h->ev[3], st)) != cudaSuccess) return cuda_fail(h, e, "profile event");
   h->prof_mode = prof;
@@ -1269,8 +1272,9 @@ ebd_status ebd_decide(ebd_handle* h, const ebd_step_args* a, void* stream) {
   if (h->w_emb == nullptr) return fail(h, EBD_ERR_STATE, "bind the token embedding first");
   if (a->rows == 0 || a->batch == 0) return EBD_OK;
   if (seq_mode(h)) {
-    cudaError_t e = launch_decide_seq(seq_params(h, a, a->conf, a->ent_norm, a->gap, a->argmax),
-                                      static_cast<cudaStream_t>(stream));
+    const SeqParams sp = seq_params(h, a, a->conf, a->ent_norm, a->gap, a->argmax);
+    cudaError_t e = launch_decide_seq_init(sp, static_cast<cudaStream_t>(stream));
+    if (e == cudaSuccess) e = launch_decide_seq(sp, static_cast<cudaStream_t>(stream), false);
     if (e != cudaSuccess) return cuda_fail(h, e, "decision launch");
     return EBD_OK;
   }

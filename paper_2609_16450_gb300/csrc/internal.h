@@ -175,7 +175,11 @@ cudaError_t launch_attention(const CUtensorMap& kc, const CUtensorMap& vc, const
                              bool pdl = false);
 cudaError_t launch_decide(const DecideParams& p, cudaStream_t st);
 // the grid-wide decision: a chain of kernels on `st` (k_decide_seq.cu)
-cudaError_t launch_decide_seq(const SeqParams& p, cudaStream_t st);
+// the grid-wide decision: the scratch reset (before the LM head, so that the
+// chain from the LM head on is unbroken), then the kernel chain; pdl_first:
+// its first kernel is a programmatic dependent of the kernel before it
+cudaError_t launch_decide_seq_init(const SeqParams& p, cudaStream_t st);
+cudaError_t launch_decide_seq(const SeqParams& p, cudaStream_t st, bool pdl_first);
 // prefix-cache append on commit: window row r of sequence b with mask[r] == 0
 // is copied (K and V, Hkv * D bf16 each) to cache position row_pos[r] < Pmax
 cudaError_t launch_kv_append(uint16_t* k_cache, uint16_t* v_cache, const uint16_t* k_win,

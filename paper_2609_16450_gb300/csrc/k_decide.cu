@@ -1171,6 +1171,10 @@ __global__ void __launch_bounds__(256) merge_stats_kernel(const float4* __restri
                                                           float* conf, float* entropy,
                                                           float* ent_norm, float* gap, int* argmax,
                                                           int* status) {
+  // as a programmatic dependent of the LM head: its partial states are read
+  // only after its grid completed; the grid-wide decision's chain follows
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   const int lane = threadIdx.x & 31;
   const int r = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
   if (r >= rows) return;
@@ -1203,10 +1207,18 @@ __global__ void __launch_bounds__(256) merge_stats_kernel(const float4* __restri
 
 cudaError_t launch_merge_stats(const float4* part_f, const int* part_i, int rows, int grid, int V,
                                float inv_log_v, float* conf, float* entropy, float* ent_norm,
-                               float* gap, int* argmax, int* status, cudaStream_t st) {
-  merge_stats_kernel<<<(rows + 7) / 8, 256, 0, st>>>(part_f, part_i, rows, grid, V, inv_log_v, conf,
-                                                    entropy, ent_norm, gap, argmax, status);
-  return cudaGetLastError();
+                               float* gap, int* argmax, int* status, cudaStream_t st, bool pdl) {
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = dim3(static_cast<unsigned>((rows + 7) / 8));
+  cfg.blockDim = dim3(256);
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, merge_stats_kernel, part_f, part_i, rows, grid, V, inv_log_v, conf,
+                            entropy, ent_norm, gap, argmax, status);
 }
 
 cudaError_t decide_configure() {

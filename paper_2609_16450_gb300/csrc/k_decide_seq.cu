@@ -43,6 +43,22 @@ constexpr int kSqNM = 0, kSqRunLbs = 1, kSqNBM = 2, kSqMetaB = 3, kSqMetaS = 4, 
 // step-wide flags after the per-sequence state: sq[8 * B + kFlagAnyLbs]
 constexpr int kFlagAnyLbs = 0;
 
+// Every kernel of the chain below is launched as a programmatic dependent of
+// the one before it.  It waits for that grid's completion (and the
+// visibility of its writes) before anything else (seq_wait), so each grid
+// completes only after the one before it did.  The per-row and per-sequence
+// kernels then let the next grid be scheduled at once (seq_release), which
+// hides its launch behind their run; the LBS GEMM and attention kernels,
+// which fill the SMs, release it only when they have no work (no LBS in the
+// step), else by exiting: the next grid's waiting CTAs would take slots their
+// own CTAs need (measured at 512 rows, step with the LBS / inside a block:
+// releasing at entry everywhere 605 / 473 us, nowhere 582.5 / 482.5 us, as
+// here 578 / 477 us).
+__device__ __forceinline__ void seq_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void seq_release() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
 __device__ __forceinline__ float gelu_f(float x) {
   return 0.5f * x * (1.0f + erff(x * 0.70710678118654752f));
 }
@@ -70,6 +86,31 @@ __device__ __forceinline__ void matvec(const float (&x)[NI], const float* __rest
       for (int o = 0; o < NO; ++o) y[o] = fmaf(xk, __ldg(w + 32 * o), y[o]);
     }
   }
+}
+
+// The same with W and b in shared memory (plain loads).
+template <int NI, int NO>
+__device__ __forceinline__ void matvec_s(const float (&x)[NI], const float* W, const float* b,
+                                         float (&y)[NO]) {
+  const int lane = threadIdx.x & 31;
+#pragma unroll
+  for (int o = 0; o < NO; ++o) y[o] = b[lane + 32 * o];
+#pragma unroll
+  for (int i = 0; i < NI; ++i) {
+#pragma unroll 8
+    for (int kk = 0; kk < 32; ++kk) {
+      const float xk = __shfl_sync(0xffffffffu, x[i], kk);
+      const float* w = W + (32 * i + kk) * (32 * NO) + lane;
+#pragma unroll
+      for (int o = 0; o < NO; ++o) y[o] = fmaf(xk, w[32 * o], y[o]);
+    }
+  }
+}
+
+// Copies n floats of the weight image from offset `off` into shared memory
+// (the whole CTA; the caller synchronises).
+__device__ __forceinline__ void stage(float* dst, const float* __restrict__ w, int off, int n) {
+  for (int i = threadIdx.x; i < n; i += blockDim.x) dst[i] = __ldg(w + off + i);
 }
 
 // LayerNorm (eps 1e-5) of a warp-spread vector of 32 * N values
@@ -108,6 +149,8 @@ __device__ __forceinline__ int block_rank(bool flag, int* warp_tot, int* total) 
 
 // ------------------------------------------------------------------ prep
 __global__ void __launch_bounds__(kSeqThreads) seq_prep_kernel(const SeqParams p) {
+  seq_wait();
+  seq_release();
   __shared__ int warp_tot[kSeqThreads / 32];
   const int b = blockIdx.x, j = threadIdx.x;
   const int r0 = p.cu_rows[b], r1 = p.cu_rows[b + 1];
@@ -302,6 +345,8 @@ __device__ __forceinline__ bool any_lbs(const SeqParams& p) {
 // F_ent hidden (Linear 1 -> 64, GELU) of H~ -> U[r][0..64), and the token
 // branch W_tok W_e[x_hat] + b (folded table) -> X[r][64..128)  (Eq. lbs_feat)
 __global__ void __launch_bounds__(256) lbs_pre_kernel(const SeqParams p) {
+  seq_wait();
+  seq_release();
   const int lane = threadIdx.x & 31;
   const int r = lbs_row(p, blockIdx.x * kWarpsPerCta + (threadIdx.x >> 5));
   if (r < 0) return;
@@ -320,7 +365,11 @@ __global__ void __launch_bounds__(256) lbs_pre_kernel(const SeqParams p) {
 
 // e = LN(W_ent2 u + b) -> X[r][0..64)  (X lives in Z; U in A)
 __global__ void __launch_bounds__(256) lbs_ent2_kernel(const SeqParams p) {
-  if (!any_lbs(p)) return;
+  seq_wait();
+  if (!any_lbs(p)) {
+    seq_release();
+    return;
+  }
   const float* w = p.w;
   gemm_rows<2>(p.A, 128, 64, w + p.o.ent2_t, 64, p.R, [&](int r, float (&acc)[2], int) {
     const int lane = threadIdx.x & 31;
@@ -336,7 +385,11 @@ __global__ void __launch_bounds__(256) lbs_ent2_kernel(const SeqParams p) {
 // z = W_combine [e; t] + b + E_pos[rank], in place in Z: a CTA owns all 128
 // columns of its rows and has read them before its epilogue
 __global__ void __launch_bounds__(256) lbs_comb_kernel(const SeqParams p) {
-  if (!any_lbs(p)) return;
+  seq_wait();
+  if (!any_lbs(p)) {
+    seq_release();
+    return;
+  }
   const float* w = p.w;
   gemm_rows<4>(p.Z, 128, 128, w + p.o.comb_t, 128, p.R, [&](int r, float (&acc)[4], int) {
     const int lane = threadIdx.x & 31;
@@ -351,7 +404,11 @@ __global__ void __launch_bounds__(256) lbs_comb_kernel(const SeqParams p) {
 }
 
 __global__ void __launch_bounds__(256) lbs_qkv_kernel(const SeqParams p, int l) {
-  if (!any_lbs(p)) return;
+  seq_wait();
+  if (!any_lbs(p)) {
+    seq_release();
+    return;
+  }
   const SeqLayer& L = p.o.l[l];
   const float* bq = p.w + L.qkv_b;
   gemm_rows<1>(p.Z, 128, 128, p.w + L.qkv_t, 384, p.R, [&](int r, float (&acc)[1], int col0) {
@@ -363,18 +420,24 @@ __global__ void __launch_bounds__(256) lbs_qkv_kernel(const SeqParams p, int l) 
 // LBS attention: CTA (x, h, b) takes 8 NQ queries of sequence b's M
 // (rank 8 NQ x + NQ w + i for warp w, i < NQ) and head h.  Blocks of 64
 // keys (k and v of head h) are staged in shared memory once for the 8
-// warps; 8 lanes share a key (4 dimensions each), 4 keys per step, with a
-// running max and sum per (query, lane group), merged at the end.
+// warps, double-buffered (the next block's loads are in flight while the
+// current one is used); 8 lanes share a key (4 dimensions each), 4 keys per
+// step, with a running max and sum per (query, lane group), merged at the end.
 constexpr int kAttnKB = 64;
 template <int NQ>
 __global__ void __launch_bounds__(256) lbs_attn_kernel(const SeqParams p) {
+  seq_wait();
   constexpr int kAttnQB = 8 * NQ;
-  __shared__ __align__(16) float Ks[kAttnKB][32];
-  __shared__ __align__(16) float Vs[kAttnKB][32];
+  __shared__ __align__(16) float Ks[2][kAttnKB][32];
+  __shared__ __align__(16) float Vs[2][kAttnKB][32];
+  static_assert(kAttnKB * 16 == 4 * 256, "four float4 of a key block per thread");
   const int b = blockIdx.z, h = blockIdx.y, qb = blockIdx.x;
   const int* sq = p.sq + 8 * b;
   const int nM = sq[kSqNM];
-  if (!sq[kSqRunLbs] || qb * kAttnQB >= nM) return;  // uniform over the CTA
+  if (!sq[kSqRunLbs] || qb * kAttnQB >= nM) {  // uniform over the CTA
+    seq_release();
+    return;
+  }
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31, grp = lane >> 3, sub = lane & 7;
   const int* rows = p.mrows + p.cu_rows[b];
   int qr[NQ];
@@ -391,24 +454,36 @@ __global__ void __launch_bounds__(256) lbs_attn_kernel(const SeqParams p) {
     l[i] = 0.f;
   }
   const float scale = rsqrtf(32.0f);
-  for (int kb = 0; kb < nM; kb += kAttnKB) {
-    __syncthreads();
-    for (int it = tid; it < kAttnKB * 16; it += 256) {
-      const int key = it >> 4, part = it & 15, c4 = part & 7;
+  float4 pre[4];
+  auto fetch = [&](int kb) {  // item it: key it / 16, float4 it % 8 of k (it % 16 < 8) or v
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int it = tid + 256 * u, key = it >> 4, part = it & 15, c4 = part & 7;
       const int kidx = kb + key;
-      float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
-      if (kidx < nM)
-        v = *reinterpret_cast<const float4*>(p.QKV + static_cast<size_t>(rows[kidx]) * 384 +
-                                             (part < 8 ? 128 : 256) + 32 * h + 4 * c4);
-      *reinterpret_cast<float4*>(part < 8 ? &Ks[key][4 * c4] : &Vs[key][4 * c4]) = v;
+      pre[u] = kidx < nM ? *reinterpret_cast<const float4*>(p.QKV + static_cast<size_t>(rows[kidx]) * 384 +
+                                                            (part < 8 ? 128 : 256) + 32 * h + 4 * c4)
+                         : make_float4(0.f, 0.f, 0.f, 0.f);
     }
-    __syncthreads();
+  };
+  auto put = [&](int buf) {
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int it = tid + 256 * u, key = it >> 4, part = it & 15, c4 = part & 7;
+      *reinterpret_cast<float4*>(part < 8 ? &Ks[buf][key][4 * c4] : &Vs[buf][key][4 * c4]) = pre[u];
+    }
+  };
+  fetch(0);
+  put(0);
+  __syncthreads();
+  for (int kb = 0, buf = 0; kb < nM; kb += kAttnKB, buf ^= 1) {
+    const bool more = kb + kAttnKB < nM;
+    if (more) fetch(kb + kAttnKB);
     const int nk = min(kAttnKB, nM - kb);
     for (int k0 = 0; k0 < nk; k0 += 4) {
       const int k = k0 + grp;
       const bool ok = k < nk;
-      const float4 kv = *reinterpret_cast<const float4*>(&Ks[k][4 * sub]);
-      const float4 vv = *reinterpret_cast<const float4*>(&Vs[k][4 * sub]);
+      const float4 kv = *reinterpret_cast<const float4*>(&Ks[buf][k][4 * sub]);
+      const float4 vv = *reinterpret_cast<const float4*>(&Vs[buf][k][4 * sub]);
       float s[NQ];
 #pragma unroll
       for (int i = 0; i < NQ; ++i) s[i] = q[i].x * kv.x + q[i].y * kv.y + q[i].z * kv.z + q[i].w * kv.w;
@@ -429,6 +504,8 @@ __global__ void __launch_bounds__(256) lbs_attn_kernel(const SeqParams p) {
         m[i] = mn;
       }
     }
+    if (more) put(buf ^ 1);  // the buffer every warp finished with before the last barrier
+    __syncthreads();
   }
 #pragma unroll
   for (int i = 0; i < NQ; ++i) {
@@ -456,7 +533,11 @@ __global__ void __launch_bounds__(256) lbs_attn_kernel(const SeqParams p) {
 
 // z = LN1(z + W_out a + b), in place (post-norm layer)
 __global__ void __launch_bounds__(256) lbs_out_kernel(const SeqParams p, int l) {
-  if (!any_lbs(p)) return;
+  seq_wait();
+  if (!any_lbs(p)) {
+    seq_release();
+    return;
+  }
   const SeqLayer& L = p.o.l[l];
   const float* w = p.w;
   gemm_rows<4>(p.A, 128, 128, w + L.out_t, 128, p.R, [&](int r, float (&acc)[4], int) {
@@ -474,7 +555,11 @@ __global__ void __launch_bounds__(256) lbs_out_kernel(const SeqParams p, int l) 
 
 // h = GELU(W_1 z + b_1) -> the QKV scratch (256 of its 384 columns)
 __global__ void __launch_bounds__(256) lbs_ff1_kernel(const SeqParams p, int l) {
-  if (!any_lbs(p)) return;
+  seq_wait();
+  if (!any_lbs(p)) {
+    seq_release();
+    return;
+  }
   const SeqLayer& L = p.o.l[l];
   const float* b1 = p.w + L.ff1_b;
   gemm_rows<1>(p.Z, 128, 128, p.w + L.ff1_t, 256, p.R, [&](int r, float (&acc)[1], int col0) {
@@ -486,7 +571,11 @@ __global__ void __launch_bounds__(256) lbs_ff1_kernel(const SeqParams p, int l) 
 // z = LN2(z + W_2 h + b_2), in place; after the last layer the LBS head
 // O = w . z + b
 __global__ void __launch_bounds__(256) lbs_ff2_kernel(const SeqParams p, int l) {
-  if (!any_lbs(p)) return;
+  seq_wait();
+  if (!any_lbs(p)) {
+    seq_release();
+    return;
+  }
   const SeqLayer& L = p.o.l[l];
   const float* w = p.w;
   gemm_rows<4>(p.QKV, 384, 256, w + L.ff2_t, 128, p.R, [&](int r, float (&acc)[4], int) {
@@ -514,6 +603,8 @@ __global__ void __launch_bounds__(256) lbs_ff2_kernel(const SeqParams p, int l) 
 // B of each sequence (App. E algorithm, block selection; Readings R8, R9),
 // then B n M in ascending position and the LPS features (Reading R13)
 __global__ void __launch_bounds__(kSeqThreads) seq_select_kernel(const SeqParams p) {
+  seq_wait();
+  seq_release();
   __shared__ int warp_tot[kSeqThreads / 32];
   __shared__ int cpos[kMaxSeqRows];
   __shared__ int s_cut, s_first;
@@ -589,6 +680,8 @@ __global__ void __launch_bounds__(kSeqThreads) seq_select_kernel(const SeqParams
 // ------------------------------------------------------------------ LPS
 // Linear(5 -> 32), LayerNorm, GELU
 __global__ void __launch_bounds__(256) lps_in_kernel(const SeqParams p) {
+  seq_wait();
+  seq_release();
   const int lane = threadIdx.x & 31;
   const int r = lps_row(p, blockIdx.x * kWarpsPerCta + (threadIdx.x >> 5));
   if (r < 0) return;
@@ -601,20 +694,33 @@ __global__ void __launch_bounds__(256) lps_in_kernel(const SeqParams p) {
   p.Zp[static_cast<size_t>(r) * 32 + lane] = gelu_f(y[0]);
 }
 
-// pre-norm block: LN1 and QKV
+// pre-norm block: LN1 and QKV.  The LPS kernels run one warp per row of
+// B n M; a CTA with any such row stages the block's weights in shared
+// memory first (a few KB, read once from L2 instead of once per row).
 __global__ void __launch_bounds__(256) lps_qkv_kernel(const SeqParams p, int l) {
+  seq_wait();
+  seq_release();
+  __shared__ float s_ln[64], s_qkv[32 * 96], s_qkvb[96];
   const int lane = threadIdx.x & 31;
   const int r = lps_row(p, blockIdx.x * kWarpsPerCta + (threadIdx.x >> 5));
-  if (r < 0) return;
+  if (!__syncthreads_or(r >= 0)) return;  // uniform over the CTA
   const SeqBlock& L = p.o.p[l];
+  stage(s_ln, p.w, L.ln1_g, 32);
+  stage(s_ln + 32, p.w, L.ln1_b, 32);
+  stage(s_qkv, p.w, L.qkv_t, 32 * 96);
+  stage(s_qkvb, p.w, L.qkv_b, 96);
+  __syncthreads();
+  if (r < 0) return;
   float y[1] = {p.Zp[static_cast<size_t>(r) * 32 + lane]}, q[3];
-  layer_norm_w<1>(y, p.w + L.ln1_g, p.w + L.ln1_b);
-  matvec<1, 3>(y, p.w + L.qkv_t, p.w + L.qkv_b, q);
+  layer_norm_w<1>(y, s_ln, s_ln + 32);
+  matvec_s<1, 3>(y, s_qkv, s_qkvb, q);
 #pragma unroll
   for (int i = 0; i < 3; ++i) p.QKVp[static_cast<size_t>(r) * 96 + lane + 32 * i] = q[i];
 }
 
 __global__ void __launch_bounds__(256) lps_attn_kernel(const SeqParams p) {
+  seq_wait();
+  seq_release();
   const int lane = threadIdx.x & 31;
   const int wid = blockIdx.x * kWarpsPerCta + (threadIdx.x >> 5);
   const int r = lps_row(p, wid >> 2), h = wid & 3;
@@ -630,20 +736,37 @@ __global__ void __launch_bounds__(256) lps_attn_kernel(const SeqParams p) {
 // output projection + residual, LN2, FFN + residual; after the last block
 // the head and p_psi = sigmoid(O_psi)
 __global__ void __launch_bounds__(256) lps_out_ffn_kernel(const SeqParams p, int l) {
+  seq_wait();
+  seq_release();
+  __shared__ float s_out[32 * 32], s_ff1[32 * 64], s_ff2[64 * 32], s_vec[32 * 4 + 64];
   const int lane = threadIdx.x & 31;
   const int r = lps_row(p, blockIdx.x * kWarpsPerCta + (threadIdx.x >> 5));
-  if (r < 0) return;
+  if (!__syncthreads_or(r >= 0)) return;  // uniform over the CTA
   const SeqBlock& L = p.o.p[l];
   const float* w = p.w;
+  float* s_outb = s_vec;
+  float* s_ln2 = s_vec + 32;  // gamma, beta
+  float* s_ff2b = s_vec + 96;
+  float* s_ff1b = s_vec + 128;
+  stage(s_out, w, L.out_t, 32 * 32);
+  stage(s_ff1, w, L.ff1_t, 32 * 64);
+  stage(s_ff2, w, L.ff2_t, 64 * 32);
+  stage(s_outb, w, L.out_b, 32);
+  stage(s_ln2, w, L.ln2_g, 32);
+  stage(s_ln2 + 32, w, L.ln2_b, 32);
+  stage(s_ff2b, w, L.ff2_b, 32);
+  stage(s_ff1b, w, L.ff1_b, 64);
+  __syncthreads();
+  if (r < 0) return;
   float a[1] = {p.Ap[static_cast<size_t>(r) * 32 + lane]}, y[1], z = p.Zp[static_cast<size_t>(r) * 32 + lane];
-  matvec<1, 1>(a, w + L.out_t, w + L.out_b, y);
+  matvec_s<1, 1>(a, s_out, s_outb, y);
   z += y[0];
   float t[1] = {z}, hdn[2], f[1];
-  layer_norm_w<1>(t, w + L.ln2_g, w + L.ln2_b);
-  matvec<1, 2>(t, w + L.ff1_t, w + L.ff1_b, hdn);
+  layer_norm_w<1>(t, s_ln2, s_ln2 + 32);
+  matvec_s<1, 2>(t, s_ff1, s_ff1b, hdn);
   hdn[0] = gelu_f(hdn[0]);
   hdn[1] = gelu_f(hdn[1]);
-  matvec<2, 1>(hdn, w + L.ff2_t, w + L.ff2_b, f);
+  matvec_s<2, 1>(hdn, s_ff2, s_ff2b, f);
   z += f[0];
   p.Zp[static_cast<size_t>(r) * 32 + lane] = z;
   if (l == 1) {
@@ -656,6 +779,8 @@ __global__ void __launch_bounds__(256) lps_out_ffn_kernel(const SeqParams p, int
 // union accept (Reading R14), anti-stall fallback, parallel commit, block
 // resolution; the baselines' rules (Reading R20) in their modes
 __global__ void __launch_bounds__(kSeqThreads) seq_accept_kernel(const SeqParams p) {
+  seq_wait();
+  seq_release();
   __shared__ float s_conf[kMaxSeqRows];
   __shared__ int s_pos[kMaxSeqRows];
   __shared__ int s_any, s_best, s_open;
@@ -728,15 +853,39 @@ __global__ void __launch_bounds__(kSeqThreads) seq_accept_kernel(const SeqParams
 
 }  // namespace
 
-cudaError_t launch_decide_seq(const SeqParams& p, cudaStream_t st) {
+namespace {
+template <typename... KArgs, typename... Args>
+cudaError_t chain(void (*k)(KArgs...), dim3 grid, dim3 block, cudaStream_t st, bool pdl, Args... args) {
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, k, args...);
+}
+}  // namespace
+
+cudaError_t launch_decide_seq_init(const SeqParams& p, cudaStream_t st) {
   if (p.B <= 0 || p.R <= 0) return cudaSuccess;
   cudaError_t e;
   if ((e = cudaMemsetAsync(p.mrank, 0xff, static_cast<size_t>(p.R) * sizeof(int), st)) != cudaSuccess) return e;
   if ((e = cudaMemsetAsync(p.bmrank, 0xff, static_cast<size_t>(p.R) * sizeof(int), st)) != cudaSuccess) return e;
-  if ((e = cudaMemsetAsync(p.sq + 8 * p.B, 0, 8 * sizeof(int), st)) != cudaSuccess) return e;
+  return cudaMemsetAsync(p.sq + 8 * p.B, 0, 8 * sizeof(int), st);
+}
+
+cudaError_t launch_decide_seq(const SeqParams& p, cudaStream_t st, bool pdl_first) {
+  if (p.B <= 0 || p.R <= 0) return cudaSuccess;
   const unsigned rows_grid = static_cast<unsigned>((p.R + kWarpsPerCta - 1) / kWarpsPerCta);
   const unsigned head_grid = static_cast<unsigned>((4 * p.R + kWarpsPerCta - 1) / kWarpsPerCta);
-  seq_prep_kernel<<<p.B, kSeqThreads, 0, st>>>(p);
+  const dim3 t256(256), tseq(kSeqThreads);
+  cudaError_t e = chain(seq_prep_kernel, dim3(p.B), tseq, st, pdl_first, p);
+  auto add = [&](cudaError_t x) {
+    if (e == cudaSuccess) e = x;
+  };
   if (p.mode == EBD_DECODE_EB) {
     const unsigned tiles = static_cast<unsigned>((p.R + kGemmRows - 1) / kGemmRows);
     // queries per warp; measured at 512 rows (384 masked): 1 -> 656 us per
@@ -745,33 +894,33 @@ cudaError_t launch_decide_seq(const SeqParams& p, cudaStream_t st) {
     if (const char* env = getenv("EBD_SEQ_ATTN_NQ")) nq = atoi(env);
     nq = nq == 2 || nq == 4 ? nq : 1;
     const dim3 attn_grid(kMaxSeqRows / (8 * nq), 4, static_cast<unsigned>(p.B));
-    lbs_pre_kernel<<<rows_grid, 256, 0, st>>>(p);
-    lbs_ent2_kernel<<<dim3(tiles, 1), 256, 0, st>>>(p);
-    lbs_comb_kernel<<<dim3(tiles, 1), 256, 0, st>>>(p);
+    add(chain(lbs_pre_kernel, dim3(rows_grid), t256, st, true, p));
+    add(chain(lbs_ent2_kernel, dim3(tiles, 1), t256, st, true, p));
+    add(chain(lbs_comb_kernel, dim3(tiles, 1), t256, st, true, p));
     for (int l = 0; l < 2; ++l) {
-      lbs_qkv_kernel<<<dim3(tiles, 12), 256, 0, st>>>(p, l);
+      add(chain(lbs_qkv_kernel, dim3(tiles, 12), t256, st, true, p, l));
       if (nq == 1)
-        lbs_attn_kernel<1><<<attn_grid, 256, 0, st>>>(p);
+        add(chain(lbs_attn_kernel<1>, attn_grid, t256, st, true, p));
       else if (nq == 4)
-        lbs_attn_kernel<4><<<attn_grid, 256, 0, st>>>(p);
+        add(chain(lbs_attn_kernel<4>, attn_grid, t256, st, true, p));
       else
-        lbs_attn_kernel<2><<<attn_grid, 256, 0, st>>>(p);
-      lbs_out_kernel<<<dim3(tiles, 1), 256, 0, st>>>(p, l);
-      lbs_ff1_kernel<<<dim3(tiles, 8), 256, 0, st>>>(p, l);
-      lbs_ff2_kernel<<<dim3(tiles, 1), 256, 0, st>>>(p, l);
+        add(chain(lbs_attn_kernel<2>, attn_grid, t256, st, true, p));
+      add(chain(lbs_out_kernel, dim3(tiles, 1), t256, st, true, p, l));
+      add(chain(lbs_ff1_kernel, dim3(tiles, 8), t256, st, true, p, l));
+      add(chain(lbs_ff2_kernel, dim3(tiles, 1), t256, st, true, p, l));
     }
   }
-  seq_select_kernel<<<p.B, kSeqThreads, 0, st>>>(p);
+  add(chain(seq_select_kernel, dim3(p.B), tseq, st, true, p));
   if (p.mode == EBD_DECODE_EB && p.lps_enabled) {
-    lps_in_kernel<<<rows_grid, 256, 0, st>>>(p);
+    add(chain(lps_in_kernel, dim3(rows_grid), t256, st, true, p));
     for (int l = 0; l < 2; ++l) {
-      lps_qkv_kernel<<<rows_grid, 256, 0, st>>>(p, l);
-      lps_attn_kernel<<<head_grid, 256, 0, st>>>(p);
-      lps_out_ffn_kernel<<<rows_grid, 256, 0, st>>>(p, l);
+      add(chain(lps_qkv_kernel, dim3(rows_grid), t256, st, true, p, l));
+      add(chain(lps_attn_kernel, dim3(head_grid), t256, st, true, p));
+      add(chain(lps_out_ffn_kernel, dim3(rows_grid), t256, st, true, p, l));
     }
   }
-  seq_accept_kernel<<<p.B, kSeqThreads, 0, st>>>(p);
-  return cudaGetLastError();
+  add(chain(seq_accept_kernel, dim3(p.B), tseq, st, true, p));
+  return e;
 }
 
 }  // namespace ebd
