@@ -417,43 +417,50 @@ __global__ void __launch_bounds__(256) lbs_qkv_kernel(const SeqParams p, int l) 
   });
 }
 
-// LBS attention: CTA (x, h, b) takes 8 NQ queries of sequence b's M
-// (rank 8 NQ x + NQ w + i for warp w, i < NQ) and head h.  Blocks of 64
-// keys (k and v of head h) are staged in shared memory once for the 8
-// warps, double-buffered (the next block's loads are in flight while the
-// current one is used); 8 lanes share a key (4 dimensions each), 4 keys per
-// step, with a running max and sum per (query, lane group), merged at the end.
+// LBS attention: CTA (x, h, b) takes 8 queries of sequence b's M (rank
+// 8 x + w for warp w) and head h (32 dimensions).  Blocks of 64 keys (k and
+// v of head h) are staged in shared memory once for the 8 warps,
+// double-buffered (the next block's loads are in flight while the current
+// one is used), rows padded to 33 floats so that 32 lanes reading 32
+// different rows hit 32 banks.  Each lane of a warp takes whole keys: the
+// full 32-dimension score, then its own running max, sum and output row
+// (no shuffles per key).  At the end the lanes' states are merged: the
+// common max, then a reduce-scatter of the 32 output dimensions that leaves
+// dimension d in lane d.
 constexpr int kAttnKB = 64;
-template <int NQ>
+constexpr int kAttnLd = 33;
 __global__ void __launch_bounds__(256) lbs_attn_kernel(const SeqParams p) {
   seq_wait();
-  constexpr int kAttnQB = 8 * NQ;
-  __shared__ __align__(16) float Ks[2][kAttnKB][32];
-  __shared__ __align__(16) float Vs[2][kAttnKB][32];
+  __shared__ float Ks[2][kAttnKB][kAttnLd];
+  __shared__ float Vs[2][kAttnKB][kAttnLd];
   static_assert(kAttnKB * 16 == 4 * 256, "four float4 of a key block per thread");
   const int b = blockIdx.z, h = blockIdx.y, qb = blockIdx.x;
   const int* sq = p.sq + 8 * b;
   const int nM = sq[kSqNM];
-  if (!sq[kSqRunLbs] || qb * kAttnQB >= nM) {  // uniform over the CTA
+  if (!sq[kSqRunLbs] || qb * 8 >= nM) {  // uniform over the CTA
     seq_release();
     return;
   }
-  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31, grp = lane >> 3, sub = lane & 7;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int* rows = p.mrows + p.cu_rows[b];
-  int qr[NQ];
-  float4 q[NQ], o[NQ];
-  float m[NQ], l[NQ];
+  const int qi = qb * 8 + warp;
+  const int qr = qi < nM ? rows[qi] : -1;
+  float q[32], o[32];
+  {
+    const float* qp = p.QKV + static_cast<size_t>(qr >= 0 ? qr : rows[0]) * 384 + 32 * h;
+    const float scale = rsqrtf(32.0f);
 #pragma unroll
-  for (int i = 0; i < NQ; ++i) {
-    const int qi = qb * kAttnQB + warp * NQ + i;
-    qr[i] = qi < nM ? rows[qi] : -1;
-    q[i] = qr[i] >= 0 ? *reinterpret_cast<const float4*>(p.QKV + static_cast<size_t>(qr[i]) * 384 + 32 * h + 4 * sub)
-                      : make_float4(0.f, 0.f, 0.f, 0.f);
-    o[i] = make_float4(0.f, 0.f, 0.f, 0.f);
-    m[i] = -INFINITY;
-    l[i] = 0.f;
+    for (int d4 = 0; d4 < 8; ++d4) {
+      const float4 v = *reinterpret_cast<const float4*>(qp + 4 * d4);
+      q[4 * d4 + 0] = v.x * scale;
+      q[4 * d4 + 1] = v.y * scale;
+      q[4 * d4 + 2] = v.z * scale;
+      q[4 * d4 + 3] = v.w * scale;
+    }
   }
-  const float scale = rsqrtf(32.0f);
+#pragma unroll
+  for (int d = 0; d < 32; ++d) o[d] = 0.f;
+  float m = -INFINITY, l = 0.f;
   float4 pre[4];
   auto fetch = [&](int kb) {  // item it: key it / 16, float4 it % 8 of k (it % 16 < 8) or v
 #pragma unroll
@@ -469,7 +476,11 @@ __global__ void __launch_bounds__(256) lbs_attn_kernel(const SeqParams p) {
 #pragma unroll
     for (int u = 0; u < 4; ++u) {
       const int it = tid + 256 * u, key = it >> 4, part = it & 15, c4 = part & 7;
-      *reinterpret_cast<float4*>(part < 8 ? &Ks[buf][key][4 * c4] : &Vs[buf][key][4 * c4]) = pre[u];
+      float* dst = part < 8 ? &Ks[buf][key][4 * c4] : &Vs[buf][key][4 * c4];
+      dst[0] = pre[u].x;
+      dst[1] = pre[u].y;
+      dst[2] = pre[u].z;
+      dst[3] = pre[u].w;
     }
   };
   fetch(0);
@@ -479,56 +490,50 @@ __global__ void __launch_bounds__(256) lbs_attn_kernel(const SeqParams p) {
     const bool more = kb + kAttnKB < nM;
     if (more) fetch(kb + kAttnKB);
     const int nk = min(kAttnKB, nM - kb);
-    for (int k0 = 0; k0 < nk; k0 += 4) {
-      const int k = k0 + grp;
-      const bool ok = k < nk;
-      const float4 kv = *reinterpret_cast<const float4*>(&Ks[buf][k][4 * sub]);
-      const float4 vv = *reinterpret_cast<const float4*>(&Vs[buf][k][4 * sub]);
-      float s[NQ];
+#pragma unroll 1
+    for (int k0 = 0; k0 < nk; k0 += 32) {
+      const int k = k0 + lane;
+      if (k < nk) {
+        const float* kr = Ks[buf][k];
+        float s = 0.f;
 #pragma unroll
-      for (int i = 0; i < NQ; ++i) s[i] = q[i].x * kv.x + q[i].y * kv.y + q[i].z * kv.z + q[i].w * kv.w;
+        for (int d = 0; d < 32; ++d) s = fmaf(q[d], kr[d], s);
+        const float mn = fmaxf(m, s);
+        const float c = expf(m - mn), e = expf(s - mn);  // m = -inf first: c = 0
+        l = fmaf(l, c, e);
+        const float* vr = Vs[buf][k];
 #pragma unroll
-      for (int off = 1; off < 8; off <<= 1)
-#pragma unroll
-        for (int i = 0; i < NQ; ++i) s[i] += __shfl_xor_sync(0xffffffffu, s[i], off);
-#pragma unroll
-      for (int i = 0; i < NQ; ++i) {
-        const float si = ok ? s[i] * scale : -INFINITY;
-        const float mn = fmaxf(m[i], si);
-        const float c = mn == -INFINITY ? 1.f : expf(m[i] - mn), e = mn == -INFINITY ? 0.f : expf(si - mn);
-        l[i] = l[i] * c + e;
-        o[i].x = fmaf(e, vv.x, o[i].x * c);
-        o[i].y = fmaf(e, vv.y, o[i].y * c);
-        o[i].z = fmaf(e, vv.z, o[i].z * c);
-        o[i].w = fmaf(e, vv.w, o[i].w * c);
-        m[i] = mn;
+        for (int d = 0; d < 32; ++d) o[d] = fmaf(e, vr[d], o[d] * c);
+        m = mn;
       }
     }
     if (more) put(buf ^ 1);  // the buffer every warp finished with before the last barrier
     __syncthreads();
   }
+  // merge the 32 lanes: common max, then sums; lanes that saw no key hold
+  // m = -inf and contribute nothing
+  float M = m;
 #pragma unroll
-  for (int i = 0; i < NQ; ++i) {
-    float M = m[i];
+  for (int off = 16; off > 0; off >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
+  const float c = m == -INFINITY ? 0.f : expf(m - M);
+  l *= c;
 #pragma unroll
-    for (int off = 8; off < 32; off <<= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
-    const float c = m[i] == -INFINITY ? 0.f : expf(m[i] - M);
-    float li = l[i] * c;
-    float4 oi = make_float4(o[i].x * c, o[i].y * c, o[i].z * c, o[i].w * c);
+  for (int off = 16; off > 0; off >>= 1) l += __shfl_xor_sync(0xffffffffu, l, off);
 #pragma unroll
-    for (int off = 8; off < 32; off <<= 1) {
-      li += __shfl_xor_sync(0xffffffffu, li, off);
-      oi.x += __shfl_xor_sync(0xffffffffu, oi.x, off);
-      oi.y += __shfl_xor_sync(0xffffffffu, oi.y, off);
-      oi.z += __shfl_xor_sync(0xffffffffu, oi.z, off);
-      oi.w += __shfl_xor_sync(0xffffffffu, oi.w, off);
-    }
-    if (lane < 8 && qr[i] >= 0) {
-      const float il = 1.0f / li;
-      *reinterpret_cast<float4*>(p.A + static_cast<size_t>(qr[i]) * 128 + 32 * h + 4 * lane) =
-          make_float4(oi.x * il, oi.y * il, oi.z * il, oi.w * il);
+  for (int d = 0; d < 32; ++d) o[d] *= c;
+  // reduce-scatter: at offset `off` a lane keeps the half of its live
+  // values selected by (lane & off) and adds its partner's copy of it
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    const bool up = (lane & off) != 0;
+#pragma unroll
+    for (int i = 0; i < off; ++i) {
+      const float give = up ? o[i] : o[i + off];
+      const float keep = up ? o[i + off] : o[i];
+      o[i] = keep + __shfl_xor_sync(0xffffffffu, give, off);
     }
   }
+  if (qr >= 0) p.A[static_cast<size_t>(qr) * 128 + 32 * h + lane] = o[0] / l;
 }
 
 // z = LN1(z + W_out a + b), in place (post-norm layer)
@@ -888,23 +893,13 @@ cudaError_t launch_decide_seq(const SeqParams& p, cudaStream_t st, bool pdl_firs
   };
   if (p.mode == EBD_DECODE_EB) {
     const unsigned tiles = static_cast<unsigned>((p.R + kGemmRows - 1) / kGemmRows);
-    // queries per warp; measured at 512 rows (384 masked): 1 -> 656 us per
-    // step, 2 -> 664, 4 -> 693 (more CTAs beat more reuse of a staged block)
-    int nq = 1;
-    if (const char* env = getenv("EBD_SEQ_ATTN_NQ")) nq = atoi(env);
-    nq = nq == 2 || nq == 4 ? nq : 1;
-    const dim3 attn_grid(kMaxSeqRows / (8 * nq), 4, static_cast<unsigned>(p.B));
+    const dim3 attn_grid(kMaxSeqRows / 8, 4, static_cast<unsigned>(p.B));
     add(chain(lbs_pre_kernel, dim3(rows_grid), t256, st, true, p));
     add(chain(lbs_ent2_kernel, dim3(tiles, 1), t256, st, true, p));
     add(chain(lbs_comb_kernel, dim3(tiles, 1), t256, st, true, p));
     for (int l = 0; l < 2; ++l) {
       add(chain(lbs_qkv_kernel, dim3(tiles, 12), t256, st, true, p, l));
-      if (nq == 1)
-        add(chain(lbs_attn_kernel<1>, attn_grid, t256, st, true, p));
-      else if (nq == 4)
-        add(chain(lbs_attn_kernel<4>, attn_grid, t256, st, true, p));
-      else
-        add(chain(lbs_attn_kernel<2>, attn_grid, t256, st, true, p));
+      add(chain(lbs_attn_kernel, attn_grid, t256, st, true, p));
       add(chain(lbs_out_kernel, dim3(tiles, 1), t256, st, true, p, l));
       add(chain(lbs_ff1_kernel, dim3(tiles, 8), t256, st, true, p, l));
       add(chain(lbs_ff2_kernel, dim3(tiles, 1), t256, st, true, p, l));
