@@ -86,6 +86,9 @@ typedef int32_t ebd_status;
 /* debug_flags bits (tests only) */
 #define EBD_DEBUG_FORCE_TIMEOUT 1 /* LM-head kernel waits on a barrier that
                                      nothing completes, with a 20 ms limit */
+#define EBD_DEBUG_FORCE_COPY_TIMEOUT 2 /* ebd_step_host: the attention waits for
+                                     a copy-stream ticket that is never
+                                     written, with a 20 ms limit */
 
 typedef struct {
   /* backbone shapes */

@@ -20,6 +20,7 @@ EBD_ERR_TIMEOUT = -4
 EBD_ERR_NONFINITE = -5
 EBD_ERR_STATE = -6
 EBD_DEBUG_FORCE_TIMEOUT = 1
+EBD_DEBUG_FORCE_COPY_TIMEOUT = 2
 EBD_DECODE_EB = 0
 EBD_DECODE_THRESHOLD = 1
 EBD_DECODE_TOPM = 2

@@ -607,6 +607,10 @@ ebd_status run_attention(ebd_handle* h, const ebd_step_args* a, cudaStream_t st,
   p.wait_prior = wait_prior ? 1 : 0;
   p.ready = ready;
   p.ready_ticket = ready_ticket;
+  if (ready != nullptr && (c.debug_flags & EBD_DEBUG_FORCE_COPY_TIMEOUT)) {
+    p.ready_ticket = ready_ticket ^ 0x80000000u;  // never written
+    p.limit_ns = 20ull * 1000 * 1000;
+  }
   cudaError_t e = launch_attention(kc, vc, kw, vw, p, st, pdl);
   if (e != cudaSuccess) return cuda_fail(h, e, "attention launch");
   return EBD_OK;

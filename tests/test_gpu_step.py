@@ -241,6 +241,39 @@ def test_timeout_is_reported_and_context_survives():
     _check(sh, inp, gpu, res)
 
 
+def test_copy_stream_timeout_is_reported_and_context_survives():
+    """ebd_step_host from pinned buffers: q and the window K/V come in on the
+    copy stream and the attention waits, time-limited, for its ticket.  A
+    ticket that never comes gives EBD_ERR_TIMEOUT; the context stays usable."""
+    from paper_2609_16450_gb300 import _ebd as E
+    from paper_2609_16450_gb300 import runtime as rt
+    sh = synth.tiny
+    inp, w, h = _setup(sh)
+    hb = rt.Handle(rt.config_for(sh, debug_flags=E.EBD_DEBUG_FORCE_COPY_TIMEOUT), w.w_emb)
+    R = inp.rows
+    pin = lambda a: torch.from_numpy(np.ascontiguousarray(a)).pin_memory()  # noqa: E731
+    ds = rt.DeviceStep(inp, w)
+    host = dict(cu_rows=pin(inp.cu_rows.astype(np.int32)), prefix_len=pin(inp.prefix_len.astype(np.int32)),
+                row_pos=pin(inp.row_pos.astype(np.int32)), hidden=pin(inp.hidden.view(np.int16)),
+                q=pin(inp.q.view(np.int16)), k_win=pin(inp.k_win.view(np.int16)),
+                v_win=pin(inp.v_win.view(np.int16)), tokens=pin(inp.tokens.astype(np.int32)),
+                mask=pin(inp.mask.astype(np.uint8)), in_block=pin(inp.in_block.astype(np.uint8)),
+                blk_meta=pin(inp.blk_meta.astype(np.int32)),
+                attn_out=torch.empty((R, sh.n_heads_q, sh.head_dim), dtype=torch.float32).pin_memory())
+    a = E.ebd_step_args()
+    a.batch, a.rows = sh.batch, R
+    for k, t in host.items():
+        setattr(a, k, t.data_ptr())
+    a.k_cache, a.v_cache, a.w_lm = ds.k_cache.data_ptr(), ds.v_cache.data_ptr(), w.w_lm.data_ptr()
+    a.w_lm_layout = w.layout
+    E.check(E.ebd_step_host(hb.h, a, rt.stream_handle(None)), hb.h)
+    assert hb.sync_status() == E.EBD_ERR_TIMEOUT
+    hb.close()
+    gpu = _run(sh, inp, w, h)
+    res = _oracle(sh, inp)
+    _check(sh, inp, gpu, res)
+
+
 def test_overlapped_and_serial_and_graph_steps_agree():
     """The production order (attention as a programmatic dependent of the
     decision), the fully serial order and a CUDA-graph replay give identical
