@@ -206,7 +206,7 @@ struct ebd_handle {
   cudaEvent_t ev[4] = {nullptr, nullptr, nullptr, nullptr};
   int profile = 0;
   int prof_mode = 0, prof_attn = 0;  // what the last ebd_step recorded
-  // ebd_step_host: the attention's inputs on a copy engine (created at first use)
+  // ebd_step_host: the attention's inputs on a copy engine (set up with the handle)
   int copy_route = -1;               // -1 not set up yet, 0 unavailable, 1 ready
   cudaStream_t s_copy = nullptr;
   cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
@@ -215,6 +215,40 @@ struct ebd_handle {
 };
 
 namespace {
+
+typedef CUresult (*WriteValue32Fn)(CUstream, CUdeviceptr, cuuint32_t, unsigned int);
+WriteValue32Fn get_write_value() {
+  static WriteValue32Fn fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* ptr = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuStreamWriteValue32", &ptr, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<WriteValue32Fn>(ptr);
+  });
+  return fn;
+}
+
+// The copy stream, its two events and the ticket word; false where the
+// driver offers no stream write (the inputs then go with the others).
+bool copy_route_ready(ebd_handle* h) {
+  if (h->copy_route >= 0) return h->copy_route == 1;
+  h->copy_route = 0;
+  if (get_write_value() == nullptr) return false;
+  if (cudaStreamCreateWithFlags(&h->s_copy, cudaStreamNonBlocking) != cudaSuccess ||
+      cudaEventCreateWithFlags(&h->ev_fork, cudaEventDisableTiming) != cudaSuccess ||
+      cudaEventCreateWithFlags(&h->ev_join, cudaEventDisableTiming) != cudaSuccess ||
+      cudaMalloc(&h->d_ready, sizeof(unsigned)) != cudaSuccess ||
+      cudaMemsetAsync(h->d_ready, 0, sizeof(unsigned), h->s_copy) != cudaSuccess ||
+      cudaStreamSynchronize(h->s_copy) != cudaSuccess) {
+    (void)cudaGetLastError();
+    return false;
+  }
+  h->copy_route = 1;
+  return true;
+}
 
 ebd_status fail(ebd_handle* h, ebd_status code, const std::string& msg) {
   if (h) h->err = msg;
@@ -869,6 +903,9 @@ ebd_status ebd_create(const ebd_config* cfg, ebd_handle** out) {
     if ((e = cudaMalloc(&h->staging, bytes)) != cudaSuccess)
       return bail(cuda_fail(h, e, "cudaMalloc(staging)"));
   }
+  // the copy stream of ebd_step_host, set up here rather than at its first
+  // call, which may come while a stream is being captured into a graph
+  if (cfg->max_window <= kMaxWindow) (void)copy_route_ready(h);
   if (cfg->max_window > kMaxWindow) {  // scratch of the grid-wide decision
     const size_t R = cfg->max_rows, B = cfg->max_batch;
     size_t bytes = 0;
@@ -1094,39 +1131,6 @@ struct StepRoute {
   int* blk_meta_out;
 };
 
-typedef CUresult (*WriteValue32Fn)(CUstream, CUdeviceptr, cuuint32_t, unsigned int);
-WriteValue32Fn get_write_value() {
-  static WriteValue32Fn fn = nullptr;
-  static std::once_flag once;
-  std::call_once(once, [] {
-    void* ptr = nullptr;
-    cudaDriverEntryPointQueryResult q;
-    if (cudaGetDriverEntryPointByVersion("cuStreamWriteValue32", &ptr, 12000, cudaEnableDefault, &q) ==
-            cudaSuccess &&
-        q == cudaDriverEntryPointSuccess)
-      fn = reinterpret_cast<WriteValue32Fn>(ptr);
-  });
-  return fn;
-}
-
-// The copy stream, its two events and the ticket word; false where the
-// driver offers no stream write (the inputs then go with the others).
-bool copy_route_ready(ebd_handle* h) {
-  if (h->copy_route >= 0) return h->copy_route == 1;
-  h->copy_route = 0;
-  if (get_write_value() == nullptr) return false;
-  if (cudaStreamCreateWithFlags(&h->s_copy, cudaStreamNonBlocking) != cudaSuccess ||
-      cudaEventCreateWithFlags(&h->ev_fork, cudaEventDisableTiming) != cudaSuccess ||
-      cudaEventCreateWithFlags(&h->ev_join, cudaEventDisableTiming) != cudaSuccess ||
-      cudaMalloc(&h->d_ready, sizeof(unsigned)) != cudaSuccess ||
-      cudaMemsetAsync(h->d_ready, 0, sizeof(unsigned), h->s_copy) != cudaSuccess ||
-      cudaStreamSynchronize(h->s_copy) != cudaSuccess) {
-    (void)cudaGetLastError();
-    return false;
-  }
-  h->copy_route = 1;
-  return true;
-}
 }  // namespace
 
 namespace {
@@ -1368,7 +1372,11 @@ ebd_status ebd_step_host(ebd_handle* h, const ebd_step_args* a, void* stream) {
   uint8_t* acc = take(RM);
   int32_t* sfx = reinterpret_cast<int32_t*>(take(BM * 8));
   const bool route = !seq_mode(h);
-  const bool dma = route && attn && copy_route_ready(h);
+  // while `stream` is being captured into a graph the attention's inputs go
+  // with the others (one capture-safe path; replays take it too)
+  cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
+  if (cudaStreamIsCapturing(st, &cap) != cudaSuccess) (void)cudaGetLastError();
+  const bool dma = route && attn && cap == cudaStreamCaptureStatusNone && copy_route_ready(h);
   HostMover in{st, true};
   in.add(hid, a->hidden, R * d * 2);
   in.add(cu, a->cu_rows, (B + 1) * 4);

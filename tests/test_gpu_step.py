@@ -250,28 +250,69 @@ def test_copy_stream_timeout_is_reported_and_context_survives():
     sh = synth.tiny
     inp, w, h = _setup(sh)
     hb = rt.Handle(rt.config_for(sh, debug_flags=E.EBD_DEBUG_FORCE_COPY_TIMEOUT), w.w_emb)
-    R = inp.rows
-    pin = lambda a: torch.from_numpy(np.ascontiguousarray(a)).pin_memory()  # noqa: E731
     ds = rt.DeviceStep(inp, w)
-    host = dict(cu_rows=pin(inp.cu_rows.astype(np.int32)), prefix_len=pin(inp.prefix_len.astype(np.int32)),
-                row_pos=pin(inp.row_pos.astype(np.int32)), hidden=pin(inp.hidden.view(np.int16)),
-                q=pin(inp.q.view(np.int16)), k_win=pin(inp.k_win.view(np.int16)),
-                v_win=pin(inp.v_win.view(np.int16)), tokens=pin(inp.tokens.astype(np.int32)),
-                mask=pin(inp.mask.astype(np.uint8)), in_block=pin(inp.in_block.astype(np.uint8)),
-                blk_meta=pin(inp.blk_meta.astype(np.int32)),
-                attn_out=torch.empty((R, sh.n_heads_q, sh.head_dim), dtype=torch.float32).pin_memory())
-    a = E.ebd_step_args()
-    a.batch, a.rows = sh.batch, R
-    for k, t in host.items():
-        setattr(a, k, t.data_ptr())
-    a.k_cache, a.v_cache, a.w_lm = ds.k_cache.data_ptr(), ds.v_cache.data_ptr(), w.w_lm.data_ptr()
-    a.w_lm_layout = w.layout
+    host, a = _pinned_host_args(sh, inp, ds, w)
     E.check(E.ebd_step_host(hb.h, a, rt.stream_handle(None)), hb.h)
     assert hb.sync_status() == E.EBD_ERR_TIMEOUT
     hb.close()
     gpu = _run(sh, inp, w, h)
     res = _oracle(sh, inp)
     _check(sh, inp, gpu, res)
+
+
+def _pinned_host_args(sh, inp, ds, w):
+    R = inp.rows
+    pin = lambda a: torch.from_numpy(np.ascontiguousarray(a)).pin_memory()  # noqa: E731
+    host = dict(cu_rows=pin(inp.cu_rows.astype(np.int32)), prefix_len=pin(inp.prefix_len.astype(np.int32)),
+                row_pos=pin(inp.row_pos.astype(np.int32)), hidden=pin(inp.hidden.view(np.int16)),
+                q=pin(inp.q.view(np.int16)), k_win=pin(inp.k_win.view(np.int16)),
+                v_win=pin(inp.v_win.view(np.int16)), tokens=pin(inp.tokens.astype(np.int32)),
+                mask=pin(inp.mask.astype(np.uint8)), in_block=pin(inp.in_block.astype(np.uint8)),
+                blk_meta=pin(inp.blk_meta.astype(np.int32)),
+                attn_out=torch.empty((R, sh.n_heads_q, sh.head_dim), dtype=torch.float32).pin_memory(),
+                conf=torch.empty(R, dtype=torch.float32).pin_memory(),
+                argmax=torch.empty(R, dtype=torch.int32).pin_memory(),
+                accepted=torch.empty(R, dtype=torch.uint8).pin_memory())
+    from paper_2609_16450_gb300 import _ebd as E
+    a = E.ebd_step_args()
+    a.batch, a.rows = sh.batch, R
+    for k, t in host.items():
+        setattr(a, k, t.data_ptr())
+    a.k_cache, a.v_cache, a.w_lm = ds.k_cache.data_ptr(), ds.v_cache.data_ptr(), w.w_lm.data_ptr()
+    a.w_lm_layout = w.layout
+    return host, a
+
+
+def test_host_step_captured_in_a_graph():
+    """ebd_step_host captured into a CUDA graph (the capture takes the
+    single-gather route) and replayed gives the uncaptured call's results."""
+    from paper_2609_16450_gb300 import _ebd as E
+    from paper_2609_16450_gb300 import runtime as rt
+    sh = synth.tiny
+    inp, w, h = _setup(sh)
+    ds = rt.DeviceStep(inp, w)
+    host, a = _pinned_host_args(sh, inp, ds, w)
+    st0 = {k: host[k].clone() for k in ("tokens", "mask", "in_block", "blk_meta")}
+    stream = torch.cuda.Stream()
+    E.check(E.ebd_step_host(h.h, a, stream.cuda_stream), h.h)
+    stream.synchronize()
+    assert h.sync_status() == 0
+    ref = {k: t.clone() for k, t in host.items()}
+    for k, v in st0.items():
+        host[k].copy_(v)
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=stream):
+        E.check(E.ebd_step_host(h.h, a, stream.cuda_stream), h.h)
+    torch.cuda.synchronize()
+    for k, v in st0.items():  # the capture ran nothing
+        host[k].copy_(v)
+    g.replay()
+    torch.cuda.synchronize()
+    assert h.sync_status() == 0
+    for k in ("tokens", "mask", "in_block", "blk_meta", "argmax", "accepted"):
+        assert torch.equal(host[k], ref[k]), k
+    for k in ("conf", "attn_out"):
+        assert torch.equal(host[k], ref[k]), k
 
 
 def test_overlapped_and_serial_and_graph_steps_agree():
