@@ -495,12 +495,14 @@ __device__ __forceinline__ void lps_attention_unit(const float* qkv, int n, int 
 // LPS (Sec. 5.2 / App. D.1): Linear(5->32) -> LayerNorm -> GELU, two pre-norm
 // blocks (4 heads of width 8, FFN 64, GELU), head Linear(32->1), p = sigmoid.
 // Over the n (<= 64) masked rows of the block (features at P + L_FEAT);
-// p_psi of row i -> P[L_PROB + i].  Called by the whole CTA.  `from` > 0
-// skips the phases of the first block before phase `from` (1 LN1, 2 QKV,
-// 3 attention, 4 output projection, 5 LN2, 6 FF1, 7 FF2; 0 the input layer);
-// only the stand-in runs of the decision kernel use it.
+// p_psi of row i -> P[L_PROB + i].  Called by the whole CTA.  Phases: 0 the
+// input layer; per block 1 LN1, 2 QKV, 3 attention, 4 output projection,
+// 5 LN2, 6 FF1, 7 FF2; 8 the second block and the head.  Only phases
+// [from, to] of the first block run (from = 8: none of it); the second
+// block and the head run when to = 8.  Only the stand-in runs of the
+// decision kernel pass anything but [0, 8].
 __device__ __noinline__ void lps_forward(float* P, int n, const __nv_bfloat16* Wlps,
-                                         const float* V, int from) {
+                                         const float* V, int from, int to) {
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const float* feats = P + L_FEAT;
   float* Z = P + L_Z;
@@ -508,7 +510,7 @@ __device__ __noinline__ void lps_forward(float* P, int n, const __nv_bfloat16* W
   const HL Y = hl_at(P + L_YH, 40);
   const HL At = hl_at(P + L_AH, 40);
   const HL Hh = hl_at(P + L_HH, 72);
-  if (from <= 0) {  // Linear(5 -> 32), LayerNorm, GELU: 8 lanes per row, 4 outputs each
+  if (from <= 0 && to >= 0) {  // Linear(5 -> 32), LayerNorm, GELU: 8 lanes per row, 4 outputs each
     const int q = lane & 7;
 #pragma unroll 1
     for (int j0 = 0; j0 < n; j0 += (blockDim.x >> 3)) {
@@ -543,43 +545,46 @@ __device__ __noinline__ void lps_forward(float* P, int n, const __nv_bfloat16* W
   __syncthreads();
 #pragma unroll 1
   for (int l = 0; l < 2; ++l) {
+    if (l == 1 && to < 8) break;
     const __nv_bfloat16* Wl = Wlps + l * PL_STRIDE;
     const float* Vl = V + VP_LAYER0 + l * VP_LAYER_STRIDE;
-    const int f = l == 0 ? from : 0;
-    if (f <= 1) ln_rows<32, false>(Z, LDQ, nullptr, 0, Y, n, Vl + VPL_LN1G, Vl + VPL_LN1B);
+    const int f = l == 0 ? from : 0, t = l == 0 ? to : 8;
+    if (f <= 1 && t >= 1) ln_rows<32, false>(Z, LDQ, nullptr, 0, Y, n, Vl + VPL_LN1G, Vl + VPL_LN1B);
     __syncthreads();
-    if (f <= 2)
+    if (f <= 2 && t >= 2)
       gemm_hl(Y, n, 32, Wl + PL_QKV, PL_LDQKV, 96, [&](int j, int o, float a, float b) {
         *reinterpret_cast<float2*>(QKV + j * 100 + o) = make_float2(a + Vl[VPL_QKVB + o], b + Vl[VPL_QKVB + o + 1]);
       });
     __syncthreads();
     const int mt = (n + 15) >> 4;
-    if (f <= 3) {
+    if (f <= 3 && t >= 3) {
 #pragma unroll 1
       for (int u = warp; u < 4 * mt; u += (blockDim.x >> 5)) lps_attention_unit(QKV, n, 16 * (u >> 2), u & 3, At);
     }
     __syncthreads();
-    if (f <= 4)
+    if (f <= 4 && t >= 4)
       gemm_hl(At, n, 32, Wl + PL_OUT, PL_LDOUT, 32, [&](int j, int o, float a, float b) {
         float2* z = reinterpret_cast<float2*>(Z + j * LDQ + o);
         const float2 zz = *z;
         *z = make_float2(zz.x + (a + Vl[VPL_OUTB + o]), zz.y + (b + Vl[VPL_OUTB + o + 1]));
       });
     __syncthreads();
-    if (f <= 5) ln_rows<32, false>(Z, LDQ, nullptr, 0, Y, n, Vl + VPL_LN2G, Vl + VPL_LN2B);
+    if (f <= 5 && t >= 5) ln_rows<32, false>(Z, LDQ, nullptr, 0, Y, n, Vl + VPL_LN2G, Vl + VPL_LN2B);
     __syncthreads();
-    if (f <= 6)
+    if (f <= 6 && t >= 6)
       gemm_hl(Y, n, 32, Wl + PL_FF1, PL_LDFF1, 64, [&](int j, int o, float a, float b) {
         hl_store2(Hh, j, o, gelu(a + Vl[VPL_FF1B + o]), gelu(b + Vl[VPL_FF1B + o + 1]));
       });
     __syncthreads();
-    gemm_hl(Hh, n, 64, Wl + PL_FF2, PL_LDFF2, 32, [&](int j, int o, float a, float b) {
-      float2* z = reinterpret_cast<float2*>(Z + j * LDQ + o);
-      const float2 zz = *z;
-      *z = make_float2(zz.x + (a + Vl[VPL_FF2B + o]), zz.y + (b + Vl[VPL_FF2B + o + 1]));
-    });
+    if (f <= 7 && t >= 7)
+      gemm_hl(Hh, n, 64, Wl + PL_FF2, PL_LDFF2, 32, [&](int j, int o, float a, float b) {
+        float2* z = reinterpret_cast<float2*>(Z + j * LDQ + o);
+        const float2 zz = *z;
+        *z = make_float2(zz.x + (a + Vl[VPL_FF2B + o]), zz.y + (b + Vl[VPL_FF2B + o + 1]));
+      });
     __syncthreads();
   }
+  if (to < 8) return;
 #pragma unroll 1
   for (int i = warp; i < n; i += (blockDim.x >> 5)) {
     const float a = warp_sum(Z[i * LDQ + lane] * V[VP_HEADW + lane]) + V[VP_HEADB];
@@ -651,6 +656,17 @@ __global__ void __cluster_dims__(kDecideCluster, 1, 1) __launch_bounds__(kDecide
     sm.f_acc[j] = 0;
     sm.f_O[j] = __int_as_float(0x7fc00000);
     sm.f_p[j] = __int_as_float(0x7fc00000);
+  }
+
+  // Every step starts with this kernel's code out of every cache.  While the
+  // LM head finishes, ranks 1..5 each run one stretch of the LPS router on a
+  // stand-in block in their own shared memory (the pool, unused until the
+  // statistics are merged; the results are discarded), so that the
+  // instructions rank 0 runs there after the LBS come from L2.
+  if (rank >= 1 && rank <= 5 && p.lps_enabled && p.mode == EBD_DECODE_EB) {
+    const int from = rank == 1 ? 0 : rank == 2 ? 1 : rank == 3 ? 3 : rank == 4 ? 4 : 6;
+    const int to = rank == 1 ? 0 : rank == 2 ? 2 : rank == 3 ? 3 : rank == 4 ? 5 : 7;
+    lps_forward(P, 32, sm.w, sm.v + V_LPS, from, to);
   }
 
   // ---------------------------------------------------------------- 1. statistics
@@ -1026,7 +1042,7 @@ __global__ void __cluster_dims__(kDecideCluster, 1, 1) __launch_bounds__(kDecide
     }
     __syncthreads();
     const float* prob = P + L_PROB;
-    lps_forward(P, nBM, sm.w, sm.v + V_LPS, lps_from);
+    lps_forward(P, nBM, sm.w, sm.v + V_LPS, lps_from, 8);
 #pragma unroll 1
     for (int i = tid; i < nBM; i += blockDim.x) sm.f_p[sm.BMrows[i]] = prob[i];
     __syncthreads();
