@@ -11,21 +11,23 @@
 //   prep      masked set M of each sequence (compaction), LBS on/off
 //   embed     F_ent hidden and the token branch (warp per row); ent2 +
 //             LayerNorm, fusion + E_pos (GEMMs)
-//   2 layers  QKV (GEMM); attention (CTA per query block and head, keys
-//             staged in shared memory); output projection + LayerNorm, FF1 +
-//             GELU, FF2 + LayerNorm (GEMMs); LBS head
+//   2 layers  QKV (GEMM); attention (CTA per 8 queries and head, key blocks
+//             staged in shared memory, one key per lane); output projection
+//             + LayerNorm, FF1 + GELU, FF2 + LayerNorm (GEMMs); LBS head
 //   select    candidates, MaxGapFilter, min-tokens fallback; B n M; LPS
 //             features                                        (CTA per sequence)
 //   LPS       input layer; 2 blocks as above (d 32, 4 heads); head, sigmoid
 //   accept    union accept, anti-stall, commit, block resolution
 // Products are fp32 FMAs on an fp32 copy of the (bf16-valued) weights stored
-// [in][out].  The LBS products are CTA-tiled GEMMs over all window rows (32
-// rows x 32*CPT columns per CTA, operands staged in shared memory) with the
+// [in][out].  The LBS products are CTA-tiled GEMMs over all window rows (8
+// rows x 32*CPT columns per CTA, k-chunks staged in shared memory) with the
 // bias, residual, LayerNorm, GELU or head fused into the epilogue: a warp
-// holds 4 whole rows of the tile.  Rows outside the LBS compute garbage in
+// holds one whole row of the tile.  Rows outside the LBS compute garbage in
 // their own scratch rows, which nothing reads.  The small LPS products run
 // one warp per row (a row's vector spread over the lanes, element lane + 32 i
-// in register i, one input broadcast at a time).
+// in register i, one input broadcast at a time) on the block's weights staged
+// in shared memory.  Each kernel is a programmatic dependent of the one
+// before it (seq_wait / seq_release below).
 #include <climits>
 #include <cstdlib>
 
