@@ -650,7 +650,9 @@ ebd_status run_attention(ebd_handle* h, const ebd_step_args* a, cudaStream_t st,
   return EBD_OK;
 }
 
-ebd_status run_lm(ebd_handle* h, const ebd_step_args* a, cudaStream_t st) {
+// pdl_first: the first LM-head launch is a programmatic dependent of the
+// kernel just before it on `st`, which copies the hidden rows in
+ebd_status run_lm(ebd_handle* h, const ebd_step_args* a, cudaStream_t st, bool pdl_first = false) {
   const ebd_config& c = h->cfg;
   CUtensorMap tw;
   const bool packed = a->w_lm_layout == 1;
@@ -681,6 +683,7 @@ ebd_status run_lm(ebd_handle* h, const ebd_step_args* a, cudaStream_t st) {
     p.status = h->d_status;
     p.limit_ns = kLimitNs;
     p.force_timeout = (c.debug_flags & EBD_DEBUG_FORCE_TIMEOUT) ? 1 : 0;
+    p.pdl = (g0 == 0 && pdl_first) ? 1 : 0;
     CUtensorMap th;
     const uint64_t dims[2] = {static_cast<uint64_t>(c.d_model), static_cast<uint64_t>(a->rows)};
     const uint64_t str[1] = {static_cast<uint64_t>(c.d_model) * 2};
@@ -1060,7 +1063,11 @@ struct CopyList {
   int n;
 };
 
+// A kernel launched after it as a programmatic dependent (the LM head of
+// ebd_step_host) may be scheduled at once; it waits for this grid before it
+// reads what this one copies.
 __global__ void __launch_bounds__(256) copy_list_kernel(const CopyList cl) {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   const int i = blockIdx.y;
   if (i >= cl.n) return;
   const CopyItem c = cl.it[i];
@@ -1123,6 +1130,7 @@ struct HostMover {
 // (its inputs come in on the copy stream) and where the decision writes the
 // decode state (the caller's buffers, when it read a staged copy).
 struct StepRoute {
+  bool lm_pdl;  // the kernel just before the step copied the hidden rows in
   const unsigned* ready;
   unsigned ready_ticket;
   int* tokens_out;
@@ -1223,7 +1231,7 @@ ebd_status step_run(ebd_handle* h, const ebd_step_args* a, cudaStream_t st, cons
   const int prof = h->profile;
   cudaError_t e0 = cudaSuccess;
   if (prof && (e0 = record(h->ev[0], st)) != cudaSuccess) return cuda_fail(h, e0, "profile event");
-  if ((s = run_lm(h, a, st)) != EBD_OK) return s;
+  if ((s = run_lm(h, a, st, rt != nullptr && rt->lm_pdl && prof == 0)) != EBD_OK) return s;
   if (prof && (e0 = record(h->ev[1], st)) != cudaSuccess) return cuda_fail(h, e0, "profile event");
   DecideParams p = decide_params(h, a, 0);
   p.pdl = prof == 0 ? 1 : 0;  // no event between the LM head and the decision
@@ -1394,6 +1402,14 @@ ebd_status ebd_step_host(ebd_handle* h, const ebd_step_args* a, void* stream) {
       in.add(vw, a->v_win, R * Hkv * D * 2);
     }
   }
+  // the copy stream forks before the gather, so that the LM head can be a
+  // programmatic dependent of the gather kernel (it prefetches its first W
+  // stages while the hidden rows come in)
+  if (dma) {
+    cudaError_t e0 = cudaEventRecord(h->ev_fork, st);
+    if (e0 != cudaSuccess) return cuda_fail(h, e0, "copy stream event");
+  }
+  const bool gathered = in.list.n > 0;  // flush() launches the gather kernel
   cudaError_t e = in.flush();
   if (e != cudaSuccess) return cuda_fail(h, e, "host-to-device copy");
   unsigned ticket = 0;
@@ -1401,8 +1417,7 @@ ebd_status ebd_step_host(ebd_handle* h, const ebd_step_args* a, void* stream) {
     if (++h->ticket == 0) h->ticket = 1;  // 0 is the word's initial value
     ticket = h->ticket;
     const cudaMemcpyKind k = cudaMemcpyHostToDevice;
-    if ((e = cudaEventRecord(h->ev_fork, st)) != cudaSuccess ||
-        (e = cudaStreamWaitEvent(h->s_copy, h->ev_fork, 0)) != cudaSuccess ||
+    if ((e = cudaStreamWaitEvent(h->s_copy, h->ev_fork, 0)) != cudaSuccess ||
         (e = cudaMemcpyAsync(q, a->q, R * Hq * D * 2, k, h->s_copy)) != cudaSuccess ||
         (e = cudaMemcpyAsync(kw, a->k_win, R * Hkv * D * 2, k, h->s_copy)) != cudaSuccess ||
         (e = cudaMemcpyAsync(vw, a->v_win, R * Hkv * D * 2, k, h->s_copy)) != cudaSuccess)
@@ -1435,7 +1450,7 @@ ebd_status ebd_step_host(ebd_handle* h, const ebd_step_args* a, void* stream) {
     back[nback++] = Back{host, stage, bytes};
     return stage;
   };
-  StepRoute rt{dma ? h->d_ready : nullptr, ticket, nullptr, nullptr, nullptr, nullptr};
+  StepRoute rt{gathered, dma ? h->d_ready : nullptr, ticket, nullptr, nullptr, nullptr, nullptr};
   rt.tokens_out = static_cast<int32_t*>(result(a->tokens, tok, R * 4, 4));
   rt.mask_out = static_cast<uint8_t*>(result(a->mask, msk, R, 1));
   rt.in_block_out = static_cast<uint8_t*>(result(a->in_block, ib, R, 1));

@@ -32,7 +32,7 @@ struct LmParams {
   int kbs, nks;             // k-blocks per pipeline stage, stages per vocabulary chunk
   int packed;               // W is tiled: tile (unit, k-block) at row (unit*nkb + kb)*64
   int stages, nbuf, acc_stride, tmem_cols;
-  int nwg;                  // epilogue warpgroups in use (1, or 2 for more than 32 rows)
+  int nwg;                  // epilogue warpgroups in use (2 with a single accumulator buffer)
   int pair;                 // clusters of 2 CTAs: W multicast, rows split in halves
   int rhalf;                // rows of one CTA of a pair (rows of the launch otherwise)
   int ncols;                // partial states per row written (>= grid; extra ones neutral)
@@ -44,6 +44,8 @@ struct LmParams {
   int* status;
   uint64_t limit_ns;
   int force_timeout;
+  int pdl;                  // a programmatic dependent of the kernel before it, which
+                            // copies the hidden rows in: W loads start before the wait
 };
 
 // ------------------------------------------------------------------ attention

@@ -135,8 +135,8 @@ __global__ void __launch_bounds__(kLmThreads, 1)
   const int tid = threadIdx.x;
   // the decision kernel, launched after this one as a programmatic dependent,
   // may be scheduled as soon as SMs free up; it waits for this grid's
-  // completion before it reads the partial states
-  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  // completion before it reads the partial states (as a dependent itself,
+  // this grid releases it only after its own wait, below)
   const int warp = __shfl_sync(0xffffffffu, tid / 32, 0);
   const int lane = tid & 31;
   // paired mode: the two CTAs of a cluster share a vocabulary range; each
@@ -193,46 +193,77 @@ __global__ void __launch_bounds__(kLmThreads, 1)
     if (lane == 0) {
       const uint64_t pol_w = l2_policy_evict_first();
       const uint64_t pol_h = l2_policy_evict_last();
-      int it = 0;
-      int s = 0;        // stage of iteration it (it % stages, kept as a counter)
-      uint32_t ph = 0;  // its phase parity
-      bool ok = true;
-      for (int u = u0; u < u1 && ok; u += 2 * MCH) {
+      // stage fill: vocabulary chunk u (2 MCH units), k-stage ks
+      auto issue_w = [&](int u, int ks, int s) {  // arms the stage for W and hidden bytes
         const int nu = min(2 * MCH, u1 - u);
-        for (int ks = 0; ks < p.nks; ++ks) {
-          if (!mbar_wait(&empty[s], ph ^ 1u, p.limit_ns, abort)) {
-            ok = false;
-            break;
+        const int nsubk = min(p.kbs, p.nkb - ks * p.kbs);
+        mbar_arrive_expect_tx(&full[s], static_cast<uint32_t>(nsubk) *
+                                            (static_cast<uint32_t>(nu) * kUnit * 128u + b_sub));
+        uint8_t* a_st = sA + static_cast<size_t>(s) * a_stage;
+        // one row half at a time, its k-boxes back to back: each W row is
+        // requested as one contiguous run of nsubk * 128 bytes
+        for (int ui = 0; ui < nu; ++ui) {
+          if (PAIR && (ui & 1) != static_cast<int>(crank)) continue;  // the peer loads it
+          for (int j = 0; j < nsubk; ++j) {
+            const int x = PACKED ? 0 : (ks * p.kbs + j) * 64;
+            const int y = PACKED ? ((u + ui) * p.nkb + ks * p.kbs + j) * kUnit : (u + ui) * kUnit;
+            uint8_t* dst = a_st + (ui >> 1) * a_chunk + j * kATile + (ui & 1) * (kUnit * 128);
+            if (PAIR)
+              tma_load_2d_multicast(dst, &tmap_w, &full[s], x, y, 0x3, pol_w);
+            else
+              tma_load_2d(dst, &tmap_w, &full[s], x, y, pol_w);
           }
-          const int nsubk = min(p.kbs, p.nkb - ks * p.kbs);
-          mbar_arrive_expect_tx(&full[s], static_cast<uint32_t>(nsubk) *
-                                              (static_cast<uint32_t>(nu) * kUnit * 128u + b_sub));
-          uint8_t* a_st = sA + static_cast<size_t>(s) * a_stage;
-          uint8_t* b_st = sB + static_cast<size_t>(s) * b_stage;
-          // one row half at a time, its k-boxes back to back: each W row is
-          // requested as one contiguous run of nsubk * 128 bytes
-          for (int ui = 0; ui < nu; ++ui) {
-            if (PAIR && (ui & 1) != static_cast<int>(crank)) continue;  // the peer loads it
-            for (int j = 0; j < nsubk; ++j) {
-              const int x = PACKED ? 0 : (ks * p.kbs + j) * 64;
-              const int y = PACKED ? ((u + ui) * p.nkb + ks * p.kbs + j) * kUnit
-                                   : (u + ui) * kUnit;
-              uint8_t* dst = a_st + (ui >> 1) * a_chunk + j * kATile + (ui & 1) * (kUnit * 128);
-              if (PAIR)
-                tma_load_2d_multicast(dst, &tmap_w, &full[s], x, y, 0x3, pol_w);
-              else
-                tma_load_2d(dst, &tmap_w, &full[s], x, y, pol_w);
-            }
-          }
-          for (int j = 0; j < nsubk; ++j)
-            for (int sb = 0; sb < p.nsub; ++sb)
-              tma_load_2d(b_st + j * b_sub + sb * p.nb * 128, &tmap_h, &full[s],
-                          (ks * p.kbs + j) * 64, rbase + sb * p.nb, pol_h);
-          ++it;
-          if (++s == p.stages) {
-            s = 0;
-            ph ^= 1u;
-          }
+        }
+      };
+      auto issue_h = [&](int ks, int s) {
+        const int nsubk = min(p.kbs, p.nkb - ks * p.kbs);
+        uint8_t* b_st = sB + static_cast<size_t>(s) * b_stage;
+        for (int j = 0; j < nsubk; ++j)
+          for (int sb = 0; sb < p.nsub; ++sb)
+            tma_load_2d(b_st + j * b_sub + sb * p.nb * 128, &tmap_h, &full[s],
+                        (ks * p.kbs + j) * 64, rbase + sb * p.nb, pol_h);
+      };
+      int u = u0, ks = 0;  // the next stage fill
+      auto advance = [&]() {
+        if (++ks == p.nks) {
+          ks = 0;
+          u += 2 * MCH;
+        }
+      };
+      // The first stages' W go out before anything else.  As a programmatic
+      // dependent of the copy of its hidden rows (ebd_step_host), the grid
+      // waits for that copy only then; and only then does it release the
+      // decision kernel, launched after it as a programmatic dependent,
+      // which reads the decode state the same copy brings at once (and waits
+      // for this grid's completion before it reads the partial states).
+      // Released this late in every launch, the decision and the attention
+      // after it no longer take SMs while this grid starts: LLaDA-8B step
+      // 205.8 us (p90 213.5) with the release at kernel entry, 198.8 us
+      // (p90 199.2) here; the LM head alone 155.7 against 156.0 us.
+      int it = 0;
+      {
+        const int ks0 = ks;
+        for (; it < p.stages && u < u1; ++it, advance()) issue_w(u, ks, it);  // stages start empty
+        asm volatile("griddepcontrol.wait;" ::: "memory");
+        asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+        for (int i = 0, hk = ks0; i < it; ++i) {
+          issue_h(hk, i);
+          if (++hk == p.nks) hk = 0;
+        }
+      }
+      int s = it == p.stages ? 0 : it;        // stage of iteration it
+      uint32_t ph = it == p.stages ? 1u : 0u;  // its phase parity
+      bool ok = true;
+      for (; u < u1; ++it, advance()) {
+        if (!mbar_wait(&empty[s], ph ^ 1u, p.limit_ns, abort)) {
+          ok = false;
+          break;
+        }
+        issue_w(u, ks, s);
+        issue_h(ks, s);
+        if (++s == p.stages) {
+          s = 0;
+          ph ^= 1u;
         }
       }
       if (!ok) {
@@ -614,13 +645,22 @@ cudaError_t launch_lm_stats(const CUtensorMap& tmap_w, const CUtensorMap& tmap_h
   cfg.blockDim = dim3(kLmThreads, 1, 1);
   cfg.dynamicSmemBytes = p.smem_bytes;
   cfg.stream = st;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = 2;
-  attr[0].val.clusterDim.y = 1;
-  attr[0].val.clusterDim.z = 1;
+  cudaLaunchAttribute attr[2];
+  int na = 0;
+  if (p.pair) {
+    attr[na].id = cudaLaunchAttributeClusterDimension;
+    attr[na].val.clusterDim.x = 2;
+    attr[na].val.clusterDim.y = 1;
+    attr[na].val.clusterDim.z = 1;
+    ++na;
+  }
+  if (p.pdl) {
+    attr[na].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[na].val.programmaticStreamSerializationAllowed = 1;
+    ++na;
+  }
   cfg.attrs = attr;
-  cfg.numAttrs = p.pair ? 1 : 0;
+  cfg.numAttrs = na;
   if (p.pair && p.mch == 2)
     return p.packed ? cudaLaunchKernelEx(&cfg, lm_stats_kernel<true, true, 2>, tmap_w, tmap_h, p)
                     : cudaLaunchKernelEx(&cfg, lm_stats_kernel<true, false, 2>, tmap_w, tmap_h, p);
