@@ -222,9 +222,13 @@ ebd_status ebd_step(ebd_handle* h, const ebd_step_args* a, void* stream);
  * Pinned, mapped buffers (cudaHostAlloc / cudaHostRegister) move by kernel
  * instead of cudaMemcpyAsync.  With max_window <= 64 the kernels also write
  * the decode state and the outputs straight into such buffers (attn_out
- * when 16-byte aligned), and q, k_win and v_win are copied while the
- * decision runs; the state and outputs then hold the step's results only
- * once the stream has passed the step, as in every other case. */
+ * when 16-byte aligned), and q, k_win and v_win come in on a copy engine on
+ * the handle's own second stream while the LM head runs (the attention waits
+ * for them, time-limited: EBD_ERR_TIMEOUT); `stream` waits for that stream
+ * at the end of the step.  While `stream` is being captured into a CUDA
+ * graph they go with the other inputs instead.  The state and outputs hold
+ * the step's results only once the stream has passed the step, as in every
+ * other case. */
 ebd_status ebd_step_host(ebd_handle* h, const ebd_step_args* a, void* stream);
 
 /* Only the decision (step 3) on caller-provided statistics: reads
