@@ -1,0 +1,147 @@
+"""The oracle's pins are sensitive: each test here plants one plausible
+mistake in the oracle (in this process only, through monkeypatch, on the CPU)
+and checks that at least one of the pins that guard that part fails.
+
+Mistakes planted: entropy in bits instead of nats; argmax ties to the highest
+index; the gap against the third logit; an attention scale of 2/sqrt(D); one
+prefix key dropped; GQA heads mapped round-robin instead of in groups; the
+MaxGapFilter cut at a gap equal to g_max; the min-tokens fallback of L_min
+rows instead of L_B; a strict kappa > tau in the accept rule."""
+import numpy as np
+import pytest
+
+from oracle import ebd_oracle as o
+from tests import test_oracle_attention as ta
+from tests import test_oracle_decision as td
+from tests import test_oracle_stats as ts
+
+
+def _some_pin_fails(pins):
+    """True if calling any of the pin callables raises AssertionError."""
+    for pin in pins:
+        try:
+            pin()
+        except AssertionError:
+            return True
+    return False
+
+
+def _stats_pins():
+    return [ts.test_golden_hand_worked,
+            lambda: ts.test_uniform_closed_form(7),
+            lambda: ts.test_one_hot_closed_form(16, 0),
+            lambda: ts.test_k_way_tie(3),
+            ts.test_against_scipy_random]
+
+
+def test_the_pins_pass_as_they_stand():
+    assert not _some_pin_fails(_stats_pins())
+    assert not _some_pin_fails([ta.test_matches_torch_sdpa, ta.test_ragged_prefix_and_batch_separation,
+                                ta.test_gqa_head_mapping])
+    assert not _some_pin_fails([td.test_maxgap_golden, td.test_select_golden, td.test_accept_golden])
+
+
+def test_entropy_in_bits_is_caught(monkeypatch):
+    real = o.softmax_stats
+
+    def bits(logits):
+        st = real(logits)
+        return o.RowStats(conf=st.conf, entropy=st.entropy / np.log(2.0), ent_norm=st.ent_norm, gap=st.gap,
+                          argmax=st.argmax, logit_gap=st.logit_gap, near_tie=st.near_tie)
+    monkeypatch.setattr(o, "softmax_stats", bits)
+    assert _some_pin_fails(_stats_pins())
+
+
+def test_argmax_ties_to_highest_index_are_caught(monkeypatch):
+    real = o.softmax_stats
+
+    def last(logits):
+        st = real(logits)
+        l = np.asarray(logits, np.float64)
+        am = l.shape[1] - 1 - np.argmax(l[:, ::-1], axis=1)
+        return o.RowStats(conf=st.conf, entropy=st.entropy, ent_norm=st.ent_norm, gap=st.gap,
+                          argmax=am.astype(np.int64), logit_gap=st.logit_gap, near_tie=st.near_tie)
+    monkeypatch.setattr(o, "softmax_stats", last)
+    assert _some_pin_fails(_stats_pins())
+
+
+def test_gap_against_the_third_logit_is_caught(monkeypatch):
+    real = o.softmax_stats
+
+    def third(logits):
+        st = real(logits)
+        l = np.sort(np.asarray(logits, np.float64), axis=1)[:, ::-1]
+        m = l[:, 0:1]
+        p = np.exp(l - m) / np.exp(l - m).sum(axis=1, keepdims=True)
+        gap = p[:, 0] - (p[:, 2] if l.shape[1] > 2 else 0.0)
+        return o.RowStats(conf=st.conf, entropy=st.entropy, ent_norm=st.ent_norm, gap=gap,
+                          argmax=st.argmax, logit_gap=st.logit_gap, near_tie=st.near_tie)
+    monkeypatch.setattr(o, "softmax_stats", third)
+    assert _some_pin_fails(_stats_pins())
+
+
+def test_wrong_attention_scale_is_caught(monkeypatch):
+    """scale 2 / sqrt(D), as from a head width taken as D / 4 (q doubled:
+    exact in bf16)"""
+    import synth
+    real = o.window_attention
+
+    def doubled(q, k_win, v_win, k_cache, v_cache, cu_rows, prefix_len, suffix=None):
+        q2 = synth.f32_to_bf16_bits((o.bf16(q) * 2.0).astype(np.float32))
+        return real(q2, k_win, v_win, k_cache, v_cache, cu_rows, prefix_len, suffix)
+    monkeypatch.setattr(o, "window_attention", doubled)
+    assert _some_pin_fails([ta.test_matches_torch_sdpa])
+
+
+def test_dropped_prefix_key_is_caught(monkeypatch):
+    real = o.window_attention
+
+    def short(q, k_win, v_win, k_cache, v_cache, cu_rows, prefix_len, suffix=None):
+        pl = np.maximum(np.asarray(prefix_len) - 1, 0)
+        return real(q, k_win, v_win, k_cache, v_cache, cu_rows, pl, suffix)
+    monkeypatch.setattr(o, "window_attention", short)
+    assert _some_pin_fails([ta.test_matches_torch_sdpa, ta.test_ragged_prefix_and_batch_separation])
+
+
+def test_round_robin_gqa_is_caught(monkeypatch):
+    real = o.window_attention
+
+    def round_robin(q, k_win, v_win, k_cache, v_cache, cu_rows, prefix_len, suffix=None):
+        Hq, Hkv = q.shape[1], k_win.shape[1]
+        # query head h reads kv head h % Hkv: permute q so that the grouped
+        # mapping of the real routine becomes the round-robin one
+        perm = np.array([(h % Hkv) * (Hq // Hkv) + h // Hkv for h in range(Hq)])
+        out = real(q[:, np.argsort(perm)], k_win, v_win, k_cache, v_cache, cu_rows, prefix_len, suffix)
+        return out[:, perm]
+    monkeypatch.setattr(o, "window_attention", round_robin)
+    assert _some_pin_fails([ta.test_gqa_head_mapping])
+
+
+def test_maxgap_cut_at_equal_gap_is_caught(monkeypatch):
+    real = o.max_gap_filter
+    monkeypatch.setattr(o, "max_gap_filter", lambda C, g: real(C, g - 1))
+    assert _some_pin_fails([td.test_maxgap_golden, td.test_select_golden])
+
+
+def test_fallback_of_l_min_rows_is_caught(monkeypatch):
+    real = o.select_block
+
+    def fallback_l_min(pos, M, O, argmax, prm):
+        return real(pos, M, O, argmax, o.DecisionParams(
+            tau=prm.tau, tau_psi=prm.tau_psi, l_min=prm.l_min, l_b=prm.l_min, g_max=prm.g_max,
+            eos_id=prm.eos_id, lps_enabled=prm.lps_enabled))
+    monkeypatch.setattr(o, "select_block", fallback_l_min)
+    assert _some_pin_fails([td.test_select_golden])
+
+
+def test_strict_kappa_threshold_is_caught(monkeypatch):
+    real = o.decide_sequence
+
+    def strict(pos, mask, tokens, in_block, meta, st, w_emb, W, prm, **kw):
+        p2 = o.DecisionParams(tau=np.nextafter(prm.tau, np.inf), tau_psi=prm.tau_psi, l_min=prm.l_min,
+                              l_b=prm.l_b, g_max=prm.g_max, eos_id=prm.eos_id,
+                              lps_enabled=prm.lps_enabled)
+        return real(pos, mask, tokens, in_block, meta, st, w_emb, W, p2, **kw)
+    monkeypatch.setattr(o, "decide_sequence", strict)
+    if not _some_pin_fails([td.test_accept_golden]):
+        pytest.fail("no accept pin has kappa exactly at tau")
