@@ -6,13 +6,16 @@ Mistakes planted: entropy in bits instead of nats; argmax ties to the highest
 index; the gap against the third logit; an attention scale of 2/sqrt(D); one
 prefix key dropped; GQA heads mapped round-robin instead of in groups; the
 MaxGapFilter cut at a gap equal to g_max; the min-tokens fallback of L_min
-rows instead of L_B; a strict kappa > tau in the accept rule."""
+rows instead of L_B; a strict kappa > tau in the accept rule; the tanh
+approximation of GELU; a LayerNorm eps of 1e-6; an attention scale of
+1/sqrt(d) instead of 1/sqrt(d/heads) in the routers."""
 import numpy as np
 import pytest
 
 from oracle import ebd_oracle as o
 from tests import test_oracle_attention as ta
 from tests import test_oracle_decision as td
+from tests import test_oracle_routers as tr
 from tests import test_oracle_stats as ts
 
 
@@ -145,3 +148,46 @@ def test_strict_kappa_threshold_is_caught(monkeypatch):
     monkeypatch.setattr(o, "decide_sequence", strict)
     if not _some_pin_fails([td.test_accept_golden]):
         pytest.fail("no accept pin has kappa exactly at tau")
+
+
+def _router_pins():
+    return [tr.test_lbs_layer_matches_torch_post_norm, tr.test_lps_block_matches_torch_pre_norm,
+            tr.test_elementary_layers_match_torch]
+
+
+def test_router_pins_pass_as_they_stand():
+    assert not _some_pin_fails(_router_pins())
+
+
+def test_tanh_gelu_is_caught(monkeypatch):
+    import math
+
+    def tanh_gelu(x):
+        return 0.5 * x * (1.0 + np.tanh(math.sqrt(2.0 / math.pi) * (x + 0.044715 * x ** 3)))
+    monkeypatch.setattr(o, "gelu", tanh_gelu)
+    assert _some_pin_fails(_router_pins())
+
+
+def test_layer_norm_eps_is_caught(monkeypatch):
+    monkeypatch.setattr(o, "LN_EPS", 1e-6)
+    assert _some_pin_fails(_router_pins())
+
+
+def test_router_attention_scale_is_caught(monkeypatch):
+    real = o.softmax_rows
+    state = {}
+
+    def wrong_scale(s):  # the scores of a head of width d / heads, rescaled as if by 1/sqrt(d)
+        return real(s * state.get("f", 1.0))
+
+    real_attn = o.self_attention
+
+    def attn(x, W, name, n_heads):
+        state["f"] = 1.0 / np.sqrt(n_heads)
+        try:
+            return real_attn(x, W, name, n_heads)
+        finally:
+            state["f"] = 1.0
+    monkeypatch.setattr(o, "softmax_rows", wrong_scale)
+    monkeypatch.setattr(o, "self_attention", attn)
+    assert _some_pin_fails(_router_pins())
