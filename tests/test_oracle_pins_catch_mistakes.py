@@ -8,7 +8,9 @@ prefix key dropped; GQA heads mapped round-robin instead of in groups; the
 MaxGapFilter cut at a gap equal to g_max; the min-tokens fallback of L_min
 rows instead of L_B; a strict kappa > tau in the accept rule; the tanh
 approximation of GELU; a LayerNorm eps of 1e-6; an attention scale of
-1/sqrt(d) instead of 1/sqrt(d/heads) in the routers."""
+1/sqrt(d) instead of 1/sqrt(d/heads) in the routers; EOS kept among the
+router candidates; the dual-cache suffix read one position late; the cache
+append writing masked rows too."""
 import numpy as np
 import pytest
 
@@ -191,3 +193,33 @@ def test_router_attention_scale_is_caught(monkeypatch):
     monkeypatch.setattr(o, "softmax_rows", wrong_scale)
     monkeypatch.setattr(o, "self_attention", attn)
     assert _some_pin_fails(_router_pins())
+
+
+def test_eos_kept_among_candidates_is_caught(monkeypatch):
+    real = o.select_block
+
+    def keep_eos(pos, M, O, argmax, prm):
+        return real(pos, M, O, argmax, o.DecisionParams(
+            tau=prm.tau, tau_psi=prm.tau_psi, l_min=prm.l_min, l_b=prm.l_b, g_max=prm.g_max,
+            eos_id=-123456, lps_enabled=prm.lps_enabled))
+    monkeypatch.setattr(o, "select_block", keep_eos)
+    assert _some_pin_fails([td.test_select_golden])
+
+
+def test_suffix_one_position_late_is_caught(monkeypatch):
+    real = o.window_attention
+
+    def late(q, k_win, v_win, k_cache, v_cache, cu_rows, prefix_len, suffix=None):
+        if suffix is not None:
+            suffix = np.asarray(suffix).copy()
+            suffix[:, 0] += 1
+        return real(q, k_win, v_win, k_cache, v_cache, cu_rows, prefix_len, suffix)
+    monkeypatch.setattr(o, "window_attention", late)
+    assert _some_pin_fails([ta.test_suffix_matches_torch_sdpa, ta.test_suffix_keys_count_once_in_any_order])
+
+
+def test_append_of_masked_rows_is_caught(monkeypatch):
+    real = o.kv_append
+    monkeypatch.setattr(o, "kv_append", lambda kc, vc, kw, vw, cu, row_pos, mask:
+                        real(kc, vc, kw, vw, cu, row_pos, np.zeros_like(mask)))
+    assert _some_pin_fails([ta.test_kv_append_writes_committed_rows_only])
