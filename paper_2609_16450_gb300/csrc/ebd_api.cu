@@ -669,9 +669,9 @@ ebd_status run_lm(ebd_handle* h, const ebd_step_args* a, cudaStream_t st, bool p
   for (int g0 = 0; g0 < a->rows; g0 += kMaxGroupRows) {
     const int rows = a->rows - g0 < kMaxGroupRows ? a->rows - g0 : kMaxGroupRows;
     LmParams p{};
-    // 257..512 rows: CTA pairs that multicast W and split the rows, which
-    // keeps each CTA's accumulator within 256 TMEM columns (double-buffered).
-    // Measured at 512 rows: 485 -> 444 us against one CTA per SM.
+    // 257..512 rows: CTA pairs that read the same W range and split the
+    // rows, which keeps each CTA's accumulator within 256 TMEM columns
+    // (double-buffered).
     bool pair = rows > 256 && rows <= 512;
     if (const char* env = getenv("EBD_LM_PAIR")) pair = pair && atoi(env) != 0;
     lm_plan(p, rows, c.vocab, c.d_model, h->num_sms, pair);

@@ -33,7 +33,7 @@ struct LmParams {
   int packed;               // W is tiled: tile (unit, k-block) at row (unit*nkb + kb)*64
   int stages, nbuf, acc_stride, tmem_cols;
   int nwg;                  // epilogue warpgroups in use (2 with a single accumulator buffer)
-  int pair;                 // clusters of 2 CTAs: W multicast, rows split in halves
+  int pair;                 // clusters of 2 CTAs: same W range, rows split in halves
   int rhalf;                // rows of one CTA of a pair (rows of the launch otherwise)
   int ncols;                // partial states per row written (>= grid; extra ones neutral)
   int mch;                  // 128-row vocabulary chunks per pipeline stage (1, or 2: one

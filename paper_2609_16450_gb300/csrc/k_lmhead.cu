@@ -139,9 +139,10 @@ __global__ void __launch_bounds__(kLmThreads, 1)
   // this grid releases it only after its own wait, below)
   const int warp = __shfl_sync(0xffffffffu, tid / 32, 0);
   const int lane = tid & 31;
-  // paired mode: the two CTAs of a cluster share a vocabulary range; each
-  // loads one of the two W units of a chunk and multicasts it to both, and
-  // accumulates half of the window rows
+  // paired mode: the two CTAs of a cluster share a vocabulary range and
+  // accumulate half of the window rows each; both load every W tile of the
+  // range with plain TMA loads into their own shared memory (the cluster
+  // keeps the two co-resident, so the second read of a tile is an L2 hit)
   const uint32_t crank = PAIR ? cluster_ctarank() : 0u;
   const int cta = PAIR ? static_cast<int>(blockIdx.x >> 1) : static_cast<int>(blockIdx.x);
   const int rbase = p.row0 + static_cast<int>(crank) * p.rhalf;  // first row of this CTA
@@ -150,7 +151,7 @@ __global__ void __launch_bounds__(kLmThreads, 1)
   if (tid == 0) {
     for (int s = 0; s < p.stages; ++s) {
       mbar_init(&full[s], 1);
-      mbar_init(&empty[s], PAIR ? 2 : 1);  // paired: both CTAs' MMAs release a stage
+      mbar_init(&empty[s], 1);
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&acc_full[b], 1);
@@ -174,10 +175,7 @@ __global__ void __launch_bounds__(kLmThreads, 1)
     }
   }
   tc_fence_before();
-  if (PAIR)
-    cluster_sync_all();  // the peer's barriers exist before anything is multicast to them
-  else
-    __syncthreads();
+  __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_holder;
 
@@ -203,15 +201,11 @@ __global__ void __launch_bounds__(kLmThreads, 1)
         // one row half at a time, its k-boxes back to back: each W row is
         // requested as one contiguous run of nsubk * 128 bytes
         for (int ui = 0; ui < nu; ++ui) {
-          if (PAIR && (ui & 1) != static_cast<int>(crank)) continue;  // the peer loads it
           for (int j = 0; j < nsubk; ++j) {
             const int x = PACKED ? 0 : (ks * p.kbs + j) * 64;
             const int y = PACKED ? ((u + ui) * p.nkb + ks * p.kbs + j) * kUnit : (u + ui) * kUnit;
             uint8_t* dst = a_st + (ui >> 1) * a_chunk + j * kATile + (ui & 1) * (kUnit * 128);
-            if (PAIR)
-              tma_load_2d_multicast(dst, &tmap_w, &full[s], x, y, 0x3, pol_w);
-            else
-              tma_load_2d(dst, &tmap_w, &full[s], x, y, pol_w);
+            tma_load_2d(dst, &tmap_w, &full[s], x, y, pol_w);
           }
         }
       };
@@ -334,10 +328,7 @@ __global__ void __launch_bounds__(kLmThreads, 1)
               }
 #undef EBD_STAGE
             }
-            if (PAIR)
-              umma_commit_multicast(&empty[s], 0x3);
-            else
-              umma_commit(&empty[s]);
+            umma_commit(&empty[s]);
             ++it;
             if (++s == p.stages) {
               s = 0;
@@ -358,10 +349,7 @@ __global__ void __launch_bounds__(kLmThreads, 1)
                 }
               }
             }
-          if (PAIR)
-            umma_commit_multicast(&empty[s], 0x3);
-          else
-            umma_commit(&empty[s]);
+          umma_commit(&empty[s]);
           ++it;
           if (++s == p.stages) {
             s = 0;
@@ -501,7 +489,6 @@ __global__ void __launch_bounds__(kLmThreads, 1)
   }
 
   __syncthreads();
-  if (PAIR) cluster_sync_all();  // no multicast or remote arrival can target a CTA that left
   if (warp == 1) {
     tc_fence_after();
     tmem_dealloc(tmem_base, p.tmem_cols);
