@@ -240,6 +240,16 @@ def lbs_router(ent_norm_seq, xhat_seq, w_emb, W) -> np.ndarray:
     n = len(ent_norm_seq)
     if n == 0:
         return np.zeros(0)
+    z = lbs_input(ent_norm_seq, xhat_seq, w_emb, W)
+    for l in range(2):
+        z = lbs_encoder_layer(z, W, f"lbs.l{l}")
+    return linear(z, W, "lbs.head")[:, 0]
+
+
+def lbs_input(ent_norm_seq, xhat_seq, w_emb, W):
+    """Z_phi of Eq. lbs_feat (App. C.1) for the n masked rows:
+    W_combine [F_ent(H~) ; W_tok W_e(x_hat)] + E_pos[:n]."""
+    n = len(ent_norm_seq)
     Ht = np.asarray(ent_norm_seq, dtype=np.float64)[:, None]           # n x 1
     # entropy branch F_ent: Linear(1->64) -> GELU -> Linear(64->64) -> LN
     e = layer_norm(linear(gelu(linear(Ht, W, "lbs.ent1")), W, "lbs.ent2"),
@@ -247,11 +257,8 @@ def lbs_router(ent_norm_seq, xhat_seq, w_emb, W) -> np.ndarray:
     # token branch: frozen embedding W_e[x_hat], projected by W_tok
     Ex = bf16(w_emb[np.asarray(xhat_seq, dtype=np.int64)])                # n x d_base
     t = linear(Ex, W, "lbs.tok")
-    # fusion + learned positional embedding indexed by rank
-    z = linear(np.concatenate([e, t], axis=1), W, "lbs.comb") + W["lbs.pos"][:n]
-    for l in range(2):
-        z = lbs_encoder_layer(z, W, f"lbs.l{l}")
-    return linear(z, W, "lbs.head")[:, 0]
+    # fusion of [e ; t], then the learned positional embedding indexed by rank
+    return linear(np.concatenate([e, t], axis=1), W, "lbs.comb") + W["lbs.pos"][:n]
 
 
 def lbs_encoder_layer(z, W, p):
@@ -282,10 +289,16 @@ def lps_router(feats, W) -> np.ndarray:
     x = np.asarray(feats, dtype=np.float64)
     if x.shape[0] == 0:
         return np.zeros(0)
-    z = gelu(layer_norm(linear(x, W, "lps.in"), W["lps.in_ln.g"], W["lps.in_ln.b"]))
+    z = lps_input(x, W)
     for l in range(2):
         z = lps_block(z, W, f"lps.l{l}")
     return linear(z, W, "lps.head")[:, 0]
+
+
+def lps_input(x, W):
+    """Z_psi (App. D.1): a linear projection of the 5 features to d = 32,
+    then LayerNorm, then GELU."""
+    return gelu(layer_norm(linear(x, W, "lps.in"), W["lps.in_ln.g"], W["lps.in_ln.b"]))
 
 
 def lps_block(z, W, p):
@@ -335,14 +348,28 @@ def select_block(pos, M, O, argmax, prm: DecisionParams):
     return B
 
 
+def lps_features(pos, mask, in_block, meta, st: RowStats):
+    """The LPS inputs of the active block (Sec. 5.2, App. E): the still-masked
+    rows BM of B in ascending position, and per row i of BM the tuple
+    (kappa_i, H~_i, Delta_i, rho, pos_i) with rho = |B n M| / |B| (Reading R4)
+    and pos_i = (i - b) / |B| (Reading R5), b and |B| from meta."""
+    BM = [i for i in range(len(pos)) if in_block[i] and mask[i]]
+    size = int(meta[1])
+    rho = len(BM) / size if BM else 0.0
+    feats = [(st.conf[i], st.ent_norm[i], st.gap[i], rho,
+              (int(pos[i]) - int(meta[0])) / size) for i in BM]
+    return BM, feats
+
+
 def decide_sequence(pos, mask, tokens, in_block, meta, st: RowStats,
-                    w_emb, W, prm: DecisionParams, lbs_fn=None) -> SeqDecision:
+                    w_emb, W, prm: DecisionParams, lbs_fn=None, lps_fn=None) -> SeqDecision:
     """One step of the App. E algorithm for one sequence, on its window rows.
 
     pos/mask/tokens/in_block are this sequence's rows (ascending position);
     meta = [b, |B|] (|B| = 0: no active block).  mask, tokens, in_block and
     meta are updated in place.  st holds the statistics of these rows.
-    lbs_fn(ent_norm_seq, xhat_seq) replaces the LBS router (tests only)."""
+    lbs_fn(ent_norm_seq, xhat_seq) replaces the LBS router and lps_fn(feats)
+    the LPS router's logit O_psi (tests only)."""
     n = len(pos)
     out = SeqDecision(lbs_logit=np.full(n, np.nan), lps_prob=np.full(n, np.nan),
                       accepted=np.zeros(n, np.uint8))
@@ -363,15 +390,13 @@ def decide_sequence(pos, mask, tokens, in_block, meta, st: RowStats,
                 in_block[i] = 1
             meta[0], meta[1] = int(pos[B[0]]), len(B)
     Bset = [i for i in range(n) if in_block[i]]
-    BM = [i for i in Bset if mask[i]]
     size = int(meta[1])
+    BM, feats = lps_features(pos, mask, in_block, meta, st)   # R4, R5, R13
     if BM:
-        rho = len(BM) / size                                   # R4
-        feats = [(st.conf[i], st.ent_norm[i], st.gap[i], rho,
-                  (int(pos[i]) - int(meta[0])) / size) for i in BM]   # R5
         p_psi = None
         if prm.lps_enabled:
-            p_psi = sigmoid(lps_router(feats, W))
+            router = lps_fn or (lambda f: lps_router(f, W))
+            p_psi = sigmoid(np.asarray(router(feats), dtype=np.float64))
             out.lps_prob[BM] = p_psi
         A = [i for j, i in enumerate(BM)                       # union accept rule
              if st.conf[i] >= prm.tau or

@@ -225,3 +225,37 @@ def test_full_sequence_loop_invariants():
         committed |= acc
     assert committed.all()
     assert any(r["lbs_ran"] for r in recs), "the LBS never ran on the whole response"
+
+
+def _lps_feature_case(c):
+    """Runs the per-sequence step on a golden case of lps_features.json with
+    the LPS logit replaced by 0 (p_psi = 1/2, below tau_psi); returns the
+    feature tuples the router received and the rows it scored."""
+    n = len(c["pos"])
+    seen = []
+
+    def capture(feats):
+        seen.append(np.array(feats, dtype=np.float64))
+        return np.zeros(len(feats))
+    st = o.RowStats(conf=np.array(c["conf"], float), entropy=np.zeros(n),
+                    ent_norm=np.array(c["ent_norm"], float), gap=np.array(c["gap"], float),
+                    argmax=np.arange(n, dtype=np.int64) + 100, logit_gap=np.ones(n),
+                    near_tie=np.zeros(n, bool))
+    prm = o.DecisionParams(tau=0.9, tau_psi=0.9, l_min=8, l_b=32, g_max=5, eos_id=-1)
+    d = o.decide_sequence(np.array(c["pos"]), np.array(c["mask"], np.uint8),
+                          np.full(n, -1, np.int32), np.array(c["in_block"], np.uint8),
+                          np.array(c["meta"], np.int32), st, None, {}, prm, lps_fn=capture)
+    assert len(seen) == 1
+    return seen[0], np.flatnonzero(~np.isnan(d.lps_prob)).tolist()
+
+
+def test_lps_feature_tuple_golden():
+    """The LPS input tuple (kappa, H~, Delta, rho, pos) of every still-masked
+    row of the block, in ascending position (Sec. 5.2, App. E; Readings R4,
+    R5, R13), against hand-worked values."""
+    g = json.load(open(os.path.join(GOLD, "lps_features.json")))
+    for c in g["cases"]:
+        feats, rows = _lps_feature_case(c)
+        assert rows == c["rows"], c["note"]
+        np.testing.assert_allclose(feats, np.array(c["features"]), rtol=0, atol=1e-15,
+                                   err_msg=c["note"])

@@ -10,7 +10,11 @@ rows instead of L_B; a strict kappa > tau in the accept rule; the tanh
 approximation of GELU; a LayerNorm eps of 1e-6; an attention scale of
 1/sqrt(d) instead of 1/sqrt(d/heads) in the routers; EOS kept among the
 router candidates; the dual-cache suffix read one position late; the cache
-append writing masked rows too."""
+append writing masked rows too; the LPS features in another order, pos
+divided by |B n M|, rho over the whole window, GELU before LayerNorm in the
+LPS input layer; in the LBS input (Eq. lbs_feat) the token branch first in
+the fusion, E_pos added before W_combine, LayerNorm and GELU swapped in
+F_ent."""
 import numpy as np
 import pytest
 
@@ -223,3 +227,91 @@ def test_append_of_masked_rows_is_caught(monkeypatch):
     monkeypatch.setattr(o, "kv_append", lambda kc, vc, kw, vw, cu, row_pos, mask:
                         real(kc, vc, kw, vw, cu, row_pos, np.zeros_like(mask)))
     assert _some_pin_fails([ta.test_kv_append_writes_committed_rows_only])
+
+
+# ---------------------------------------------------------------- router inputs
+def _input_pins():
+    return [td.test_lps_feature_tuple_golden, tr.test_lps_router_matches_torch_modules,
+            tr.test_lbs_router_matches_torch_modules]
+
+
+def test_input_pins_pass_as_they_stand():
+    assert not _some_pin_fails(_input_pins())
+
+
+@pytest.mark.parametrize("order", [(1, 0, 2, 3, 4), (0, 1, 2, 4, 3), (4, 0, 1, 2, 3)])
+def test_lps_features_in_another_order_are_caught(monkeypatch, order):
+    real = o.lps_features
+
+    def reordered(pos, mask, in_block, meta, st):
+        BM, feats = real(pos, mask, in_block, meta, st)
+        return BM, [tuple(f[k] for k in order) for f in feats]
+    monkeypatch.setattr(o, "lps_features", reordered)
+    assert _some_pin_fails([td.test_lps_feature_tuple_golden])
+
+
+def test_pos_over_the_masked_count_is_caught(monkeypatch):
+    """pos = (i - b) / |B n M| instead of / |B|"""
+    real = o.lps_features
+
+    def pos_masked(pos, mask, in_block, meta, st):
+        BM, feats = real(pos, mask, in_block, meta, st)
+        return BM, [f[:4] + (f[4] * int(meta[1]) / len(BM),) for f in feats]
+    monkeypatch.setattr(o, "lps_features", pos_masked)
+    assert _some_pin_fails([td.test_lps_feature_tuple_golden])
+
+
+def test_rho_over_the_window_is_caught(monkeypatch):
+    """rho = |M| / window rows (a window-wide mask ratio) instead of |B n M| / |B|"""
+    real = o.lps_features
+
+    def rho_window(pos, mask, in_block, meta, st):
+        BM, feats = real(pos, mask, in_block, meta, st)
+        rho = float(np.count_nonzero(mask)) / len(mask)
+        return BM, [f[:3] + (rho, f[4]) for f in feats]
+    monkeypatch.setattr(o, "lps_features", rho_window)
+    assert _some_pin_fails([td.test_lps_feature_tuple_golden])
+
+
+def test_gelu_before_layer_norm_in_the_lps_input_is_caught(monkeypatch):
+    monkeypatch.setattr(o, "lps_input", lambda x, W: o.layer_norm(
+        o.gelu(o.linear(x, W, "lps.in")), W["lps.in_ln.g"], W["lps.in_ln.b"]))
+    assert _some_pin_fails(_input_pins())
+
+
+def _lbs_parts(ent_norm_seq, xhat_seq, w_emb, W, ent_order="lin-gelu-lin-ln"):
+    Ht = np.asarray(ent_norm_seq, dtype=np.float64)[:, None]
+    if ent_order == "lin-gelu-lin-ln":
+        e = o.layer_norm(o.linear(o.gelu(o.linear(Ht, W, "lbs.ent1")), W, "lbs.ent2"),
+                         W["lbs.ent_ln.g"], W["lbs.ent_ln.b"])
+    else:  # LayerNorm and GELU swapped
+        e = o.gelu(o.linear(o.layer_norm(o.linear(Ht, W, "lbs.ent1"), W["lbs.ent_ln.g"],
+                                         W["lbs.ent_ln.b"]), W, "lbs.ent2"))
+    t = o.linear(o.bf16(w_emb[np.asarray(xhat_seq, dtype=np.int64)]), W, "lbs.tok")
+    return e, t
+
+
+def test_token_branch_first_in_the_fusion_is_caught(monkeypatch):
+    """[t ; e] instead of [e ; t] (Eq. lbs_feat)"""
+    def swapped(h, x, w_emb, W):
+        e, t = _lbs_parts(h, x, w_emb, W)
+        return o.linear(np.concatenate([t, e], axis=1), W, "lbs.comb") + W["lbs.pos"][:len(h)]
+    monkeypatch.setattr(o, "lbs_input", swapped)
+    assert _some_pin_fails(_input_pins())
+
+
+def test_position_table_before_the_fusion_is_caught(monkeypatch):
+    """W_combine([e ; t] + E_pos) instead of W_combine [e ; t] + E_pos"""
+    def pos_first(h, x, w_emb, W):
+        e, t = _lbs_parts(h, x, w_emb, W)
+        return o.linear(np.concatenate([e, t], axis=1) + W["lbs.pos"][:len(h)], W, "lbs.comb")
+    monkeypatch.setattr(o, "lbs_input", pos_first)
+    assert _some_pin_fails(_input_pins())
+
+
+def test_layer_norm_and_gelu_swapped_in_the_entropy_branch_are_caught(monkeypatch):
+    def swapped(h, x, w_emb, W):
+        e, t = _lbs_parts(h, x, w_emb, W, ent_order="lin-ln-lin-gelu")
+        return o.linear(np.concatenate([e, t], axis=1), W, "lbs.comb") + W["lbs.pos"][:len(h)]
+    monkeypatch.setattr(o, "lbs_input", swapped)
+    assert _some_pin_fails(_input_pins())

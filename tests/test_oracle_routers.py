@@ -5,8 +5,10 @@ paper is unpinned; what is pinned here: the parameter count the paper states
 for LBS ("600k", App. C.1), the zero-weight closed form (all weights zero but
 the head bias c gives O = c at every row), the layer structure against
 PyTorch's own nn.TransformerEncoderLayer / LayerNorm / GELU (post-norm for
-LBS, pre-norm for LPS), and permutation equivariance where the architecture
-has no positional table.
+LBS, pre-norm for LPS), both whole routers against torch.nn modules assembled
+from the sizes and the order of App. C.1 (F_ent, the [e ; t] fusion, E_pos
+after W_combine) and App. D.1 (Linear, LayerNorm, GELU input layer), and
+permutation equivariance where the architecture has no positional table.
 """
 import numpy as np
 import pytest
@@ -153,3 +155,75 @@ def test_splitmix64_published_vectors():
         [0xE220A8397B1DCDAF, 0x6E789E6AA1B965F4, 0x06C45D188009454F]
     assert [r._mix_int((1234567 + k * G) % 2 ** 64) for k in (1, 2, 3)] == \
         [6457827717110365317, 3203168211198807973, 9817491932198370423]
+
+
+def _lin(W, name, fan_in, fan_out):
+    m = torch.nn.Linear(fan_in, fan_out, dtype=torch.float64)
+    m.load_state_dict({"weight": torch.from_numpy(np.array(W[name + ".w"])),
+                       "bias": torch.from_numpy(np.array(W[name + ".b"]))})
+    return m
+
+
+def _ln(W, name, width):
+    m = torch.nn.LayerNorm(width, eps=1e-5, dtype=torch.float64)
+    m.load_state_dict({"weight": torch.from_numpy(np.array(W[name + ".g"])),
+                       "bias": torch.from_numpy(np.array(W[name + ".b"]))})
+    return m
+
+
+def torch_lps_router(feats, W):
+    """The LPS router of App. D.1 assembled from torch.nn modules at the
+    stated sizes: Linear(5 -> 32) -> LayerNorm -> GELU, two pre-norm encoder
+    blocks (4 heads, FFN 64, GELU), Linear(32 -> 1)."""
+    net = torch.nn.Sequential(_lin(W, "lps.in", 5, 32), _ln(W, "lps.in_ln", 32),
+                              torch.nn.GELU(),
+                              _torch_layer(W, "lps.l0", 32, 4, 64, norm_first=True),
+                              _torch_layer(W, "lps.l1", 32, 4, 64, norm_first=True),
+                              _lin(W, "lps.head", 32, 1))
+    net.eval()
+    with torch.no_grad():
+        return net(torch.from_numpy(np.asarray(feats, np.float64))[None])[0, :, 0].numpy()
+
+
+def torch_lbs_router(ent_norm_seq, xhat_seq, w_emb, W):
+    """The LBS router of App. C.1 assembled from torch.nn modules at the
+    stated sizes: F_ent = Linear(1 -> 64) -> GELU -> Linear(64 -> 64) ->
+    LayerNorm; token branch W_tok W_e(x_hat) with W_e a frozen nn.Embedding;
+    Z = W_combine [F_ent ; token] + E_pos (Eq. lbs_feat); two post-norm
+    encoder layers (4 heads, FFN 256, GELU); Linear(128 -> 1)."""
+    d_base = w_emb.shape[1]
+    f_ent = torch.nn.Sequential(_lin(W, "lbs.ent1", 1, 64), torch.nn.GELU(),
+                                _lin(W, "lbs.ent2", 64, 64), _ln(W, "lbs.ent_ln", 64))
+    emb = torch.nn.Embedding.from_pretrained(torch.from_numpy(o.bf16(w_emb)), freeze=True)
+    tok = _lin(W, "lbs.tok", d_base, 64)
+    comb = _lin(W, "lbs.comb", 128, 128)
+    enc = torch.nn.Sequential(_torch_layer(W, "lbs.l0", 128, 4, 256, norm_first=False),
+                              _torch_layer(W, "lbs.l1", 128, 4, 256, norm_first=False))
+    enc.eval()
+    head = _lin(W, "lbs.head", 128, 1)
+    h = torch.from_numpy(np.asarray(ent_norm_seq, np.float64))[:, None]
+    x = torch.from_numpy(np.asarray(xhat_seq, np.int64))
+    with torch.no_grad():
+        z = comb(torch.cat([f_ent(h), tok(emb(x))], dim=-1))
+        z = z + torch.from_numpy(np.array(W["lbs.pos"]))[:len(x)]
+        return head(enc(z[None])[0])[:, 0].numpy()
+
+
+def test_lps_router_matches_torch_modules():
+    """The whole LPS router, input layer order included (Linear, then
+    LayerNorm, then GELU), against torch.nn modules built from App. D.1."""
+    W = _perturb_ln(_W())
+    f = np.random.default_rng(21).random((7, 5)) * np.array([1, 1, 1, 1, 1.6])
+    np.testing.assert_allclose(o.lps_router(f, W), torch_lps_router(f, W), rtol=1e-10, atol=1e-10)
+
+
+def test_lbs_router_matches_torch_modules():
+    """The whole LBS router, Eq. lbs_feat included (F_ent's order, the [e ; t]
+    concatenation, E_pos added after W_combine), against torch.nn modules
+    built from App. C.1."""
+    W = _perturb_ln(_W())
+    emb = synth.f32_to_bf16_bits(np.random.default_rng(22).standard_normal((60, 64)))
+    h = np.random.default_rng(23).random(13)
+    x = np.random.default_rng(24).integers(0, 60, 13)
+    np.testing.assert_allclose(o.lbs_router(h, x, emb, W), torch_lbs_router(h, x, emb, W),
+                               rtol=1e-10, atol=1e-10)
