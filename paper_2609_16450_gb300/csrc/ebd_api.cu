@@ -190,7 +190,8 @@ struct ebd_handle {
   const uint16_t* w_emb = nullptr;
   float4* part_f = nullptr;
   int* part_i = nullptr;
-  int grid_lm = 0;
+  int grid_lm = 0;       // LM-head partial states per row
+  int lm_units = 0;      // 64-row vocabulary units
   float* attn_part = nullptr;
   float* attn_part_ml = nullptr;
   int* tickets = nullptr;
@@ -669,12 +670,13 @@ ebd_status run_lm(ebd_handle* h, const ebd_step_args* a, cudaStream_t st, bool p
   for (int g0 = 0; g0 < a->rows; g0 += kMaxGroupRows) {
     const int rows = a->rows - g0 < kMaxGroupRows ? a->rows - g0 : kMaxGroupRows;
     LmParams p{};
-    // 257..512 rows: CTA pairs that read the same W range and split the
-    // rows, which keeps each CTA's accumulator within 256 TMEM columns
-    // (double-buffered).
-    bool pair = rows > 256 && rows <= 512;
-    if (const char* env = getenv("EBD_LM_PAIR")) pair = pair && atoi(env) != 0;
+    // from kLmPairMinRows rows on, CTA pairs run cta_group::2 MMAs of
+    // M = 256: each SM receives half of the hidden rows per MMA
+    int pair_min = kLmPairMinRows;
+    if (const char* env = getenv("EBD_LM_PAIR_MIN")) pair_min = atoi(env) > 0 ? atoi(env) : kMaxGroupRows + 1;
+    const bool pair = rows >= pair_min && h->grid_lm >= lm_pair_grid(h->num_sms, h->lm_units);
     lm_plan(p, rows, c.vocab, c.d_model, h->num_sms, pair);
+    p.ncols = h->grid_lm;
     if (p.stages < 2) return fail(h, EBD_ERR_UNSUPPORTED, "LM head: shared memory plan failed");
     p.row0 = g0;
     p.packed = packed ? 1 : 0;
@@ -687,7 +689,8 @@ ebd_status run_lm(ebd_handle* h, const ebd_step_args* a, cudaStream_t st, bool p
     CUtensorMap th;
     const uint64_t dims[2] = {static_cast<uint64_t>(c.d_model), static_cast<uint64_t>(a->rows)};
     const uint64_t str[1] = {static_cast<uint64_t>(c.d_model) * 2};
-    const uint32_t box[2] = {64, static_cast<uint32_t>(p.nb)};
+    // a CTA of a pair loads half of each N sub-tile of hidden rows
+    const uint32_t box[2] = {64, static_cast<uint32_t>(p.pair ? p.nb / 2 : p.nb)};
     if (!encode_bf16(&th, a->hidden, 2, dims, str, box))
       return fail(h, EBD_ERR_CUDA, "cuTensorMapEncodeTiled (hidden) failed");
     cudaError_t e = launch_lm_stats(tw, th, p, st);
@@ -859,7 +862,14 @@ ebd_status ebd_create(const ebd_config* cfg, ebd_handle** out) {
   if ((s = upload_router(h)) != EBD_OK) return bail(s);
 
   // LM-head partials: one state per (row, CTA)
-  h->grid_lm = lm_grid(h->num_sms, (cfg->vocab + kUnit - 1) / kUnit);
+  h->lm_units = (cfg->vocab + kUnit - 1) / kUnit;
+  h->grid_lm = lm_grid(h->num_sms, h->lm_units);
+  {  // a handle whose steps may take the paired LM head leaves room for its partials
+    int pair_min = kLmPairMinRows;
+    if (const char* env = getenv("EBD_LM_PAIR_MIN")) pair_min = atoi(env) > 0 ? atoi(env) : kMaxGroupRows + 1;
+    const int pg = lm_pair_grid(h->num_sms, h->lm_units);
+    if (cfg->max_rows >= pair_min && pg > h->grid_lm) h->grid_lm = pg;
+  }
   const size_t np = static_cast<size_t>(cfg->max_rows) * h->grid_lm;
   if ((e = cudaMalloc(&h->part_f, np * sizeof(float4))) != cudaSuccess)
     return bail(cuda_fail(h, e, "cudaMalloc(partials)"));

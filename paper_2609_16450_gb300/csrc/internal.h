@@ -27,17 +27,15 @@ struct LmParams {
   int row0, rows;           // rows [row0, row0 + rows) of this launch
   int nb, nsub, n_pad;      // MMA N per sub-tile, sub-tiles, padded N = nb * nsub
   int n_units;              // ceil(V / 64)
-  int grid;                 // CTAs (partials per row)
+  int grid;                 // CTAs (each writes one partial per row)
   int nkb;                  // ceil(d / 64) k-blocks of 64 columns
   int kbs, nks;             // k-blocks per pipeline stage, stages per vocabulary chunk
   int packed;               // W is tiled: tile (unit, k-block) at row (unit*nkb + kb)*64
   int stages, nbuf, acc_stride, tmem_cols;
   int nwg;                  // epilogue warpgroups in use (2 with a single accumulator buffer)
-  int pair;                 // clusters of 2 CTAs: same W range, rows split in halves
-  int rhalf;                // rows of one CTA of a pair (rows of the launch otherwise)
+  int pair;                 // CTA pairs (clusters of 2) running cta_group::2 MMAs, M = 256
+  int nwork;                // owners of vocabulary ranges: CTAs, or pairs
   int ncols;                // partial states per row written (>= grid; extra ones neutral)
-  int mch;                  // 128-row vocabulary chunks per pipeline stage (1, or 2: one
-                            // hidden tile feeds two accumulators)
   uint32_t off_a, off_b, off_t, off_st, off_bar, smem_bytes;
   float4* part_f;           // [R][grid] (max, sum exp, sum exp*(l-max), second logit)
   int* part_i;              // [R][grid] argmax
@@ -167,7 +165,10 @@ struct SeqParams {
 // host launchers (defined next to their kernels)
 cudaError_t launch_lm_stats(const CUtensorMap& tmap_w, const CUtensorMap& tmap_h,
                             const LmParams& p, cudaStream_t st);
-int lm_grid(int num_sms, int n_units);  // partial states per row of the LM head
+int lm_grid(int num_sms, int n_units);       // CTAs of the unpaired LM head
+int lm_pair_grid(int num_sms, int n_units);  // CTAs of the paired (cta_group::2) LM head
+// rows of an LM-head launch from which CTA pairs run it (and up to kMaxGroupRows)
+constexpr int kLmPairMinRows = 65;
 void lm_plan(LmParams& p, int rows, int V, int d, int num_sms, bool pair = false);
 // pdl: launched as a programmatic dependent of the kernel before it on
 // `st` (that kernel's CTAs release it early; the attention reads nothing the

@@ -14,7 +14,9 @@
 // (A = W rows, K-major, streamed by TMA with an evict-first L2 policy), the
 // window rows are N (B = hidden rows, K-major), the fp32 accumulator lives
 // in TMEM as 128 lanes (vocabulary) x N columns (rows).  Warp 0 issues TMA,
-// warp 1 issues tcgen05.mma, warps 2..5 drain TMEM and run the statistics.
+// warp 1 issues tcgen05.mma, warps 2..5 (and 6..9) drain TMEM and run the
+// statistics.  Where the rows make the tensor cores the bound, CTA pairs run
+// cta_group::2 MMAs with M = 256 (two SMs, one accumulator tile).
 #include <climits>
 #include <cstdlib>
 
@@ -27,7 +29,7 @@ namespace {
 
 constexpr uint32_t kATile = 128 * 128;  // 128 rows x 64 bf16
 constexpr int kTLd = 132;               // transpose buffer row stride (floats)
-constexpr uint32_t kTBytes = 32 * kTLd * 4;
+constexpr uint32_t kTBytes = 32 * kTLd * 4;  // transpose buffer of one epilogue warpgroup
 
 __device__ __forceinline__ void state_merge(float& m, float& s, float& t, float& l2, int& idx,
                                             float bm, float bs, float bt, float bl2, int bidx) {
@@ -63,7 +65,7 @@ __device__ __forceinline__ bool named_barrier_and(uint32_t id, uint32_t n, bool 
 // descriptors advanced by immediates (k16 step = 32 bytes = 2 in the
 // descriptor's address field; k-box = kATile bytes of A, b_step of B; N
 // sub-tile sb at sb * sub_desc of B and sb * sub_cols TMEM columns).
-template <int KBS, int NSUB>
+template <int KBS, int NSUB, bool PAIR>
 __device__ __forceinline__ void mma_stage(uint32_t d, uint32_t a_lo, uint32_t b_lo,
                                           uint32_t b_step, uint32_t sub_desc, uint32_t sub_cols,
                                           uint32_t hi, uint32_t idesc, uint32_t acc0) {
@@ -72,12 +74,16 @@ __device__ __forceinline__ void mma_stage(uint32_t d, uint32_t a_lo, uint32_t b_
 #pragma unroll
     for (int kk = 0; kk < 4; ++kk)
 #pragma unroll
-      for (int sb = 0; sb < NSUB; ++sb)
-        umma_bf16_lo(d + static_cast<uint32_t>(sb) * sub_cols,
-                     a_lo + static_cast<uint32_t>(j * (kATile >> 4) + kk * 2),
-                     b_lo + static_cast<uint32_t>(j) * b_step + static_cast<uint32_t>(sb) * sub_desc +
-                         static_cast<uint32_t>(kk * 2),
-                     hi, idesc, (j | kk) != 0 ? 1u : acc0);
+      for (int sb = 0; sb < NSUB; ++sb) {
+        const uint32_t dd = d + static_cast<uint32_t>(sb) * sub_cols;
+        const uint32_t al = a_lo + static_cast<uint32_t>(j * (kATile >> 4) + kk * 2);
+        const uint32_t bl = b_lo + static_cast<uint32_t>(j) * b_step +
+                            static_cast<uint32_t>(sb) * sub_desc + static_cast<uint32_t>(kk * 2);
+        if (PAIR)
+          umma_bf16_lo_pair(dd, al, bl, hi, idesc, (j | kk) != 0 ? 1u : acc0);
+        else
+          umma_bf16_lo(dd, al, bl, hi, idesc, (j | kk) != 0 ? 1u : acc0);
+      }
 }
 
 // Waits with a back-off between polls: for warps whose wait is long and not
@@ -100,14 +106,101 @@ __device__ __forceinline__ void record_error(int* status, volatile int* abort, i
   atomicCAS(status, 0, code);
 }
 
+// Statistics of one accumulator buffer by one epilogue warpgroup, in slices
+// of 32 columns (window rows): each slice goes TMEM -> registers -> a
+// transpose in shared memory, after which 4 threads share a column and scan
+// its 128 vocabulary lanes (32 each); the column's state is merged into the
+// running state of its row.  `release` is called once this thread has
+// loaded its last slice (the MMAs may then overwrite the buffer).  Returns
+// whether it was called.
+template <typename Release>
+__device__ __forceinline__ bool epilogue_buffer(uint32_t taddr0, int wg, int nwg, int n_pad,
+                                                float* sTw, int lanev, int et, uint32_t bar_id,
+                                                int vbase, int valid, float* st_m, float* st_s,
+                                                float* st_t, float* st_l2, int* st_i,
+                                                Release release) {
+  bool released = false;
+  const bool lv = lanev < valid;
+  for (int cc = 32 * wg; cc < n_pad; cc += 32 * nwg) {
+    float v[32];
+    if (n_pad - cc >= 32)
+      tmem_ld_32x32b_x32(taddr0 + static_cast<uint32_t>(cc), v);
+    else
+      tmem_ld_32x32b_x16(taddr0 + static_cast<uint32_t>(cc), v);
+    if (cc + 32 * nwg >= n_pad) {  // this warpgroup's last slice is in registers
+      release();
+      released = true;
+    }
+#pragma unroll
+    for (int j = 0; j < 32; ++j) sTw[j * kTLd + lanev] = lv ? v[j] : -INFINITY;
+    named_barrier(bar_id, 128);
+    {
+      const int j = et >> 2, q = et & 3;
+      float x[32];
+#pragma unroll
+      for (int i = 0; i < 32; ++i) x[i] = sTw[j * kTLd + q + 4 * i];
+      // branch-free scan: the threads of a warp see different data
+      float m = -INFINITY, l2 = -INFINITY;
+      int ii = -1;
+#pragma unroll
+      for (int i = 0; i < 32; ++i) {
+        l2 = fmaxf(l2, fminf(m, x[i]));
+        ii = x[i] > m ? i : ii;  // strict: the first (lowest) index of the maximum
+        m = fmaxf(m, x[i]);
+      }
+      int idx = ii < 0 ? INT_MAX : vbase + q + 4 * ii;
+      float s = 0.f, t = 0.f;
+      if (m != -INFINITY) {
+#pragma unroll
+        for (int i = 0; i < 32; ++i) {
+          const float dl = x[i] - m;
+          const float e = __expf(dl);
+          s += e;
+          t = fmaf(e, e > 0.f ? dl : 0.f, t);  // masked lanes: e = 0, dl = -inf
+        }
+      }
+#pragma unroll
+      for (int off = 1; off <= 2; off <<= 1) {
+        const float bm = __shfl_xor_sync(0xffffffffu, m, off);
+        const float bs = __shfl_xor_sync(0xffffffffu, s, off);
+        const float bt = __shfl_xor_sync(0xffffffffu, t, off);
+        const float bl = __shfl_xor_sync(0xffffffffu, l2, off);
+        const int bi = __shfl_xor_sync(0xffffffffu, idx, off);
+        state_merge(m, s, t, l2, idx, bm, bs, bt, bl, bi);
+      }
+      const int r = cc + j;
+      if (q == 0 && r < n_pad) {
+        float M = st_m[r], S = st_s[r], T = st_t[r], L2 = st_l2[r];
+        int I = st_i[r];
+        state_merge(M, S, T, L2, I, m, s, t, l2, idx);
+        st_m[r] = M;
+        st_s[r] = S;
+        st_t[r] = T;
+        st_l2[r] = L2;
+        st_i[r] = I;
+      }
+    }
+    named_barrier(bar_id, 128);
+  }
+  return released;
+}
+
 }  // namespace
 
-// PAIR (p.pair), PACKED (p.packed) and MCH (p.mch) are template parameters:
-// a runtime branch in the single-thread producer or MMA loop costs
-// measurable time.  With MCH = 2 a pipeline stage holds two 128-row chunks of
-// W and one tile of hidden rows; the chunks accumulate into two TMEM regions,
-// which halves the hidden bytes per MMA where the tensor cores are the bound.
-template <bool PAIR, bool PACKED, int MCH>
+// PAIR (p.pair) and PACKED (p.packed) are template parameters: a runtime
+// branch in the single-thread producer or MMA loop costs measurable time.
+//
+// PAIR: the CTAs of a cluster of 2 form a pair that runs cta_group::2 MMAs
+// of M = 256 vocabulary rows.  A vocabulary chunk is 4 units: the even CTA
+// (the leader) loads units 0-1 of it, the odd CTA units 2-3, each into its
+// own shared memory; each loads its half of every N sub-tile of hidden rows.
+// The leader's thread issues the MMAs, whose 256 x N accumulator lands as
+// 128 lanes x N columns in each CTA's TMEM, and its commits arrive on both
+// CTAs' barriers.  Both CTAs' copies complete on the leader's stage
+// barriers; both epilogues release the accumulator on the leader's barrier.
+// Each SM thus receives half of the hidden rows per MMA, which halves the
+// operand bytes per flop against a 128-row tile over the same rows.
+template <bool PAIR, bool PACKED>
 __global__ void __launch_bounds__(kLmThreads, 1)
     lm_stats_kernel(const __grid_constant__ CUtensorMap tmap_w,
                     const __grid_constant__ CUtensorMap tmap_h, const LmParams p) {
@@ -132,6 +225,7 @@ __global__ void __launch_bounds__(kLmThreads, 1)
   uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(dummy + 1);
   volatile int* abort = reinterpret_cast<volatile int*>(tmem_holder + 1);
 
+  constexpr int kChunkUnits = PAIR ? 4 : 2;  // vocabulary units per accumulator
   const int tid = threadIdx.x;
   // the decision kernel, launched after this one as a programmatic dependent,
   // may be scheduled as soon as SMs free up; it waits for this grid's
@@ -139,14 +233,13 @@ __global__ void __launch_bounds__(kLmThreads, 1)
   // this grid releases it only after its own wait, below)
   const int warp = __shfl_sync(0xffffffffu, tid / 32, 0);
   const int lane = tid & 31;
-  // paired mode: the two CTAs of a cluster share a vocabulary range and
-  // accumulate half of the window rows each; both load every W tile of the
-  // range with plain TMA loads into their own shared memory (the cluster
-  // keeps the two co-resident, so the second read of a tile is an L2 hit)
   const uint32_t crank = PAIR ? cluster_ctarank() : 0u;
-  const int cta = PAIR ? static_cast<int>(blockIdx.x >> 1) : static_cast<int>(blockIdx.x);
-  const int rbase = p.row0 + static_cast<int>(crank) * p.rhalf;  // first row of this CTA
-  const int rows_c = min(p.rhalf, p.rows - static_cast<int>(crank) * p.rhalf);
+  const bool leader = crank == 0;
+  const int owner = PAIR ? static_cast<int>(blockIdx.x >> 1) : static_cast<int>(blockIdx.x);
+  const int rbase = p.row0;  // first row of the launch
+  // hidden rows of one N sub-tile that this CTA holds: all of them, or its
+  // half in a pair
+  const int hrows = PAIR ? p.nb / 2 : p.nb;
 
   if (tid == 0) {
     for (int s = 0; s < p.stages; ++s) {
@@ -155,7 +248,7 @@ __global__ void __launch_bounds__(kLmThreads, 1)
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&acc_full[b], 1);
-      mbar_init(&acc_empty[b], 128 * p.nwg);
+      mbar_init(&acc_empty[b], (PAIR ? 2 : 1) * 128 * p.nwg);  // both CTAs' epilogues
     }
     mbar_init(drain, 1);
     mbar_init(dummy, 1);
@@ -164,7 +257,12 @@ __global__ void __launch_bounds__(kLmThreads, 1)
     tma_prefetch_desc(&tmap_w);
     tma_prefetch_desc(&tmap_h);
   }
-  if (warp == 1) tmem_alloc(tmem_holder, p.tmem_cols);
+  if (warp == 1) {
+    if (PAIR)
+      tmem_alloc_pair(tmem_holder, p.tmem_cols);
+    else
+      tmem_alloc(tmem_holder, p.tmem_cols);
+  }
   if (tid >= 64) {
     for (int r = tid - 64; r < p.n_pad; r += kLmThreads - 64) {
       st_m[r] = -INFINITY;
@@ -175,37 +273,49 @@ __global__ void __launch_bounds__(kLmThreads, 1)
     }
   }
   tc_fence_before();
-  __syncthreads();
+  if (PAIR)
+    cluster_sync_all();  // the peer's barriers exist before anything arrives on them
+  else
+    __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_holder;
 
-  const int u0 = static_cast<int>((static_cast<long long>(cta) * p.n_units) / p.grid);
-  const int u1 = static_cast<int>((static_cast<long long>(cta + 1) * p.n_units) / p.grid);
-  const uint32_t b_sub = static_cast<uint32_t>(p.n_pad) * 128u;  // one k-box of hidden rows
-  const uint32_t a_chunk = static_cast<uint32_t>(p.kbs) * kATile;  // one chunk's k-boxes
-  const uint32_t a_stage = static_cast<uint32_t>(MCH) * a_chunk;
+  const int u0 = static_cast<int>((static_cast<long long>(owner) * p.n_units) / p.nwork);
+  const int u1 = static_cast<int>((static_cast<long long>(owner + 1) * p.n_units) / p.nwork);
+  const uint32_t b_sub = static_cast<uint32_t>(p.nsub * hrows) * 128u;  // one k-box of hidden rows here
+  const uint32_t a_stage = static_cast<uint32_t>(p.kbs) * kATile;
   const uint32_t b_stage = static_cast<uint32_t>(p.kbs) * b_sub;
+  // W units of a chunk that this CTA loads and accumulates: [ulo, ulo + 2)
+  const int ulo = PAIR ? 2 * static_cast<int>(crank) : 0;
 
   if (warp == 0) {
     // ------------------------------------------------------------ TMA producer
     if (lane == 0) {
       const uint64_t pol_w = l2_policy_evict_first();
       const uint64_t pol_h = l2_policy_evict_last();
-      // stage fill: vocabulary chunk u (2 MCH units), k-stage ks
-      auto issue_w = [&](int u, int ks, int s) {  // arms the stage for W and hidden bytes
-        const int nu = min(2 * MCH, u1 - u);
+      auto load = [&](void* dst, const CUtensorMap* map, int s, int x, int y, uint64_t pol) {
+        if (PAIR)
+          tma_load_2d_pair(dst, map, mapa_shared(smem_u32(&full[s]), 0), x, y, pol);
+        else
+          tma_load_2d(dst, map, &full[s], x, y, pol);
+      };
+      // stage fill: vocabulary chunk u (kChunkUnits units), k-stage ks; the
+      // leader arms the stage for the W and hidden bytes of both CTAs
+      auto issue_w = [&](int u, int ks, int s) {
+        const int nu = min(kChunkUnits, u1 - u);
         const int nsubk = min(p.kbs, p.nkb - ks * p.kbs);
-        mbar_arrive_expect_tx(&full[s], static_cast<uint32_t>(nsubk) *
-                                            (static_cast<uint32_t>(nu) * kUnit * 128u + b_sub));
+        if (leader)
+          mbar_arrive_expect_tx(&full[s], static_cast<uint32_t>(nsubk) *
+                                              (static_cast<uint32_t>(nu) * kUnit * 128u +
+                                               static_cast<uint32_t>(p.n_pad) * 128u));
         uint8_t* a_st = sA + static_cast<size_t>(s) * a_stage;
-        // one row half at a time, its k-boxes back to back: each W row is
+        // one unit at a time, its k-boxes back to back: each W row is
         // requested as one contiguous run of nsubk * 128 bytes
-        for (int ui = 0; ui < nu; ++ui) {
+        for (int ui = ulo; ui < min(ulo + 2, nu); ++ui) {
           for (int j = 0; j < nsubk; ++j) {
             const int x = PACKED ? 0 : (ks * p.kbs + j) * 64;
             const int y = PACKED ? ((u + ui) * p.nkb + ks * p.kbs + j) * kUnit : (u + ui) * kUnit;
-            uint8_t* dst = a_st + (ui >> 1) * a_chunk + j * kATile + (ui & 1) * (kUnit * 128);
-            tma_load_2d(dst, &tmap_w, &full[s], x, y, pol_w);
+            load(a_st + j * kATile + (ui - ulo) * (kUnit * 128), &tmap_w, s, x, y, pol_w);
           }
         }
       };
@@ -214,14 +324,14 @@ __global__ void __launch_bounds__(kLmThreads, 1)
         uint8_t* b_st = sB + static_cast<size_t>(s) * b_stage;
         for (int j = 0; j < nsubk; ++j)
           for (int sb = 0; sb < p.nsub; ++sb)
-            tma_load_2d(b_st + j * b_sub + sb * p.nb * 128, &tmap_h, &full[s],
-                        (ks * p.kbs + j) * 64, rbase + sb * p.nb, pol_h);
+            load(b_st + j * b_sub + sb * hrows * 128, &tmap_h, s, (ks * p.kbs + j) * 64,
+                 rbase + sb * p.nb + static_cast<int>(crank) * hrows, pol_h);
       };
       int u = u0, ks = 0;  // the next stage fill
       auto advance = [&]() {
         if (++ks == p.nks) {
           ks = 0;
-          u += 2 * MCH;
+          u += kChunkUnits;
         }
       };
       // The first stages' W go out before anything else.  As a programmatic
@@ -262,23 +372,35 @@ __global__ void __launch_bounds__(kLmThreads, 1)
       }
       if (!ok) {
         if (!*abort) record_error(p.status, abort, EBD_ERR_TIMEOUT);
-        // let the copies already in flight land before the CTA can exit
-        for (int j = max(0, it - p.stages); j < it; ++j)
-          mbar_wait(&full[j % p.stages], static_cast<uint32_t>(j / p.stages) & 1u, p.limit_ns,
-                    nullptr);
+        if (leader) {
+          // let the copies already in flight land before the CTA can exit
+          for (int j = max(0, it - p.stages); j < it; ++j)
+            mbar_wait(&full[j % p.stages], static_cast<uint32_t>(j / p.stages) & 1u, p.limit_ns,
+                      nullptr);
+        } else {
+          // the peer's copies complete on the leader's barriers: give those
+          // in flight time to land (a stage lands in a few microseconds)
+          const uint64_t t0 = global_timer_ns();
+          while (global_timer_ns() - t0 < 200ull * 1000) __nanosleep(1000);
+        }
       }
     }
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
-    if (lane == 0) {
-      const uint32_t idesc = umma_idesc_bf16(128, static_cast<uint32_t>(p.nb));
+    if (lane == 0 && leader) {
+      const uint32_t idesc = umma_idesc_bf16(PAIR ? 256 : 128, static_cast<uint32_t>(p.nb));
       const uint32_t desc_hi = static_cast<uint32_t>(umma_desc_sw128(0) >> 32);
       int it = 0, c = 0;
       int s = 0;        // stage of iteration it, as in the producer
       uint32_t ph = 0;
       bool ok = true;
-      for (int u = u0; u < u1 && ok; u += 2 * MCH, ++c) {
-        const int nch = MCH == 1 ? 1 : (min(2 * MCH, u1 - u) + 1) >> 1;  // chunks holding W
+      auto commit_stage = [&](int st) {
+        if (PAIR)
+          umma_commit_pair_mc(&empty[st], 0x3);
+        else
+          umma_commit(&empty[st]);
+      };
+      for (int u = u0; u < u1 && ok; u += kChunkUnits, ++c) {
         const int buf = c % p.nbuf;
         const uint32_t bph = static_cast<uint32_t>(c / p.nbuf) & 1u;
         if (!mbar_wait(&acc_empty[buf], bph ^ 1u, p.limit_ns, abort)) {
@@ -286,7 +408,7 @@ __global__ void __launch_bounds__(kLmThreads, 1)
           break;
         }
         tc_fence_after();
-        const uint32_t d0 = tmem_base + static_cast<uint32_t>(buf * MCH * p.acc_stride);
+        const uint32_t d0 = tmem_base + static_cast<uint32_t>(buf * p.acc_stride);
         for (int ks = 0; ks < p.nks; ++ks) {
           if (!mbar_wait(&full[s], ph, p.limit_ns, abort)) {
             ok = false;
@@ -298,58 +420,51 @@ __global__ void __launch_bounds__(kLmThreads, 1)
           const uint32_t b_addr = smem_u32(sB + static_cast<size_t>(s) * b_stage);
           if (p.nsub <= 2 && nsubk >= 1 && nsubk <= 5) {
             // the unrolled issue path
+            const uint32_t a_lo = static_cast<uint32_t>(umma_desc_sw128(a_addr));
             const uint32_t b_lo = static_cast<uint32_t>(umma_desc_sw128(b_addr));
             const uint32_t b_step = b_sub >> 4;
-            const uint32_t sub_desc = static_cast<uint32_t>(p.nb) * 8u;  // nb rows x 128 B >> 4
+            const uint32_t sub_desc = static_cast<uint32_t>(hrows) * 8u;  // hrows x 128 B >> 4
             const uint32_t sub_cols = static_cast<uint32_t>(p.nb);
             const uint32_t acc0 = ks != 0 ? 1u : 0u;
-#pragma unroll
-            for (int ch = 0; ch < MCH; ++ch) {
-              if (ch >= nch) break;
-              const uint32_t a_lo = static_cast<uint32_t>(umma_desc_sw128(a_addr + ch * a_chunk));
-              const uint32_t dc = d0 + static_cast<uint32_t>(ch * p.acc_stride);
-#define EBD_STAGE(K, S) mma_stage<K, S>(dc, a_lo, b_lo, b_step, sub_desc, sub_cols, desc_hi, idesc, acc0)
-              if (p.nsub == 1) {
-                switch (nsubk) {
-                  case 1: EBD_STAGE(1, 1); break;
-                  case 2: EBD_STAGE(2, 1); break;
-                  case 3: EBD_STAGE(3, 1); break;
-                  case 4: EBD_STAGE(4, 1); break;
-                  default: EBD_STAGE(5, 1); break;
-                }
-              } else {
-                switch (nsubk) {
-                  case 1: EBD_STAGE(1, 2); break;
-                  case 2: EBD_STAGE(2, 2); break;
-                  case 3: EBD_STAGE(3, 2); break;
-                  case 4: EBD_STAGE(4, 2); break;
-                  default: EBD_STAGE(5, 2); break;
-                }
+#define EBD_STAGE(K, S) \
+  mma_stage<K, S, PAIR>(d0, a_lo, b_lo, b_step, sub_desc, sub_cols, desc_hi, idesc, acc0)
+            if (p.nsub == 1) {
+              switch (nsubk) {
+                case 1: EBD_STAGE(1, 1); break;
+                case 2: EBD_STAGE(2, 1); break;
+                case 3: EBD_STAGE(3, 1); break;
+                case 4: EBD_STAGE(4, 1); break;
+                default: EBD_STAGE(5, 1); break;
               }
+            } else {
+              switch (nsubk) {
+                case 1: EBD_STAGE(1, 2); break;
+                case 2: EBD_STAGE(2, 2); break;
+                case 3: EBD_STAGE(3, 2); break;
+                case 4: EBD_STAGE(4, 2); break;
+                default: EBD_STAGE(5, 2); break;
+              }
+            }
 #undef EBD_STAGE
-            }
-            umma_commit(&empty[s]);
-            ++it;
-            if (++s == p.stages) {
-              s = 0;
-              ph ^= 1u;
-            }
-            continue;
-          }
-          for (int ch = 0; ch < nch; ++ch)
+          } else {
             for (int j = 0; j < nsubk; ++j) {
 #pragma unroll
               for (int kk = 0; kk < 4; ++kk) {
-                const uint64_t ad = umma_desc_sw128(a_addr + ch * a_chunk + j * kATile + kk * 32);
+                const uint64_t ad = umma_desc_sw128(a_addr + j * kATile + kk * 32);
                 for (int sb = 0; sb < p.nsub; ++sb) {
-                  const uint64_t bd =
-                      umma_desc_sw128(b_addr + j * b_sub + sb * p.nb * 128 + kk * 32);
-                  umma_bf16(d0 + static_cast<uint32_t>(ch * p.acc_stride + sb * p.nb), ad, bd, idesc,
-                            (ks | j | kk) != 0 ? 1u : 0u);
+                  const uint64_t bd = umma_desc_sw128(b_addr + j * b_sub + sb * hrows * 128 + kk * 32);
+                  const uint32_t acc = (ks | j | kk) != 0 ? 1u : 0u;
+                  const uint32_t dd = d0 + static_cast<uint32_t>(sb * p.nb);
+                  if (PAIR)
+                    umma_bf16_lo_pair(dd, static_cast<uint32_t>(ad), static_cast<uint32_t>(bd),
+                                      desc_hi, idesc, acc);
+                  else
+                    umma_bf16(dd, ad, bd, idesc, acc);
                 }
               }
             }
-          umma_commit(&empty[s]);
+          }
+          commit_stage(s);
           ++it;
           if (++s == p.stages) {
             s = 0;
@@ -357,19 +472,26 @@ __global__ void __launch_bounds__(kLmThreads, 1)
           }
         }
         if (!ok) break;
-        umma_commit(&acc_full[buf]);
+        if (PAIR)
+          umma_commit_pair_mc(&acc_full[buf], 0x3);
+        else
+          umma_commit(&acc_full[buf]);
       }
       if (!ok) {
         if (!*abort) record_error(p.status, abort, EBD_ERR_TIMEOUT);
-        umma_commit(drain);  // completes once every MMA issued so far is done
+        // completes once every MMA issued so far is done
+        if (PAIR)
+          umma_commit_pair(drain);
+        else
+          umma_commit(drain);
         mbar_wait(drain, 0, p.limit_ns, nullptr);
       }
     }
   } else {
     // ------------------------------------------------------------ epilogue
     // p.nwg warpgroups of 4 warps (one per TMEM lane quadrant) take the
-    // 32-row column slices of the accumulator in turn; a second warpgroup is
-    // used when the accumulator is wider than one slice.
+    // 32-row column slices of the accumulator in turn; a second warpgroup
+    // is used when the accumulator has a single buffer.
     const int wg = (tid - 64) >> 7;
     const int et = (tid - 64) & 127;  // thread within the warpgroup
     const int quad = warp & 3;        // TMEM lane quadrant this warp may read
@@ -383,10 +505,16 @@ __global__ void __launch_bounds__(kLmThreads, 1)
       if (!ok && et == 0 && wg == 0) record_error(p.status, abort, EBD_ERR_TIMEOUT);
     }
     const bool active = ok;
+    auto release = [&](int buf) {  // this thread's reads of the accumulator are done
+      tc_fence_before();
+      if (PAIR)
+        mbar_arrive_cluster(mapa_shared(smem_u32(&acc_empty[buf]), 0));
+      else
+        mbar_arrive(&acc_empty[buf]);
+    };
     int c = 0;
-    for (int u = u0; u < u1 && ok; u += 2 * MCH, ++c) {
-      const int nu = min(2 * MCH, u1 - u);
-      const int nch = MCH == 1 ? 1 : (nu + 1) >> 1;
+    for (int u = u0; u < u1 && ok; u += kChunkUnits, ++c) {
+      const int nu = min(kChunkUnits, u1 - u);
       const int buf = c % p.nbuf;
       const uint32_t bph = static_cast<uint32_t>(c / p.nbuf) & 1u;
       bool w = mbar_wait_sleepy(&acc_full[buf], bph, p.limit_ns, abort);
@@ -396,86 +524,22 @@ __global__ void __launch_bounds__(kLmThreads, 1)
         break;
       }
       tc_fence_after();
-      bool released = false;
-      for (int ch = 0; ch < nch; ++ch) {
-      const int vbase = (u + 2 * ch) * kUnit;
-      const int valid = min(min(2, nu - 2 * ch) * kUnit, p.V - vbase);
-      for (int cc = 32 * wg; cc < p.n_pad; cc += 32 * p.nwg) {
-        float v[32];
-        const uint32_t taddr = tmem_base + (static_cast<uint32_t>(quad * 32) << 16) +
-                               static_cast<uint32_t>((buf * MCH + ch) * p.acc_stride + cc);
-        if (p.n_pad - cc >= 32)
-          tmem_ld_32x32b_x32(taddr, v);
-        else
-          tmem_ld_32x32b_x16(taddr, v);
-        if (ch == nch - 1 && cc + 32 * p.nwg >= p.n_pad) {  // this warpgroup's last slice is in registers
-          tc_fence_before();
-          mbar_arrive(&acc_empty[buf]);
-          released = true;
-        }
-        const bool lv = lanev < valid;
-#pragma unroll
-        for (int j = 0; j < 32; ++j) sTw[j * kTLd + lanev] = lv ? v[j] : -INFINITY;
-        named_barrier(bar_id, 128);
-        {
-          const int j = et >> 2, q = et & 3;
-          float x[32];
-#pragma unroll
-          for (int i = 0; i < 32; ++i) x[i] = sTw[j * kTLd + q + 4 * i];
-          // branch-free scan: the threads of a warp see different data
-          float m = -INFINITY, l2 = -INFINITY;
-          int ii = -1;
-#pragma unroll
-          for (int i = 0; i < 32; ++i) {
-            l2 = fmaxf(l2, fminf(m, x[i]));
-            ii = x[i] > m ? i : ii;  // strict: the first (lowest) index of the maximum
-            m = fmaxf(m, x[i]);
-          }
-          int idx = ii < 0 ? INT_MAX : vbase + q + 4 * ii;
-          float s = 0.f, t = 0.f;
-          if (m != -INFINITY) {
-#pragma unroll
-            for (int i = 0; i < 32; ++i) {
-              const float dl = x[i] - m;
-              const float e = __expf(dl);
-              s += e;
-              t = fmaf(e, e > 0.f ? dl : 0.f, t);  // masked lanes: e = 0, dl = -inf
-            }
-          }
-#pragma unroll
-          for (int off = 1; off <= 2; off <<= 1) {
-            const float bm = __shfl_xor_sync(0xffffffffu, m, off);
-            const float bs = __shfl_xor_sync(0xffffffffu, s, off);
-            const float bt = __shfl_xor_sync(0xffffffffu, t, off);
-            const float bl = __shfl_xor_sync(0xffffffffu, l2, off);
-            const int bi = __shfl_xor_sync(0xffffffffu, idx, off);
-            state_merge(m, s, t, l2, idx, bm, bs, bt, bl, bi);
-          }
-          const int r = cc + j;
-          if (q == 0 && r < p.n_pad) {
-            float M = st_m[r], S = st_s[r], T = st_t[r], L2 = st_l2[r];
-            int I = st_i[r];
-            state_merge(M, S, T, L2, I, m, s, t, l2, idx);
-            st_m[r] = M;
-            st_s[r] = S;
-            st_t[r] = T;
-            st_l2[r] = L2;
-            st_i[r] = I;
-          }
-        }
-        named_barrier(bar_id, 128);
-      }
-      }
-      if (!released) {  // no slice of these chunks for this warpgroup
-        tc_fence_before();
-        mbar_arrive(&acc_empty[buf]);
-      }
+      // this CTA's vocabulary rows of the chunk: units [u + ulo, u + ulo + 2)
+      const int vbase = (u + ulo) * kUnit;
+      const int valid = min(min(2, nu - ulo) * kUnit, p.V - vbase);
+      const uint32_t taddr0 = tmem_base + (static_cast<uint32_t>(quad * 32) << 16) +
+                              static_cast<uint32_t>(buf * p.acc_stride);
+      auto rel = [&]() { release(buf); };
+      const bool released = epilogue_buffer(taddr0, wg, p.nwg, p.n_pad, sTw, lanev, et, bar_id,
+                                            vbase, valid, st_m, st_s, st_t, st_l2, st_i, rel);
+      if (!released) release(buf);  // no slice of this chunk for this warpgroup
     }
     if (ok && active) {
-      // the rows of this warpgroup's slices (its threads updated them last);
-      // in paired mode the pair's partial goes to column cta and a neutral
-      // state to column grid + cta, so that every row has ncols partials
-      for (int r = et; r < rows_c; r += 128) {
+      // the rows of this warpgroup's slices (its threads updated them last):
+      // this CTA's partial goes to column blockIdx.x, and neutral states to
+      // the columns [grid, ncols) that no CTA of this launch owns
+      const int cta = static_cast<int>(blockIdx.x);
+      for (int r = et; r < p.rows; r += 128) {
         if (((r >> 5) % p.nwg) != wg) continue;
         const size_t o = static_cast<size_t>(rbase + r) * p.ncols + cta;
         p.part_f[o] = make_float4(st_m[r], st_s[r], st_t[r], st_l2[r]);
@@ -489,9 +553,14 @@ __global__ void __launch_bounds__(kLmThreads, 1)
   }
 
   __syncthreads();
+  // the peer's MMAs, copies and arrivals that target this CTA are over
+  if (PAIR) cluster_sync_all();
   if (warp == 1) {
     tc_fence_after();
-    tmem_dealloc(tmem_base, p.tmem_cols);
+    if (PAIR)
+      tmem_dealloc_pair(tmem_base, p.tmem_cols);
+    else
+      tmem_dealloc(tmem_base, p.tmem_cols);
   }
 }
 
@@ -509,66 +578,78 @@ int lm_grid(int num_sms, int n_units) {
   return 10 * g >= 9 * num_sms ? g : num_sms;
 }
 
+// CTAs of the paired launch: one pair per two SMs, at most one per 4-unit
+// chunk of the vocabulary
+int lm_pair_grid(int num_sms, int n_units) {
+  int np = num_sms / 2;
+  const int chunks = (n_units + 3) / 4;
+  if (np > chunks) np = chunks;
+  if (np < 1) np = 1;
+  return 2 * np;
+}
+
 void lm_plan(LmParams& p, int rows, int V, int d, int num_sms, bool pair) {
   p.V = V;
   p.d = d;
   p.rows = rows;
   p.pair = pair ? 1 : 0;
-  p.rhalf = pair ? (rows + 1) / 2 : rows;
-  const int rc = p.rhalf;  // rows one CTA accumulates
-  p.nsub = (rc + 255) / 256;
+  p.nsub = (rows + 255) / 256;
   if (p.nsub < 1) p.nsub = 1;
-  p.nb = ((rc + p.nsub - 1) / p.nsub + 15) / 16 * 16;
+  p.nb = ((rows + p.nsub - 1) / p.nsub + 15) / 16 * 16;
   if (p.nb < 16) p.nb = 16;
   p.n_pad = p.nb * p.nsub;
   p.acc_stride = (p.n_pad + 31) / 32 * 32;
-  // two W chunks per stage in paired mode when both accumulators fit in
-  // TMEM below 256 columns each.  They lose the second accumulator buffer,
-  // so the epilogue no longer overlaps the MMAs; measured: 390 rows (208 per
-  // CTA) 408 -> 401 us, but 512 rows (256 per CTA) 444 -> 498 us.
-  p.mch = (pair && p.n_pad >= 128 && p.acc_stride < 256) ? 2 : 1;
-  if (const char* env = getenv("EBD_LM_MCH")) p.mch = (atoi(env) == 2 && pair && 2 * p.acc_stride <= 512) ? 2 : 1;
-  p.nbuf = (2 * p.mch * p.acc_stride <= 512) ? 2 : 1;
-  int cols = p.nbuf * p.mch * p.acc_stride;
+  p.nbuf = (2 * p.acc_stride <= 512) ? 2 : 1;
+  int cols = p.nbuf * p.acc_stride;
   int tc = 32;
   while (tc < cols) tc <<= 1;
   p.tmem_cols = tc;
   p.n_units = (V + kUnit - 1) / kUnit;
-  p.grid = lm_grid(num_sms, p.n_units);
-  p.ncols = p.grid;  // partial states per row: the same in both modes
-  if (pair) {         // one pair per two SMs; each pair leaves one partial per row
-    p.grid = num_sms / 2 < p.n_units ? num_sms / 2 : p.n_units;
-    if (p.grid < 1) p.grid = 1;
+  if (pair) {  // 4 units per accumulator
+    p.grid = lm_pair_grid(num_sms, p.n_units);
+    p.nwork = p.grid / 2;
+  } else {
+    p.grid = lm_grid(num_sms, p.n_units);
+    p.nwork = p.grid;
   }
-  p.nkb = (d + 63) / 64;
+  p.ncols = p.grid;  // partial states per row (a caller may raise it: neutral states)
   // a second epilogue warpgroup (and its transpose buffer) only pays where
   // the epilogue is exposed, i.e. with a single accumulator buffer; with two,
   // one warpgroup keeps up with the MMAs and its buffer is worth more as
-  // pipeline stages (measured: 256 rows 270.7 -> 247.2 us, 512 rows in CTA
-  // pairs 445 -> 408.5 us; two chunks per stage (one buffer) 405 -> 432 us
-  // with one warpgroup)
-  p.nwg = p.mch == 2 ? 2 : 1;
+  // pipeline stages (measured with 128-row tiles: 256 rows 270.7 -> 247.2 us)
+  p.nwg = p.nbuf == 1 ? 2 : 1;
+  if (const char* env = getenv("EBD_LM_NWG")) p.nwg = atoi(env) == 2 ? 2 : 1;
   const uint32_t st_bytes = static_cast<uint32_t>(p.n_pad) * 20u;
   const uint32_t tail = kTBytes * static_cast<uint32_t>(p.nwg) + ((st_bytes + 7) / 8 * 8) +
                         (2 * 8 + 6) * 8 + 16;
   const uint32_t budget = 232448u - 1024u - tail;
-  // k-boxes (64 columns each) per pipeline stage: longer contiguous runs of
-  // each W row per request, while keeping at least two stages in flight
-  int kbs = 5;
+  p.nkb = (d + 63) / 64;
+  // hidden bytes per k-box in one CTA: all rows, or half of them in a pair
+  const uint32_t b_box = static_cast<uint32_t>(pair ? p.n_pad / 2 : p.n_pad) * 128u;
+  // k-boxes (64 columns each) per pipeline stage, while keeping at least two
+  // stages in flight.  Unpaired (few rows, HBM bound): up to 5, for longer
+  // contiguous runs of each W row per request.  Paired: about 512 / N, so
+  // that a stage's MMAs keep the tensor cores busy for about as long at any
+  // N: measured at 128 rows 4 k-boxes x 2 stages 172 us, 2 x 4 197 us; 256
+  // rows 2 x 3 214 us, 3 x 2 223 us, 1 x 6 272 us; 390 rows 1 x 4 360 us,
+  // 2 x 2 367 us.  Smaller stages cost more in hand-offs than their depth
+  // gains (one k-box per stage in separate W and hidden-row rings: 256 rows
+  // 434 us).
+  int kbs = pair ? 512 / p.n_pad : 5;
   if (const char* env = getenv("EBD_LM_KBS")) kbs = atoi(env);
   if (kbs < 1) kbs = 1;
+  if (kbs > 5) kbs = 5;
   if (kbs > p.nkb) kbs = p.nkb;
-  const uint32_t a_box = static_cast<uint32_t>(p.mch) * kATile;
-  while (kbs > 1 && budget / (static_cast<uint32_t>(kbs) * (a_box + p.n_pad * 128u)) < 2) --kbs;
+  while (kbs > 1 && budget / (static_cast<uint32_t>(kbs) * (kATile + b_box)) < 2) --kbs;
   p.kbs = kbs;
   p.nks = (p.nkb + kbs - 1) / kbs;
-  const uint32_t stage = static_cast<uint32_t>(kbs) * (a_box + static_cast<uint32_t>(p.n_pad) * 128u);
+  const uint32_t stage = static_cast<uint32_t>(kbs) * (kATile + b_box);
   int stages = static_cast<int>(budget / stage);
   if (stages > 8) stages = 8;
   p.stages = stages;
   p.off_a = 0;
-  p.off_b = p.off_a + static_cast<uint32_t>(stages) * kbs * a_box;
-  p.off_t = p.off_b + static_cast<uint32_t>(stages) * kbs * static_cast<uint32_t>(p.n_pad) * 128u;
+  p.off_b = p.off_a + static_cast<uint32_t>(stages) * kbs * kATile;
+  p.off_t = p.off_b + static_cast<uint32_t>(stages) * kbs * b_box;
   p.off_st = p.off_t + kTBytes * static_cast<uint32_t>(p.nwg);
   p.off_bar = (p.off_st + st_bytes + 7) / 8 * 8;
   p.smem_bytes = p.off_bar + static_cast<uint32_t>(2 * stages + 6) * 8u + 16u + 1024u;
@@ -617,18 +698,16 @@ cudaError_t launch_pack_lm(const __nv_bfloat16* w, __nv_bfloat16* out, int V, in
 cudaError_t lm_configure() {
   const cudaFuncAttribute a = cudaFuncAttributeMaxDynamicSharedMemorySize;
   cudaError_t e;
-  if ((e = cudaFuncSetAttribute(lm_stats_kernel<true, true, 1>, a, 232448)) != cudaSuccess) return e;
-  if ((e = cudaFuncSetAttribute(lm_stats_kernel<true, false, 1>, a, 232448)) != cudaSuccess) return e;
-  if ((e = cudaFuncSetAttribute(lm_stats_kernel<true, true, 2>, a, 232448)) != cudaSuccess) return e;
-  if ((e = cudaFuncSetAttribute(lm_stats_kernel<true, false, 2>, a, 232448)) != cudaSuccess) return e;
-  if ((e = cudaFuncSetAttribute(lm_stats_kernel<false, true, 1>, a, 232448)) != cudaSuccess) return e;
-  return cudaFuncSetAttribute(lm_stats_kernel<false, false, 1>, a, 232448);
+  if ((e = cudaFuncSetAttribute(lm_stats_kernel<true, true>, a, 232448)) != cudaSuccess) return e;
+  if ((e = cudaFuncSetAttribute(lm_stats_kernel<true, false>, a, 232448)) != cudaSuccess) return e;
+  if ((e = cudaFuncSetAttribute(lm_stats_kernel<false, true>, a, 232448)) != cudaSuccess) return e;
+  return cudaFuncSetAttribute(lm_stats_kernel<false, false>, a, 232448);
 }
 
 cudaError_t launch_lm_stats(const CUtensorMap& tmap_w, const CUtensorMap& tmap_h,
                             const LmParams& p, cudaStream_t st) {
   cudaLaunchConfig_t cfg{};
-  cfg.gridDim = dim3(p.pair ? 2 * p.grid : p.grid, 1, 1);
+  cfg.gridDim = dim3(p.grid, 1, 1);
   cfg.blockDim = dim3(kLmThreads, 1, 1);
   cfg.dynamicSmemBytes = p.smem_bytes;
   cfg.stream = st;
@@ -648,14 +727,11 @@ cudaError_t launch_lm_stats(const CUtensorMap& tmap_w, const CUtensorMap& tmap_h
   }
   cfg.attrs = attr;
   cfg.numAttrs = na;
-  if (p.pair && p.mch == 2)
-    return p.packed ? cudaLaunchKernelEx(&cfg, lm_stats_kernel<true, true, 2>, tmap_w, tmap_h, p)
-                    : cudaLaunchKernelEx(&cfg, lm_stats_kernel<true, false, 2>, tmap_w, tmap_h, p);
   if (p.pair)
-    return p.packed ? cudaLaunchKernelEx(&cfg, lm_stats_kernel<true, true, 1>, tmap_w, tmap_h, p)
-                    : cudaLaunchKernelEx(&cfg, lm_stats_kernel<true, false, 1>, tmap_w, tmap_h, p);
-  return p.packed ? cudaLaunchKernelEx(&cfg, lm_stats_kernel<false, true, 1>, tmap_w, tmap_h, p)
-                  : cudaLaunchKernelEx(&cfg, lm_stats_kernel<false, false, 1>, tmap_w, tmap_h, p);
+    return p.packed ? cudaLaunchKernelEx(&cfg, lm_stats_kernel<true, true>, tmap_w, tmap_h, p)
+                    : cudaLaunchKernelEx(&cfg, lm_stats_kernel<true, false>, tmap_w, tmap_h, p);
+  return p.packed ? cudaLaunchKernelEx(&cfg, lm_stats_kernel<false, true>, tmap_w, tmap_h, p)
+                  : cudaLaunchKernelEx(&cfg, lm_stats_kernel<false, false>, tmap_w, tmap_h, p);
 }
 
 }  // namespace ebd
