@@ -3,7 +3,8 @@ sweep, through the C ABI.  At these sizes the oracle's full logits rows take
 minutes, so:
   * the window attention is compared in full (Dream) or on sampled sequences;
   * the statistics are compared on sampled rows (first, middle and last row
-    of every sequence, at most 48 rows);
+    of every sequence, at most 48 rows) and, for Dream, on every masked row
+    of its shortest and its longest sequence;
   * the decision is compared with the GPU's statistics fed to the oracle's
     decision (bit-exact apart from sequences flagged for a near-tie), which
     checks the routers, the filters and the commit at full size."""
@@ -44,8 +45,18 @@ def _sample_rows(cu_rows, cap=48):
     return rows
 
 
-def _check_stats_sampled(inp, gpu):
-    rows = _sample_rows(inp.cu_rows)
+def _whole_sequences(inp, seqs):
+    """Every masked row of the given sequences."""
+    rows = []
+    for b in seqs:
+        r0, r1 = int(inp.cu_rows[b]), int(inp.cu_rows[b + 1])
+        rows += [r for r in range(r0, r1) if inp.mask[r]]
+    return rows
+
+
+def _check_stats_sampled(inp, gpu, whole=()):
+    rows = np.array(sorted(set(_sample_rows(inp.cu_rows).tolist()) |
+                           set(_whole_sequences(inp, whole))), dtype=np.int64)
     st = o.softmax_stats(o.lm_logits(inp.hidden.reshape(inp.rows, -1)[rows],
                                      inp.w_lm.reshape(inp.shape.vocab, -1)))
     return parity.compare_stats(st, {k: gpu[k][rows] for k in
@@ -72,7 +83,7 @@ def _check_decision_injected(inp, gpu, sh):
     W = o.weights_f64(synth.router_weights(sh.seed, sh.d_base, sh.gen_len))
     res = o.decide(inp.cu_rows, inp.row_pos, inp.tokens, inp.mask, inp.in_block, inp.blk_meta,
                    st, inp.w_emb, W, _prm(sh))
-    return parity.compare_decision(res, gpu, inp.mask, inp.cu_rows)
+    return parity.compare_decision(res, gpu, inp, _prm(sh))
 
 
 _cache = {}
@@ -100,7 +111,10 @@ def test_dream_step(state):
     if state == "inblock":
         synth.preset_in_block(inp, 20)
     gpu = _gpu_step(sh, inp, h, w)
-    rep = {"stats": _check_stats_sampled(inp, gpu)}
+    # every masked row of the shortest and the longest sequence, and the
+    # first, middle and last row of every other
+    lens = np.diff(inp.cu_rows)
+    rep = {"stats": _check_stats_sampled(inp, gpu, whole=(int(np.argmin(lens)), int(np.argmax(lens))))}
     _check_attention(inp, gpu, range(sh.batch))
     rep["decision"] = _check_decision_injected(inp, gpu, sh)
     print(state, rep)

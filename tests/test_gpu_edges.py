@@ -76,7 +76,7 @@ def test_degenerate_sequences_match_oracle(state, max_window):
     parity.compare_stats(res.stats, gpu)
     if attention:
         parity._close("attn_out", gpu["attn_out"], res.attn_out)
-    rep = parity.compare_decision(res, gpu, inp.mask, inp.cu_rows)
+    rep = parity.compare_decision(res, gpu, inp, _prm(sh))
     assert rep["flagged_sequences"] <= 2, rep
     cu = inp.cu_rows
     # nothing masked: no commit, no block

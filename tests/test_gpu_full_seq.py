@@ -67,7 +67,7 @@ def test_tiny_full_step_matches_oracle(state):
     gpu = _gpu_step(sh, inp)
     res = o.step(inp, _weights(sh), _prm(sh), attention=False)
     parity.compare_stats(res.stats, gpu)
-    rep = parity.compare_decision(res, gpu, inp.mask, inp.cu_rows)
+    rep = parity.compare_decision(res, gpu, inp, _prm(sh))
     assert rep["flagged_sequences"] < rep["sequences"]
     if state == "select":
         assert np.any(np.isfinite(gpu["lbs_logit"])), "the LBS did not run"
@@ -103,7 +103,7 @@ def test_llada_full_step_512_rows():
     parity.compare_stats(st, {k: gpu[k][rows] for k in ("conf", "entropy", "ent_norm", "gap", "argmax")})
     res = o.decide(inp.cu_rows, inp.row_pos, inp.tokens, inp.mask, inp.in_block, inp.blk_meta,
                    _injected(inp, gpu, sh), inp.w_emb, _weights(sh), _prm(sh))
-    parity.compare_decision(res, gpu, inp.mask, inp.cu_rows)
+    parity.compare_decision(res, gpu, inp, _prm(sh))
     assert np.isfinite(gpu["lbs_logit"][inp.mask == 1]).all()
 
 

@@ -64,6 +64,16 @@ def test_loop_tiny_matches_oracle():
         sh, W, _prm(sh), lambda s, p: synth.loop_window_inputs(sh, s, p),
         lambda p: synth.loop_kv(sh, p), inp.w_lm, inp.w_emb, attention=True)
     compared = 0
+    prm = _prm(sh)
+    for g in res.records:  # every GPU step is the rules' decision on its own features
+        lo, hi = g.window
+        b = g.before
+        out = {"conf": g.conf, "argmax": g.argmax, "lbs_logit": g.lbs_logit,
+               "lps_prob": g.lps_prob, "accepted": g.accepted, "tokens": g.after["tokens"],
+               "mask": g.after["mask"], "in_block": g.after["in_block"]}
+        parity.check_decision_valid(sh.prefix + np.arange(lo, hi), b["mask"], b["tokens"],
+                                    b["in_block"], b["meta"], out, g.after["meta"], prm)
+    first_flag = None
     for g, r in zip(res.records, recs):
         assert g.window == r["window"], (g.step, g.window, r["window"])
         parity._close(f"attn step {g.step}", g.attn_out, r["attn"])
@@ -73,6 +83,7 @@ def test_loop_tiny_matches_oracle():
         nt = st.near_tie
         assert np.array_equal(g.argmax[~nt], st.argmax[~nt]), g.step
         if r["flag"] or r["flag_lbs"]:
+            first_flag = g.step
             break  # a near-tie decision: the runs may part from here
         assert np.array_equal(g.accepted, r["accepted"]), (g.step, g.accepted, r["accepted"])
         compared += 1
@@ -83,8 +94,10 @@ def test_loop_tiny_matches_oracle():
             lo, hi = g.window
             ties[lo:hi] |= r["stats"].near_tie & r["accepted"].astype(bool)
         assert np.array_equal(res.tokens[~ties], toks[~ties])
-    print("steps", res.steps, "oracle", steps, "compared", compared)
-    assert compared >= 1
+    print("steps", res.steps, "oracle", steps, "compared", compared, "first flagged", first_flag)
+    # every step up to the first flagged one (or all of them) was compared
+    assert compared == (res.steps if first_flag is None else first_flag)
+    assert compared >= min(10, res.steps)
 
 
 def test_loop_llada_full_size():
@@ -107,6 +120,11 @@ def test_loop_llada_full_size():
         d = o.decide_sequence(sh.prefix + np.arange(lo, hi), m, t, ib, meta, st, inp.w_emb, W, prm)
         if d.flag_accept or d.flag_lbs:
             flagged += 1
+            out = {"conf": g.conf, "argmax": g.argmax, "lbs_logit": g.lbs_logit,
+                   "lps_prob": g.lps_prob, "accepted": g.accepted, "tokens": g.after["tokens"],
+                   "mask": g.after["mask"], "in_block": g.after["in_block"]}
+            parity.check_decision_valid(sh.prefix + np.arange(lo, hi), b["mask"], b["tokens"],
+                                        b["in_block"], b["meta"], out, g.after["meta"], prm)
             continue
         a = g.after
         assert np.array_equal(g.accepted, d.accepted), g.step

@@ -50,7 +50,7 @@ def _check(sh, inp, gpu, res, attention=True):
     rep = parity.compare_stats(res.stats, gpu)
     if attention:
         rep["attn"] = parity._close("attn_out", gpu["attn_out"], res.attn_out)
-    rep.update(parity.compare_decision(res, gpu, inp.mask, inp.cu_rows))
+    rep.update(parity.compare_decision(res, gpu, inp, _prm(sh)))
     return rep
 
 
