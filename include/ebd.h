@@ -241,6 +241,37 @@ ebd_status ebd_decide(ebd_handle* h, const ebd_step_args* a, void* stream);
  * writes conf, entropy, ent_norm, gap, argmax (any may be NULL). */
 ebd_status ebd_lm_stats(ebd_handle* h, const ebd_step_args* a, void* stream);
 
+/* ---- Vocabulary-parallel LM head (several GPUs) --------------------------
+ * Step 2 sharded by vocabulary: GPU g holds rows [v_off_g, v_off_g +
+ * v_count_g) of W_lm.  The statistics of App. B (Eq. app-confidence: kappa =
+ * max_v p(v)), Sec. 5.1 (H~, x_hat) and Sec. 5.2 (Delta) are taken over the
+ * whole vocabulary; the online-softmax state of a row over a vocabulary
+ * range, (m = max logit, S = sum exp(l - m), T = sum exp(l - m)(l - m),
+ * l2 = second largest logit, idx = lowest index of the maximum), merges
+ * associatively, so each GPU reduces its range to one state per row, the
+ * states are all-gathered (the caller's collective, e.g. NCCL), and every
+ * GPU merges them into the statistics and runs the decision (ebd_decide)
+ * on identical inputs.
+ *
+ * ebd_lm_shard_state: a->hidden and a->rows as for ebd_lm_stats; a->w_lm
+ * points at this GPU's rows of W_lm (row-major [v_count][d_model], or the
+ * tiled copy of those rows, which for v_off a multiple of 64 is the
+ * contiguous slice of ebd_pack_lm_head's output starting at tile row
+ * (v_off / 64) * ceil(d_model / 64) * 64); v_off must be a multiple of 64
+ * and v_off + v_count <= vocab of the handle (the whole vocabulary).
+ *   state  device float [a->rows][8], 16-byte aligned, caller-owned: per row
+ *          m, S, T, l2, idx (int32 bits of a vocabulary index), 0, 0, 0.
+ * ebd_merge_shard_states: states = device float [shards][a->rows][8] (the
+ * gathered states, any shard order), 16-byte aligned; writes a->conf,
+ * a->entropy, a->ent_norm, a->gap, a->argmax (any may be NULL), with
+ * H~ = H / ln(vocab); a non-finite row records EBD_ERR_NONFINITE.
+ * Both only enqueue on `stream`; argument errors return EBD_ERR_INVALID_ARG
+ * and enqueue nothing. */
+ebd_status ebd_lm_shard_state(ebd_handle* h, const ebd_step_args* a, int32_t v_off,
+                              int32_t v_count, float* state, void* stream);
+ebd_status ebd_merge_shard_states(ebd_handle* h, const float* states, int32_t shards,
+                                  const ebd_step_args* a, void* stream);
+
 /* Only step 1 (window attention): writes a->attn_out. */
 ebd_status ebd_attention(ebd_handle* h, const ebd_step_args* a, void* stream);
 

@@ -13,6 +13,9 @@ Everything is the plain definition, in float64, on bf16-decoded inputs:
   * cache append:       the K/V of the rows committed in a step written into
     the cache at their positions (Sec. 6.3);
   * LM head:            full logits row l = W h, materialised;
+  * vocabulary ranges:  the softmax state of a row over a range of the
+    vocabulary and the merge of the ranges' states into the statistics (the
+    vocabulary-parallel LM head);
   * statistics:         softmax in two passes (max, then sum), then
     kappa = max_v p(v)  (App. B, Eq. app-confidence), x_hat = argmax_v p(v),
     H~ = (-sum_v p log p) / log|V|  (Sec. 5.1), Delta = p(top1) - p(top2)
@@ -229,6 +232,63 @@ def softmax_stats(logits) -> RowStats:
     ent_norm = ent / math.log(V)
     return RowStats(conf=conf, entropy=ent, ent_norm=ent_norm, gap=gap,
                     argmax=am, logit_gap=lg, near_tie=lg < NEAR_TIE)
+
+
+# ----------------------------------------------------------------------------
+# (2b) the statistics from vocabulary ranges (the vocabulary-parallel LM head)
+# ----------------------------------------------------------------------------
+@dataclass
+class RangeState:
+    """Softmax state of each row over a range of the vocabulary: m = max
+    logit, S = sum exp(l - m), T = sum exp(l - m)(l - m), l2 = second largest
+    logit (duplicates count; -inf for a one-entry range), idx = vocabulary
+    index of the first maximum."""
+    m: np.ndarray
+    S: np.ndarray
+    T: np.ndarray
+    l2: np.ndarray
+    idx: np.ndarray
+
+
+def range_state(logits_range, v0: int) -> RangeState:
+    """The state of each row over logits_range[:, j] = l[v0 + j], by its
+    definition."""
+    L = np.atleast_2d(np.asarray(logits_range, dtype=np.float64))
+    n, w = L.shape
+    m = L.max(axis=1)
+    e = np.exp(L - m[:, None])
+    S = e.sum(axis=1)
+    T = (e * (L - m[:, None])).sum(axis=1)
+    l2 = np.partition(L, w - 2, axis=1)[:, w - 2] if w >= 2 else np.full(n, -np.inf)
+    idx = v0 + np.argmax(L, axis=1)
+    return RangeState(m=m, S=S, T=T, l2=l2, idx=idx.astype(np.int64))
+
+
+def merge_range_states(states: List[RangeState], V: int) -> RowStats:
+    """The statistics of the whole vocabulary from the states of ranges that
+    partition it: with the common maximum M = max_g m_g,
+    S = sum_g S_g exp(m_g - M), T = sum_g exp(m_g - M)(T_g + (m_g - M) S_g)
+    (each range's sums re-centred on M), kappa = 1/S, H = ln S - T/S,
+    Delta = (1 - exp(l2 - M))/S with l2 the largest of the argmax range's l2
+    and the other ranges' maxima, x_hat = the lowest index among the ranges
+    whose maximum is M (Readings R1-R3)."""
+    m = np.stack([s.m for s in states])          # G x n
+    M = m.max(axis=0)
+    w = np.exp(m - M)
+    S = (np.stack([s.S for s in states]) * w).sum(axis=0)
+    T = (w * (np.stack([s.T for s in states]) + (m - M) * np.stack([s.S for s in states]))).sum(axis=0)
+    idx = np.where(m == M, np.stack([s.idx for s in states]), np.iinfo(np.int64).max).min(axis=0)
+    n = len(M)
+    l2 = np.empty(n)
+    for r in range(n):
+        win = [g for g in range(len(states)) if m[g, r] == M[r] and states[g].idx[r] == idx[r]][0]
+        others = [m[g, r] for g in range(len(states)) if g != win]
+        l2[r] = max([states[win].l2[r]] + others)
+    conf = 1.0 / S
+    ent = np.log(S) - T / S
+    p2 = np.exp(l2 - M) / S
+    return RowStats(conf=conf, entropy=ent, ent_norm=ent / math.log(V), gap=conf - p2,
+                    argmax=idx, logit_gap=M - l2, near_tie=(M - l2) < NEAR_TIE)
 
 
 # ----------------------------------------------------------------------------

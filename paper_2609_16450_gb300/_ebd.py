@@ -60,7 +60,7 @@ EXPORTS = ["ebd_create", "ebd_destroy", "ebd_bind_embedding", "ebd_step", "ebd_s
            "ebd_weight_count", "ebd_lm_head_packed_bytes", "ebd_pack_lm_head",
            "ebd_profile_enable", "ebd_profile_read", "ebd_last_error",
            "ebd_version", "ebd_lm_stats_noalloc", "ebd_loop_window",
-           "ebd_loop_block_window"]
+           "ebd_loop_block_window", "ebd_lm_shard_state", "ebd_merge_shard_states"]
 
 _lib = None
 
@@ -109,6 +109,9 @@ def load(path: str = LIB_PATH):
     lib.ebd_loop_window.restype = c_int32
     lib.ebd_loop_block_window.argtypes = [c_void_p, c_int32, c_int32, P(c_int32), P(c_int32)]
     lib.ebd_loop_block_window.restype = c_int32
+    lib.ebd_lm_shard_state.argtypes = [c_void_p, P(ebd_step_args), c_int32, c_int32, c_void_p,
+                                       c_void_p]
+    lib.ebd_merge_shard_states.argtypes = [c_void_p, c_void_p, c_int32, P(ebd_step_args), c_void_p]
     lib.ebd_version.restype = c_char_p
     for fn in EXPORTS:
         if getattr(lib, fn).restype is ctypes.c_int:
@@ -152,6 +155,18 @@ def ebd_decide(h, args: ebd_step_args, stream: int = 0) -> int:
 
 def ebd_lm_stats(h, args: ebd_step_args, stream: int = 0) -> int:
     return load().ebd_lm_stats(h, ctypes.byref(args), c_void_p(stream))
+
+
+def ebd_lm_shard_state(h, args: ebd_step_args, v_off: int, v_count: int, state_ptr: int,
+                       stream: int = 0) -> int:
+    return load().ebd_lm_shard_state(h, ctypes.byref(args), v_off, v_count, c_void_p(state_ptr),
+                                     c_void_p(stream))
+
+
+def ebd_merge_shard_states(h, states_ptr: int, shards: int, args: ebd_step_args,
+                           stream: int = 0) -> int:
+    return load().ebd_merge_shard_states(h, c_void_p(states_ptr), shards, ctypes.byref(args),
+                                         c_void_p(stream))
 
 
 def ebd_attention(h, args: ebd_step_args, stream: int = 0) -> int:

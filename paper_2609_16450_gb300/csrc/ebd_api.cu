@@ -652,16 +652,20 @@ ebd_status run_attention(ebd_handle* h, const ebd_step_args* a, cudaStream_t st,
 }
 
 // pdl_first: the first LM-head launch is a programmatic dependent of the
-// kernel just before it on `st`, which copies the hidden rows in
-ebd_status run_lm(ebd_handle* h, const ebd_step_args* a, cudaStream_t st, bool pdl_first = false) {
+// kernel just before it on `st`, which copies the hidden rows in.
+// v_off, v_count: a->w_lm holds the vocabulary rows [v_off, v_off + v_count)
+// (a shard of the vocabulary-parallel LM head); v_count < 0: all of them.
+ebd_status run_lm(ebd_handle* h, const ebd_step_args* a, cudaStream_t st, bool pdl_first = false,
+                  int v_off = 0, int v_count = -1) {
   const ebd_config& c = h->cfg;
+  const int V = v_count < 0 ? c.vocab : v_count;
   CUtensorMap tw;
   const bool packed = a->w_lm_layout == 1;
   {
-    const uint64_t units = (static_cast<uint64_t>(c.vocab) + kUnit - 1) / kUnit;
+    const uint64_t units = (static_cast<uint64_t>(V) + kUnit - 1) / kUnit;
     const uint64_t nkb = (static_cast<uint64_t>(c.d_model) + 63) / 64;
     const uint64_t dims[2] = {packed ? 64ull : static_cast<uint64_t>(c.d_model),
-                              packed ? units * nkb * 64 : static_cast<uint64_t>(c.vocab)};
+                              packed ? units * nkb * 64 : static_cast<uint64_t>(V)};
     const uint64_t str[1] = {packed ? 128ull : static_cast<uint64_t>(c.d_model) * 2};
     const uint32_t box[2] = {64, 64};
     if (!encode_bf16(&tw, a->w_lm, 2, dims, str, box))
@@ -674,9 +678,14 @@ ebd_status run_lm(ebd_handle* h, const ebd_step_args* a, cudaStream_t st, bool p
     // M = 256: each SM receives half of the hidden rows per MMA
     int pair_min = kLmPairMinRows;
     if (const char* env = getenv("EBD_LM_PAIR_MIN")) pair_min = atoi(env) > 0 ? atoi(env) : kMaxGroupRows + 1;
-    const bool pair = rows >= pair_min && h->grid_lm >= lm_pair_grid(h->num_sms, h->lm_units);
-    lm_plan(p, rows, c.vocab, c.d_model, h->num_sms, pair);
+    const int units = (V + kUnit - 1) / kUnit;
+    const bool pair = rows >= pair_min && h->grid_lm >= lm_pair_grid(h->num_sms, units);
+    lm_plan(p, rows, V, c.d_model, h->num_sms, pair);
+    // a shard's own grid may exceed the partial columns of the handle
+    if (p.grid > h->grid_lm) lm_plan(p, rows, V, c.d_model, h->grid_lm, pair);
+    if (p.grid > h->grid_lm) return fail(h, EBD_ERR_UNSUPPORTED, "LM head: grid exceeds the partials");
     p.ncols = h->grid_lm;
+    p.v_off = v_off;
     if (p.stages < 2) return fail(h, EBD_ERR_UNSUPPORTED, "LM head: shared memory plan failed");
     p.row0 = g0;
     p.packed = packed ? 1 : 0;
@@ -1324,6 +1333,43 @@ ebd_status ebd_lm_stats(ebd_handle* h, const ebd_step_args* a, void* stream) {
                                      a->conf, a->entropy, a->ent_norm, a->gap, a->argmax,
                                      h->d_status, st);
   if (e != cudaSuccess) return cuda_fail(h, e, "merge launch");
+  return EBD_OK;
+}
+
+ebd_status ebd_lm_shard_state(ebd_handle* h, const ebd_step_args* a, int32_t v_off,
+                              int32_t v_count, float* state, void* stream) {
+  if (h == nullptr) return EBD_ERR_INVALID_ARG;
+  ebd_status s = check_device(h);
+  if (s != EBD_OK) return s;
+  if ((s = check_args(h, a, false, true, false)) != EBD_OK) return s;
+  if (v_off < 0 || v_count < 1 || v_off % kUnit != 0 || v_count > h->cfg.vocab - v_off)
+    return fail(h, EBD_ERR_INVALID_ARG, "shard range: v_off a multiple of 64, within the vocabulary");
+  if (a->rows == 0) return EBD_OK;
+  if (state == nullptr || !aligned(state, 16))
+    return fail(h, EBD_ERR_INVALID_ARG, "state must be a 16-byte aligned device pointer");
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  if ((s = run_lm(h, a, st, false, v_off, v_count)) != EBD_OK) return s;
+  cudaError_t e = launch_shard_state(h->part_f, h->part_i, a->rows, h->grid_lm, state, st);
+  if (e != cudaSuccess) return cuda_fail(h, e, "shard state launch");
+  return EBD_OK;
+}
+
+ebd_status ebd_merge_shard_states(ebd_handle* h, const float* states, int32_t shards,
+                                  const ebd_step_args* a, void* stream) {
+  if (h == nullptr) return EBD_ERR_INVALID_ARG;
+  ebd_status s = check_device(h);
+  if (s != EBD_OK) return s;
+  if (a == nullptr) return fail(h, EBD_ERR_INVALID_ARG, "args is NULL");
+  if (a->rows < 0 || a->rows > h->cfg.max_rows) return fail(h, EBD_ERR_INVALID_ARG, "rows out of range");
+  if (shards < 1) return fail(h, EBD_ERR_INVALID_ARG, "shards must be >= 1");
+  if (a->rows == 0) return EBD_OK;
+  if (states == nullptr || !aligned(states, 16))
+    return fail(h, EBD_ERR_INVALID_ARG, "states must be a 16-byte aligned device pointer");
+  const float inv = static_cast<float>(1.0 / std::log(static_cast<double>(h->cfg.vocab)));
+  cudaError_t e = launch_merge_shards(states, shards, a->rows, h->cfg.vocab, inv, a->conf, a->entropy,
+                                      a->ent_norm, a->gap, a->argmax, h->d_status,
+                                      static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(h, e, "shard merge launch");
   return EBD_OK;
 }
 

@@ -23,7 +23,8 @@ constexpr int kMaxAttnSplits = 8;
 
 // ------------------------------------------------------------------ LM head
 struct LmParams {
-  int V, d;                 // vocabulary, hidden size
+  int V, d;                 // vocabulary rows of this launch's W, hidden size
+  int v_off;                // vocabulary index of W's first row (a shard's offset; 0 otherwise)
   int row0, rows;           // rows [row0, row0 + rows) of this launch
   int nb, nsub, n_pad;      // MMA N per sub-tile, sub-tiles, padded N = nb * nsub
   int n_units;              // ceil(V / 64)
@@ -177,6 +178,13 @@ cudaError_t launch_attention(const CUtensorMap& kc, const CUtensorMap& vc, const
                              const CUtensorMap& vw, const AttnParams& p, cudaStream_t st,
                              bool pdl = false);
 cudaError_t launch_decide(const DecideParams& p, cudaStream_t st);
+// vocabulary-parallel LM head: one state per row from a launch's partials,
+// and the statistics from the states of several shards (k_decide.cu)
+cudaError_t launch_shard_state(const float4* part_f, const int* part_i, int rows, int grid,
+                               float* state, cudaStream_t st);
+cudaError_t launch_merge_shards(const float* states, int shards, int rows, int V, float inv_log_v,
+                                float* conf, float* entropy, float* ent_norm, float* gap,
+                                int* argmax, int* status, cudaStream_t st);
 // the grid-wide decision: a chain of kernels on `st` (k_decide_seq.cu)
 // the grid-wide decision: the scratch reset (before the LM head, so that the
 // chain from the LM head on is unbroken), then the kernel chain; pdl_first:

@@ -1237,6 +1237,101 @@ cudaError_t launch_merge_stats(const float4* part_f, const int* part_i, int rows
                             entropy, ent_norm, gap, argmax, status);
 }
 
+// Vocabulary-parallel LM head (several GPUs, each holding a range of W's
+// rows).  The softmax statistics of App. B (Eq. app-confidence), Sec. 5.1
+// and Sec. 5.2 are functions of the whole vocabulary; each shard reduces its
+// range to one online-softmax state per row (m, S, T, l2, x_hat), and the
+// merge of states is associative, so the states of the shards, gathered on
+// every GPU, merge into the statistics of the whole vocabulary.
+//
+// shard_state_kernel: one warp per row merges the row's `grid` LM-head
+// partials into one state, stored as 8 words: m, S, T, l2, idx (int32 bits),
+// and three zero words (32-byte rows).
+__global__ void __launch_bounds__(256) shard_state_kernel(const float4* __restrict__ part_f,
+                                                          const int* __restrict__ part_i, int rows,
+                                                          int grid, float* __restrict__ state) {
+  const int lane = threadIdx.x & 31;
+  const int r = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  if (r >= rows) return;
+  const size_t base = static_cast<size_t>(r) * grid;
+  float m = -INFINITY, s = 0.f, t = 0.f, l2 = -INFINITY;
+  int idx = INT_MAX;
+  for (int g = lane; g < grid; g += 32) {
+    const float4 f = part_f[base + g];
+    merge_state(m, s, t, l2, idx, f.x, f.y, f.z, f.w, part_i[base + g]);
+  }
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    const float bm = __shfl_xor_sync(0xffffffffu, m, off);
+    const float bs = __shfl_xor_sync(0xffffffffu, s, off);
+    const float bt = __shfl_xor_sync(0xffffffffu, t, off);
+    const float bl = __shfl_xor_sync(0xffffffffu, l2, off);
+    const int bi = __shfl_xor_sync(0xffffffffu, idx, off);
+    merge_state(m, s, t, l2, idx, bm, bs, bt, bl, bi);
+  }
+  if (lane != 0) return;
+  float4* o = reinterpret_cast<float4*>(state + static_cast<size_t>(r) * 8);
+  o[0] = make_float4(m, s, t, l2);
+  o[1] = make_float4(__int_as_float(idx), 0.f, 0.f, 0.f);
+}
+
+// merge_shards_kernel: one warp per row merges the row's state from each of
+// `shards` shards (states[shard][row][8]) and writes the statistics as the
+// merge of the single-GPU path does (kappa = 1/S, H = ln S - T/S,
+// H~ = H / ln V with V the whole vocabulary, Delta = (1 - exp(l2 - m)) / S,
+// x_hat = idx); a non-finite state records EBD_ERR_NONFINITE.
+__global__ void __launch_bounds__(256) merge_shards_kernel(const float* __restrict__ states,
+                                                           int shards, int rows, int V,
+                                                           float inv_log_v, float* conf,
+                                                           float* entropy, float* ent_norm,
+                                                           float* gap, int* argmax, int* status) {
+  const int lane = threadIdx.x & 31;
+  const int r = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  if (r >= rows) return;
+  float m = -INFINITY, s = 0.f, t = 0.f, l2 = -INFINITY;
+  int idx = INT_MAX;
+  for (int g = lane; g < shards; g += 32) {
+    const float4* q = reinterpret_cast<const float4*>(
+        states + (static_cast<size_t>(g) * rows + r) * 8);
+    const float4 f = q[0];
+    const float4 i4 = q[1];
+    merge_state(m, s, t, l2, idx, f.x, f.y, f.z, f.w, __float_as_int(i4.x));
+  }
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    const float bm = __shfl_xor_sync(0xffffffffu, m, off);
+    const float bs = __shfl_xor_sync(0xffffffffu, s, off);
+    const float bt = __shfl_xor_sync(0xffffffffu, t, off);
+    const float bl = __shfl_xor_sync(0xffffffffu, l2, off);
+    const int bi = __shfl_xor_sync(0xffffffffu, idx, off);
+    merge_state(m, s, t, l2, idx, bm, bs, bt, bl, bi);
+  }
+  if (lane != 0) return;
+  const float ent = logf(s) - t / s;
+  const bool bad = !(isfinite(m) && isfinite(s) && isfinite(t) && s >= 1.0f) || idx < 0 || idx >= V;
+  if (conf) conf[r] = 1.0f / s;
+  if (entropy) entropy[r] = ent;
+  if (ent_norm) ent_norm[r] = ent * inv_log_v;
+  if (gap) gap[r] = (1.0f - expf(l2 - m)) / s;
+  if (argmax) argmax[r] = bad ? -1 : idx;
+  if (bad) atomicCAS(status, 0, EBD_ERR_NONFINITE);
+}
+
+cudaError_t launch_shard_state(const float4* part_f, const int* part_i, int rows, int grid,
+                               float* state, cudaStream_t st) {
+  shard_state_kernel<<<static_cast<unsigned>((rows + 7) / 8), 256, 0, st>>>(part_f, part_i, rows,
+                                                                            grid, state);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_merge_shards(const float* states, int shards, int rows, int V, float inv_log_v,
+                                float* conf, float* entropy, float* ent_norm, float* gap,
+                                int* argmax, int* status, cudaStream_t st) {
+  merge_shards_kernel<<<static_cast<unsigned>((rows + 7) / 8), 256, 0, st>>>(
+      states, shards, rows, V, inv_log_v, conf, entropy, ent_norm, gap, argmax, status);
+  return cudaGetLastError();
+}
+
 cudaError_t decide_configure() {
   return cudaFuncSetAttribute(decide_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                               static_cast<int>(sizeof(Smem) + 16));

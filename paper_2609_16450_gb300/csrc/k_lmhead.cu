@@ -148,7 +148,7 @@ __device__ __forceinline__ bool epilogue_buffer(uint32_t taddr0, int wg, int nwg
         ii = x[i] > m ? i : ii;  // strict: the first (lowest) index of the maximum
         m = fmaxf(m, x[i]);
       }
-      int idx = ii < 0 ? INT_MAX : vbase + q + 4 * ii;
+      int idx = ii < 0 ? INT_MAX : vbase + q + 4 * ii;  // vbase includes the shard offset
       float s = 0.f, t = 0.f;
       if (m != -INFINITY) {
 #pragma unroll
@@ -525,8 +525,10 @@ __global__ void __launch_bounds__(kLmThreads, 1)
       }
       tc_fence_after();
       // this CTA's vocabulary rows of the chunk: units [u + ulo, u + ulo + 2)
-      const int vbase = (u + ulo) * kUnit;
-      const int valid = min(min(2, nu - ulo) * kUnit, p.V - vbase);
+      // of W, i.e. vocabulary indices from p.v_off + (u + ulo) * kUnit
+      const int wbase = (u + ulo) * kUnit;
+      const int valid = min(min(2, nu - ulo) * kUnit, p.V - wbase);
+      const int vbase = p.v_off + wbase;
       const uint32_t taddr0 = tmem_base + (static_cast<uint32_t>(quad * 32) << 16) +
                               static_cast<uint32_t>(buf * p.acc_stride);
       auto rel = [&]() { release(buf); };

@@ -315,3 +315,43 @@ def test_layer_norm_and_gelu_swapped_in_the_entropy_branch_are_caught(monkeypatc
         return o.linear(np.concatenate([e, t], axis=1), W, "lbs.comb") + W["lbs.pos"][:len(h)]
     monkeypatch.setattr(o, "lbs_input", swapped)
     assert _some_pin_fails(_input_pins())
+
+
+# ---------------------------------------------------------------- vocabulary ranges
+def _range_pins():
+    return [lambda: ts.test_range_states_merge_to_the_whole_row(3),
+            ts.test_range_state_single_entry_ranges]
+
+
+def test_range_pins_pass_as_they_stand():
+    assert not _some_pin_fails(_range_pins())
+
+
+def test_merge_without_the_recentring_term_is_caught(monkeypatch):
+    """T merged as sum exp(m_g - M) T_g, dropping (m_g - M) S_g"""
+    real = o.merge_range_states
+
+    def no_shift(states, V):
+        shifted = []
+        M = np.stack([s.m for s in states]).max(axis=0)
+        for s in states:  # fold the dropped term back out of T so the merge loses it
+            shifted.append(o.RangeState(m=s.m, S=s.S, T=s.T - (s.m - M) * s.S, l2=s.l2, idx=s.idx))
+        return real(shifted, V)
+    monkeypatch.setattr(o, "merge_range_states", no_shift)
+    assert _some_pin_fails(_range_pins())
+
+
+def test_second_logit_from_the_argmax_range_only_is_caught(monkeypatch):
+    """l2 taken from the argmax range alone, ignoring the other ranges' maxima"""
+    real = o.merge_range_states
+
+    def l2_local(states, V):
+        st = real(states, V)
+        m = np.stack([s.m for s in states])
+        win = np.argmax(m, axis=0)
+        l2 = np.array([states[win[r]].l2[r] for r in range(m.shape[1])])
+        p2 = np.exp(l2 - m.max(axis=0)) * st.conf
+        return o.RowStats(conf=st.conf, entropy=st.entropy, ent_norm=st.ent_norm, gap=st.conf - p2,
+                          argmax=st.argmax, logit_gap=st.logit_gap, near_tie=st.near_tie)
+    monkeypatch.setattr(o, "merge_range_states", l2_local)
+    assert _some_pin_fails(_range_pins())

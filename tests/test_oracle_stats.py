@@ -105,3 +105,52 @@ def test_lm_logits_exact_rationals():
 def test_bf16_decode():
     assert o.bf16(np.array([0x3F80, 0xBF80, 0x4049, 0x0000], np.uint16)).tolist() == \
         [1.0, -1.0, 3.140625, 0.0]
+
+
+# ---------------------------------------------------------------- vocabulary ranges
+def _split_points(V, k, rng):
+    cuts = np.sort(rng.choice(np.arange(1, V), size=k - 1, replace=False))
+    return [0] + cuts.tolist() + [V]
+
+
+@pytest.mark.parametrize("k", [1, 2, 3, 7])
+def test_range_states_merge_to_the_whole_row(k):
+    """The statistics merged from the states of any partition of the
+    vocabulary equal the statistics of the whole row (scipy's softmax and
+    entropy), whatever the order of the ranges."""
+    rng = np.random.default_rng(40 + k)
+    V = 997
+    L = rng.standard_normal((5, V)) * np.array([[0.5], [2], [8], [20], [1]])
+    L[4, 10] = L[4, 900] = L[4].max() + 3.0       # a duplicated maximum across ranges
+    pts = _split_points(V, k, rng)
+    states = [o.range_state(L[:, a:b], a) for a, b in zip(pts[:-1], pts[1:])]
+    for order in (states, states[::-1]):
+        st = o.merge_range_states(order, V)
+        p = sp_softmax(L, axis=1)
+        np.testing.assert_allclose(st.conf, p.max(axis=1), rtol=1e-12)
+        np.testing.assert_allclose(st.entropy, sp_entropy(p, axis=1), rtol=1e-10, atol=1e-12)
+        srt = np.sort(p, axis=1)
+        np.testing.assert_allclose(st.gap, srt[:, -1] - srt[:, -2], rtol=1e-10, atol=1e-15)
+        assert st.argmax.tolist() == np.argmax(L, axis=1).tolist()
+    assert st.argmax[4] == 10 and st.gap[4] == 0.0  # lowest index of the duplicated maximum
+
+
+def test_range_state_of_one_range_is_the_row():
+    rng = np.random.default_rng(5)
+    L = rng.standard_normal((3, 50)) * 4
+    st = o.merge_range_states([o.range_state(L, 0)], 50)
+    ref = o.softmax_stats(L)
+    for k in ("conf", "entropy", "ent_norm", "gap"):
+        np.testing.assert_allclose(getattr(st, k), getattr(ref, k), rtol=1e-12, atol=1e-15)
+    assert st.argmax.tolist() == ref.argmax.tolist()
+
+
+def test_range_state_single_entry_ranges():
+    """Ranges of one entry each: m = the logit, S = 1, T = 0, l2 = -inf."""
+    L = np.array([[1.0, 4.0, 4.0, -2.0]])
+    states = [o.range_state(L[:, j:j + 1], j) for j in range(4)]
+    assert states[2].S[0] == 1.0 and states[2].T[0] == 0.0 and states[2].l2[0] == -np.inf
+    st = o.merge_range_states(states, 4)
+    assert st.argmax[0] == 1 and st.gap[0] == 0.0
+    np.testing.assert_allclose(st.conf[0], math.exp(4) / (math.exp(1) + 2 * math.exp(4) + math.exp(-2)),
+                               rtol=1e-14)
