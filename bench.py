@@ -200,6 +200,23 @@ def lm_grid(num_sms, n_units):
     return g if 10 * g >= 9 * num_sms else num_sms
 
 
+PAIR_MIN_ROWS = 65  # LM-head launches of at least this many rows run in CTA pairs
+
+
+def lm_pair_grid(num_sms, n_units):
+    """CTAs of the library's paired (cta_group::2) LM-head launch: one pair
+    per two SMs, at most one per 4-unit chunk of the vocabulary."""
+    return 2 * max(1, min(num_sms // 2, -(-n_units // 4)))
+
+
+def partials_per_row(num_sms, n_units, max_rows):
+    """LM-head partial states per row that a handle with max_rows rows per
+    step keeps (the library's rule): room for the paired launch when a step
+    may take it."""
+    g = lm_grid(num_sms, n_units)
+    return max(g, lm_pair_grid(num_sms, n_units)) if max_rows >= PAIR_MIN_ROWS else g
+
+
 def step_work(sh, rows, masked, grid_lm, lbs_runs, suffix=0, append=False):
     """Algorithmic bytes and flops of one step (each input read once); suffix:
     cached keys after each window (dual cache); append: committed rows'
@@ -406,7 +423,7 @@ def run_ours(args, rank, world, local_rank):
     out["suffix"] = None if sfx is None else sfx
     out["fetch"] = ds.fetch()
     h_sms = torch.cuda.get_device_properties(local_rank).multi_processor_count
-    out["grid_lm"] = lm_grid(h_sms, (sh.vocab + 63) // 64)
+    out["grid_lm"] = partials_per_row(h_sms, (sh.vocab + 63) // 64, h.cfg.max_rows)
     out["num_sms"] = h_sms
     h.close()
     return out
@@ -484,7 +501,8 @@ def run_e2e(args, h, ds, inp, sh, stream, world, sfx=None):
 # ----------------------------------------------------------------------------- oracle arm
 def oracle_step_sample(sh, inp, budget_s, suffix=None):
     """Times the CPU oracle on the step's inputs: full steps until budget_s
-    has passed (at least one).  Returns (positions/s, steps, seconds)."""
+    has passed (at least one).  Returns (positions/s, steps, seconds, the
+    oracle's result of the step)."""
     from oracle import ebd_oracle as o
     import synth
     W = o.weights_f64(synth.router_weights(sh.seed, sh.d_base, sh.gen_len))
@@ -492,12 +510,58 @@ def oracle_step_sample(sh, inp, budget_s, suffix=None):
                            g_max=sh.g_max, eos_id=sh.eos_id, lps_enabled=bool(sh.lps_enabled))
     n, t0 = 0, time.perf_counter()
     while True:
-        o.step(inp, W, prm, suffix=suffix)
+        res = o.step(inp, W, prm, suffix=suffix)
         n += 1
         el = time.perf_counter() - t0
         if el >= budget_s:
             break
-    return inp.rows * n / el, n, el
+    return inp.rows * n / el, n, el, res
+
+
+def parity_summary(sh, inp, res, gpu, tol=2e-3):
+    """The GPU step's outputs (one step from the same state) against the
+    oracle's: near-ties counted as the benchmark spec defines them (top-2 logit gap,
+    or a decision margin, below 1e-3), argmax mismatches outside near-ties,
+    decision mismatches in sequences the oracle does not flag, and the
+    largest differences of the floating-point outputs."""
+    NT = 1e-3
+    st = res.stats
+    masked = inp.mask.astype(bool)
+    scored = ~np.isnan(res.lps_prob)
+    routed = ~np.isnan(res.lbs_logit)
+    nt = st.logit_gap < NT
+    out = {"against": "the CPU oracle (float64) on the same inputs, one step",
+           "tolerance_abs": tol,
+           "near_ties": {"top2_logit_gap": int(nt.sum()),
+                         "kappa_vs_tau": int((masked & (np.abs(st.conf - sh.tau) < NT)).sum()),
+                         "p_psi_vs_tau_psi": int((scored & (np.abs(res.lps_prob - sh.tau_psi) < NT)).sum()),
+                         "lbs_logit_vs_0": int((routed & (np.abs(res.lbs_logit) < NT)).sum())},
+           "argmax_mismatch": int(((gpu["argmax"].astype(np.int64) != st.argmax) & ~nt).sum())}
+    B = len(inp.cu_rows) - 1
+    flagged = 0
+    mism = {"accepted": 0, "tokens": 0, "mask": 0, "in_block": 0, "blk_meta": 0}
+    for b in range(B):
+        if res.flag_accept[b] or res.flag_lbs[b]:
+            flagged += 1
+            continue
+        sl = slice(int(inp.cu_rows[b]), int(inp.cu_rows[b + 1]))
+        for k in ("accepted", "tokens", "mask", "in_block"):
+            mism[k] += int((np.asarray(gpu[k][sl]).astype(np.int64) !=
+                            np.asarray(getattr(res, k)[sl]).astype(np.int64)).sum())
+        mism["blk_meta"] += int(not np.array_equal(gpu["blk_meta"][b], res.blk_meta[b]))
+    out["flagged_sequences"] = flagged
+    out["sequences"] = B
+    out["decision_mismatch"] = mism
+    diff = {}
+    for k, ref in (("conf", st.conf), ("entropy", st.entropy), ("ent_norm", st.ent_norm),
+                   ("gap", st.gap)):
+        diff[k] = float(np.abs(gpu[k].astype(np.float64) - ref).max())
+    if "attn_out" in gpu and res.attn_out is not None:
+        diff["attn_out"] = float(np.abs(gpu["attn_out"].astype(np.float64) - res.attn_out).max())
+    out["max_abs_diff"] = {k: float(f"{v:.3g}") for k, v in diff.items()}
+    out["within_tolerance"] = bool(max(diff.values()) <= tol and out["argmax_mismatch"] == 0 and
+                                   not any(mism.values()))
+    return out
 
 
 def run_loop_bench(args):
@@ -560,6 +624,21 @@ def run_loop_bench(args):
     print(json.dumps(line))
 
 
+def config_dict(sh, args, rows, masked, world):
+    """The workload of a bench line, the same for both arms."""
+    return {"workload": workload_text(sh, args.state), "state": args.state,
+            "rows": rows, "masked": masked,
+            "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
+            "l2": "flushed before every timed step: 256 MB write, then 256 MB read (write-back "
+                  "done outside the timed region); W_lm (1 GB) > L2",
+            "launch": "cuda_graph" if not args.no_graph else "stream",
+            "kv_cache": (f"dual: prefix + window + {suffix_len(sh)} cached positions after "
+                         f"the window" if args.cache == "dual" else "prefix") +
+                        ("; committed rows appended every step" if args.append else ""),
+            "w_lm": ("64x64 tiles, unit-major (ebd_pack_lm_head, once at load)"
+                     if args.w_layout == "packed" else "row-major [V][d]")}
+
+
 def run_reference(args, rank, world):
     """The CPU oracle as the reference arm: rank 0 only."""
     if rank != 0:
@@ -598,7 +677,7 @@ def run_reference(args, rank, world):
             "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": round(ms, 3), "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": {"workload": workload_text(sh, args.state), "state": args.state},
+            "config": config_dict(sh, args, inp.rows, int(inp.mask.sum()), world),
             "cpu_baseline": {"value": round(value, 3), "unit": UNIT, "cores": cores,
                              "kind": "oracle", "sample": sample},
             "e2e": {"value": round(value, 3), "unit": UNIT, "h2d_bytes_per_step": 0,
@@ -695,17 +774,7 @@ def main():
                                     for q in (10, 50, 90)],
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic (seeded; LLaDA-8B/Dream-7B shapes, random-init routers)",
-        "config": {"workload": workload_text(sh, args.state), "state": args.state,
-                   "rows": r["rows"], "masked": r["masked"],
-                   "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
-                   "l2": "flushed before every timed step: 256 MB write, then 256 MB read (write-back "
-                         "done outside the timed region); W_lm (1 GB) > L2",
-                   "launch": "cuda_graph" if not args.no_graph else "stream",
-                   "kv_cache": (f"dual: prefix + window + {suffix_len(sh)} cached positions after "
-                                f"the window" if args.cache == "dual" else "prefix") +
-                               ("; committed rows appended every step" if args.append else ""),
-                   "w_lm": ("64x64 tiles, unit-major (ebd_pack_lm_head, once at load)"
-                            if args.w_layout == "packed" else "row-major [V][d]")},
+        "config": config_dict(sh, args, r["rows"], r["masked"], world),
         "roofline": roof,
         "step_roofline": {"bytes": wk["step_bytes"], "flops": wk["step_flops"],
                           "t_roofline_us": round(t_roof * 1e6, 2),
@@ -742,11 +811,12 @@ def main():
                        "d2h_bytes_per_step": e["d2h"], "ms_per_step": round(e["mean_ms"], 4),
                        "api": "ebd_step_host"}
     if not args.skip_cpu and world == 1:
-        v, n, el = oracle_step_sample(sh, r["inp"], args.cpu_budget, r["suffix"])
+        v, n, el, res = oracle_step_sample(sh, r["inp"], args.cpu_budget, r["suffix"])
         line["cpu_baseline"] = {"value": round(v, 3), "unit": UNIT, "cores": os.cpu_count(),
                                 "kind": "oracle",
                                 "sample": f"{n} full oracle steps of {sh.name} "
                                           f"({r['rows']} rows each) in {el:.1f} s"}
+        line["parity"] = parity_summary(sh, r["inp"], res, r["fetch"])
     print(json.dumps(line))
     if world > 1:
         import torch.distributed as dist

@@ -63,3 +63,44 @@ def test_lm_grid_rule():
     for units in (153, 1000, 1976, 2376, 5000):
         g = b.lm_grid(152, units)
         assert -(-units // g) <= -(-units // 152) + 1
+
+
+def test_partials_per_row_rule():
+    """The partial states per row a handle keeps: the unpaired grid, or the
+    paired one (one pair per two SMs) when a step may take it."""
+    b = _bench()
+    assert b.lm_pair_grid(152, 1976) == 152 and b.lm_pair_grid(152, 64) == 32
+    assert b.partials_per_row(152, 1976, 32) == 142       # LLaDA-8B step: unpaired
+    assert b.partials_per_row(152, 2376, 512) == 152      # Dream-7B: pairs possible
+    assert b.partials_per_row(152, 64, 512) == 64         # tiny vocabulary
+
+
+def test_parity_summary_of_the_oracle_itself():
+    """bench.py's parity block, given the oracle's own outputs as the GPU's,
+    reports no mismatch; a changed argmax and a changed commit are counted."""
+    from oracle import ebd_oracle as o
+    b = _bench()
+    sh = synth.tiny
+    inp = synth.make_step_inputs(sh)
+    W = o.weights_f64(synth.router_weights(sh.seed, sh.d_base, sh.gen_len))
+    prm = o.DecisionParams(tau=sh.tau, tau_psi=sh.tau_psi, l_min=sh.l_min, l_b=sh.l_b,
+                           g_max=sh.g_max, eos_id=sh.eos_id, lps_enabled=bool(sh.lps_enabled))
+    res = o.step(inp, W, prm)
+    gpu = dict(conf=res.stats.conf.astype(np.float32), entropy=res.stats.entropy.astype(np.float32),
+               ent_norm=res.stats.ent_norm.astype(np.float32), gap=res.stats.gap.astype(np.float32),
+               argmax=res.stats.argmax.astype(np.int32), accepted=res.accepted.copy(),
+               tokens=res.tokens.copy(), mask=res.mask.copy(), in_block=res.in_block.copy(),
+               blk_meta=res.blk_meta.copy(), attn_out=res.attn_out.astype(np.float32))
+    rep = b.parity_summary(sh, inp, res, gpu)
+    assert rep["argmax_mismatch"] == 0 and not any(rep["decision_mismatch"].values())
+    assert rep["within_tolerance"] and rep["max_abs_diff"]["conf"] < 1e-6
+    assert set(rep["near_ties"]) == {"top2_logit_gap", "kappa_vs_tau", "p_psi_vs_tau_psi",
+                                     "lbs_logit_vs_0"}
+    r = int(np.flatnonzero(~res.stats.near_tie)[0])
+    gpu["argmax"][r] += 1
+    acc = int(np.flatnonzero(res.accepted)[0])
+    gpu["accepted"][acc] = 0
+    rep = b.parity_summary(sh, inp, res, gpu)
+    assert rep["argmax_mismatch"] == 1
+    if rep["flagged_sequences"] == 0:
+        assert rep["decision_mismatch"]["accepted"] == 1 and not rep["within_tolerance"]
