@@ -87,7 +87,7 @@ def workload_text(sh, state):
 
 def lm_kernel_hash():
     h = hashlib.sha256()
-    for f in ("k_lmhead.cu", "ptx.cuh", "internal.h"):
+    for f in ("k_lmhead.cu", "ptx.cuh", "lm_params.h"):
         with open(os.path.join(ROOT, "paper_2609_16450_gb300", "csrc", f), "rb") as fh:
             h.update(fh.read())
     return h.hexdigest()[:16]
