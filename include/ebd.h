@@ -69,6 +69,9 @@ typedef int32_t ebd_status;
 #define EBD_ERR_TIMEOUT (-4)     /* a device-side bounded wait gave up       */
 #define EBD_ERR_NONFINITE (-5)   /* NaN/Inf logit statistic; row not committed */
 #define EBD_ERR_STATE (-6)       /* call order: e.g. LBS needs a bound W_e   */
+#define EBD_ERR_BOUNDS (-7)      /* checked builds (EBD_CHECKS) only: a device
+                                    index outside its buffer; the access was
+                                    skipped                                   */
 
 /* decode_mode: which decision step 3 applies.  EBD_DECODE_EB is the EB
  * decision (LBS + LPS, App. E).  The other two are the fixed-block update

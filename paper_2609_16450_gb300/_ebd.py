@@ -19,6 +19,7 @@ EBD_ERR_CUDA = -3
 EBD_ERR_TIMEOUT = -4
 EBD_ERR_NONFINITE = -5
 EBD_ERR_STATE = -6
+EBD_ERR_BOUNDS = -7
 EBD_DEBUG_FORCE_TIMEOUT = 1
 EBD_DEBUG_FORCE_COPY_TIMEOUT = 2
 EBD_DECODE_EB = 0
@@ -27,7 +28,7 @@ EBD_DECODE_TOPM = 2
 
 STATUS_NAMES = {0: "EBD_OK", -1: "EBD_ERR_INVALID_ARG", -2: "EBD_ERR_UNSUPPORTED",
                 -3: "EBD_ERR_CUDA", -4: "EBD_ERR_TIMEOUT", -5: "EBD_ERR_NONFINITE",
-                -6: "EBD_ERR_STATE"}
+                -6: "EBD_ERR_STATE", -7: "EBD_ERR_BOUNDS"}
 
 
 class ebd_config(Structure):
@@ -72,10 +73,12 @@ class EbdError(RuntimeError):
 
 
 def load(path: str = LIB_PATH):
-    """Loads libebd.so; raises if it has not been built."""
+    """Loads libebd.so (or the library named by the EBD_LIBRARY environment
+    variable, e.g. the checked build); raises if it has not been built."""
     global _lib
     if _lib is not None:
         return _lib
+    path = os.environ.get("EBD_LIBRARY", path)
     if not os.path.exists(path):
         raise RuntimeError(f"{path} is missing: build it with paper_2609_16450_gb300.build.build()")
     lib = ctypes.CDLL(path)

@@ -622,6 +622,7 @@ ebd_status run_attention(ebd_handle* h, const ebd_step_args* a, cudaStream_t st,
   }
   AttnParams p{};
   p.B = a->batch;
+  p.R = a->rows;
   p.Hq = c.n_heads_q;
   p.Hkv = Hkv;
   p.D = D;
@@ -685,6 +686,7 @@ ebd_status run_lm(ebd_handle* h, const ebd_step_args* a, cudaStream_t st, bool p
     if (p.grid > h->grid_lm) lm_plan(p, rows, V, c.d_model, h->grid_lm, pair);
     if (p.grid > h->grid_lm) return fail(h, EBD_ERR_UNSUPPORTED, "LM head: grid exceeds the partials");
     p.ncols = h->grid_lm;
+    p.part_rows = c.max_rows;
     p.v_off = v_off;
     if (p.stages < 2) return fail(h, EBD_ERR_UNSUPPORTED, "LM head: shared memory plan failed");
     p.row0 = g0;
@@ -1681,6 +1683,7 @@ extern "C" ebd_status ebd_lm_stats_noalloc(const uint16_t* hidden, const uint16_
           nd->num_sms < EBD_NOALLOC_MAX_PARTS ? nd->num_sms : EBD_NOALLOC_MAX_PARTS);
   if (p.stages < 2 || p.grid > EBD_NOALLOC_MAX_PARTS) return EBD_ERR_UNSUPPORTED;
   p.row0 = 0;
+  p.part_rows = EBD_NOALLOC_MAX_ROWS;
   p.packed = packed ? 1 : 0;
   p.part_f = nd->part_f;
   p.part_i = nd->part_i;

@@ -10,6 +10,24 @@
 
 namespace ebd {
 
+// Checked builds (compiled with -DEBD_CHECKS): a global access whose index
+// comes from device data (row offsets, positions, counts) is preceded by a
+// check of the index against the buffer's extent; a failed check records
+// EBD_ERR_BOUNDS in the status word and the access is skipped (nothing traps
+// or waits).  In other builds the check compiles away.
+__device__ __forceinline__ bool in_bounds(long long i, long long n, int* status) {
+#ifdef EBD_CHECKS
+  if (i >= 0 && i < n) return true;
+  if (status != nullptr) atomicCAS(status, 0, EBD_ERR_BOUNDS);
+  return false;
+#else
+  (void)i;
+  (void)n;
+  (void)status;
+  return true;
+#endif
+}
+
 constexpr int kMaxWindow = 64;        // window rows per sequence of the cluster decision
 constexpr int kMaxSeqRows = 512;      // window rows per sequence of the grid-wide decision
 constexpr int kUnit = 64;             // vocabulary rows per work unit of the LM head
@@ -25,6 +43,7 @@ constexpr int kMaxAttnSplits = 8;
 // ------------------------------------------------------------------ attention
 struct AttnParams {
   int B, Hq, Hkv, D, group;
+  int R;                    // rows of the step (extent of q and out)
   int max_prefix;
   int max_qtiles, splits;
   const int* cu_rows;

@@ -48,6 +48,7 @@ __device__ __forceinline__ void attn_body(const CUtensorMap& tm_kc, const CUtens
   const int wb = p.cu_rows[b + 1] - r0;
   const int m_total = wb * p.group;
   if (wb <= 0 || wb > kMaxWindow || qt * 64 >= m_total) return;
+  if (!in_bounds(r0, p.R, p.status) || !in_bounds(r0 + wb - 1, p.R, p.status)) return;
   int P = p.prefix_len[b];
   P = P < 0 ? 0 : (P > p.max_prefix ? p.max_prefix : P);
   int S0 = 0, S = 0;  // suffix range of the cache (dual cache)
@@ -244,9 +245,9 @@ __device__ __forceinline__ void attn_body(const CUtensorMap& tm_kc, const CUtens
 #pragma unroll
       for (int t = 0; t < NT; ++t) {
         const int d = t * 8 + 2 * (lane & 3);
-        if (mrow_lo < m_total)
+        if (mrow_lo < m_total && in_bounds(r0 + mrow_lo % wb, p.R, p.status))
           *reinterpret_cast<float2*>(out_row(mrow_lo) + d) = make_float2(o[t][0] * il, o[t][1] * il);
-        if (mrow_hi < m_total)
+        if (mrow_hi < m_total && in_bounds(r0 + mrow_hi % wb, p.R, p.status))
           *reinterpret_cast<float2*>(out_row(mrow_hi) + d) = make_float2(o[t][2] * ih, o[t][3] * ih);
       }
     }
@@ -310,7 +311,8 @@ __device__ __forceinline__ void attn_body(const CUtensorMap& tm_kc, const CUtens
         acc.w = fmaf(wgt, v.w, acc.w);
       }
     }
-    *reinterpret_cast<float4*>(out_row(qt * 64 + r) + d) = acc;
+    if (in_bounds(r0 + (qt * 64 + r) % wb, p.R, p.status))
+      *reinterpret_cast<float4*>(out_row(qt * 64 + r) + d) = acc;
   }
   if (tid == 0) p.tickets[slot] = 0;
 }

@@ -719,7 +719,7 @@ __global__ void __cluster_dims__(kDecideCluster, 1, 1) __launch_bounds__(kDecide
       const float gap = (1.0f - expf(l2 - m)) / s;
       const bool bad = !(isfinite(m) && isfinite(s) && isfinite(t) && s >= 1.0f) || idx < 0 ||
                        idx >= p.V;
-      if (lane == 0) {
+      if (lane == 0 && in_bounds(r0 + j, p.rows_expected, p.status)) {
         const int r = r0 + j;
         if (p.conf) p.conf[r] = conf;
         if (p.entropy) p.entropy[r] = ent;
@@ -1130,6 +1130,7 @@ __global__ void __cluster_dims__(kDecideCluster, 1, 1) __launch_bounds__(kDecide
   if (shadow) return;
   for (int j = tid; j < nr; j += blockDim.x) {
     const int r = r0 + j;
+    if (!in_bounds(r, p.rows_expected, p.status)) continue;
     p.tokens_out[r] = sm.f_tok[j];
     p.mask_out[r] = sm.f_mask[j];
     p.in_block_out[r] = sm.f_ib[j];

@@ -836,7 +836,7 @@ __global__ void __launch_bounds__(kSeqThreads) seq_accept_kernel(const SeqParams
     acc = bm && k == s_best;
   }
   bool msk = row && p.mask[r] != 0;
-  if (acc) {
+  if (acc && in_bounds(r, p.R, p.status)) {
     p.tokens[r] = p.argmax[r];
     msk = false;
   }
@@ -844,7 +844,7 @@ __global__ void __launch_bounds__(kSeqThreads) seq_accept_kernel(const SeqParams
   if (inb && msk) atomicOr(&s_open, 1);
   __syncthreads();
   const bool resolve = p.mode == EBD_DECODE_EB && meta_s > 0 && !s_open;
-  if (row) {
+  if (row && in_bounds(r, p.R, p.status)) {
     p.mask[r] = msk ? 1 : 0;
     if (p.mode == EBD_DECODE_EB) p.in_block[r] = (inb && !resolve) ? 1 : 0;
     if (p.accepted) p.accepted[r] = acc ? 1 : 0;

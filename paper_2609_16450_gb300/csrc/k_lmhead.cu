@@ -543,6 +543,7 @@ __global__ void __launch_bounds__(kLmThreads, 1)
       const int cta = static_cast<int>(blockIdx.x);
       for (int r = et; r < p.rows; r += 128) {
         if (((r >> 5) % p.nwg) != wg) continue;
+        if (!in_bounds(rbase + r, p.part_rows, p.status) || !in_bounds(cta, p.ncols, p.status)) continue;
         const size_t o = static_cast<size_t>(rbase + r) * p.ncols + cta;
         p.part_f[o] = make_float4(st_m[r], st_s[r], st_t[r], st_l2[r]);
         p.part_i[o] = st_i[r];

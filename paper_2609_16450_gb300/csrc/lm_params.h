@@ -21,6 +21,7 @@ struct LmParams {
   int pair;                 // CTA pairs (clusters of 2) running cta_group::2 MMAs, M = 256
   int nwork;                // owners of vocabulary ranges: CTAs, or pairs
   int ncols;                // partial states per row written (>= grid; extra ones neutral)
+  int part_rows;            // rows the partial buffers hold
   uint32_t off_a, off_b, off_t, off_st, off_bar, smem_bytes;
   float4* part_f;           // [R][grid] (max, sum exp, sum exp*(l-max), second logit)
   int* part_i;              // [R][grid] argmax
