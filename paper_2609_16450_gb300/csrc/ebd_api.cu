@@ -9,9 +9,20 @@
 #include <string>
 #include <vector>
 
+#include <nvtx3/nvToolsExt.h>
+
 #include "ebd.h"
 #include "internal.h"
 #include "router_image.h"
+
+namespace {
+// An NVTX range around the host side of an entry point (visible in Nsight
+// Systems timelines; a no-op when no tool is attached).
+struct NvtxRange {
+  explicit NvtxRange(const char* name) { nvtxRangePushA(name); }
+  ~NvtxRange() { nvtxRangePop(); }
+};
+}  // namespace
 
 namespace ebd {
 cudaError_t decide_configure();
@@ -1286,6 +1297,7 @@ ebd_status step_run(ebd_handle* h, const ebd_step_args* a, cudaStream_t st, cons
 }  // namespace
 
 ebd_status ebd_step(ebd_handle* h, const ebd_step_args* a, void* stream) {
+  NvtxRange nvtx("ebd_step");
   if (h == nullptr) return EBD_ERR_INVALID_ARG;
   ebd_status s = check_device(h);
   if (s != EBD_OK) return s;
@@ -1300,6 +1312,7 @@ ebd_status ebd_step(ebd_handle* h, const ebd_step_args* a, void* stream) {
 }
 
 ebd_status ebd_decide(ebd_handle* h, const ebd_step_args* a, void* stream) {
+  NvtxRange nvtx("ebd_decide");
   if (h == nullptr) return EBD_ERR_INVALID_ARG;
   ebd_status s = check_device(h);
   if (s != EBD_OK) return s;
@@ -1323,6 +1336,7 @@ ebd_status ebd_decide(ebd_handle* h, const ebd_step_args* a, void* stream) {
 }
 
 ebd_status ebd_lm_stats(ebd_handle* h, const ebd_step_args* a, void* stream) {
+  NvtxRange nvtx("ebd_lm_stats");
   if (h == nullptr) return EBD_ERR_INVALID_ARG;
   ebd_status s = check_device(h);
   if (s != EBD_OK) return s;
@@ -1340,6 +1354,7 @@ ebd_status ebd_lm_stats(ebd_handle* h, const ebd_step_args* a, void* stream) {
 
 ebd_status ebd_lm_shard_state(ebd_handle* h, const ebd_step_args* a, int32_t v_off,
                               int32_t v_count, float* state, void* stream) {
+  NvtxRange nvtx("ebd_lm_shard_state");
   if (h == nullptr) return EBD_ERR_INVALID_ARG;
   ebd_status s = check_device(h);
   if (s != EBD_OK) return s;
@@ -1358,6 +1373,7 @@ ebd_status ebd_lm_shard_state(ebd_handle* h, const ebd_step_args* a, int32_t v_o
 
 ebd_status ebd_merge_shard_states(ebd_handle* h, const float* states, int32_t shards,
                                   const ebd_step_args* a, void* stream) {
+  NvtxRange nvtx("ebd_merge_shard_states");
   if (h == nullptr) return EBD_ERR_INVALID_ARG;
   ebd_status s = check_device(h);
   if (s != EBD_OK) return s;
@@ -1376,6 +1392,7 @@ ebd_status ebd_merge_shard_states(ebd_handle* h, const float* states, int32_t sh
 }
 
 ebd_status ebd_attention(ebd_handle* h, const ebd_step_args* a, void* stream) {
+  NvtxRange nvtx("ebd_attention");
   if (h == nullptr) return EBD_ERR_INVALID_ARG;
   ebd_status s = check_device(h);
   if (s != EBD_OK) return s;
@@ -1394,6 +1411,7 @@ ebd_status ebd_attention(ebd_handle* h, const ebd_step_args* a, void* stream) {
 // step's ticket, which the attention waits for; `stream` waits for that
 // stream at the end of the step.
 ebd_status ebd_step_host(ebd_handle* h, const ebd_step_args* a, void* stream) {
+  NvtxRange nvtx("ebd_step_host");
   if (h == nullptr) return EBD_ERR_INVALID_ARG;
   ebd_status s = check_device(h);
   if (s != EBD_OK) return s;
