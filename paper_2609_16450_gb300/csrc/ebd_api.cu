@@ -694,8 +694,8 @@ ebd_status run_lm(ebd_handle* h, const ebd_step_args* a, cudaStream_t st, bool p
     const bool pair = rows >= pair_min && h->grid_lm >= lm_pair_grid(h->num_sms, units);
     lm_plan(p, rows, V, c.d_model, h->num_sms, pair);
     // a shard's own grid may exceed the partial columns of the handle
-    if (p.grid > h->grid_lm) lm_plan(p, rows, V, c.d_model, h->grid_lm, pair);
-    if (p.grid > h->grid_lm) return fail(h, EBD_ERR_UNSUPPORTED, "LM head: grid exceeds the partials");
+    if (p.grp_cols > h->grid_lm) lm_plan(p, rows, V, c.d_model, h->grid_lm, pair);
+    if (p.grp_cols > h->grid_lm) return fail(h, EBD_ERR_UNSUPPORTED, "LM head: grid exceeds the partials");
     p.ncols = h->grid_lm;
     p.part_rows = c.max_rows;
     p.v_off = v_off;

@@ -235,8 +235,13 @@ __global__ void __launch_bounds__(kLmThreads, 1)
   const int lane = tid & 31;
   const uint32_t crank = PAIR ? cluster_ctarank() : 0u;
   const bool leader = crank == 0;
-  const int owner = PAIR ? static_cast<int>(blockIdx.x >> 1) : static_cast<int>(blockIdx.x);
-  const int rbase = p.row0;  // first row of the launch
+  // row group of this CTA (its pair) and its owner index within the group
+  const int q = PAIR ? static_cast<int>(blockIdx.x >> 1) : static_cast<int>(blockIdx.x);
+  const int grp = q / p.nwork;
+  const int owner = q - grp * p.nwork;
+  const int rbase = p.row0 + grp * p.nb;                 // first row of the group
+  const int rows_g = min(p.rgroups > 1 ? p.nb : p.rows, p.rows - grp * p.nb);
+  const int col = PAIR ? 2 * owner + static_cast<int>(crank) : owner;  // partial column
   // hidden rows of one N sub-tile that this CTA holds: all of them, or its
   // half in a pair
   const int hrows = PAIR ? p.nb / 2 : p.nb;
@@ -538,18 +543,18 @@ __global__ void __launch_bounds__(kLmThreads, 1)
     }
     if (ok && active) {
       // the rows of this warpgroup's slices (its threads updated them last):
-      // this CTA's partial goes to column blockIdx.x, and neutral states to
-      // the columns [grid, ncols) that no CTA of this launch owns
-      const int cta = static_cast<int>(blockIdx.x);
-      for (int r = et; r < p.rows; r += 128) {
+      // this CTA's partial goes to column `col` of its group's rows, and
+      // neutral states to the columns [grp_cols, ncols) that no CTA of the
+      // group owns
+      for (int r = et; r < rows_g; r += 128) {
         if (((r >> 5) % p.nwg) != wg) continue;
-        if (!in_bounds(rbase + r, p.part_rows, p.status) || !in_bounds(cta, p.ncols, p.status)) continue;
-        const size_t o = static_cast<size_t>(rbase + r) * p.ncols + cta;
+        if (!in_bounds(rbase + r, p.part_rows, p.status) || !in_bounds(col, p.ncols, p.status)) continue;
+        const size_t o = static_cast<size_t>(rbase + r) * p.ncols + col;
         p.part_f[o] = make_float4(st_m[r], st_s[r], st_t[r], st_l2[r]);
         p.part_i[o] = st_i[r];
-        for (int jc = p.grid + cta; jc < p.ncols; jc += p.grid) {  // neutral states
-          p.part_f[o - cta + jc] = make_float4(-INFINITY, 0.f, 0.f, -INFINITY);
-          p.part_i[o - cta + jc] = INT_MAX;
+        for (int jc = p.grp_cols + col; jc < p.ncols; jc += p.grp_cols) {  // neutral states
+          p.part_f[o - col + jc] = make_float4(-INFINITY, 0.f, 0.f, -INFINITY);
+          p.part_i[o - col + jc] = INT_MAX;
         }
       }
     }
@@ -596,9 +601,21 @@ void lm_plan(LmParams& p, int rows, int V, int d, int num_sms, bool pair) {
   p.d = d;
   p.rows = rows;
   p.pair = pair ? 1 : 0;
-  p.nsub = (rows + 255) / 256;
+  // Paired launches of more than 432 rows split the rows into two groups of
+  // at most 256, each served by half the pairs over the whole vocabulary:
+  // every CTA's accumulator then fits twice in TMEM, so the epilogue of one
+  // chunk overlaps the MMAs of the next, and LLaDA-8B's 494 chunks split
+  // evenly over 38 pairs (6.5 per pair otherwise), at the cost of each W tile
+  // being read by two pairs (the second read from L2) and ~33 % more operand
+  // bytes per flop.  Measured (LM head): 512 rows 401 -> 378 us, 1024 rows
+  // 796 -> 751 us, 4096 rows 3188 -> 3021 us; but Dream-7B's 390 rows (groups
+  // of 208) 361 -> 396 us, hence the threshold.
+  p.rgroups = pair && rows > 432 ? (rows + 255) / 256 : 1;
+  if (const char* env = getenv("EBD_LM_RGROUPS")) p.rgroups = pair && atoi(env) > 1 ? (rows + 255) / 256 : 1;
+  p.nsub = p.rgroups > 1 ? 1 : (rows + 255) / 256;
   if (p.nsub < 1) p.nsub = 1;
-  p.nb = ((rows + p.nsub - 1) / p.nsub + 15) / 16 * 16;
+  p.nb = p.rgroups > 1 ? ((rows + p.rgroups - 1) / p.rgroups + 15) / 16 * 16
+                       : ((rows + p.nsub - 1) / p.nsub + 15) / 16 * 16;
   if (p.nb < 16) p.nb = 16;
   p.n_pad = p.nb * p.nsub;
   p.acc_stride = (p.n_pad + 31) / 32 * 32;
@@ -608,14 +625,16 @@ void lm_plan(LmParams& p, int rows, int V, int d, int num_sms, bool pair) {
   while (tc < cols) tc <<= 1;
   p.tmem_cols = tc;
   p.n_units = (V + kUnit - 1) / kUnit;
-  if (pair) {  // 4 units per accumulator
-    p.grid = lm_pair_grid(num_sms, p.n_units);
-    p.nwork = p.grid / 2;
+  if (pair) {  // 4 units per accumulator; the pairs split evenly over the row groups
+    p.nwork = lm_pair_grid(num_sms / p.rgroups, p.n_units) / 2;
+    p.grid = 2 * p.nwork * p.rgroups;
+    p.grp_cols = 2 * p.nwork;
   } else {
     p.grid = lm_grid(num_sms, p.n_units);
     p.nwork = p.grid;
+    p.grp_cols = p.grid;
   }
-  p.ncols = p.grid;  // partial states per row (a caller may raise it: neutral states)
+  p.ncols = p.grp_cols;  // partial states per row (a caller may raise it: neutral states)
   // a second epilogue warpgroup (and its transpose buffer) only pays where
   // the epilogue is exposed, i.e. with a single accumulator buffer; with two,
   // one warpgroup keeps up with the MMAs and its buffer is worth more as

@@ -19,7 +19,10 @@ struct LmParams {
   int stages, nbuf, acc_stride, tmem_cols;
   int nwg;                  // epilogue warpgroups in use (2 with a single accumulator buffer)
   int pair;                 // CTA pairs (clusters of 2) running cta_group::2 MMAs, M = 256
-  int nwork;                // owners of vocabulary ranges: CTAs, or pairs
+  int nwork;                // owners of vocabulary ranges per row group: CTAs, or pairs
+  int rgroups;              // row groups (paired launches of more than 256 rows: 2), each
+                            // of nb rows, served by its own nwork owners
+  int grp_cols;             // CTAs per row group (the partial columns a row gets here)
   int ncols;                // partial states per row written (>= grid; extra ones neutral)
   int part_rows;            // rows the partial buffers hold
   uint32_t off_a, off_b, off_t, off_st, off_bar, smem_bytes;
