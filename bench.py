@@ -85,11 +85,26 @@ def workload_text(sh, state):
             f"window rows {int(w.sum())} ({'no active block: LBS runs' if state == 'select' else 'active block'})")
 
 
-def lm_kernel_hash():
+def strip_comments(src: str) -> str:
+    """C/C++ source without its comments and blank lines (string literals in
+    these files hold no comment markers)."""
+    import re
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    src = re.sub(r"//[^\n]*", "", src)
+    return "\n".join(l.rstrip() for l in src.splitlines() if l.strip())
+
+
+def lm_kernel_hash(read=None):
+    """Hash of the LM head's sources (k_lmhead.cu, ptx.cuh, lm_params.h)
+    without comments: the kernel a profile was captured on."""
     h = hashlib.sha256()
     for f in ("k_lmhead.cu", "ptx.cuh", "lm_params.h"):
-        with open(os.path.join(ROOT, "paper_2609_16450_gb300", "csrc", f), "rb") as fh:
-            h.update(fh.read())
+        if read is None:
+            with open(os.path.join(ROOT, "paper_2609_16450_gb300", "csrc", f)) as fh:
+                text = fh.read()
+        else:
+            text = read(f)
+        h.update(strip_comments(text).encode())
     return h.hexdigest()[:16]
 
 

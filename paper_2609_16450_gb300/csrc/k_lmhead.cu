@@ -200,6 +200,11 @@ __device__ __forceinline__ bool epilogue_buffer(uint32_t taddr0, int wg, int nwg
 // barriers; both epilogues release the accumulator on the leader's barrier.
 // Each SM thus receives half of the hidden rows per MMA, which halves the
 // operand bytes per flop against a 128-row tile over the same rows.
+//
+// Row groups (p.rgroups = 2, paired launches of more than 432 rows): pair q
+// serves rows [row0 + g nb, row0 + (g + 1) nb) of group g = q / nwork over
+// the vocabulary range of owner q % nwork, and writes its partials to
+// columns [0, grp_cols) of those rows.
 template <bool PAIR, bool PACKED>
 __global__ void __launch_bounds__(kLmThreads, 1)
     lm_stats_kernel(const __grid_constant__ CUtensorMap tmap_w,
@@ -227,10 +232,6 @@ __global__ void __launch_bounds__(kLmThreads, 1)
 
   constexpr int kChunkUnits = PAIR ? 4 : 2;  // vocabulary units per accumulator
   const int tid = threadIdx.x;
-  // the decision kernel, launched after this one as a programmatic dependent,
-  // may be scheduled as soon as SMs free up; it waits for this grid's
-  // completion before it reads the partial states (as a dependent itself,
-  // this grid releases it only after its own wait, below)
   const int warp = __shfl_sync(0xffffffffu, tid / 32, 0);
   const int lane = tid & 31;
   const uint32_t crank = PAIR ? cluster_ctarank() : 0u;

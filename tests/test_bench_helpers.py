@@ -104,3 +104,14 @@ def test_parity_summary_of_the_oracle_itself():
     assert rep["argmax_mismatch"] == 1
     if rep["flagged_sequences"] == 0:
         assert rep["decision_mismatch"]["accepted"] == 1 and not rep["within_tolerance"]
+
+
+def test_kernel_hash_ignores_comments_only():
+    """The profiled-traffic hash follows the LM head's code, not its
+    comments: a comment-only change keeps it, a code change does not."""
+    b = _bench()
+    import os as _os
+    base = lambda f: open(_os.path.join(ROOT, "paper_2609_16450_gb300", "csrc", f)).read()
+    h0 = b.lm_kernel_hash(base)
+    assert b.lm_kernel_hash(lambda f: "// a note\n/* and\n another */\n" + base(f) + "\n// end\n") == h0
+    assert b.lm_kernel_hash(lambda f: base(f).replace("kUnit", "kUnit ", 1) + "\nint x;\n") != h0
