@@ -22,7 +22,8 @@ LIB = os.path.join(PKG, "libebd.so")
 # EBD_ERR_BOUNDS and skip the access), a separate library for tests
 BUILD_CHECKED = os.path.join(PKG, "_build_checked")
 LIB_CHECKED = os.path.join(PKG, "libebd_checked.so")
-SOURCES = ["ebd_api.cu", "k_lmhead.cu", "k_attn.cu", "k_decide.cu", "k_decide_seq.cu"]
+SOURCES = ["ebd_api.cu", "k_lmhead.cu", "k_attn.cu", "k_decide.cu", "k_decide_cta.cu",
+           "k_decide_seq.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

@@ -26,6 +26,7 @@ struct NvtxRange {
 
 namespace ebd {
 cudaError_t decide_configure();
+cudaError_t decide_cta_configure();
 cudaError_t attn_configure();
 cudaError_t lm_configure();
 cudaError_t launch_merge_stats(const float4* part_f, const int* part_i, int rows, int grid,
@@ -202,6 +203,7 @@ struct ebd_handle {
   float4* part_f = nullptr;
   int* part_i = nullptr;
   int grid_lm = 0;       // LM-head partial states per row
+  int lm_ctas = 0;       // CTAs of the last LM-head launch (one SM each)
   int lm_units = 0;      // 64-row vocabulary units
   float* attn_part = nullptr;
   float* attn_part_ml = nullptr;
@@ -527,17 +529,77 @@ ebd_status upload_router(ebd_handle* h) {
     for (int k = 0; k < 64; ++k)
       for (int o = 0; o < 32; ++o) wl[PL_FF2 + k * PL_LDFF2 + o] = at(pre + ".ff2.w", o, k);
   }
+  // the one-CTA kernel's image (rcta): 128 x 64 swizzled A tiles of W [out][in]
+  std::vector<uint16_t> cw(static_cast<size_t>(rcta::kChunks) * rcta::kChunkElems, 0);
+  std::vector<float> cv(rcta::S_ELEMS, 0.f);
+  {
+    using namespace rcta;
+    auto chunk = [&](int c) { return cw.data() + static_cast<size_t>(c) * kChunkElems; };
+    // chunks c0 + t * nkb + kb: rows [128 t, 128 t + 128) (< outs), inputs [64 kb, 64 kb + 64)
+    auto tiles = [&](int c0, const std::string& n, int outs, int ins) {
+      const int nt = (outs + 127) / 128, nkb = ins / 64;
+      for (int t = 0; t < nt; ++t)
+        for (int kb = 0; kb < nkb; ++kb)
+          for (int m = 0; m < 128 && 128 * t + m < outs; ++m)
+            for (int k = 0; k < 64; ++k)
+              chunk(c0 + t * nkb + kb)[tile_off(m, k)] = at(n, 128 * t + m, 64 * kb + k);
+    };
+    tiles(C_ENT, "lbs.ent2.w", 64, 64);
+    tiles(C_COMB, "lbs.comb.w", 128, 128);
+    for (int l = 0; l < 2; ++l) {
+      const std::string pre = "lbs.l" + std::to_string(l);
+      const int base = C_LAYER0 + l * CL_CHUNKS;
+      tiles(base + CL_QKV, pre + ".qkv.w", 384, 128);
+      tiles(base + CL_OUT, pre + ".out.w", 128, 128);
+      tiles(base + CL_FF1, pre + ".ff1.w", 256, 128);
+      tiles(base + CL_FF2, pre + ".ff2.w", 128, 256);
+      float* vl = cv.data() + S_LAYER0 + l * S_LAYER_STRIDE;
+      for (int o = 0; o < 384; ++o) vl[SL_QKVB + o] = atf(pre + ".qkv.b", 0, o);
+      for (int o = 0; o < 256; ++o) vl[SL_FF1B + o] = atf(pre + ".ff1.b", 0, o);
+      for (int o = 0; o < 128; ++o) {
+        vl[SL_OUTB + o] = atf(pre + ".out.b", 0, o);
+        vl[SL_FF2B + o] = atf(pre + ".ff2.b", 0, o);
+        vl[SL_LN1G + o] = atf(pre + ".ln1.g", 0, o);
+        vl[SL_LN1B + o] = atf(pre + ".ln1.b", 0, o);
+        vl[SL_LN2G + o] = atf(pre + ".ln2.g", 0, o);
+        vl[SL_LN2B + o] = atf(pre + ".ln2.b", 0, o);
+      }
+    }
+    uint16_t* pos = reinterpret_cast<uint16_t*>(cv.data() + S_POS);
+    for (int j = 0; j < rcta::kPosRows; ++j)
+      for (int o = 0; o < 128; ++o) pos[j * 128 + o] = j < gen_len ? at("lbs.pos", j, o) : 0;
+    std::copy(lps.begin(), lps.end(), chunk(C_LPS));
+    for (int o = 0; o < 64; ++o) {
+      cv[S_ENT1W + o] = atf("lbs.ent1.w", o, 0);
+      cv[S_ENT1B + o] = atf("lbs.ent1.b", 0, o);
+      cv[S_ENT2B + o] = atf("lbs.ent2.b", 0, o);
+      cv[S_ENTLNG + o] = atf("lbs.ent_ln.g", 0, o);
+      cv[S_ENTLNB + o] = atf("lbs.ent_ln.b", 0, o);
+      cv[S_TOKB + o] = atf("lbs.tok.b", 0, o);
+    }
+    for (int o = 0; o < 128; ++o) {
+      cv[S_COMBB + o] = atf("lbs.comb.b", 0, o);
+      cv[S_HEADW + o] = atf("lbs.head.w", 0, o);
+    }
+    cv[S_HEADB] = atf("lbs.head.b", 0, 0);
+    // the LPS vectors: the same as every rank's copy above
+    std::copy(vec.begin() + V_LPS, vec.begin() + V_ELEMS, cv.begin() + S_LPS);
+  }
   const size_t b_lbs = lbs.size() * 2, b_lps = lps.size() * 2, b_vec = vec.size() * 4;
   const size_t o_lps = (b_lbs + 255) / 256 * 256;
   const size_t o_vec = o_lps + (b_lps + 255) / 256 * 256;
-  const size_t total = o_vec + b_vec;
+  const size_t o_cw = o_vec + (b_vec + 255) / 256 * 256;
+  const size_t o_cv = o_cw + (cw.size() * 2 + 255) / 256 * 256;
+  const size_t total = o_cv + cv.size() * 4;
   if (h->d_image) cudaFree(h->d_image);
   h->d_image = nullptr;
   cudaError_t e = cudaMalloc(&h->d_image, total);
   if (e != cudaSuccess) return cuda_fail(h, e, "cudaMalloc(router image)");
   if ((e = cudaMemcpy(h->d_image, lbs.data(), b_lbs, cudaMemcpyHostToDevice)) != cudaSuccess ||
       (e = cudaMemcpy(h->d_image + o_lps, lps.data(), b_lps, cudaMemcpyHostToDevice)) != cudaSuccess ||
-      (e = cudaMemcpy(h->d_image + o_vec, vec.data(), b_vec, cudaMemcpyHostToDevice)) != cudaSuccess)
+      (e = cudaMemcpy(h->d_image + o_vec, vec.data(), b_vec, cudaMemcpyHostToDevice)) != cudaSuccess ||
+      (e = cudaMemcpy(h->d_image + o_cw, cw.data(), cw.size() * 2, cudaMemcpyHostToDevice)) != cudaSuccess ||
+      (e = cudaMemcpy(h->d_image + o_cv, cv.data(), cv.size() * 4, cudaMemcpyHostToDevice)) != cudaSuccess)
     return cuda_fail(h, e, "cudaMemcpy(router image)");
   e = cudaMemcpy(h->d_blob, h->h_blob.data(), h->h_blob.size() * 2, cudaMemcpyHostToDevice);
   if (e != cudaSuccess) return cuda_fail(h, e, "cudaMemcpy(router blob)");
@@ -545,6 +607,8 @@ ebd_status upload_router(ebd_handle* h) {
   h->img.lps_w = reinterpret_cast<const __nv_bfloat16*>(h->d_image + o_lps);
   h->img.vec = reinterpret_cast<const float*>(h->d_image + o_vec);
   h->img.tok_table = h->d_tok;
+  h->img.cta_w = reinterpret_cast<const __nv_bfloat16*>(h->d_image + o_cw);
+  h->img.cta_vec = reinterpret_cast<const float*>(h->d_image + o_cv);
   return upload_seq_weights(h);
 }
 
@@ -717,8 +781,27 @@ ebd_status run_lm(ebd_handle* h, const ebd_step_args* a, cudaStream_t st, bool p
       return fail(h, EBD_ERR_CUDA, "cuTensorMapEncodeTiled (hidden) failed");
     cudaError_t e = launch_lm_stats(tw, th, p, st);
     if (e != cudaSuccess) return cuda_fail(h, e, "LM-head launch");
+    h->lm_ctas = p.grid;
   }
   return EBD_OK;
+}
+
+// Which kernel decides a launch of `batch` sequences with windows of up to
+// kCtaWindow rows: the one-CTA kernel from kCtaMinBatch sequences on, the
+// cluster kernel below.  Measured on the LLaDA-8B head shape (µs per step,
+// one-CTA against cluster): 1 x 32 rows 209 / 197, 4 x 32 245 / 214,
+// 16 x 8 200 / 212, 16 x 32 454 / 465, 64 x 8 464 / 515, 64 x 32 1638 /
+// 1749: one sequence decides faster on eight SMs, while many sequences
+// need several waves of 8-CTA clusters.  EBD_DECIDE_KERNEL=cta or cluster
+// overrides the rule (a measurement knob).
+constexpr int kCtaMinBatch = 16;
+bool cta_decision(const ebd_handle* h, int batch) {
+  if (h->cfg.max_window > kCtaWindow) return false;
+  if (const char* env = getenv("EBD_DECIDE_KERNEL")) {
+    if (strcmp(env, "cta") == 0) return true;
+    if (strcmp(env, "cluster") == 0) return false;
+  }
+  return batch >= kCtaMinBatch;
 }
 
 DecideParams decide_params(ebd_handle* h, const ebd_step_args* a, int features_in) {
@@ -872,7 +955,8 @@ ebd_status ebd_create(const ebd_config* cfg, ebd_handle** out) {
     return bail(fail(h, EBD_ERR_CUDA, "cuTensorMapEncodeTiled is unavailable"));
   if ((e = lm_configure()) != cudaSuccess) return bail(cuda_fail(h, e, "LM-head attributes"));
   if ((e = attn_configure()) != cudaSuccess) return bail(cuda_fail(h, e, "attention attributes"));
-  if ((e = decide_configure()) != cudaSuccess) return bail(cuda_fail(h, e, "decision attributes"));
+  if ((e = decide_configure()) != cudaSuccess || (e = decide_cta_configure()) != cudaSuccess)
+    return bail(cuda_fail(h, e, "decision attributes"));
 
   h->layout = router_layout(cfg->d_base, cfg->gen_len);
   h->h_blob.resize(layout_count(h->layout));
@@ -1273,7 +1357,11 @@ ebd_status step_run(ebd_handle* h, const ebd_step_args* a, cudaStream_t st, cons
     p.in_block_out = rt->in_block_out;
     p.blk_meta_out = rt->blk_meta_out;
   }
-  cudaError_t e = launch_decide(p, st);
+  const bool cta = cta_decision(h, a->batch);
+  // the LM head's CTAs hold one SM each: the decision's CTAs are placed while
+  // it runs if enough SMs are left, and then warm up on a stand-in window
+  p.warm = (p.pdl && cta && h->num_sms - h->lm_ctas >= a->batch) ? 1 : 0;
+  cudaError_t e = cta ? launch_decide_cta(p, st) : launch_decide(p, st);
   if (e != cudaSuccess) return cuda_fail(h, e, "decision launch");
   if (prof == 1 && (e0 = record(h->ev[2], st)) != cudaSuccess)
     return cuda_fail(h, e0, "profile event");
@@ -1330,7 +1418,8 @@ ebd_status ebd_decide(ebd_handle* h, const ebd_step_args* a, void* stream) {
   }
   DecideParams p = decide_params(h, a, 1);
   p.entropy = nullptr;
-  cudaError_t e = launch_decide(p, static_cast<cudaStream_t>(stream));
+  cudaError_t e = cta_decision(h, a->batch) ? launch_decide_cta(p, static_cast<cudaStream_t>(stream))
+                                  : launch_decide(p, static_cast<cudaStream_t>(stream));
   if (e != cudaSuccess) return cuda_fail(h, e, "decision launch");
   return EBD_OK;
 }

@@ -35,6 +35,8 @@ constexpr int kLmThreads = 320;  // TMA warp, MMA warp, two epilogue warpgroups 
 constexpr int kMaxGroupRows = 512;    // rows per LM-head launch (TMEM: 512 columns)
 constexpr int kDecideCluster = 8;     // CTAs per sequence in the decision kernel
 constexpr int kDecideThreads = 256;
+constexpr int kCtaWindow = 32;        // window rows per sequence of the one-CTA decision
+constexpr int kCtaThreads = 512;
 constexpr int kAttnThreads = 128;
 constexpr int kAttnChunk = 64;        // keys per K/V tile
 constexpr int kAttnStages = 3;
@@ -68,12 +70,17 @@ struct RouterImage {
   const __nv_bfloat16* lps_w;  // [LPS_W_ELEMS]
   const float* vec;            // [8 ranks][V_ELEMS]
   const float* tok_table;      // [V][64] = W_tok W_e[v] (no bias)
+  const __nv_bfloat16* cta_w;  // [rcta::kChunks][rcta::kChunkElems] (one-CTA kernel)
+  const float* cta_vec;        // [rcta::S_ELEMS]
 };
 
 struct DecideParams {
   int B, V, grid_lm;        // grid_lm: LM-head partials per row
   int features_in;          // 1: conf/ent_norm/gap/argmax are inputs
   int pdl;                  // launched as a programmatic dependent of the LM head
+  int warm;                 // one-CTA kernel: its CTAs find free SMs while the LM head
+                            // runs, and each runs the decision once on a stand-in window
+                            // before it waits for the LM head
   int mode, top_m;          // EBD_DECODE_*; commits per step of the Top-m rule
   int gen_len, g_max, l_min, l_b, eos_id, lps_enabled;
   float tau, tau_psi, inv_log_v;
@@ -172,6 +179,9 @@ cudaError_t launch_attention(const CUtensorMap& kc, const CUtensorMap& vc, const
                              const CUtensorMap& vw, const AttnParams& p, cudaStream_t st,
                              bool pdl = false);
 cudaError_t launch_decide(const DecideParams& p, cudaStream_t st);
+// the same decision with one CTA per sequence, for windows of up to
+// kCtaWindow rows (k_decide_cta.cu)
+cudaError_t launch_decide_cta(const DecideParams& p, cudaStream_t st);
 // vocabulary-parallel LM head: one state per row from a launch's partials,
 // and the statistics from the states of several shards (k_decide.cu)
 cudaError_t launch_shard_state(const float4* part_f, const int* part_i, int rows, int grid,

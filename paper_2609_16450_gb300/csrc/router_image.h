@@ -71,5 +71,53 @@ static_assert((LBS_W_ELEMS * 2) % 16 == 0 && (LPS_W_ELEMS * 2) % 16 == 0 &&
                   (V_ELEMS * 4) % 16 == 0,
               "bulk copies move multiples of 16 bytes");
 
+// ---- the one-CTA decision kernel (windows of up to 32 rows).  Its LBS
+// products run on the tcgen05 tensor cores with the weights as the A operand:
+// every matrix W [out][in] is cut into tiles of 128 output rows x 64 inputs,
+// each stored as the K-major, 128-byte-swizzled shared-memory image the MMA
+// reads (row m at m * 128 bytes; its 16-byte chunk c at chunk c ^ (m & 7)),
+// 16 KB, so that one bulk copy moves one tile into a slot of a ring.  The
+// tiles are stored in the order the kernel consumes them; a tile of a
+// product with T output tiles and K / 64 input boxes is at chunk t * (K / 64)
+// + kb.  Rows beyond a matrix's outputs are zero.
+namespace rcta {
+
+constexpr int kChunkElems = 8192;  // bf16 elements per chunk (16 KB)
+constexpr int kPosRows = 32;       // E_pos rows a window can use
+constexpr int C_ENT = 0;           // ent2: 64 output rows of 128, K = 64
+constexpr int C_COMB = 1;          // 2 chunks: combine, 128 outputs, K = 128
+constexpr int C_LAYER0 = 3;        // encoder layer l at C_LAYER0 + l * CL_CHUNKS
+constexpr int CL_QKV = 0;          // 6 chunks: 384 outputs (3 tiles), K = 128
+constexpr int CL_OUT = 6;          // 2 chunks: output projection, K = 128
+constexpr int CL_FF1 = 8;          // 4 chunks: 256 hidden units (2 tiles), K = 128
+constexpr int CL_FF2 = 12;         // 4 chunks: 128 outputs, K = 256
+constexpr int CL_CHUNKS = 16;
+constexpr int C_LPS = C_LAYER0 + 2 * CL_CHUNKS;  // the LPS weights (PL_* layout above)
+constexpr int LPS_CHUNKS = (LPS_W_ELEMS + kChunkElems - 1) / kChunkElems;
+constexpr int kChunks = C_LPS + LPS_CHUNKS;
+
+// element (m, k) of a 128 x 64 tile, in bf16 elements from the tile start
+__host__ __device__ constexpr int tile_off(int m, int k) {
+  return m * 64 + ((((k >> 3) ^ (m & 7)) << 3) | (k & 7));
+}
+
+// fp32 vectors, whole; then E_pos [32][128] as bf16 (S_POS, in floats)
+constexpr int S_ENT1W = 0, S_ENT1B = 64, S_ENT2B = 128, S_ENTLNG = 192, S_ENTLNB = 256;
+constexpr int S_TOKB = 320, S_COMBB = 384, S_HEADW = 512, S_HEADB = 640;
+constexpr int S_LAYER0 = 656, S_LAYER_STRIDE = 1408;
+constexpr int SL_QKVB = 0, SL_OUTB = 384, SL_FF1B = 512, SL_FF2B = 768;
+constexpr int SL_LN1G = 896, SL_LN1B = 1024, SL_LN2G = 1152, SL_LN2B = 1280;
+constexpr int S_LPS = S_LAYER0 + 2 * S_LAYER_STRIDE;  // the LPS vectors (VP_* layout above)
+constexpr int S_POS = S_LPS + 1008;
+constexpr int S_ELEMS = S_POS + kPosRows * 128 / 2;
+
+static_assert(S_LPS + VP_LAYER0 + 2 * VP_LAYER_STRIDE <= S_POS, "vector layout");
+static_assert(S_LAYER0 % 4 == 0 && S_LAYER_STRIDE % 4 == 0 && S_LPS % 4 == 0 &&
+                  S_POS % 4 == 0 && (S_ELEMS * 4) % 16 == 0,
+              "float4 alignment of LayerNorm vectors, bulk copy size");
+static_assert(LPS_CHUNKS == 3, "the LPS weights take three chunks");
+
+}  // namespace rcta
+
 }  // namespace rimg
 }  // namespace ebd
