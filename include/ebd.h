@@ -41,7 +41,10 @@
  *     rows of a step <= max_rows <= 4096.  Anything else returns
  *     EBD_ERR_UNSUPPORTED.
  *   - max_window <= 64: the decision runs as one thread-block cluster per
- *     sequence.  max_window > 64 (the full-sequence setting, where every
+ *     sequence; with max_window <= 32, a launch of 16 or more sequences runs
+ *     it as one CTA per sequence instead (the same results; the environment
+ *     variable EBD_DECIDE_KERNEL = "cta" or "cluster" forces either kernel
+ *     for max_window <= 32).  max_window > 64 (the full-sequence setting, where every
  *     position of the response is a row, App. E with M = all masked
  *     positions): the decision runs as a chain of grid-wide kernels, and a
  *     step takes no window attention (attn_out and kv_append must be unset:
