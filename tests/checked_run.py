@@ -14,9 +14,9 @@ def run_cases():
     from paper_2609_16450_gb300 import _ebd as E
     from paper_2609_16450_gb300 import runtime as rt
     from tests import guards
-    from tests.test_gpu_guards import CASES
+    from tests.test_gpu_guards import CASES, decide_kernel
     res = {}
-    for name, state, attention, append in CASES:
+    for name, state, attention, append, kernel in CASES:
         sh = synth.SHAPES[name]
         inp = synth.make_step_inputs(sh)
         if state == "inblock":
@@ -26,8 +26,10 @@ def run_cases():
         try:
             if name != "tiny":
                 w = rt.pack_weights(h, w)
-            status, out, g = guards.guarded_step(E, rt, h, inp, w, attention=attention, append=append)
-            key = f"{name}_{state}"
+            with decide_kernel(kernel):
+                status, out, g = guards.guarded_step(E, rt, h, inp, w, attention=attention,
+                                                     append=append)
+            key = f"{name}_{state}" + (f"_{kernel}" if kernel else "")
             res[key + "/status"] = np.array(status)
             res[key + "/guards"] = np.array(all(v.intact() for v in g.values()))
             for k, v in out.items():

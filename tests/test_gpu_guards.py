@@ -1,6 +1,11 @@
 """Guard words around every buffer a step writes (outputs, decode state,
 K/V cache with the append), checked after steps of the tiny, LLaDA-8B and
-Dream-7B shapes, with and without an active block, on both decision paths."""
+Dream-7B shapes, with and without an active block, on the cluster and the
+grid-wide decision paths and, forced with EBD_DECIDE_KERNEL, on the one-CTA
+decision kernel."""
+import contextlib
+import os
+
 import numpy as np
 import pytest
 
@@ -11,13 +16,35 @@ pytestmark = pytest.mark.gpu
 
 torch = pytest.importorskip("torch")
 
-CASES = [("tiny", "select", True, False), ("tiny", "inblock", True, True),
-         ("llada8b", "select", True, False), ("dream7b", "select", True, True),
-         ("tiny_full", "select", False, False), ("tiny_full", "inblock", False, False)]
+# (shape, state, window attention, cache append, decision kernel forced or "")
+CASES = [("tiny", "select", True, False, ""), ("tiny", "inblock", True, True, ""),
+         ("llada8b", "select", True, False, ""), ("dream7b", "select", True, True, ""),
+         ("tiny_full", "select", False, False, ""), ("tiny_full", "inblock", False, False, ""),
+         ("tiny", "select", True, False, "cta"), ("tiny", "inblock", True, True, "cta"),
+         ("llada8b", "select", True, False, "cta")]
 
 
-@pytest.mark.parametrize("name,state,attention,append", CASES)
-def test_step_writes_stay_inside_its_buffers(name, state, attention, append):
+@contextlib.contextmanager
+def decide_kernel(kernel):
+    """EBD_DECIDE_KERNEL set to `kernel` (unset for "") inside the block."""
+    old = os.environ.pop("EBD_DECIDE_KERNEL", None)
+    if kernel:
+        os.environ["EBD_DECIDE_KERNEL"] = kernel
+    try:
+        yield
+    finally:
+        os.environ.pop("EBD_DECIDE_KERNEL", None)
+        if old is not None:
+            os.environ["EBD_DECIDE_KERNEL"] = old
+
+
+@pytest.mark.parametrize("name,state,attention,append,kernel", CASES)
+def test_step_writes_stay_inside_its_buffers(name, state, attention, append, kernel):
+    with decide_kernel(kernel):
+        _guarded(name, state, attention, append)
+
+
+def _guarded(name, state, attention, append):
     from paper_2609_16450_gb300 import _ebd as E
     from paper_2609_16450_gb300 import runtime as rt
     sh = synth.SHAPES[name]
