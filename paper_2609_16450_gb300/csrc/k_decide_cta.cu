@@ -702,7 +702,7 @@ __device__ __noinline__ void decide_window(int q, bool lbs) {
           bj = oj;
         }
       }
-      if (lane == 0) sm.f_acc[bj] = 1;
+      if (lane == 0 && bj < nr) sm.f_acc[bj] = 1;
     }
     __syncwarp();
     bool open = false;
