@@ -535,8 +535,8 @@ def oracle_step_sample(sh, inp, budget_s, suffix=None):
 
 def parity_summary(sh, inp, res, gpu, tol=2e-3):
     """The GPU step's outputs (one step from the same state) against the
-    oracle's: near-ties counted as the benchmark spec defines them (top-2 logit gap,
-    or a decision margin, below 1e-3), argmax mismatches outside near-ties,
+    oracle's: near-ties counted (a top-2 logit gap, or a decision margin,
+    below 1e-3), argmax mismatches outside near-ties,
     decision mismatches in sequences the oracle does not flag, and the
     largest differences of the floating-point outputs."""
     NT = 1e-3
