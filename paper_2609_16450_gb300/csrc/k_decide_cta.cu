@@ -152,13 +152,6 @@ __device__ __forceinline__ void b_store2(uint8_t* buf, int r, int k, float x, fl
   *reinterpret_cast<uint32_t*>(buf + b_off(r, k)) = hi;
   *reinterpret_cast<uint32_t*>(buf + b_off(r + 32, k)) = lo;
 }
-// x as column k of activation row r
-__device__ __forceinline__ void b_store1(uint8_t* buf, int r, int k, float x) {
-  const __nv_bfloat16 h = __float2bfloat16_rn(x);
-  const __nv_bfloat16 l = __float2bfloat16_rn(x - __bfloat162float(h));
-  *reinterpret_cast<__nv_bfloat16*>(buf + b_off(r, k)) = h;
-  *reinterpret_cast<__nv_bfloat16*>(buf + b_off(r + 32, k)) = l;
-}
 
 // One unit of the LBS attention: query rows [16 qt, 16 qt + 16) of head h
 // (width 32) over all n <= 32 keys, output columns [16 hf, 16 hf + 16) of
@@ -344,10 +337,13 @@ __device__ __forceinline__ void mma_wait(CtaSmem& sm, uint32_t parity) {
   tc_fence_after();
 }
 
-// The epilogue of T accumulator tiles: epi(r, f, value) for output feature
-// f = 128 t + (TMEM lane) < fmax and row r < n, value = W hi + W lo of that
-// row (columns r and 32 + r).  Warpgroup g takes the (tile, 8-row group)
-// units g, g + 4, ...; a warp reads its TMEM lane quadrant.
+// The epilogue of T accumulator tiles: epi(r, f, x, y) for the output
+// features f and f + 1 (f even, < fmax, a multiple of 64) of row r < n,
+// each value W hi + W lo of that row (columns r and 32 + r).  Warpgroup g
+// takes the (tile, 8-row group) units g, g + 4, ...; a warp reads its TMEM
+// lane quadrant (a lane one feature, 8 rows), then lanes 2k and 2k + 1 swap
+// halves so that each holds 4 rows of the feature pair: stores of two
+// adjacent bf16 or fp32 values.
 template <class Epi>
 __device__ __forceinline__ void mma_epilogue(const CtaSmem& sm, int T, int n, int fmax, Epi epi) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -369,11 +365,17 @@ __device__ __forceinline__ void mma_epilogue(const CtaSmem& sm, int T, int n, in
         : "r"(ta), "r"(ta + 32u)
         : "memory");
     const int f = 128 * t + 32 * quad + lane;
-    if (f >= fmax) continue;
+    if (f >= fmax) continue;  // the whole warp: fmax is a multiple of 64
+    const bool odd = (lane & 1) != 0;
+    const int fe = f & ~1;
 #pragma unroll
-    for (int i = 0; i < 8; ++i) {
-      const int r = 8 * g8 + i;
-      if (r < n) epi(r, f, __uint_as_float(rh[i]) + __uint_as_float(rl[i]));
+    for (int i = 0; i < 4; ++i) {
+      const float lo_row = __uint_as_float(rh[i]) + __uint_as_float(rl[i]);          // row i
+      const float hi_row = __uint_as_float(rh[4 + i]) + __uint_as_float(rl[4 + i]);  // row 4 + i
+      const float got = __shfl_xor_sync(0xffffffffu, odd ? lo_row : hi_row, 1);
+      // even lane: row i of features (f, f + 1); odd lane: row 4 + i of (f - 1, f)
+      const int r = 8 * g8 + (odd ? 4 + i : i);
+      if (r < n) epi(r, fe, odd ? got : lo_row, odd ? hi_row : got);
     }
   }
 }
@@ -430,7 +432,9 @@ __device__ __noinline__ void lbs_forward(int n, int q) {
   if (tid == 0) mma_issue(sm, q, 1, 1, br);
   mma_wait(sm, ph);
   ph ^= 1u;
-  mma_epilogue(sm, 1, n, 64, [&](int r, int f, float v) { Z[r * LDZ + f] = v + Vv[S_ENT2B + f]; });
+  mma_epilogue(sm, 1, n, 64, [&](int r, int f, float x, float y) {
+    *reinterpret_cast<float2*>(Z + r * LDZ + f) = make_float2(x + Vv[S_ENT2B + f], y + Vv[S_ENT2B + f + 1]);
+  });
   tc_fence_before();
   __syncthreads();
   // 3. e = LayerNorm(ent2) -> columns 0..63 of [e; t], t -> 64..127
@@ -449,10 +453,11 @@ __device__ __noinline__ void lbs_forward(int n, int q) {
   if (tid == 0) mma_issue(sm, q + 1, 1, 2, bx);
   mma_wait(sm, ph);
   ph ^= 1u;
-  mma_epilogue(sm, 1, n, 128, [&](int r, int f, float v) {
-    const float z = v + Vv[S_COMBB + f] + __bfloat162float(pos[r * 128 + f]);
-    Z[r * LDZ + f] = z;
-    b_store1(bz, r, f, z);
+  mma_epilogue(sm, 1, n, 128, [&](int r, int f, float x, float y) {
+    const float2 pe = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(pos + r * 128 + f));
+    const float z0 = x + Vv[S_COMBB + f] + pe.x, z1 = y + Vv[S_COMBB + f + 1] + pe.y;
+    *reinterpret_cast<float2*>(Z + r * LDZ + f) = make_float2(z0, z1);
+    b_store2(bz, r, f, z0, z1);
   });
   fence_proxy_async_smem();
   tc_fence_before();
@@ -470,8 +475,8 @@ __device__ __noinline__ void lbs_forward(int n, int q) {
     }
     mma_wait(sm, ph);
     ph ^= 1u;
-    mma_epilogue(sm, 3, n, 384, [&](int r, int f, float v) {
-      b_store1(f < 128 ? bq : (f < 256 ? bk : bv), r, f & 127, v + Vl[SL_QKVB + f]);
+    mma_epilogue(sm, 3, n, 384, [&](int r, int f, float x, float y) {
+      b_store2(f < 128 ? bq : (f < 256 ? bk : bv), r, f & 127, x + Vl[SL_QKVB + f], y + Vl[SL_QKVB + f + 1]);
     });
     // v rows n..31: zeros (the products with key blocks that end past n read them)
 #pragma unroll 1
@@ -493,7 +498,11 @@ __device__ __noinline__ void lbs_forward(int n, int q) {
     if (tid == 0) mma_issue(sm, q, 1, 2, bx);
     mma_wait(sm, ph);
     ph ^= 1u;
-    mma_epilogue(sm, 1, n, 128, [&](int r, int f, float v) { Z[r * LDZ + f] += v + Vl[SL_OUTB + f]; });
+    mma_epilogue(sm, 1, n, 128, [&](int r, int f, float x, float y) {
+      float2* z = reinterpret_cast<float2*>(Z + r * LDZ + f);
+      const float2 zz = *z;
+      *z = make_float2(zz.x + (x + Vl[SL_OUTB + f]), zz.y + (y + Vl[SL_OUTB + f + 1]));
+    });
     tc_fence_before();
     __syncthreads();
     q += 2;
@@ -506,7 +515,9 @@ __device__ __noinline__ void lbs_forward(int n, int q) {
     if (tid == 0) mma_issue(sm, q, 2, 2, bz);
     mma_wait(sm, ph);
     ph ^= 1u;
-    mma_epilogue(sm, 2, n, 256, [&](int r, int f, float v) { b_store1(br, r, f, gelu(v + Vl[SL_FF1B + f])); });
+    mma_epilogue(sm, 2, n, 256, [&](int r, int f, float x, float y) {
+      b_store2(br, r, f, gelu(x + Vl[SL_FF1B + f]), gelu(y + Vl[SL_FF1B + f + 1]));
+    });
     fence_proxy_async_smem();
     tc_fence_before();
     __syncthreads();
@@ -518,7 +529,11 @@ __device__ __noinline__ void lbs_forward(int n, int q) {
     }
     mma_wait(sm, ph);
     ph ^= 1u;
-    mma_epilogue(sm, 1, n, 128, [&](int r, int f, float v) { Z[r * LDZ + f] += v + Vl[SL_FF2B + f]; });
+    mma_epilogue(sm, 1, n, 128, [&](int r, int f, float x, float y) {
+      float2* z = reinterpret_cast<float2*>(Z + r * LDZ + f);
+      const float2 zz = *z;
+      *z = make_float2(zz.x + (x + Vl[SL_FF2B + f]), zz.y + (y + Vl[SL_FF2B + f + 1]));
+    });
     tc_fence_before();
     __syncthreads();
     q += 4;
