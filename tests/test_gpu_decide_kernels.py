@@ -12,7 +12,9 @@ EBD_DECIDE_KERNEL (without it, the launch's batch size picks the kernel).
 * the router branches forced both ways by the head biases, EOS removal;
 * the baselines' threshold and Top-m rules;
 * sweep points of 16 and 64 sequences, where the batch rule picks the
-  one-CTA kernel."""
+  one-CTA kernel;
+* ebd_decide (statistics as inputs) on a step's own statistics takes that
+  step's decision bit for bit."""
 import numpy as np
 import pytest
 
@@ -107,3 +109,33 @@ def test_baseline_modes(kernel, mode, top_m):
 @pytest.mark.parametrize("point", [(16, 256, 32), (64, 256, 8)])
 def test_many_sequences(kernel, point):
     C.test_sweep_point(point)
+
+
+@pytest.mark.parametrize("state", ["select", "inblock"])
+def test_decide_entry_takes_the_steps_decision(kernel, state):
+    """ebd_decide (statistics as inputs) on the statistics a step produced, from
+    the same decode state, takes exactly that step's decision."""
+    from paper_2609_16450_gb300 import _ebd as E
+    from paper_2609_16450_gb300 import runtime as rt
+    sh = synth.llada
+    inp = synth.make_step_inputs(sh)
+    if state == "inblock":
+        synth.preset_in_block(inp, 20)
+    w = rt.upload_weights(inp)
+    h = rt.Handle(rt.config_for(sh), w.w_emb)
+    try:
+        ds = rt.DeviceStep(inp, w, attention=False)
+        E.check(E.ebd_step(h.h, ds.args(), rt.stream_handle(None)), h.h)
+        assert h.sync_status() == 0
+        step = ds.fetch()
+        ds.restore_state()
+        E.check(E.ebd_decide(h.h, ds.args(), rt.stream_handle(None)), h.h)
+        assert h.sync_status() == 0
+        dec = ds.fetch()
+        for k in ("tokens", "mask", "in_block", "blk_meta", "accepted"):
+            np.testing.assert_array_equal(dec[k], step[k], err_msg=k)
+        for k in ("lbs_logit", "lps_prob"):
+            np.testing.assert_array_equal(dec[k], step[k], err_msg=k)  # NaN where not scored
+        assert step["accepted"].sum() >= 1
+    finally:
+        h.close()
