@@ -227,7 +227,6 @@ __device__ __forceinline__ void lbs_attention(cg::cluster_group& cluster, float*
 }
 
 
-
 }  // namespace
 
 __global__ void __cluster_dims__(kDecideCluster, 1, 1) __launch_bounds__(kDecideThreads, 1)
@@ -281,8 +280,6 @@ __global__ void __cluster_dims__(kDecideCluster, 1, 1) __launch_bounds__(kDecide
   // shared-memory access; this also orders the block-level setup above
   cluster.sync();
   const int r0 = sm.r0, nr = sm.n_rows;
-  // meta_s as read from the decode state (rank 0 changes it only after the LBS)
-  const bool lbs_possible = p.mode == EBD_DECODE_EB && sm.meta_s == 0;
 
 #pragma unroll 1
   for (int j = tid; j < nr; j += blockDim.x) {
@@ -324,27 +321,9 @@ __global__ void __cluster_dims__(kDecideCluster, 1, 1) __launch_bounds__(kDecide
       sm.f_bad[j] = !(isfinite(c) && isfinite(e) && isfinite(g)) || a < 0 || a >= p.V;
     }
   } else {
-    // With the LBS possible, row j is merged by warp (j / 8) of rank (j % 8)
-    // and broadcast to every rank.  Otherwise (a block is active, or a
-    // baseline rule) only rank 0 needs the statistics: it merges every row
-    // itself, one per warp at a time, and no cluster barrier follows, so the
-    // other ranks' stand-in runs no longer hold it up; they take finite
-    // stand-in statistics.  One loop serves both, keeping the code compact.
-    const bool solo = !lbs_possible;
-    if (solo && rank != 0) {
+    // row j is merged by warp (j / 8) of rank (j % 8) and broadcast
 #pragma unroll 1
-      for (int j = tid; j < nr; j += blockDim.x) {
-        sm.f_conf[j] = 0.5f;
-        sm.f_ent[j] = 0.5f;
-        sm.f_gap[j] = 0.1f;
-        sm.f_arg[j] = j % p.V;
-        sm.f_bad[j] = 0;
-      }
-    }
-    const int nw = blockDim.x >> 5;
-    const int jstep = solo ? nw : kDecideCluster * nw;
-#pragma unroll 1
-    for (int j = solo ? (rank == 0 ? warp : nr) : warp * kDecideCluster + rank; j < nr; j += jstep) {
+    for (int j = warp * kDecideCluster + rank; j < nr; j += kDecideCluster * (blockDim.x >> 5)) {
       const size_t base = static_cast<size_t>(r0 + j) * p.grid_lm;
       float m = -INFINITY, s = 0.f, t = 0.f, l2 = -INFINITY;
       int idx = INT_MAX;
@@ -383,8 +362,8 @@ __global__ void __cluster_dims__(kDecideCluster, 1, 1) __launch_bounds__(kDecide
         if (p.argmax) p.argmax[r] = bad ? -1 : idx;
         if (bad) atomicCAS(p.status, 0, EBD_ERR_NONFINITE);
       }
-      if (lane < (solo ? 1 : kDecideCluster)) {
-        Smem* dst = cluster.map_shared_rank(&sm, solo ? rank : lane);
+      if (lane < kDecideCluster) {
+        Smem* dst = cluster.map_shared_rank(&sm, lane);
         dst->f_conf[j] = conf;
         dst->f_ent[j] = entn;
         dst->f_gap[j] = gap;
@@ -396,13 +375,7 @@ __global__ void __cluster_dims__(kDecideCluster, 1, 1) __launch_bounds__(kDecide
   // the weight copy must have landed before any use (and before exit)
   if (!mbar_wait(&sm.bar, 0, 1000ull * 1000 * 1000, nullptr) && tid == 0)
     atomicCAS(p.status, 0, EBD_ERR_TIMEOUT);
-  // with the LBS possible, every rank has pushed its rows' statistics to all
-  // (and the LBS exchanges follow); otherwise no rank touches another's
-  // shared memory from here on
-  if (lbs_possible)
-    cluster.sync();
-  else
-    __syncthreads();
+  cluster.sync();
 
   // ---------------------------------------------------------------- 2. masked set
   if (warp == 0) {
@@ -762,7 +735,7 @@ __global__ void __cluster_dims__(kDecideCluster, 1, 1) __launch_bounds__(kDecide
           bj = oj;
         }
       }
-      if (lane == 0 && bj < nr) sm.f_acc[bj] = 1;
+      if (lane == 0) sm.f_acc[bj] = 1;
     }
     __syncwarp();
     bool open = false;
