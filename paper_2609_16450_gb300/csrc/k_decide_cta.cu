@@ -90,6 +90,12 @@ static_assert(offsetof(CtaSmem, pool) % 1024 == 0, "B operands on 1024-byte boun
 extern __shared__ __align__(1024) uint8_t cta_dsmem[];
 __device__ __forceinline__ CtaSmem& cta_smem() { return *reinterpret_cast<CtaSmem*>(cta_dsmem); }
 
+// Orders this thread's earlier shared-memory accesses (generic proxy) before
+// later accesses by the async proxy (bulk copies, tcgen05.mma operand reads).
+__device__ __forceinline__ void fence_proxy_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
 __device__ __forceinline__ void bulk_copy_keep(void* smem_dst, const void* gsrc, uint32_t bytes,
                                                uint64_t* bar, uint64_t policy) {
   asm volatile(
