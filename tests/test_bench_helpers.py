@@ -115,3 +115,12 @@ def test_kernel_hash_ignores_comments_only():
     h0 = b.lm_kernel_hash(base)
     assert b.lm_kernel_hash(lambda f: "// a note\n/* and\n another */\n" + base(f) + "\n// end\n") == h0
     assert b.lm_kernel_hash(lambda f: base(f).replace("kUnit", "kUnit ", 1) + "\nint x;\n") != h0
+
+
+def test_headline_profile_matches_the_lm_head_sources():
+    """The committed ncu capture of the headline LM head was taken on the
+    current LM-head sources (else bench.py reports no traffic): a code change
+    to k_lmhead.cu, ptx.cuh or lm_params.h needs a new capture."""
+    b = _bench()
+    t = b.profiled_traffic("llada8b")
+    assert t is not None and t > 1.0e9
