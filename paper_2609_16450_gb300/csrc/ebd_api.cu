@@ -209,6 +209,7 @@ struct ebd_handle {
   float* attn_part_ml = nullptr;
   int* tickets = nullptr;
   int attn_splits = 1, attn_max_qtiles = 1;
+  int attn_tc = 1;         // window attention on tcgen05 (else the mma.sync kernel)
   int* d_status = nullptr;
   uint8_t* staging = nullptr;
   size_t staging_bytes = 0;
@@ -705,6 +706,7 @@ ebd_status run_attention(ebd_handle* h, const ebd_step_args* a, cudaStream_t st,
   p.max_prefix = c.max_prefix;
   p.max_qtiles = h->attn_max_qtiles;
   p.splits = h->attn_splits;
+  p.tc = h->attn_tc;
   p.cu_rows = a->cu_rows;
   p.prefix_len = a->prefix_len;
   p.suffix = c.max_prefix > 0 ? a->suffix : nullptr;
@@ -983,21 +985,46 @@ ebd_status ebd_create(const ebd_config* cfg, ebd_handle** out) {
     return bail(cuda_fail(h, e, "cudaMalloc(partials)"));
   // attention split-KV workspace
   {
+    // Both attention kernels take 64-row query tiles.  The tcgen05 kernel
+    // holds an SM alone (one CTA per SM) and pays a fixed setup and drain
+    // per CTA (TMEM, barriers, the query tile, its output), which long key
+    // ranges amortise; the mma.sync kernel runs two CTAs per SM and keeps
+    // launches of many short key ranges (measured, attention alone, LLaDA-8B
+    // heads, us, mma.sync against tcgen05: 16 x 256 x 32 rows 41.6 / 47.8,
+    // 64 x 1024 x 8 211.6 / 230.0; but 16 x 4096 x 32 305.8 / 203.4,
+    // 64 x 4096 x 32 1032.9 / 690.8, 4 x 1024 x 32 45.7 / 27.3, LLaDA-8B
+    // 21.2 / 17.1, Dream-7B 53.9 / 39.6).  EBD_ATTN_KERNEL=tc|mma forces one,
+    // EBD_ATTN_SPLITS the split count (measurement sweeps).
+    const int tile = 64;
     const int group = cfg->n_heads_q / cfg->n_heads_kv;
     const int aw = cfg->max_window < kMaxWindow ? cfg->max_window : kMaxWindow;
-    h->attn_max_qtiles = (aw * group + 63) / 64;
+    h->attn_max_qtiles = (aw * group + tile - 1) / tile;
     const int slots = cfg->max_batch * cfg->n_heads_kv * h->attn_max_qtiles;
     const int nch = (cfg->max_prefix + kAttnChunk - 1) / kAttnChunk + 1;
-    int splits = (2 * h->num_sms + slots - 1) / slots;
+    h->attn_tc = (slots <= 2 * h->num_sms || nch >= 65 || (nch >= 17 && aw >= 32)) ? 1 : 0;
+    if (const char* env = getenv("EBD_ATTN_KERNEL")) h->attn_tc = strcmp(env, "mma") == 0 ? 0 : 1;
+    int splits;
+    if (h->attn_tc) {
+      // one split, unless few tiles leave most SMs idle: then about one
+      // CTA per SM, but at least 8 key chunks per split
+      splits = 1;
+      if (2 * slots < h->num_sms) {
+        splits = (h->num_sms + slots - 1) / slots;
+        if (splits > nch / 8) splits = nch / 8;
+      }
+    } else {
+      splits = (2 * h->num_sms + slots - 1) / slots;
+    }
+    if (const char* env = getenv("EBD_ATTN_SPLITS")) splits = atoi(env);
     if (splits > kMaxSplits) splits = kMaxSplits;
     if (splits > nch) splits = nch;
     if (splits < 1) splits = 1;
     h->attn_splits = splits;
     if (splits > 1) {
-      const size_t bytes = static_cast<size_t>(slots) * splits * 64 * (cfg->head_dim + 2) * 4;
+      const size_t bytes = static_cast<size_t>(slots) * splits * tile * (cfg->head_dim + 2) * 4;
       if ((e = cudaMalloc(&h->attn_part, bytes)) != cudaSuccess)
         return bail(cuda_fail(h, e, "cudaMalloc(attention partials)"));
-      h->attn_part_ml = h->attn_part + static_cast<size_t>(slots) * splits * 64 * cfg->head_dim;
+      h->attn_part_ml = h->attn_part + static_cast<size_t>(slots) * splits * tile * cfg->head_dim;
     }
     if ((e = cudaMalloc(&h->tickets, static_cast<size_t>(slots) * sizeof(int))) != cudaSuccess)
       return bail(cuda_fail(h, e, "cudaMalloc(tickets)"));

@@ -41,6 +41,8 @@ constexpr int kAttnThreads = 128;
 constexpr int kAttnChunk = 64;        // keys per K/V tile
 constexpr int kAttnStages = 3;
 constexpr int kMaxAttnSplits = 8;
+constexpr int kAttnTcThreads = 352;   // tcgen05 attention: K and V load warps, MMA warp, 8 softmax warps
+constexpr int kAttnTcRows = 64;       // query rows per tile of the tcgen05 attention
 
 // ------------------------------------------------------------------ attention
 struct AttnParams {
@@ -48,13 +50,14 @@ struct AttnParams {
   int R;                    // rows of the step (extent of q and out)
   int max_prefix;
   int max_qtiles, splits;
+  int tc;                   // 1: the tcgen05 kernel, 0: the mma.sync kernel (64-row tiles)
   const int* cu_rows;
   const int* prefix_len;
   const int* suffix;        // [B][2] {s0, S} cached keys after the window, or null
   const __nv_bfloat16* q;   // [R][Hq][D]
   float* out;               // [R][Hq][D]
-  float* part;              // [B*Hkv*max_qtiles*splits][64][D] unnormalised O
-  float* part_ml;           // [B*Hkv*max_qtiles*splits][64][2] (max, sum) in log2 units
+  float* part;              // [B*Hkv*max_qtiles*splits][tile rows][D] unnormalised O
+  float* part_ml;           // [B*Hkv*max_qtiles*splits][tile rows][2] (max, sum) in log2 units
   int* tickets;             // [B*Hkv*max_qtiles]
   int* status;
   uint64_t limit_ns;
