@@ -278,7 +278,13 @@ ebd_status ebd_lm_shard_state(ebd_handle* h, const ebd_step_args* a, int32_t v_o
 ebd_status ebd_merge_shard_states(ebd_handle* h, const float* states, int32_t shards,
                                   const ebd_step_args* a, void* stream);
 
-/* Only step 1 (window attention): writes a->attn_out. */
+/* Only step 1 (window attention): writes a->attn_out.  The handle picks one
+ * of two kernels when it is created: the tcgen05 kernel (S and O in tensor
+ * memory, one CTA per SM) for long key ranges or launches of few query
+ * tiles, the mma.sync kernel (two CTAs per SM) for many tiles with short key
+ * ranges; both compute the same attention.  The environment variables
+ * EBD_ATTN_KERNEL = "tc" or "mma" and EBD_ATTN_SPLITS (key splits per query
+ * tile, 1..8), read at ebd_create, override the choices. */
 ebd_status ebd_attention(ebd_handle* h, const ebd_step_args* a, void* stream);
 
 /* Synchronises `stream`, returns the first device-side failure recorded
