@@ -10,6 +10,8 @@ the window; Sec. 6.3: prefix and dual cache).
 * Dream-7B heads (GQA 28 / 4, up to 448 query rows per kv head: several
   query tiles), ragged windows, a suffix per sequence;
 * degenerate windows: no prefix, one row, splits that get no key chunk;
+* 64-dim heads with GQA 8 / 2 at the query-tile boundaries (64, 65, 128 and 4
+  query rows per kv head) and ragged;
 * sixteen sequences (one split per tile) and a long prefix (4096);
 * the key range forced into 3 and 8 splits per query tile;
 * scores that grow from chunk to chunk by far more than the tcgen05 kernel's
@@ -146,3 +148,17 @@ def test_key_splits(kernel, monkeypatch, splits):
     sh = synth.tiny.with_(name="attn_edge", batch=6, windows=(0, 1, 64, 7, 20, 33), seed=23)
     inp = synth.make_step_inputs(sh, weights=False, prefix_lens=np.array([128, 0, 128, 5, 64, 1]))
     _check(f"degenerate splits={splits}", inp)
+
+
+@pytest.mark.parametrize("windows", [(32, 33, 64, 1), (31, 17, 48, 40)])
+def test_gqa_tile_boundaries(kernel, windows):
+    """64-dim heads with GQA 8 / 2 (4 query heads per kv head): windows of
+    32, 33, 64 and 1 rows give 128, 132, 256 and 4 query rows per kv head,
+    i.e. tiles of exactly 64 rows, a tile of 4 after two full ones, and a
+    lone short tile (the tcgen05 kernel repeats 32- and 64-row tiles over
+    its lane quadrants differently); the second set is ragged throughout."""
+    sh = synth.tiny.with_(name="attn_gqa", batch=len(windows), windows=windows,
+                          n_heads_q=8, n_heads_kv=2, seed=31)
+    inp = synth.make_step_inputs(sh, weights=False,
+                                 prefix_lens=np.array([128, 77, 0, 128][:len(windows)]))
+    _check(f"gqa {windows}", inp)
