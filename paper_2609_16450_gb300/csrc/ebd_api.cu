@@ -176,17 +176,17 @@ bool encode_bf16(CUtensorMap* m, const void* base, int rank, const uint64_t* dim
 
 // Tensor map of W_lm in boxes of 64 columns by 64 rows: row-major [V][d], or
 // the packed layout ([unit][k-box][64 rows][64 columns], ebd_pack_lm_head).
-// For CTA pairs (pair_boxes) the packed layout is read as a 3-D tensor
-// (column, row of the unit's k-box rows, unit) in boxes of two units: one box
-// is a CTA's 128 W rows of one k-box.
-bool encode_w_lm(CUtensorMap* m, const void* w, int V, int d, bool packed, bool pair_boxes) {
+// For CTA pairs (pair_kbs > 0 k-boxes per stage) the packed layout is read as
+// a 4-D tensor (column, row, unit, k-box) in boxes of two units by pair_kbs
+// k-boxes: one box is a CTA's 128 W rows of a whole pipeline stage.
+bool encode_w_lm(CUtensorMap* m, const void* w, int V, int d, bool packed, int pair_kbs) {
   const uint64_t units = (static_cast<uint64_t>(V) + kUnit - 1) / kUnit;
   const uint64_t nkb = (static_cast<uint64_t>(d) + 63) / 64;
-  if (packed && pair_boxes) {
-    const uint64_t dims[3] = {64ull, nkb * 64, units};
-    const uint64_t str[2] = {128ull, nkb * 64 * 128};
-    const uint32_t box[3] = {64, 64, 2};
-    return encode_bf16(m, w, 3, dims, str, box);
+  if (packed && pair_kbs > 0) {
+    const uint64_t dims[4] = {64ull, 64ull, units, nkb};
+    const uint64_t str[3] = {128ull, nkb * 64 * 128, 64 * 128};
+    const uint32_t box[4] = {64, 64, 2, static_cast<uint32_t>(pair_kbs)};
+    return encode_bf16(m, w, 4, dims, str, box);
   }
   const uint64_t dims[2] = {packed ? 64ull : static_cast<uint64_t>(d),
                             packed ? units * nkb * 64 : static_cast<uint64_t>(V)};
@@ -760,9 +760,7 @@ ebd_status run_lm(ebd_handle* h, const ebd_step_args* a, cudaStream_t st, bool p
   const int V = v_count < 0 ? c.vocab : v_count;
   CUtensorMap tw;
   const bool packed = a->w_lm_layout == 1;
-  CUtensorMap tw3;  // the paired launches' view of packed W
-  if (!encode_w_lm(&tw, a->w_lm, V, c.d_model, packed, false) ||
-      !encode_w_lm(&tw3, a->w_lm, V, c.d_model, packed, true))
+  if (!encode_w_lm(&tw, a->w_lm, V, c.d_model, packed, 0))
     return fail(h, EBD_ERR_CUDA, "cuTensorMapEncodeTiled (W_lm) failed");
   for (int g0 = 0; g0 < a->rows; g0 += kMaxGroupRows) {
     const int rows = a->rows - g0 < kMaxGroupRows ? a->rows - g0 : kMaxGroupRows;
@@ -796,7 +794,10 @@ ebd_status run_lm(ebd_handle* h, const ebd_step_args* a, cudaStream_t st, bool p
     const uint32_t box[2] = {64, static_cast<uint32_t>(p.pair ? p.nb / 2 : p.nb)};
     if (!encode_bf16(&th, a->hidden, 2, dims, str, box))
       return fail(h, EBD_ERR_CUDA, "cuTensorMapEncodeTiled (hidden) failed");
-    cudaError_t e = launch_lm_stats(p.pair && packed ? tw3 : tw, th, p, st);
+    CUtensorMap tw4;  // the paired launches' view of packed W: one box per stage
+    if (p.pair && packed && !encode_w_lm(&tw4, a->w_lm, V, c.d_model, packed, p.kbs))
+      return fail(h, EBD_ERR_CUDA, "cuTensorMapEncodeTiled (W_lm) failed");
+    cudaError_t e = launch_lm_stats(p.pair && packed ? tw4 : tw, th, p, st);
     if (e != cudaSuccess) return cuda_fail(h, e, "LM-head launch");
     h->lm_ctas = p.grid;
   }
@@ -1822,7 +1823,7 @@ extern "C" ebd_status ebd_lm_stats_noalloc(const uint16_t* hidden, const uint16_
   CUtensorMap tw, th;
   (void)units;
   (void)nkb;
-  if (!encode_w_lm(&tw, w_lm, vocab, d_model, packed, false)) return EBD_ERR_CUDA;
+  if (!encode_w_lm(&tw, w_lm, vocab, d_model, packed, 0)) return EBD_ERR_CUDA;
   LmParams p{};
   lm_plan(p, rows, vocab, d_model,
           nd->num_sms < EBD_NOALLOC_MAX_PARTS ? nd->num_sms : EBD_NOALLOC_MAX_PARTS);

@@ -305,35 +305,33 @@ __global__ void __launch_bounds__(kLmThreads, 1)
         else
           tma_load_2d(dst, map, &full[s], x, y, pol);
       };
-      auto load3 = [&](void* dst, const CUtensorMap* map, int s, int x, int y, int z, uint64_t pol) {
-        if (PAIR)
-          tma_load_3d_pair(dst, map, mapa_shared(smem_u32(&full[s]), 0), x, y, z, pol);
-        else
-          tma_load_3d_hint(dst, map, &full[s], x, y, z, pol);
+      auto load4 = [&](void* dst, const CUtensorMap* map, int s, int z, int w, uint64_t pol) {
+        tma_load_4d_pair(dst, map, mapa_shared(smem_u32(&full[s]), 0), 0, 0, z, w, pol);
       };
       // stage fill: vocabulary chunk u (kChunkUnits units), k-stage ks; the
       // leader arms the stage for the W and hidden bytes of both CTAs.
-      // A pair reads packed W as a 3-D tensor (column, row of a unit's k-box
-      // rows, unit): one box of two units by one k-box is a CTA's 128 W rows
-      // of that k-box, 16 KB in one copy (the copies, not L2, set the paired
-      // kernel's operand feed: two 8 KB boxes per k-box took 1522 us against
-      // 1394 us for one 16 KB box at 64 x 32 rows).  A CTA with one unit of
-      // the chunk still reads two (the second is the next pair's, or zeros
-      // past the last unit) and its epilogue ignores the second.  Unpaired,
-      // HBM-bound launches read one unit at a time (no such extra reads).
+      // A pair reads packed W as a 4-D tensor (column, row, unit, k-box):
+      // one box of two units by the stage's kbs k-boxes is a CTA's 128 W
+      // rows of the whole stage in one copy, laid out as the MMAs read it
+      // (the copies, not L2, set the paired kernel's operand feed: at 64 x 32
+      // rows the LM head took 1522 us with two 8 KB boxes per k-box, 1394 us
+      // with one 16 KB box, 1317 us with one box per stage).  A CTA with one
+      // unit of the chunk still reads two (the second is the next pair's, or
+      // zeros past the last unit) and its epilogue ignores the second.
+      // Unpaired, HBM-bound launches read one unit at a time.
       auto issue_w = [&](int u, int ks, int s) {
         const int nu = min(kChunkUnits, u1 - u);
         const int nsubk = min(p.kbs, p.nkb - ks * p.kbs);
-        const uint32_t w_bytes = (PACKED && PAIR) ? (nu > 2 ? 2u : 1u) * (2u * kUnit * 128u)
-                                                  : static_cast<uint32_t>(nu) * kUnit * 128u;
+        // W bytes of the stage: one box of kbs k-boxes by two units per CTA
+        // with units in the chunk (a stage past the last k-box reads zeros)
+        const uint32_t w_bytes = (PACKED && PAIR)
+                                     ? (nu > 2 ? 2u : 1u) * static_cast<uint32_t>(p.kbs) * kATile
+                                     : static_cast<uint32_t>(nsubk * nu) * kUnit * 128u;
         if (leader)
-          mbar_arrive_expect_tx(&full[s], static_cast<uint32_t>(nsubk) *
-                                              (w_bytes + static_cast<uint32_t>(p.n_pad) * 128u));
+          mbar_arrive_expect_tx(&full[s], w_bytes + static_cast<uint32_t>(nsubk * p.n_pad) * 128u);
         uint8_t* a_st = sA + static_cast<size_t>(s) * a_stage;
         if (PACKED && PAIR) {
-          if (nu > ulo)
-            for (int j = 0; j < nsubk; ++j)
-              load3(a_st + j * kATile, &tmap_w, s, 0, (ks * p.kbs + j) * 64, u + ulo, pol_w);
+          if (nu > ulo) load4(a_st, &tmap_w, s, u + ulo, ks * p.kbs, pol_w);
         } else {
           // one unit at a time, its k-boxes back to back: each W row is
           // requested as one contiguous run of nsubk * 128 bytes

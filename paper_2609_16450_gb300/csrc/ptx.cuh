@@ -123,24 +123,15 @@ __device__ __forceinline__ void tma_load_3d(void* smem_dst, const void* tmap, ui
       "l"(tmap), "r"(x), "r"(y), "r"(z), "r"(smem_u32(bar))
       : "memory");
 }
-// 3-D tiled load with an L2 cache hint; and its cta_group::2 form (the bytes
-// counted on the mbarrier at cluster address `bar_cluster`).  x as in
-// tma_load_2d.
-__device__ __forceinline__ void tma_load_3d_hint(void* smem_dst, const void* tmap, uint64_t* bar,
-                                                 int32_t x, int32_t y, int32_t z, uint64_t policy) {
-  asm volatile(
-      "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint"
-      " [%0], [%1, {%2, %3, %4}], [%5], %6;" ::"r"(smem_u32(smem_dst)),
-      "l"(tmap), "r"(x), "r"(y), "r"(z), "r"(smem_u32(bar)), "l"(policy)
-      : "memory");
-}
-__device__ __forceinline__ void tma_load_3d_pair(void* smem_dst, const void* tmap,
+// 4-D tiled load for a CTA pair (cta_group::2): the bytes are counted on the
+// mbarrier at cluster address `bar_cluster`.  x as in tma_load_2d.
+__device__ __forceinline__ void tma_load_4d_pair(void* smem_dst, const void* tmap,
                                                  uint32_t bar_cluster, int32_t x, int32_t y,
-                                                 int32_t z, uint64_t policy) {
+                                                 int32_t z, int32_t w, uint64_t policy) {
   asm volatile(
-      "cp.async.bulk.tensor.3d.cta_group::2.shared::cluster.global.mbarrier::complete_tx::bytes"
-      ".L2::cache_hint [%0], [%1, {%2, %3, %4}], [%5], %6;" ::"r"(smem_u32(smem_dst)),
-      "l"(tmap), "r"(x), "r"(y), "r"(z), "r"(bar_cluster), "l"(policy)
+      "cp.async.bulk.tensor.4d.cta_group::2.shared::cluster.global.mbarrier::complete_tx::bytes"
+      ".L2::cache_hint [%0], [%1, {%2, %3, %4, %5}], [%6], %7;" ::"r"(smem_u32(smem_dst)),
+      "l"(tmap), "r"(x), "r"(y), "r"(z), "r"(w), "r"(bar_cluster), "l"(policy)
       : "memory");
 }
 __device__ __forceinline__ void tma_load_4d(void* smem_dst, const void* tmap, uint64_t* bar,
