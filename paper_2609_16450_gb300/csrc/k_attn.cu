@@ -447,7 +447,9 @@ __device__ __forceinline__ bool named_barrier_and(uint32_t id, uint32_t n, bool 
 // The same attention on the 5th-generation tensor cores.  A CTA takes 64
 // query rows of one (sequence, kv head) -- rows past the group's window
 // rows are zero -- and one split of the key chunks, in steps of 128 keys.
-//   warp 0: TMA producer, K and V tiles through two rings of 2 steps;
+//   warps 0 and 10: TMA loads of the K steps and of the V steps, each into
+//           its own ring of 2 steps (a K slot frees after its Q K^T, a V slot
+//           after its P V);
 //   warp 1: TMEM allocation and the MMA thread: S = Q K^T (M = 128, N = 128,
 //           both operands K-major) into one of two 128-column TMEM buffers,
 //           then O += P V with M = 128: rows 0..63 of P hold the
